@@ -1,0 +1,385 @@
+"""Benchmark of the PCS hot path on GB300.
+
+A step = one pass of the batched path over the windowed-KV population:
+checkpoint of every session (gather of the paged ring into contiguous PCS1
+records, fingerprint of every section fused into the copy, headers) and a
+verified restore into a freshly permuted page pool (scatter, fingerprints
+recomputed and checked), then delete.
+
+Workload (default): 256 sessions x 24 layers x 16 heads x 64, bf16 K and V,
+window 1024 tokens in 16-token pages randomly permuted in one pool, ring
+start ~ U[0,1023].  Algorithmic bytes per step: pack reads and writes
+25.77 GB, restore reads and writes 25.77 GB -> 103.1 GB.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl pcs|reference]
+                    [--sessions S] [--layers L] [--no-cpu-baseline] [--no-e2e]
+
+Prints one JSON line (rank 0).  Under torchrun each rank runs the same
+workload on its own GPU (sessions are independent: weak scaling, no data
+collective); the timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "snapshot+restore GB/s and sessions/s on 1 GB300; % of HBM (PCIe) roofline"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="pcs", choices=["pcs", "reference"])
+    ap.add_argument("--sessions", type=int, default=256)
+    ap.add_argument("--layers", type=int, default=24)
+    ap.add_argument("--heads", type=int, default=16)
+    ap.add_argument("--head-dim", type=int, default=64)
+    ap.add_argument("--window", type=int, default=1024)
+    ap.add_argument("--page-rows", type=int, default=16)
+    ap.add_argument("--no-verify", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+def workload_name(a) -> str:
+    return ("kv-window %d sessions x %d layers x %d heads x %d, bf16, window %d, %d-token pages"
+            % (a.sessions, a.layers, a.heads, a.head_dim, a.window, a.page_rows))
+
+
+def step_bytes(a) -> int:
+    """Algorithmic bytes per step: pack R+W and restore R+W of every section."""
+    sec = a.window * a.heads * a.head_dim * 2
+    meta = 32
+    payload = a.sessions * (2 * a.layers * sec + meta)
+    return 4 * payload
+
+
+def load_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            threading.Thread(target=self._read, daemon=True).start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle leg (bounded sample of the same workload)
+# ---------------------------------------------------------------------------
+
+def cpu_oracle_rate(a, seconds: float) -> dict:
+    """Oracle checkpoint + verified restore of whole sessions, one core."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_21686_gb300 import synth
+
+    oracle.build()
+    pages = a.window // a.page_rows
+    kv = synth.kv(seed=synth.seed_for(3), sessions=1, layers=a.layers, heads=a.heads,
+                  head_dim=a.head_dim, window=a.window, page_rows=a.page_rows, device="cpu")
+    kp = kv.k_pool.view(torch.int16).numpy().view(np.uint16)
+    vp = kv.v_pool.view(torch.int16).numpy().view(np.uint16)
+    pt = kv.page_table[0].numpy()
+    pt2 = synth.page_permutation(7, 1, a.layers, pages)[0].numpy()
+    kp2, vp2 = np.zeros_like(kp), np.zeros_like(vp)
+    meta = kv.meta[0].numpy().copy()
+    meta2 = np.zeros_like(meta)
+    per_session = step_bytes(a) // a.sessions
+    done, t0 = 0, time.perf_counter()
+    while True:
+        rec = oracle.pack(oracle.kv_session(0, meta, kp, vp, pt, kv.ring_start[0], a.window,
+                                            a.page_rows, kv.row_bytes))
+        t = oracle.kv_session(0, meta2, kp2, vp2, pt2, 0, a.window, a.page_rows, kv.row_bytes,
+                              ring_start_override=oracle.RING_START_FROM_RECORD)
+        assert oracle.restore(rec, t, verify=True) == 0
+        done += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or done >= 64:
+            break
+    gbs = done * per_session / el / 1e9
+    return {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": "%d whole session(s) of the same geometry (checkpoint + verified restore, "
+                      "%.1f MB each), %.1f s" % (done, per_session / 1e6, el),
+            "sessions_per_s": round(done / el, 4)}
+
+
+# ---------------------------------------------------------------------------
+# GPU leg
+# ---------------------------------------------------------------------------
+
+def run_reference(a, rank, world):
+    """The oracle timed on the host cores: K steps of a bounded sample each."""
+    if rank != 0:
+        return None
+    per_step = max(1.0, min(a.cpu_seconds, 120.0 / max(1, a.steps + a.warmup)))
+    for _ in range(a.warmup):
+        cpu_oracle_rate(a, per_step / 4)
+    rates = [cpu_oracle_rate(a, per_step) for _ in range(a.steps)]
+    v = statistics.median(r["value"] for r in rates)
+    sps = statistics.median(r["sessions_per_s"] for r in rates)
+    line = {"metric": METRIC, "value": v, "unit": "GB/s", "n_gpus": world, "steps": a.steps,
+            "warmup": a.warmup, "ms_per_step": round(a.sessions / sps * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": workload_name(a), "sessions": a.sessions,
+                       "l2": "inputs larger than L2"},
+            "sessions_per_s": sps,
+            "cpu_baseline": dict(rates[-1], value=v),
+            "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    return line
+
+
+def run_pcs(a, rank, world, local_rank):
+    from paper_2607_21686_gb300 import build, pcs, synth
+
+    build.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    ctx = pcs.Context(local_rank)
+    stream = torch.cuda.current_stream()
+    pages = a.window // a.page_rows
+
+    kv = synth.kv(seed=synth.seed_for(3) + 1000 * rank, sessions=a.sessions, layers=a.layers,
+                  heads=a.heads, head_dim=a.head_dim, window=a.window, page_rows=a.page_rows,
+                  device=dev)
+    pt2 = synth.page_permutation(synth.seed_for(3) + 7, a.sessions, a.layers, pages, device=dev)
+    k2, v2 = torch.empty_like(kv.k_pool), torch.empty_like(kv.v_pool)
+    meta2 = torch.empty_like(kv.meta)
+    src = [pcs.kv_session(s, kv.meta[s], kv.k_pool, kv.v_pool, kv.page_table[s], kv.ring_start[s],
+                          a.window) for s in range(a.sessions)]
+    dst = [pcs.kv_session(s, meta2[s], k2, v2, pt2[s], pcs.PCS_RING_START_FROM_SNAPSHOT,
+                          a.window) for s in range(a.sessions)]
+    verify = not a.no_verify
+
+    def step():
+        snaps = ctx.checkpoint(src)
+        ctx.restore(snaps, dst, verify=verify)
+        for s in snaps:
+            ctx.delete(s)
+
+    for _ in range(a.warmup):
+        step()
+    ctx.sync()
+    # Spot-check the restore of the warm-up (full parity lives in the tests).
+    s0 = 0
+    j = torch.arange(a.window, device=dev)
+    slot = (kv.ring_start[s0] + j) % a.window
+    for l in (0, a.layers - 1):
+        orig = kv.k_pool[kv.page_table[s0, l].long()[slot // a.page_rows], slot % a.page_rows]
+        back = k2[pt2[s0, l].long()[slot // a.page_rows], slot % a.page_rows]
+        assert torch.equal(orig, back), "restore mismatch"
+
+    launches0 = ctx.stats().kernel_launches
+    ctx.timing(True)
+    clocks = ClockSampler(local_rank)
+    clocks.start()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(a.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    ktimes = ctx.kernel_times()
+    ctx.timing(False)
+    launches = ctx.stats().kernel_launches - launches0
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # End to end through the public API with the state coming from host memory.
+    e2e = None
+    if not a.no_e2e:
+        e2e = run_e2e(a, ctx, kv, src, dst, stream, dev)
+
+    res = {"ms": ms, "ktimes": ktimes, "launches": launches, "clocks": clk, "e2e": e2e}
+    ctx.close()
+    return res
+
+
+def run_e2e(a, ctx, kv, src, dst, stream, dev):
+    """Each step: H2D of the KV pools from pinned memory, checkpoint, verified
+    restore, D2H of the session fingerprints; events on the same stream."""
+    from paper_2607_21686_gb300 import pcs
+
+    try:
+        kh = torch.empty(kv.k_pool.shape, dtype=kv.k_pool.dtype, pin_memory=True)
+        vh = torch.empty(kv.v_pool.shape, dtype=kv.v_pool.dtype, pin_memory=True)
+    except Exception as ex:  # pinned memory could not be had
+        return {"value": None, "unit": "GB/s", "note": "pinned allocation failed: %s" % ex}
+    kh.copy_(kv.k_pool)
+    vh.copy_(kv.v_pool)
+    fps_h = torch.empty(a.sessions, dtype=torch.int64, pin_memory=True)
+    fps_d = torch.empty(a.sessions, dtype=torch.int64, device=dev)
+    steps = max(2, min(a.steps, 5))
+
+    def one():
+        kv.k_pool.copy_(kh, non_blocking=True)
+        kv.v_pool.copy_(vh, non_blocking=True)
+        snaps = ctx.checkpoint(src)
+        ctx.restore(snaps, dst, verify=not a.no_verify)
+        for i, s in enumerate(snaps):
+            ctx.copy_out(s, 24, 8, fps_d[i:i + 1])
+        fps_h.copy_(fps_d, non_blocking=True)
+        for s in snaps:
+            ctx.delete(s)
+
+    one()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    h2d = kh.numel() * kh.element_size() * 2
+    d2h = fps_h.numel() * 8
+    del kh, vh
+    return {"value": round(step_bytes(a) / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms, 3),
+            "sessions_per_s": round(a.sessions / (ms / 1e3), 2), "steps": steps}
+
+
+def main():
+    a = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        backend = "nccl" if a.impl == "pcs" else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group(backend=backend)
+
+    if a.impl == "reference":
+        line = run_reference(a, rank, world)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return
+
+    r = run_pcs(a, rank, world, local_rank)
+    if rank == 0:
+        peaks = load_peaks()
+        bytes_step = step_bytes(a) * world
+        ms_step = r["ms"] / a.steps
+        gbs = bytes_step / (ms_step / 1e3) / 1e9
+        sps = a.sessions * world / (ms_step / 1e3)
+        # Roofline of the dominant kernel: pack or restore stream pass.
+        kt = r["ktimes"]
+        cand = {k: v for k, v in kt.items() if k.startswith("k_stream")}
+        top = max(cand, key=lambda k: cand[k][1]) if cand else None
+        roof = None
+        if top:
+            n_l, tot = cand[top]
+            per_launch_ms = tot / n_l
+            algo = step_bytes(a) // 2     # one pass: read + write of every payload byte
+            achieved = algo / (per_launch_ms / 1e3) / 1e9
+            roof = {"bound": "hbm", "kernel": top, "achieved": round(achieved, 1),
+                    "peak": peaks["hbm_gbs"], "peak_source": peaks["source"], "unit": "GB/s",
+                    "frac": round(achieved / peaks["hbm_gbs"], 4),
+                    "bytes_per_launch": algo, "ms_per_launch": round(per_launch_ms, 4),
+                    "traffic": None}
+        cpu = None
+        if not a.no_cpu_baseline:
+            cpu = cpu_oracle_rate(a, a.cpu_seconds)
+        line = {"metric": METRIC, "value": round(gbs, 2), "unit": "GB/s", "n_gpus": world,
+                "steps": a.steps, "warmup": a.warmup, "ms_per_step": round(ms_step, 4),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
+                "data": "synthetic",
+                "config": {"workload": workload_name(a), "sessions": a.sessions * world,
+                           "layers": a.layers, "verify": not a.no_verify,
+                           "l2": "inputs larger than L2 (24 GiB pools)"},
+                "sessions_per_s": round(sps, 2),
+                "frac_of_nominal_8tbs": round(gbs / 8000.0, 4),
+                "roofline": roof, "cpu_baseline": cpu, "e2e": r["e2e"],
+                "gpu_launches": r["launches"], "clocks": r["clocks"],
+                "kernel_ms": {k: [v[0], round(v[1], 3)] for k, v in r["ktimes"].items()}}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,354 @@
+/*
+ * pcs.h -- C ABI of libpcs, the GB300 (sm_103a) data-parallel hot path of
+ * Persistent Computational State (PCS).
+ *
+ * PCS is the minimal non-recomputable state a generative session must keep
+ * across requests (Sec. 3, Definition 1).  The paper's runtime exposes four
+ * operations over sessions and opaque snapshot handles -- checkpoint,
+ * restore, fork, delete (Sec. 3 "The contract") -- with four invariants:
+ *   I1 round-trip      restore(checkpoint(s)) reproduces s (here: byte-exact)
+ *   I2 durability      a snapshot is immutable; it survives later work and,
+ *                      through a file, the death of the process that made it
+ *   I3 fork independence   a fork is an independent copy
+ *   I4 completeness    a snapshot holds exactly the selected sections
+ * This library implements those operations for many sessions per call, plus
+ * the content fingerprint that decides must-snapshot vs derivable (Sec. 4,
+ * procedure FINGERPRINT, step 1 at epsilon = 0) and the relevance-keyed
+ * pruning of memory banks (Sec. 5 "The two semantic decisions"; Sec. 7.5).
+ *
+ * Conventions for every call
+ *   - Return value: PCS_OK (0) or a negative pcs_status.  pcs_last_error()
+ *     gives a message for the calling thread's last failure.
+ *   - Argument errors are detected on the host before anything is enqueued.
+ *     Errors found by a kernel (an index out of range) are recorded on the
+ *     device and returned by the next pcs_sync() as PCS_E_RANGE; the kernel
+ *     skips the offending access instead of performing it.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  All device work is enqueued on it; calls return before it
+ *     finishes unless documented otherwise.
+ *   - Pointers marked "device" must be device (or mapped pinned host) memory
+ *     reachable from the GPU of the context; the caller owns every buffer it
+ *     passes.  Buffers are read or written only by work enqueued on `stream`.
+ *   - Alignment: every contiguous buffer, row base and row size must be a
+ *     multiple of 16 bytes (else PCS_E_ALIGN).  Byte counts may be any size.
+ *   - Snapshots are owned by the library (device or pinned host arenas) and
+ *     are immutable after checkpoint; a handle is valid until pcs_delete.
+ *   - A context may be used from several host threads; calls are serialised
+ *     internally.  Work from different streams that uses the same snapshot
+ *     is ordered by the library (events), so a restore on stream B after a
+ *     checkpoint on stream A reads the finished record.
+ */
+#ifndef PCS_H
+#define PCS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t pcs_status;
+
+#define PCS_OK 0
+#define PCS_E_INVAL (-1)    /* bad argument (null, size, count, layout)      */
+#define PCS_E_ALIGN (-2)    /* pointer or row size not a multiple of 16 B   */
+#define PCS_E_NOMEM (-3)    /* device or pinned host allocation failed      */
+#define PCS_E_CUDA (-4)     /* a CUDA runtime call failed                   */
+#define PCS_E_BUDGET (-5)   /* a byte budget cannot be met                  */
+#define PCS_E_CORRUPT (-6)  /* verified restore / file: fingerprint mismatch */
+#define PCS_E_HANDLE (-7)   /* unknown or deleted snapshot handle           */
+#define PCS_E_IO (-8)       /* file could not be opened, read or written    */
+#define PCS_E_TIMEOUT (-9)  /* a bounded device wait gave up                */
+#define PCS_E_RANGE (-10)   /* a device-side index was out of range         */
+
+/* Element type tags recorded in section entries (informational). */
+#define PCS_DT_RAW 0
+#define PCS_DT_U8 1
+#define PCS_DT_I32 2
+#define PCS_DT_I64 3
+#define PCS_DT_F16 4
+#define PCS_DT_BF16 5
+#define PCS_DT_F32 6
+#define PCS_DT_U64 7
+
+/* Section type tags (caller-chosen; these are the conventional ones). */
+#define PCS_SEC_OBS 1       /* uint8 observation (Markovian model)          */
+#define PCS_SEC_RNG 2       /* generator state: seed u64, offset u64        */
+#define PCS_SEC_KEPT_IDX 3  /* int32 indices of the kept bank entries       */
+#define PCS_SEC_KEYS 4      /* bank keys of the kept entries                */
+#define PCS_SEC_VALUES 5    /* bank values (latents) of the kept entries    */
+#define PCS_SEC_META 6      /* position indices of a KV context             */
+#define PCS_SEC_K 7         /* one layer's keys of a KV window              */
+#define PCS_SEC_V 8         /* one layer's values of a KV window            */
+
+/* Session kinds (recorded in the record header; informational). */
+#define PCS_KIND_MARKOV 1   /* {OBS, RNG}                                   */
+#define PCS_KIND_BANK 2     /* {KEPT_IDX, KEYS, VALUES}                     */
+#define PCS_KIND_KV 3       /* {META, K_0, V_0, K_1, V_1, ...}              */
+
+/* How a section's logical bytes map onto memory. */
+#define PCS_LAYOUT_CONTIG 0 /* bytes [0, bytes) at base                     */
+#define PCS_LAYOUT_ROWS 1   /* row r at base + index[r] * row_bytes         */
+#define PCS_LAYOUT_RING 2   /* paged ring: row r in ring slot               */
+                            /* q = (ring_start + r) mod window, on page     */
+                            /* index[q / page_rows], row q mod page_rows:   */
+                            /* base + (page * page_rows + q % page_rows)    */
+                            /*        * row_bytes                           */
+
+/* Where a snapshot lives. */
+#define PCS_PLACE_DEVICE 0       /* HBM of the context's GPU                */
+#define PCS_PLACE_PINNED_HOST 1  /* page-locked host memory, GPU-mapped     */
+
+/* Ring start meaning "the one stored in the snapshot" (restore targets). */
+#define PCS_RING_START_FROM_SNAPSHOT 0xFFFFFFFFu
+
+/* k-rules of pcs_prune. */
+#define PCS_K_FIXED 0     /* k = min(n, k_max)                               */
+#define PCS_K_BUDGET 1    /* T = sum n_s*entry_bytes_s; k_s = n_s if T <= B, */
+                          /* else floor(n_s * B / T)  (Sec. 7.5)             */
+#define PCS_K_FRACTION 2  /* k = round-half-even(fraction * n)              */
+                          /* (Table tab:keepfrac)                           */
+
+typedef struct pcs_ctx pcs_ctx;
+typedef struct pcs_snapshot pcs_snapshot;
+
+/* A runtime buffer to fingerprint: `bytes` bytes at device pointer `ptr`. */
+typedef struct pcs_buf {
+    const void *ptr;   /* device, 16-byte aligned (may be NULL if bytes==0) */
+    uint64_t bytes;
+    uint32_t dtype;    /* PCS_DT_* (informational)                          */
+    uint32_t flags;    /* reserved, 0                                       */
+} pcs_buf;
+
+/*
+ * One section of a session.  For pcs_checkpoint `base` is read; for
+ * pcs_restore it is written.  Logical bytes of the section:
+ *   CONTIG: `bytes` bytes at base.
+ *   ROWS:   bytes / row_bytes rows; row r at base + index[r] * row_bytes;
+ *           every index[r] must lie in [0, base_rows).
+ *   RING:   window rows (bytes == window * row_bytes); see PCS_LAYOUT_RING;
+ *           every page id must lie in [0, base_rows); window must be a
+ *           multiple of page_rows; ring_start < window (restore targets may
+ *           pass PCS_RING_START_FROM_SNAPSHOT).
+ * row_bytes and base must be multiples of 16; `index` is device int32.
+ */
+typedef struct pcs_section {
+    uint32_t type;        /* PCS_SEC_*                                      */
+    uint32_t dtype;       /* PCS_DT_*                                       */
+    uint32_t layer;       /* layer number (KV) or 0                         */
+    uint32_t layout;      /* PCS_LAYOUT_*                                   */
+    void *base;           /* device                                         */
+    uint64_t bytes;       /* logical payload bytes                          */
+    uint64_t row_bytes;   /* ROWS / RING                                    */
+    const int32_t *index; /* device: ROWS row ids / RING page table         */
+    uint64_t base_rows;   /* ROWS: rows at base; RING: pages at base        */
+    uint32_t ring_start;  /* RING                                           */
+    uint32_t window;      /* RING: ring slots (rows)                        */
+    uint32_t page_rows;   /* RING: rows per page                            */
+    uint32_t reserved;    /* 0                                              */
+    uint64_t dim0, dim1;  /* shape recorded in the snapshot (informational) */
+} pcs_section;
+
+/* A session: an ordered list of 1..65535 sections. */
+typedef struct pcs_session {
+    uint32_t session_id;
+    uint32_t kind;                 /* PCS_KIND_*                             */
+    int32_t n_sections;
+    int32_t reserved;              /* 0                                      */
+    const pcs_section *sections;   /* host array of n_sections               */
+} pcs_session;
+
+/* A memory bank to prune: n_entries keys of key_dim fp16/bf16 elements. */
+typedef struct pcs_bank {
+    const void *keys;      /* device [n_entries][key_dim], 16-byte aligned  */
+    const void *query;     /* device [key_dim]: the return viewpoint        */
+    int32_t n_entries;
+    int32_t key_dim;       /* multiple of 8                                 */
+    uint32_t key_dtype;    /* PCS_DT_F16 or PCS_DT_BF16                     */
+    uint32_t reserved;     /* 0                                             */
+    uint64_t entry_bytes;  /* bytes one kept entry costs (PCS_K_BUDGET)     */
+} pcs_bank;
+
+typedef struct pcs_prune_params {
+    int32_t rule;          /* PCS_K_*                                       */
+    int32_t k_max;         /* PCS_K_FIXED                                   */
+    uint64_t budget_bytes; /* PCS_K_BUDGET: host byte budget B              */
+    double fraction;       /* PCS_K_FRACTION, in [0, 1]                     */
+} pcs_prune_params;
+
+typedef struct pcs_snapshot_info {
+    uint32_t session_id;
+    uint32_t kind;
+    int32_t n_sections;
+    uint32_t placement;    /* PCS_PLACE_*                                   */
+    uint64_t total_bytes;  /* record bytes (multiple of 256)                */
+    uint64_t session_fp;   /* fmix(tree(section fps) ^ n_sections)          */
+    const void *data;      /* record address (read-only for the caller)     */
+} pcs_snapshot_info;
+
+typedef struct pcs_section_info {
+    uint32_t type, dtype, layer, layout;
+    uint64_t offset;       /* payload offset within the record              */
+    uint64_t bytes;
+    uint64_t fp;           /* PCSFP64-v1 of the payload                     */
+    uint64_t dim0, dim1;
+    uint64_t aux;          /* RING: ring start at checkpoint; else 0        */
+} pcs_section_info;
+
+/* Counters of a context. */
+typedef struct pcs_stats {
+    uint64_t kernel_launches;  /* kernels this context has launched         */
+    uint64_t device_reserved;  /* bytes of HBM held by the snapshot arena   */
+    uint64_t host_reserved;    /* bytes of pinned host memory held          */
+    int32_t live_snapshots;    /* handles not yet deleted                   */
+    int32_t sm_count;          /* SMs of the context's GPU                  */
+} pcs_stats;
+
+/* Accumulated device time of one kernel (see pcs_timing_enable). */
+typedef struct pcs_kernel_time {
+    char name[32];             /* kernel name, NUL-terminated               */
+    uint64_t launches;         /* launches timed                            */
+    double total_ms;           /* sum of CUDA-event durations               */
+} pcs_kernel_time;
+
+/* Message of the calling thread's last error ("" if none). */
+const char *pcs_last_error(void);
+/* Name of a status code. */
+const char *pcs_status_string(pcs_status s);
+
+/*
+ * Create a context on CUDA device `device`: it owns the snapshot arenas,
+ * the workspace of the kernels and the snapshot table.  PCS_E_CUDA if the
+ * device cannot be used.
+ */
+pcs_status pcs_create(int32_t device, pcs_ctx **out);
+/* Destroy a context: waits for its work, frees every snapshot it owns. */
+pcs_status pcs_destroy(pcs_ctx *ctx);
+/* Fill `out` with the context's counters (host only, no synchronisation). */
+pcs_status pcs_get_stats(pcs_ctx *ctx, pcs_stats *out);
+
+/*
+ * Per-kernel timing: with on != 0 every kernel launch of the context is
+ * bracketed by CUDA events on its own stream; on == 0 stops.  Either call
+ * clears the accumulated times.
+ */
+pcs_status pcs_timing_enable(pcs_ctx *ctx, int32_t on);
+/*
+ * Wait for the timed launches and write up to `max` per-kernel totals to
+ * `out` (host); *n = number of kernels with at least one timed launch.
+ */
+pcs_status pcs_timing_read(pcs_ctx *ctx, pcs_kernel_time *out, int32_t max, int32_t *n);
+
+/*
+ * Wait for `stream`, then report errors recorded by kernels since the last
+ * pcs_sync (PCS_E_RANGE) or by CUDA (PCS_E_CUDA).  Clears them.
+ */
+pcs_status pcs_sync(pcs_ctx *ctx, void *stream);
+
+/*
+ * Content fingerprint PCSFP64-v1 of n buffers (the measurement that decides
+ * must-snapshot, Sec. 4 step 1 at epsilon = 0).  fp_out: device uint64[n].
+ * Definition: 4096-byte chunks (bytes past the end read as 0); in chunk c,
+ * lane l in [0,32) hashes 16-byte segments l+32k (k = 0..7) with
+ * h = fmix(SEED ^ (32c + l)), h = (rotl(h,23) ^ w) * P per little-endian
+ * word, a_l = fmix(h); a lane tree comb(a,b) = fmix(a*P + rotl(b,31)) gives
+ * the chunk hash; a pairwise tree over chunks (odd item carried up) gives
+ * the root; fp = fmix(root ^ bytes * P).  fmix = SplitMix64 finaliser,
+ * P = 0x9E3779B97F4A7C15, SEED = 0x5043534650363401.
+ */
+pcs_status pcs_fingerprint(pcs_ctx *ctx, const pcs_buf *bufs, int32_t n, uint64_t *fp_out,
+                           void *stream);
+
+/*
+ * Classify n buffers after a recompute (Sec. 3 "The partition"): fingerprint
+ * them again and write must_snapshot[i] = (fp_before[i] != fp_after[i]):
+ * 1 = non-derivable, must be snapshotted; 0 = derivable.
+ * fp_before: device uint64[n]; fp_after: device uint64[n] or NULL;
+ * must_snapshot: device uint8[n].
+ */
+pcs_status pcs_classify(pcs_ctx *ctx, const pcs_buf *bufs, int32_t n, const uint64_t *fp_before,
+                        uint64_t *fp_after, uint8_t *must_snapshot, void *stream);
+
+/*
+ * Host only: how many entries each bank keeps under `params`.  k_out: host
+ * int32[n].  PCS_E_INVAL on a bad rule or fraction.
+ */
+pcs_status pcs_prune_counts(const pcs_bank *banks, int32_t n, const pcs_prune_params *params,
+                            int32_t *k_out);
+
+/*
+ * Relevance-keyed pruning (Sec. 5; Sec. 7.5): score every entry of every
+ * bank by cos(query, key) in fp32 (fixed order: lane floor(e/8) mod 32 owns
+ * element e, separately rounded multiply and add, lane tree, RN sqrt and
+ * division, 0 if a norm is 0), keep per bank the k_s entries with the
+ * largest (score, -index) -- ties to the lower index, NaN lowest, -0 == +0 --
+ * and write their indices in ascending order.
+ *   scores:   device float[sum n] (CSR by bank) or NULL
+ *   kept_idx: device int32[sum k] (CSR by bank, k from pcs_prune_counts)
+ *   kept_off: device int32[n + 1] or NULL: CSR offsets of kept_idx
+ */
+pcs_status pcs_prune(pcs_ctx *ctx, const pcs_bank *banks, int32_t n,
+                     const pcs_prune_params *params, float *scores, int32_t *kept_idx,
+                     int32_t *kept_off, void *stream);
+
+/*
+ * Host only: bytes of the PCS1 record a session of these sections packs to:
+ * 256-byte aligned header + 64-byte entries, then each payload at a
+ * 256-byte aligned offset.
+ */
+pcs_status pcs_record_bytes(const pcs_section *sections, int32_t n_sections, uint64_t *out);
+
+/*
+ * checkpoint(s) for n sessions (Sec. 3 "The contract"): gather every
+ * section into one contiguous PCS1 record per session in a new snapshot of
+ * the given placement, with the fingerprint of every section payload fused
+ * into the copy, and write the record header (session fp) and section
+ * table.  out: host array receiving n handles.  Asynchronous; the live
+ * buffers may be changed once `stream` has passed this call (I2).
+ */
+pcs_status pcs_checkpoint(pcs_ctx *ctx, const pcs_session *sessions, int32_t n,
+                          uint32_t placement, pcs_snapshot **out, void *stream);
+
+/*
+ * fork(c): an independent byte copy of a snapshot, same placement (I3).
+ */
+pcs_status pcs_fork(pcs_ctx *ctx, const pcs_snapshot *parent, pcs_snapshot **child,
+                    void *stream);
+
+/*
+ * restore(c) for n snapshots (I1): scatter each section payload to the
+ * target section of targets[i] (same section count and byte counts; any
+ * layout).  verify != 0 also recomputes every section fingerprint and the
+ * session fp, waits for `stream`, and returns PCS_E_CORRUPT if any differs
+ * from the record (the bytes have been written by then).
+ */
+pcs_status pcs_restore(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n,
+                       const pcs_session *targets, int32_t verify, void *stream);
+
+/* delete(c): release a snapshot (its memory is reused once pending work
+ * that reads it has finished). */
+pcs_status pcs_delete(pcs_ctx *ctx, pcs_snapshot *snap);
+
+/* Header fields of a snapshot; waits for the work that wrote it. */
+pcs_status pcs_snapshot_get_info(pcs_ctx *ctx, const pcs_snapshot *snap, pcs_snapshot_info *out);
+/* Section entry i of a snapshot; waits for the work that wrote it. */
+pcs_status pcs_snapshot_get_section(pcs_ctx *ctx, const pcs_snapshot *snap, int32_t i,
+                                pcs_section_info *out);
+/* Copy record bytes [offset, offset + bytes) to dst (device or host),
+ * enqueued on stream. */
+pcs_status pcs_snapshot_copy_out(pcs_ctx *ctx, const pcs_snapshot *snap, uint64_t offset,
+                                 uint64_t bytes, void *dst, void *stream);
+
+/* Durability across processes (I2): write the record to `path` (written to
+ * a temporary file, flushed, then renamed); read one back into a new
+ * snapshot after validating its header and section table (PCS_E_CORRUPT on
+ * a malformed record, PCS_E_IO on a file error). */
+pcs_status pcs_snapshot_write_file(pcs_ctx *ctx, const pcs_snapshot *snap, const char *path);
+pcs_status pcs_snapshot_read_file(pcs_ctx *ctx, const char *path, uint32_t placement,
+                                  pcs_snapshot **out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PCS_H */

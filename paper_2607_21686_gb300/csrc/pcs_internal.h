@@ -1,0 +1,123 @@
+// pcs_internal.h -- descriptors shared by the host runtime (pcs_runtime.cpp)
+// and the sm_103a kernels (pcs_kernels.cu).  Plain structs copied to the
+// device once per call; no torch types.
+#pragma once
+
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace pcs {
+
+constexpr uint32_t kChunkBytes = 4096;   // fingerprint chunk
+constexpr uint32_t kRecordAlign = 256;   // record / payload alignment
+constexpr uint32_t kHeaderBytes = 64;
+constexpr uint32_t kEntryBytes = 64;
+constexpr uint32_t kMagic = 0x31534350u;  // "PCS1"
+constexpr uint32_t kVersion = 1;
+constexpr int kMaxGroupLog2 = 5;         // at most 32 chunks per warp task
+
+// Errors a kernel records (OR-ed into the context's device error word).
+constexpr uint32_t kDevErrIndex = 1u;    // a row / page id out of range
+
+enum Layout : uint32_t { kContig = 0, kRows = 1, kRing = 2 };
+
+// Work modes of the streaming kernel.
+enum Mode : int {
+  kModeHash = 0,       // read a contiguous buffer, fingerprint it
+  kModePack = 1,       // gather layout side -> payload, fingerprint
+  kModeRestore = 2,    // payload -> scatter layout side (no hashing)
+  kModeRestoreV = 3,   // payload -> scatter layout side, fingerprint payload
+};
+
+// One fingerprinted stream of bytes (a buffer, or a section payload).
+// "Layout side" = where the bytes live in the session (source of a pack,
+// target of a restore, the buffer itself when hashing); the other side is
+// the contiguous payload inside a record.
+struct alignas(16) SecDesc {
+  uint8_t* lbase;          // layout-side base
+  uint8_t* payload;        // contiguous side (record payload), or null
+  const int32_t* index;    // ROWS row ids / RING page table
+  uint64_t bytes;          // logical bytes L
+  uint64_t row_bytes;      // ROWS / RING
+  uint64_t base_rows;      // bound on index values
+  uint32_t layout;
+  int32_t rb_shift;        // log2(row_bytes) if a power of two, else -1
+  uint32_t ring_start;
+  uint32_t window;
+  uint32_t page_rows;
+  int32_t pr_shift;        // log2(page_rows) if a power of two, else -1
+  uint32_t task_begin;     // first warp task (= node slot) of this stream
+  uint32_t n_tasks;
+  uint64_t n_chunks;
+  uint64_t pad0;
+};
+static_assert(sizeof(SecDesc) == 96, "SecDesc layout");
+
+// One session: a record and the contiguous range of its sections.
+struct alignas(16) SessDesc {
+  uint8_t* record;         // record base (pack: written; restore: read)
+  uint64_t total_bytes;
+  uint64_t payload_start;  // header + table, rounded up to 256
+  uint32_t sec_begin;
+  uint32_t n_sections;
+  uint32_t session_id;
+  uint32_t kind;
+};
+static_assert(sizeof(SessDesc) == 40 || sizeof(SessDesc) == 48, "SessDesc layout");
+
+// Section entry exactly as stored in a record (64 bytes, little-endian).
+struct alignas(16) Entry {
+  uint32_t type, dtype, layer, layout;
+  uint64_t offset, bytes, fp, dim0, dim1, aux;
+};
+static_assert(sizeof(Entry) == 64, "Entry layout");
+
+// One memory bank to score / prune.
+struct alignas(16) BankDesc {
+  const uint16_t* keys;    // [n][D] fp16 / bf16 bits
+  const uint16_t* query;   // [D]
+  uint64_t entry_begin;    // CSR offset of this bank's scores
+  uint64_t kept_begin;     // CSR offset of this bank's kept indices
+  int32_t n;
+  int32_t D;
+  int32_t k;
+  uint32_t is_bf16;
+};
+static_assert(sizeof(BankDesc) == 48, "BankDesc layout");
+
+// Kernel launchers (pcs_kernels.cu).  All enqueue on `stream`, return the
+// CUDA error of the launch.
+struct LaunchShape {
+  int blocks;
+  int threads;
+};
+
+cudaError_t launch_stream(int mode, const SecDesc* secs, int n_secs, uint32_t n_tasks,
+                          int group_log2, uint64_t* nodes, uint32_t* dev_err, int sm_count,
+                          int blocks_per_sm, cudaStream_t stream);
+
+// Section fps from the warp-task nodes (in place), then per mode:
+//   kModeHash: fp_out[i] = fp; if fp_before: flags[i] = fp != fp_before[i]
+//   kModePack: header + section table of each session's record
+//   kModeRestoreV: compare with the record's stored fps; corrupt[s] = 1 and
+//                  ++*bad on mismatch
+cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess, int n_sess,
+                            const Entry* entries, uint64_t* nodes, uint64_t* fp_out,
+                            const uint64_t* fp_before, uint8_t* flags, uint32_t* bad,
+                            cudaStream_t stream);
+
+cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
+                         const uint64_t* entry_begin_sorted, float* scores, int sm_count,
+                         cudaStream_t stream);
+
+cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
+                        int32_t* kept_idx, cudaStream_t stream);
+
+cudaError_t launch_copy(const void* src, void* dst, uint64_t bytes, int sm_count,
+                        cudaStream_t stream);
+
+// Occupancy of the streaming kernel (blocks per SM) for the launch shape.
+int stream_blocks_per_sm();
+
+}  // namespace pcs

@@ -1,0 +1,1359 @@
+// pcs_runtime.cpp -- host side of libpcs: argument validation, planning of
+// records and kernel work, the snapshot table, the arena allocator, files.
+//
+// The paper's runtime (Sec. 5, Sec. 8) is a single-process Python service
+// that keeps, per session, the PCS a later restore needs; the byte movement
+// is delegated to the layer below.  This file is that layer's host half: it
+// turns a batch of sessions into one launch of the streaming kernel over
+// every section of every session, and owns the snapshots behind opaque
+// handles (Sec. 3 "The contract": checkpoint / restore / fork / delete).
+#include <cuda_runtime.h>
+#include <fcntl.h>
+#include <unistd.h>
+
+#include <algorithm>
+#include <cerrno>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <memory>
+#include <mutex>
+#include <string>
+#include <unordered_set>
+#include <vector>
+
+#include "../../include/pcs.h"
+#include "pcs_internal.h"
+
+using namespace pcs;
+
+// ---------------------------------------------------------------------------
+// Errors
+// ---------------------------------------------------------------------------
+
+namespace {
+
+thread_local std::string g_err;
+
+pcs_status fail(pcs_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return s;
+}
+
+pcs_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(PCS_E_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define PCS_CUDA(call)                                  \
+  do {                                                  \
+    cudaError_t e_ = (call);                            \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call); \
+  } while (0)
+
+uint64_t round_up(uint64_t x, uint64_t a) { return (x + a - 1) / a * a; }
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+int log2_exact(uint64_t x) {
+  if (x == 0 || (x & (x - 1)) != 0) return -1;
+  int s = 0;
+  while ((1ull << s) != x) ++s;
+  return s;
+}
+
+// ---------------------------------------------------------------------------
+// Events: pooled, shared; a range of freed memory keeps the events of the
+// work that last used it, and whoever reuses it first waits for them on its
+// own stream (stream-ordered reuse; the host never blocks for it).
+// ---------------------------------------------------------------------------
+
+struct EventPool {
+  std::vector<cudaEvent_t> free_;
+  ~EventPool() {
+    for (auto e : free_) cudaEventDestroy(e);
+  }
+  cudaEvent_t get() {
+    if (!free_.empty()) {
+      cudaEvent_t e = free_.back();
+      free_.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return nullptr;
+    return e;
+  }
+  void put(cudaEvent_t e) { free_.push_back(e); }
+};
+
+struct Event {
+  cudaEvent_t ev = nullptr;
+  std::shared_ptr<EventPool> pool;
+  ~Event() {
+    if (ev) pool->put(ev);
+  }
+  bool done() const { return cudaEventQuery(ev) == cudaSuccess; }
+};
+using Ev = std::shared_ptr<Event>;
+
+Ev record_event(const std::shared_ptr<EventPool>& pool, cudaStream_t s) {
+  auto e = std::make_shared<Event>();
+  e->pool = pool;
+  e->ev = pool->get();
+  if (!e->ev || cudaEventRecord(e->ev, s) != cudaSuccess) return nullptr;
+  return e;
+}
+
+void prune_done(std::vector<Ev>& deps) {
+  deps.erase(std::remove_if(deps.begin(), deps.end(), [](const Ev& e) { return !e || e->done(); }),
+             deps.end());
+}
+
+// ---------------------------------------------------------------------------
+// Arena allocator: slabs of device (HBM) or pinned, GPU-mapped host memory,
+// first fit with coalescing, 256-byte granules.
+// ---------------------------------------------------------------------------
+
+struct Range {
+  uint64_t size = 0;
+  std::vector<Ev> deps;  // work that must finish before the bytes are reused
+};
+
+struct Slab {
+  uint8_t* base = nullptr;  // device-usable address
+  uint64_t size = 0;
+  uint64_t used = 0;
+  std::map<uint64_t, Range> free;  // offset -> free range
+};
+
+struct Block {
+  Slab* slab = nullptr;
+  uint64_t off = 0;
+  uint64_t size = 0;
+  uint8_t* ptr = nullptr;
+  uint32_t placement = PCS_PLACE_DEVICE;
+  int refs = 0;
+  Ev written;                                 // completion of the write
+  std::map<cudaStream_t, Ev> uses;            // latest use per stream
+};
+
+class Arena {
+ public:
+  Arena(uint32_t placement, std::shared_ptr<EventPool> pool) : placement_(placement), pool_(pool) {}
+  ~Arena() { release_all(); }
+
+  // Reserve `bytes`; `stream` is made to wait for earlier users of the range.
+  pcs_status alloc(uint64_t bytes, cudaStream_t stream, Block** out) {
+    bytes = round_up(std::max<uint64_t>(bytes, kRecordAlign), kRecordAlign);
+    for (int attempt = 0; attempt < 3; ++attempt) {
+      for (auto& sp : slabs_) {
+        Slab* s = sp.get();
+        for (auto it = s->free.begin(); it != s->free.end(); ++it) {
+          if (it->second.size < bytes) continue;
+          const uint64_t off = it->first;
+          Range r = std::move(it->second);
+          s->free.erase(it);
+          prune_done(r.deps);
+          for (auto& e : r.deps)
+            if (cudaStreamWaitEvent(stream, e->ev, 0) != cudaSuccess)
+              return fail(PCS_E_CUDA, "cudaStreamWaitEvent failed");
+          if (r.size > bytes) {
+            Range rest;
+            rest.size = r.size - bytes;
+            rest.deps = r.deps;
+            s->free.emplace(off + bytes, std::move(rest));
+          }
+          auto* b = new Block();
+          b->slab = s;
+          b->off = off;
+          b->size = bytes;
+          b->ptr = s->base + off;
+          b->placement = placement_;
+          s->used += bytes;
+          *out = b;
+          return PCS_OK;
+        }
+      }
+      if (attempt == 0) {
+        if (new_slab(bytes) == PCS_OK) continue;
+        // Out of memory: return empty slabs, then try once more.
+        trim();
+        cudaGetLastError();
+      } else if (attempt == 1) {
+        if (new_slab(bytes) == PCS_OK) continue;
+        cudaGetLastError();
+      }
+    }
+    return fail(PCS_E_NOMEM, "cannot allocate %llu bytes of %s memory",
+                static_cast<unsigned long long>(bytes),
+                placement_ == PCS_PLACE_DEVICE ? "device" : "pinned host");
+  }
+
+  // Return a block; its bytes are reused only after its recorded uses.
+  void free(Block* b) {
+    Slab* s = b->slab;
+    Range r;
+    r.size = b->size;
+    for (auto& kv : b->uses) r.deps.push_back(kv.second);
+    if (b->written) r.deps.push_back(b->written);
+    prune_done(r.deps);
+    uint64_t off = b->off;
+    s->used -= b->size;
+    delete b;
+    // Coalesce with the following and preceding free ranges.
+    auto next = s->free.lower_bound(off);
+    if (next != s->free.end() && next->first == off + r.size) {
+      r.size += next->second.size;
+      r.deps.insert(r.deps.end(), next->second.deps.begin(), next->second.deps.end());
+      s->free.erase(next);
+    }
+    auto it = s->free.lower_bound(off);
+    if (it != s->free.begin()) {
+      auto prev = std::prev(it);
+      if (prev->first + prev->second.size == off) {
+        prev->second.size += r.size;
+        prev->second.deps.insert(prev->second.deps.end(), r.deps.begin(), r.deps.end());
+        prune_done(prev->second.deps);
+        return;
+      }
+    }
+    prune_done(r.deps);
+    s->free.emplace(off, std::move(r));
+  }
+
+  void trim() {
+    for (auto it = slabs_.begin(); it != slabs_.end();) {
+      Slab* s = it->get();
+      if (s->used == 0) {
+        for (auto& kv : s->free)
+          for (auto& e : kv.second.deps) cudaEventSynchronize(e->ev);
+        free_memory(s->base);
+        it = slabs_.erase(it);
+      } else {
+        ++it;
+      }
+    }
+  }
+
+  void release_all() {
+    for (auto& s : slabs_) free_memory(s->base);
+    slabs_.clear();
+  }
+
+  uint64_t reserved() const {
+    uint64_t t = 0;
+    for (auto& s : slabs_) t += s->size;
+    return t;
+  }
+
+ private:
+  pcs_status new_slab(uint64_t bytes) {
+    const uint64_t min_slab = placement_ == PCS_PLACE_DEVICE ? (256ull << 20) : (64ull << 20);
+    const uint64_t size = round_up(std::max(bytes, min_slab), 2ull << 20);
+    void* p = nullptr;
+    if (placement_ == PCS_PLACE_DEVICE) {
+      if (cudaMalloc(&p, size) != cudaSuccess) return PCS_E_NOMEM;
+    } else {
+      void* h = nullptr;
+      if (cudaHostAlloc(&h, size, cudaHostAllocMapped | cudaHostAllocPortable) != cudaSuccess)
+        return PCS_E_NOMEM;
+      if (cudaHostGetDevicePointer(&p, h, 0) != cudaSuccess) {
+        cudaFreeHost(h);
+        return PCS_E_NOMEM;
+      }
+      host_of_[p] = h;
+    }
+    auto s = std::make_unique<Slab>();
+    s->base = static_cast<uint8_t*>(p);
+    s->size = size;
+    Range r;
+    r.size = size;
+    s->free.emplace(0, std::move(r));
+    slabs_.push_back(std::move(s));
+    return PCS_OK;
+  }
+
+  void free_memory(uint8_t* p) {
+    if (placement_ == PCS_PLACE_DEVICE) {
+      cudaFree(p);
+    } else {
+      auto it = host_of_.find(p);
+      if (it != host_of_.end()) {
+        cudaFreeHost(it->second);
+        host_of_.erase(it);
+      }
+    }
+  }
+
+  uint32_t placement_;
+  std::shared_ptr<EventPool> pool_;
+  std::vector<std::unique_ptr<Slab>> slabs_;
+  std::map<void*, void*> host_of_;
+};
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Snapshots and the context
+// ---------------------------------------------------------------------------
+
+struct pcs_snapshot {
+  Block* block = nullptr;
+  uint64_t offset = 0;         // record offset within the block
+  uint64_t total_bytes = 0;
+  uint64_t payload_start = 0;
+  uint32_t session_id = 0;
+  uint32_t kind = 0;
+  std::vector<Entry> table;    // host copy of the section table (fp = 0)
+  uint8_t* record() const { return block->ptr + offset; }
+};
+
+struct pcs_ctx {
+  int device = 0;
+  int sm_count = 0;
+  int stream_bps = 1;          // resident blocks per SM of the streaming kernel
+  std::mutex mu;
+  std::shared_ptr<EventPool> events = std::make_shared<EventPool>();
+  std::unique_ptr<Arena> dev_arena, host_arena;
+  std::unordered_set<pcs_snapshot*> live;
+  // Workspace: descriptors and tree nodes of one call.
+  uint8_t* ws = nullptr;
+  uint64_t ws_bytes = 0;
+  Ev ws_busy;
+  // Small device words: [0] kernel error bits, [1] verification failures.
+  uint32_t* words = nullptr;
+  std::vector<uint8_t> plan;   // host staging of the descriptors
+  uint8_t* stage = nullptr;    // pinned staging for file I/O
+  uint64_t stage_bytes = 0;
+  uint64_t launches = 0;       // kernels launched by this context
+  // Per-kernel CUDA-event timing (pcs_timing_enable).
+  bool timing = false;
+  struct Timed {
+    int kind;
+    cudaEvent_t start, stop;
+  };
+  std::vector<Timed> timed;
+  std::vector<cudaEvent_t> timing_events;  // free timing-capable events
+  double kernel_ms[16] = {};
+  uint64_t kernel_n[16] = {};
+};
+
+namespace {
+
+constexpr uint64_t kStageBytes = 64ull << 20;
+
+pcs_status set_device(pcs_ctx* c) {
+  PCS_CUDA(cudaSetDevice(c->device));
+  return PCS_OK;
+}
+
+// Kernels the context launches, for counting and timing.
+enum KernelKind {
+  kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
+  kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKCopy, kKernelKinds
+};
+const char* kKernelNames[kKernelKinds] = {
+    "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
+    "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
+    "k_copy"};
+
+cudaEvent_t timing_event(pcs_ctx* c) {
+  if (!c->timing_events.empty()) {
+    cudaEvent_t e = c->timing_events.back();
+    c->timing_events.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+// Brackets one kernel launch: counts it and, when timing is on, records
+// CUDA events around it on the launching stream.
+struct LaunchScope {
+  pcs_ctx* c;
+  int kind;
+  cudaStream_t stream;
+  cudaEvent_t start = nullptr;
+  LaunchScope(pcs_ctx* c_, int kind_, cudaStream_t s) : c(c_), kind(kind_), stream(s) {
+    c->launches += 1;
+    if (c->timing) {
+      start = timing_event(c);
+      if (start) cudaEventRecord(start, stream);
+    }
+  }
+  ~LaunchScope() {
+    if (!start) return;
+    cudaEvent_t stop = timing_event(c);
+    if (!stop) return;
+    cudaEventRecord(stop, stream);
+    c->timed.push_back({kind, start, stop});
+  }
+};
+
+int stream_kind(int mode) {
+  switch (mode) {
+    case kModeHash: return kKStreamHash;
+    case kModePack: return kKStreamPack;
+    case kModeRestore: return kKStreamRestore;
+    default: return kKStreamRestoreV;
+  }
+}
+
+Arena* arena_of(pcs_ctx* c, uint32_t placement) {
+  return placement == PCS_PLACE_DEVICE ? c->dev_arena.get() : c->host_arena.get();
+}
+
+// Make `stream` wait for the previous call's use of the workspace, grow it
+// if needed.  Returns the workspace base.
+pcs_status ws_acquire(pcs_ctx* c, uint64_t bytes, cudaStream_t stream, uint8_t** out) {
+  bytes = round_up(std::max<uint64_t>(bytes, 1), kRecordAlign);
+  if (bytes > c->ws_bytes) {
+    if (c->ws_busy) PCS_CUDA(cudaEventSynchronize(c->ws_busy->ev));
+    c->ws_busy.reset();
+    if (c->ws) cudaFree(c->ws);
+    c->ws = nullptr;
+    c->ws_bytes = 0;
+    const uint64_t want = round_up(std::max<uint64_t>(bytes, 1ull << 20) * 5 / 4, 2ull << 20);
+    if (cudaMalloc(&c->ws, want) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(PCS_E_NOMEM, "cannot allocate %llu bytes of workspace",
+                  static_cast<unsigned long long>(want));
+    }
+    c->ws_bytes = want;
+  } else if (c->ws_busy && !c->ws_busy->done()) {
+    PCS_CUDA(cudaStreamWaitEvent(stream, c->ws_busy->ev, 0));
+  }
+  *out = c->ws;
+  return PCS_OK;
+}
+
+pcs_status ws_release(pcs_ctx* c, cudaStream_t stream) {
+  c->ws_busy = record_event(c->events, stream);
+  if (!c->ws_busy) return fail(PCS_E_CUDA, "cudaEventRecord failed");
+  return PCS_OK;
+}
+
+// Record a use of a block on `stream` (kept until the block is freed).
+pcs_status note_use(pcs_ctx* c, Block* b, cudaStream_t stream) {
+  auto it = b->uses.find(stream);
+  if (it != b->uses.end() && it->second.use_count() == 1) {
+    PCS_CUDA(cudaEventRecord(it->second->ev, stream));
+    return PCS_OK;
+  }
+  Ev e = record_event(c->events, stream);
+  if (!e) return fail(PCS_E_CUDA, "cudaEventRecord failed");
+  b->uses[stream] = e;
+  return PCS_OK;
+}
+
+pcs_status wait_written(Block* b, cudaStream_t stream) {
+  if (b->written && !b->written->done()) PCS_CUDA(cudaStreamWaitEvent(stream, b->written->ev, 0));
+  return PCS_OK;
+}
+
+void release_block(pcs_ctx* c, Block* b) {
+  if (--b->refs == 0) arena_of(c, b->placement)->free(b);
+}
+
+// Layout of one call's descriptors inside the workspace.
+struct WsLayout {
+  uint64_t secs = 0, sess = 0, entries = 0, banks = 0, nodes = 0, total = 0;
+};
+
+// Choose 2^g chunks per warp task: at least ~4 tasks per resident warp,
+// at most 32 chunks per task.
+int choose_group_log2(const pcs_ctx* c, uint64_t total_chunks) {
+  const uint64_t warps = static_cast<uint64_t>(c->sm_count) * c->stream_bps * 8;
+  int g = 0;
+  while (g < kMaxGroupLog2 && (total_chunks >> (g + 1)) >= 4 * warps) ++g;
+  return g;
+}
+
+uint64_t n_chunks_of(uint64_t bytes) { return bytes == 0 ? 1 : (bytes + kChunkBytes - 1) / kChunkBytes; }
+
+// Validate a section used as a checkpoint source or a restore target.
+pcs_status check_section(const pcs_section& s, int sess, int i, bool target) {
+  if (s.layout > PCS_LAYOUT_RING)
+    return fail(PCS_E_INVAL, "session %d section %d: unknown layout %u", sess, i, s.layout);
+  if (s.layout == PCS_LAYOUT_CONTIG) {
+    if (s.bytes > 0 && !s.base)
+      return fail(PCS_E_INVAL, "session %d section %d: null base", sess, i);
+    if (s.bytes > 0 && !aligned16(s.base))
+      return fail(PCS_E_ALIGN, "session %d section %d: base not 16-byte aligned", sess, i);
+    return PCS_OK;
+  }
+  if (s.row_bytes == 0 || s.row_bytes % 16 != 0)
+    return fail(PCS_E_ALIGN, "session %d section %d: row_bytes %llu not a positive multiple of 16",
+                sess, i, static_cast<unsigned long long>(s.row_bytes));
+  if (s.bytes % s.row_bytes != 0)
+    return fail(PCS_E_INVAL, "session %d section %d: bytes not a multiple of row_bytes", sess, i);
+  if (s.bytes == 0) return PCS_OK;
+  if (!s.base || !s.index)
+    return fail(PCS_E_INVAL, "session %d section %d: null base or index", sess, i);
+  if (!aligned16(s.base))
+    return fail(PCS_E_ALIGN, "session %d section %d: base not 16-byte aligned", sess, i);
+  if ((reinterpret_cast<uintptr_t>(s.index) & 3u) != 0)
+    return fail(PCS_E_ALIGN, "session %d section %d: index not 4-byte aligned", sess, i);
+  if (s.base_rows == 0)
+    return fail(PCS_E_INVAL, "session %d section %d: base_rows must bound the index values", sess, i);
+  if (s.layout == PCS_LAYOUT_ROWS) {
+    if (s.bytes / s.row_bytes > 0x7FFFFFFFull)
+      return fail(PCS_E_INVAL, "session %d section %d: too many rows", sess, i);
+    return PCS_OK;
+  }
+  if (s.page_rows == 0 || s.window == 0 || s.window % s.page_rows != 0)
+    return fail(PCS_E_INVAL, "session %d section %d: window must be a positive multiple of page_rows",
+                sess, i);
+  if (s.bytes != static_cast<uint64_t>(s.window) * s.row_bytes)
+    return fail(PCS_E_INVAL, "session %d section %d: bytes != window * row_bytes", sess, i);
+  if (s.ring_start >= s.window && !(target && s.ring_start == PCS_RING_START_FROM_SNAPSHOT))
+    return fail(PCS_E_INVAL, "session %d section %d: ring_start %u >= window %u", sess, i,
+                s.ring_start, s.window);
+  return PCS_OK;
+}
+
+SecDesc make_desc(const pcs_section& s, uint8_t* payload, uint32_t ring_start) {
+  SecDesc d{};
+  d.lbase = static_cast<uint8_t*>(s.base);
+  d.payload = payload;
+  d.index = s.index;
+  d.bytes = s.bytes;
+  d.layout = s.layout;
+  d.row_bytes = s.layout == PCS_LAYOUT_CONTIG ? 0 : s.row_bytes;
+  d.rb_shift = s.layout == PCS_LAYOUT_CONTIG ? 0 : log2_exact(s.row_bytes);
+  d.base_rows = s.base_rows;
+  d.ring_start = ring_start;
+  d.window = s.window;
+  d.page_rows = s.page_rows;
+  d.pr_shift = s.layout == PCS_LAYOUT_RING ? log2_exact(s.page_rows) : 0;
+  d.n_chunks = n_chunks_of(s.bytes);
+  return d;
+}
+
+// Assign warp tasks to descriptors for a given group size.
+uint64_t assign_tasks(std::vector<SecDesc>& d, int glog2) {
+  uint64_t t = 0;
+  for (auto& x : d) {
+    x.task_begin = static_cast<uint32_t>(t);
+    x.n_tasks = static_cast<uint32_t>((x.n_chunks + (1ull << glog2) - 1) >> glog2);
+    t += x.n_tasks;
+  }
+  return t;
+}
+
+template <class T>
+void put(std::vector<uint8_t>& plan, uint64_t off, const std::vector<T>& v) {
+  if (!v.empty()) std::memcpy(plan.data() + off, v.data(), v.size() * sizeof(T));
+}
+
+// Fingerprint (and optionally classify) contiguous buffers.
+pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t* fp_out,
+                            const uint64_t* fp_before, uint8_t* flags, void* stream_) {
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  if (n < 0 || (n > 0 && !bufs)) return fail(PCS_E_INVAL, "bad buffer list");
+  if (n == 0) return PCS_OK;
+  std::vector<SecDesc> d(n);
+  uint64_t chunks = 0;
+  for (int i = 0; i < n; ++i) {
+    if (bufs[i].bytes > 0 && !bufs[i].ptr) return fail(PCS_E_INVAL, "buffer %d: null pointer", i);
+    if (bufs[i].bytes > 0 && !aligned16(bufs[i].ptr))
+      return fail(PCS_E_ALIGN, "buffer %d: pointer not 16-byte aligned", i);
+    pcs_section s{};
+    s.layout = PCS_LAYOUT_CONTIG;
+    s.base = const_cast<void*>(bufs[i].ptr);
+    s.bytes = bufs[i].bytes;
+    d[i] = make_desc(s, nullptr, 0);
+    chunks += d[i].n_chunks;
+  }
+  const int g = choose_group_log2(c, chunks);
+  const uint64_t tasks = assign_tasks(d, g);
+  if (tasks >= (1ull << 32)) return fail(PCS_E_INVAL, "too much data in one call");
+  WsLayout L;
+  L.secs = 0;
+  L.nodes = round_up(L.secs + sizeof(SecDesc) * n, kRecordAlign);
+  L.total = L.nodes + 8 * tasks;
+  uint8_t* ws = nullptr;
+  pcs_status st = ws_acquire(c, L.total, stream, &ws);
+  if (st) return st;
+  c->plan.resize(L.nodes);
+  put(c->plan, L.secs, d);
+  PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
+  auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
+  auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
+  {
+    LaunchScope ls(c, kKStreamHash, stream);
+    PCS_CUDA(launch_stream(kModeHash, dsecs, n, static_cast<uint32_t>(tasks), g, nodes, c->words,
+                           c->sm_count, c->stream_bps, stream));
+  }
+  {
+    LaunchScope ls(c, kKFinalizeHash, stream);
+    PCS_CUDA(launch_finalize(kModeHash, dsecs, nullptr, n, nullptr, nodes, fp_out, fp_before,
+                             flags, nullptr, stream));
+  }
+  return ws_release(c, stream);
+}
+
+pcs_snapshot* check_handle(pcs_ctx* c, const pcs_snapshot* h) {
+  auto* p = const_cast<pcs_snapshot*>(h);
+  return c->live.count(p) ? p : nullptr;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+
+extern "C" {
+
+const char* pcs_last_error(void) { return g_err.c_str(); }
+
+const char* pcs_status_string(pcs_status s) {
+  switch (s) {
+    case PCS_OK: return "PCS_OK";
+    case PCS_E_INVAL: return "PCS_E_INVAL";
+    case PCS_E_ALIGN: return "PCS_E_ALIGN";
+    case PCS_E_NOMEM: return "PCS_E_NOMEM";
+    case PCS_E_CUDA: return "PCS_E_CUDA";
+    case PCS_E_BUDGET: return "PCS_E_BUDGET";
+    case PCS_E_CORRUPT: return "PCS_E_CORRUPT";
+    case PCS_E_HANDLE: return "PCS_E_HANDLE";
+    case PCS_E_IO: return "PCS_E_IO";
+    case PCS_E_TIMEOUT: return "PCS_E_TIMEOUT";
+    case PCS_E_RANGE: return "PCS_E_RANGE";
+    default: return "PCS_E_UNKNOWN";
+  }
+}
+
+pcs_status pcs_create(int32_t device, pcs_ctx** out) {
+  if (!out) return fail(PCS_E_INVAL, "out is null");
+  *out = nullptr;
+  int count = 0;
+  cudaError_t e = cudaGetDeviceCount(&count);
+  if (e != cudaSuccess || count == 0) {
+    cudaGetLastError();
+    return fail(PCS_E_CUDA, "no CUDA device available (%s)", cudaGetErrorString(e));
+  }
+  if (device < 0 || device >= count) return fail(PCS_E_INVAL, "device %d out of range", device);
+  auto c = std::make_unique<pcs_ctx>();
+  c->device = device;
+  PCS_CUDA(cudaSetDevice(device));
+  PCS_CUDA(cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, device));
+  c->stream_bps = stream_blocks_per_sm();
+  c->dev_arena = std::make_unique<Arena>(PCS_PLACE_DEVICE, c->events);
+  c->host_arena = std::make_unique<Arena>(PCS_PLACE_PINNED_HOST, c->events);
+  PCS_CUDA(cudaMalloc(&c->words, 256));
+  PCS_CUDA(cudaMemset(c->words, 0, 256));
+  *out = c.release();
+  return PCS_OK;
+}
+
+pcs_status pcs_destroy(pcs_ctx* c) {
+  if (!c) return PCS_OK;
+  {
+    std::lock_guard<std::mutex> lk(c->mu);
+    cudaSetDevice(c->device);
+    cudaDeviceSynchronize();
+    for (auto* h : c->live) {
+      release_block(c, h->block);
+      delete h;
+    }
+    c->live.clear();
+    c->ws_busy.reset();
+    if (c->ws) cudaFree(c->ws);
+    if (c->words) cudaFree(c->words);
+    if (c->stage) cudaFreeHost(c->stage);
+    for (auto& t : c->timed) {
+      cudaEventDestroy(t.start);
+      cudaEventDestroy(t.stop);
+    }
+    for (auto e : c->timing_events) cudaEventDestroy(e);
+    c->dev_arena.reset();
+    c->host_arena.reset();
+  }
+  delete c;
+  return PCS_OK;
+}
+
+pcs_status pcs_get_stats(pcs_ctx* c, pcs_stats* out) {
+  if (!c || !out) return fail(PCS_E_INVAL, "null argument");
+  std::lock_guard<std::mutex> lk(c->mu);
+  out->kernel_launches = c->launches;
+  out->device_reserved = c->dev_arena->reserved();
+  out->host_reserved = c->host_arena->reserved();
+  out->live_snapshots = static_cast<int32_t>(c->live.size());
+  out->sm_count = c->sm_count;
+  return PCS_OK;
+}
+
+pcs_status pcs_timing_enable(pcs_ctx* c, int32_t on) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  for (auto& t : c->timed) {
+    cudaEventSynchronize(t.stop);
+    c->timing_events.push_back(t.start);
+    c->timing_events.push_back(t.stop);
+  }
+  c->timed.clear();
+  for (int i = 0; i < kKernelKinds; ++i) {
+    c->kernel_ms[i] = 0;
+    c->kernel_n[i] = 0;
+  }
+  c->timing = on != 0;
+  return PCS_OK;
+}
+
+pcs_status pcs_timing_read(pcs_ctx* c, pcs_kernel_time* out, int32_t max, int32_t* n) {
+  if (!c || !n || (max > 0 && !out)) return fail(PCS_E_INVAL, "null argument");
+  std::lock_guard<std::mutex> lk(c->mu);
+  for (auto& t : c->timed) {
+    float ms = 0;
+    PCS_CUDA(cudaEventSynchronize(t.stop));
+    PCS_CUDA(cudaEventElapsedTime(&ms, t.start, t.stop));
+    c->kernel_ms[t.kind] += ms;
+    c->kernel_n[t.kind] += 1;
+    c->timing_events.push_back(t.start);
+    c->timing_events.push_back(t.stop);
+  }
+  c->timed.clear();
+  int32_t k = 0;
+  for (int i = 0; i < kKernelKinds; ++i) {
+    if (c->kernel_n[i] == 0) continue;
+    if (k < max) {
+      std::snprintf(out[k].name, sizeof out[k].name, "%s", kKernelNames[i]);
+      out[k].launches = c->kernel_n[i];
+      out[k].total_ms = c->kernel_ms[i];
+    }
+    ++k;
+  }
+  *n = k;
+  return PCS_OK;
+}
+
+pcs_status pcs_sync(pcs_ctx* c, void* stream) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  PCS_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  uint32_t w = 0;
+  PCS_CUDA(cudaMemcpy(&w, c->words, 4, cudaMemcpyDeviceToHost));
+  if (w != 0) {
+    PCS_CUDA(cudaMemset(c->words, 0, 4));
+    return fail(PCS_E_RANGE, "a kernel met a row or page id out of range (error bits 0x%x)", w);
+  }
+  return PCS_OK;
+}
+
+pcs_status pcs_fingerprint(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t* fp_out,
+                           void* stream) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  if (n > 0 && !fp_out) return fail(PCS_E_INVAL, "fp_out is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  return fingerprint_impl(c, bufs, n, fp_out, nullptr, nullptr, stream);
+}
+
+pcs_status pcs_classify(pcs_ctx* c, const pcs_buf* bufs, int32_t n, const uint64_t* fp_before,
+                        uint64_t* fp_after, uint8_t* must_snapshot, void* stream) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  if (n > 0 && (!fp_before || !must_snapshot))
+    return fail(PCS_E_INVAL, "fp_before and must_snapshot are required");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  return fingerprint_impl(c, bufs, n, fp_after, fp_before, must_snapshot, stream);
+}
+
+pcs_status pcs_prune_counts(const pcs_bank* banks, int32_t n, const pcs_prune_params* p,
+                            int32_t* k_out) {
+  if (n < 0 || (n > 0 && (!banks || !k_out)) || !p) return fail(PCS_E_INVAL, "bad arguments");
+  for (int s = 0; s < n; ++s)
+    if (banks[s].n_entries < 0) return fail(PCS_E_INVAL, "bank %d: negative n_entries", s);
+  switch (p->rule) {
+    case PCS_K_FIXED:
+      if (p->k_max < 0) return fail(PCS_E_INVAL, "k_max < 0");
+      for (int s = 0; s < n; ++s) k_out[s] = std::min(banks[s].n_entries, p->k_max);
+      return PCS_OK;
+    case PCS_K_BUDGET: {
+      unsigned __int128 T = 0;
+      for (int s = 0; s < n; ++s)
+        T += static_cast<unsigned __int128>(static_cast<uint64_t>(banks[s].n_entries)) *
+             banks[s].entry_bytes;
+      for (int s = 0; s < n; ++s) {
+        if (T <= p->budget_bytes) {
+          k_out[s] = banks[s].n_entries;
+        } else {
+          const unsigned __int128 num =
+              static_cast<unsigned __int128>(static_cast<uint64_t>(banks[s].n_entries)) *
+              p->budget_bytes;
+          k_out[s] = static_cast<int32_t>(num / T);
+        }
+      }
+      return PCS_OK;
+    }
+    case PCS_K_FRACTION: {
+      if (!(p->fraction >= 0.0 && p->fraction <= 1.0))
+        return fail(PCS_E_INVAL, "fraction must lie in [0, 1]");
+      for (int s = 0; s < n; ++s) {
+        // Round to nearest, ties to even (default rounding mode).
+        double v = __builtin_nearbyint(p->fraction * static_cast<double>(banks[s].n_entries));
+        v = std::min<double>(std::max(v, 0.0), banks[s].n_entries);
+        k_out[s] = static_cast<int32_t>(v);
+      }
+      return PCS_OK;
+    }
+    default:
+      return fail(PCS_E_INVAL, "unknown k-rule %d", p->rule);
+  }
+}
+
+pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_prune_params* p,
+                     float* scores, int32_t* kept_idx, int32_t* kept_off, void* stream_) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::vector<int32_t> k(std::max(n, 0));
+  pcs_status st = pcs_prune_counts(banks, n, p, k.data());
+  if (st) return st;
+  if (n == 0) return PCS_OK;
+  std::vector<BankDesc> d(n);
+  std::vector<int32_t> koff(n + 1, 0);
+  uint64_t entries = 0, kept = 0;
+  for (int s = 0; s < n; ++s) {
+    const pcs_bank& b = banks[s];
+    if (b.key_dtype != PCS_DT_F16 && b.key_dtype != PCS_DT_BF16)
+      return fail(PCS_E_INVAL, "bank %d: key_dtype must be F16 or BF16", s);
+    if (b.key_dim <= 0 || b.key_dim % 8 != 0)
+      return fail(PCS_E_ALIGN, "bank %d: key_dim must be a positive multiple of 8", s);
+    if (b.n_entries > 0 && (!b.keys || !b.query))
+      return fail(PCS_E_INVAL, "bank %d: null keys or query", s);
+    if (b.n_entries > 0 && (!aligned16(b.keys) || !aligned16(b.query)))
+      return fail(PCS_E_ALIGN, "bank %d: keys / query not 16-byte aligned", s);
+    d[s].keys = static_cast<const uint16_t*>(b.keys);
+    d[s].query = static_cast<const uint16_t*>(b.query);
+    d[s].entry_begin = entries;
+    d[s].kept_begin = kept;
+    d[s].n = b.n_entries;
+    d[s].D = b.key_dim;
+    d[s].k = k[s];
+    d[s].is_bf16 = b.key_dtype == PCS_DT_BF16;
+    entries += b.n_entries;
+    kept += k[s];
+    koff[s + 1] = static_cast<int32_t>(kept);
+  }
+  if (kept > 0 && !kept_idx) return fail(PCS_E_INVAL, "kept_idx is null");
+  if (entries > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many entries in one call");
+  std::lock_guard<std::mutex> lk(c->mu);
+  st = set_device(c);
+  if (st) return st;
+  WsLayout L;
+  L.banks = 0;
+  L.secs = round_up(sizeof(BankDesc) * n, kRecordAlign);       // kept offsets (int32)
+  L.nodes = round_up(L.secs + 4ull * (n + 1), kRecordAlign);   // scores if caller gives none
+  L.total = L.nodes + (scores ? 0 : 4 * entries);
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, L.total, stream, &ws);
+  if (st) return st;
+  c->plan.resize(L.nodes);
+  put(c->plan, L.banks, d);
+  put(c->plan, L.secs, koff);
+  PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
+  if (kept_off)
+    PCS_CUDA(cudaMemcpyAsync(kept_off, ws + L.secs, 4ull * (n + 1), cudaMemcpyDeviceToDevice, stream));
+  float* sc = scores ? scores : reinterpret_cast<float*>(ws + L.nodes);
+  auto* dbanks = reinterpret_cast<const BankDesc*>(ws + L.banks);
+  {
+    LaunchScope ls(c, kKScore, stream);
+    PCS_CUDA(launch_score(dbanks, n, entries, nullptr, sc, c->sm_count, stream));
+  }
+  {
+    LaunchScope ls(c, kKTopk, stream);
+    PCS_CUDA(launch_topk(dbanks, n, sc, kept_idx, stream));
+  }
+  return ws_release(c, stream);
+}
+
+pcs_status pcs_record_bytes(const pcs_section* sections, int32_t n, uint64_t* out) {
+  if (!out || n < 1 || n > 65535 || !sections) return fail(PCS_E_INVAL, "bad section list");
+  uint64_t off = round_up(kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * n, kRecordAlign);
+  for (int i = 0; i < n; ++i) off = round_up(off + sections[i].bytes, kRecordAlign);
+  *out = off;
+  return PCS_OK;
+}
+
+pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, uint32_t placement,
+                          pcs_snapshot** out, void* stream_) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  if (n < 0 || (n > 0 && (!sessions || !out))) return fail(PCS_E_INVAL, "bad session list");
+  if (placement != PCS_PLACE_DEVICE && placement != PCS_PLACE_PINNED_HOST)
+    return fail(PCS_E_INVAL, "unknown placement %u", placement);
+  if (n == 0) return PCS_OK;
+  // Plan records: sizes, offsets, entries.
+  std::vector<uint64_t> rec_off(n + 1, 0), pstart(n);
+  uint64_t total_secs = 0;
+  for (int s = 0; s < n; ++s) {
+    const pcs_session& S = sessions[s];
+    if (S.n_sections < 1 || S.n_sections > 65535 || !S.sections)
+      return fail(PCS_E_INVAL, "session %d: needs 1..65535 sections", s);
+    for (int i = 0; i < S.n_sections; ++i) {
+      pcs_status st = check_section(S.sections[i], s, i, false);
+      if (st) return st;
+    }
+    uint64_t bytes = 0;
+    pcs_record_bytes(S.sections, S.n_sections, &bytes);
+    pstart[s] = round_up(kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * S.n_sections, kRecordAlign);
+    rec_off[s + 1] = rec_off[s] + bytes;
+    total_secs += S.n_sections;
+  }
+  if (total_secs > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many sections in one call");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  Block* blk = nullptr;
+  st = arena_of(c, placement)->alloc(rec_off[n], stream, &blk);
+  if (st) return st;
+  std::vector<SecDesc> d;
+  std::vector<SessDesc> sd(n);
+  std::vector<Entry> ent;
+  d.reserve(total_secs);
+  ent.reserve(total_secs);
+  std::vector<std::unique_ptr<pcs_snapshot>> handles(n);
+  uint64_t chunks = 0;
+  for (int s = 0; s < n; ++s) {
+    const pcs_session& S = sessions[s];
+    uint8_t* rec = blk->ptr + rec_off[s];
+    auto h = std::make_unique<pcs_snapshot>();
+    h->block = blk;
+    h->offset = rec_off[s];
+    h->total_bytes = rec_off[s + 1] - rec_off[s];
+    h->payload_start = pstart[s];
+    h->session_id = S.session_id;
+    h->kind = S.kind;
+    sd[s].record = rec;
+    sd[s].total_bytes = h->total_bytes;
+    sd[s].payload_start = pstart[s];
+    sd[s].sec_begin = static_cast<uint32_t>(d.size());
+    sd[s].n_sections = static_cast<uint32_t>(S.n_sections);
+    sd[s].session_id = S.session_id;
+    sd[s].kind = S.kind;
+    uint64_t off = pstart[s];
+    for (int i = 0; i < S.n_sections; ++i) {
+      const pcs_section& x = S.sections[i];
+      SecDesc desc = make_desc(x, rec + off, x.ring_start);
+      chunks += desc.n_chunks;
+      d.push_back(desc);
+      Entry e{};
+      e.type = x.type;
+      e.dtype = x.dtype;
+      e.layer = x.layer;
+      e.layout = x.layout;
+      e.offset = off;
+      e.bytes = x.bytes;
+      e.fp = 0;
+      e.dim0 = x.dim0;
+      e.dim1 = x.dim1;
+      e.aux = x.layout == PCS_LAYOUT_RING ? x.ring_start : 0;
+      ent.push_back(e);
+      h->table.push_back(e);
+      off = round_up(off + x.bytes, kRecordAlign);
+    }
+    handles[s] = std::move(h);
+  }
+  const int g = choose_group_log2(c, chunks);
+  const uint64_t tasks = assign_tasks(d, g);
+  WsLayout L;
+  L.secs = 0;
+  L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
+  L.entries = round_up(L.sess + sizeof(SessDesc) * n, kRecordAlign);
+  L.nodes = round_up(L.entries + sizeof(Entry) * ent.size(), kRecordAlign);
+  L.total = L.nodes + 8 * tasks;
+  auto undo = [&](pcs_status s) {
+    arena_of(c, placement)->free(blk);
+    return s;
+  };
+  if (tasks >= (1ull << 32)) return undo(fail(PCS_E_INVAL, "too much data in one call"));
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, L.total, stream, &ws);
+  if (st) return undo(st);
+  c->plan.resize(L.nodes);
+  put(c->plan, L.secs, d);
+  put(c->plan, L.sess, sd);
+  put(c->plan, L.entries, ent);
+  cudaError_t e = cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream);
+  auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
+  auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
+  auto* dent = reinterpret_cast<const Entry*>(ws + L.entries);
+  auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
+  if (e == cudaSuccess) {
+    LaunchScope ls(c, kKStreamPack, stream);
+    e = launch_stream(kModePack, dsecs, static_cast<int>(d.size()), static_cast<uint32_t>(tasks), g,
+                      nodes, c->words, c->sm_count, c->stream_bps, stream);
+  }
+  if (e == cudaSuccess) {
+    LaunchScope ls(c, kKFinalizePack, stream);
+    e = launch_finalize(kModePack, dsecs, dsess, n, dent, nodes, nullptr, nullptr, nullptr, nullptr,
+                        stream);
+  }
+  if (e != cudaSuccess) return undo(cuda_fail(e, "checkpoint launch"));
+  blk->written = record_event(c->events, stream);
+  st = ws_release(c, stream);
+  if (st) return undo(st);
+  blk->refs = n;
+  for (int s = 0; s < n; ++s) {
+    out[s] = handles[s].release();
+    c->live.insert(out[s]);
+  }
+  return PCS_OK;
+}
+
+pcs_status pcs_fork(pcs_ctx* c, const pcs_snapshot* parent, pcs_snapshot** child, void* stream_) {
+  if (!c || !child) return fail(PCS_E_INVAL, "null argument");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_snapshot* p = check_handle(c, parent);
+  if (!p) return fail(PCS_E_HANDLE, "unknown snapshot handle");
+  pcs_status st = set_device(c);
+  if (st) return st;
+  Block* blk = nullptr;
+  st = arena_of(c, p->block->placement)->alloc(p->total_bytes, stream, &blk);
+  if (st) return st;
+  st = wait_written(p->block, stream);
+  if (st) {
+    arena_of(c, blk->placement)->free(blk);
+    return st;
+  }
+  cudaError_t e;
+  {
+    LaunchScope ls(c, kKCopy, stream);
+    e = launch_copy(p->record(), blk->ptr, p->total_bytes, c->sm_count, stream);
+  }
+  if (e != cudaSuccess) {
+    arena_of(c, blk->placement)->free(blk);
+    return cuda_fail(e, "fork copy");
+  }
+  note_use(c, p->block, stream);
+  blk->written = record_event(c->events, stream);
+  blk->refs = 1;
+  auto h = std::make_unique<pcs_snapshot>(*p);
+  h->block = blk;
+  h->offset = 0;
+  *child = h.release();
+  c->live.insert(*child);
+  return PCS_OK;
+}
+
+pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const pcs_session* targets,
+                       int32_t verify, void* stream_) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  if (n < 0 || (n > 0 && (!snaps || !targets))) return fail(PCS_E_INVAL, "bad arguments");
+  if (n == 0) return PCS_OK;
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  std::vector<SecDesc> d;
+  std::vector<SessDesc> sd(n);
+  uint64_t chunks = 0;
+  for (int s = 0; s < n; ++s) {
+    pcs_snapshot* h = check_handle(c, snaps[s]);
+    if (!h) return fail(PCS_E_HANDLE, "snapshot %d: unknown handle", s);
+    const pcs_session& T = targets[s];
+    if (T.n_sections != static_cast<int32_t>(h->table.size()) || !T.sections)
+      return fail(PCS_E_INVAL, "session %d: target has %d sections, snapshot %zu", s,
+                  T.n_sections, h->table.size());
+    sd[s].record = h->record();
+    sd[s].total_bytes = h->total_bytes;
+    sd[s].payload_start = h->payload_start;
+    sd[s].sec_begin = static_cast<uint32_t>(d.size());
+    sd[s].n_sections = static_cast<uint32_t>(T.n_sections);
+    sd[s].session_id = h->session_id;
+    sd[s].kind = h->kind;
+    for (int i = 0; i < T.n_sections; ++i) {
+      const pcs_section& x = T.sections[i];
+      st = check_section(x, s, i, true);
+      if (st) return st;
+      const Entry& e = h->table[i];
+      if (x.bytes != e.bytes)
+        return fail(PCS_E_INVAL, "session %d section %d: target bytes %llu != snapshot %llu", s, i,
+                    static_cast<unsigned long long>(x.bytes), static_cast<unsigned long long>(e.bytes));
+      uint32_t rs = x.ring_start;
+      if (x.layout == PCS_LAYOUT_RING && rs == PCS_RING_START_FROM_SNAPSHOT) {
+        if (e.layout != PCS_LAYOUT_RING || e.aux >= x.window)
+          return fail(PCS_E_INVAL, "session %d section %d: no stored ring start fits", s, i);
+        rs = static_cast<uint32_t>(e.aux);
+      }
+      SecDesc desc = make_desc(x, h->record() + e.offset, rs);
+      chunks += desc.n_chunks;
+      d.push_back(desc);
+    }
+  }
+  for (int s = 0; s < n; ++s) {
+    st = wait_written(snaps[s]->block, stream);
+    if (st) return st;
+  }
+  const int g = choose_group_log2(c, chunks);
+  const uint64_t tasks = assign_tasks(d, g);
+  if (tasks >= (1ull << 32)) return fail(PCS_E_INVAL, "too much data in one call");
+  WsLayout L;
+  L.secs = 0;
+  L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
+  L.nodes = round_up(L.sess + sizeof(SessDesc) * n, kRecordAlign);
+  L.total = L.nodes + (verify ? 8 * tasks : 0);
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, L.total, stream, &ws);
+  if (st) return st;
+  c->plan.resize(L.nodes);
+  put(c->plan, L.secs, d);
+  put(c->plan, L.sess, sd);
+  PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
+  auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
+  auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
+  auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
+  if (verify) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
+  {
+    const int mode = verify ? kModeRestoreV : kModeRestore;
+    LaunchScope ls(c, stream_kind(mode), stream);
+    PCS_CUDA(launch_stream(mode, dsecs, static_cast<int>(d.size()), static_cast<uint32_t>(tasks), g,
+                           nodes, c->words, c->sm_count, c->stream_bps, stream));
+  }
+  if (verify) {
+    LaunchScope ls(c, kKFinalizeRestoreV, stream);
+    PCS_CUDA(launch_finalize(kModeRestoreV, dsecs, dsess, n, nullptr, nodes, nullptr, nullptr,
+                             nullptr, c->words + 1, stream));
+  }
+  for (int s = 0; s < n; ++s) {
+    st = note_use(c, snaps[s]->block, stream);
+    if (st) return st;
+  }
+  st = ws_release(c, stream);
+  if (st) return st;
+  if (verify) {
+    uint32_t bad = 0;
+    PCS_CUDA(cudaMemcpyAsync(&bad, c->words + 1, 4, cudaMemcpyDeviceToHost, stream));
+    PCS_CUDA(cudaStreamSynchronize(stream));
+    if (bad) return fail(PCS_E_CORRUPT, "%u of %d restored sessions failed verification", bad, n);
+  }
+  return PCS_OK;
+}
+
+pcs_status pcs_delete(pcs_ctx* c, pcs_snapshot* h) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  if (!check_handle(c, h)) return fail(PCS_E_HANDLE, "unknown snapshot handle");
+  c->live.erase(h);
+  release_block(c, h->block);
+  delete h;
+  return PCS_OK;
+}
+
+static pcs_status read_record(pcs_ctx* c, pcs_snapshot* h, uint64_t off, uint64_t bytes, void* dst) {
+  if (h->block->written) PCS_CUDA(cudaEventSynchronize(h->block->written->ev));
+  PCS_CUDA(cudaMemcpy(dst, h->record() + off, bytes, cudaMemcpyDefault));
+  (void)c;
+  return PCS_OK;
+}
+
+pcs_status pcs_snapshot_get_info(pcs_ctx* c, const pcs_snapshot* snap, pcs_snapshot_info* out) {
+  if (!c || !out) return fail(PCS_E_INVAL, "null argument");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_snapshot* h = check_handle(c, snap);
+  if (!h) return fail(PCS_E_HANDLE, "unknown snapshot handle");
+  pcs_status st = set_device(c);
+  if (st) return st;
+  uint8_t hdr[64];
+  st = read_record(c, h, 0, 64, hdr);
+  if (st) return st;
+  out->session_id = h->session_id;
+  out->kind = h->kind;
+  out->n_sections = static_cast<int32_t>(h->table.size());
+  out->placement = h->block->placement;
+  out->total_bytes = h->total_bytes;
+  std::memcpy(&out->session_fp, hdr + 24, 8);
+  out->data = h->record();
+  return PCS_OK;
+}
+
+pcs_status pcs_snapshot_get_section(pcs_ctx* c, const pcs_snapshot* snap, int32_t i,
+                                pcs_section_info* out) {
+  if (!c || !out) return fail(PCS_E_INVAL, "null argument");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_snapshot* h = check_handle(c, snap);
+  if (!h) return fail(PCS_E_HANDLE, "unknown snapshot handle");
+  if (i < 0 || i >= static_cast<int32_t>(h->table.size()))
+    return fail(PCS_E_INVAL, "section %d out of range", i);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  Entry e;
+  st = read_record(c, h, kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * i, sizeof e, &e);
+  if (st) return st;
+  out->type = e.type;
+  out->dtype = e.dtype;
+  out->layer = e.layer;
+  out->layout = e.layout;
+  out->offset = e.offset;
+  out->bytes = e.bytes;
+  out->fp = e.fp;
+  out->dim0 = e.dim0;
+  out->dim1 = e.dim1;
+  out->aux = e.aux;
+  return PCS_OK;
+}
+
+pcs_status pcs_snapshot_copy_out(pcs_ctx* c, const pcs_snapshot* snap, uint64_t offset,
+                                 uint64_t bytes, void* dst, void* stream_) {
+  if (!c || (bytes > 0 && !dst)) return fail(PCS_E_INVAL, "null argument");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_snapshot* h = check_handle(c, snap);
+  if (!h) return fail(PCS_E_HANDLE, "unknown snapshot handle");
+  if (offset > h->total_bytes || bytes > h->total_bytes - offset)
+    return fail(PCS_E_INVAL, "range outside the record");
+  pcs_status st = set_device(c);
+  if (st) return st;
+  if (bytes == 0) return PCS_OK;
+  st = wait_written(h->block, stream);
+  if (st) return st;
+  PCS_CUDA(cudaMemcpyAsync(dst, h->record() + offset, bytes, cudaMemcpyDefault, stream));
+  return note_use(c, h->block, stream);
+}
+
+static pcs_status ensure_stage(pcs_ctx* c) {
+  if (c->stage) return PCS_OK;
+  if (cudaHostAlloc(&c->stage, kStageBytes, cudaHostAllocDefault) != cudaSuccess) {
+    cudaGetLastError();
+    c->stage = nullptr;
+    return fail(PCS_E_NOMEM, "cannot allocate the pinned staging buffer");
+  }
+  c->stage_bytes = kStageBytes;
+  return PCS_OK;
+}
+
+pcs_status pcs_snapshot_write_file(pcs_ctx* c, const pcs_snapshot* snap, const char* path) {
+  if (!c || !path) return fail(PCS_E_INVAL, "null argument");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_snapshot* h = check_handle(c, snap);
+  if (!h) return fail(PCS_E_HANDLE, "unknown snapshot handle");
+  pcs_status st = set_device(c);
+  if (st) return st;
+  if (h->block->written) PCS_CUDA(cudaEventSynchronize(h->block->written->ev));
+  st = ensure_stage(c);
+  if (st) return st;
+  std::string tmp = std::string(path) + ".tmp";
+  FILE* f = std::fopen(tmp.c_str(), "wb");
+  if (!f) return fail(PCS_E_IO, "cannot open %s: %s", tmp.c_str(), std::strerror(errno));
+  for (uint64_t off = 0; off < h->total_bytes; off += c->stage_bytes) {
+    const uint64_t nb = std::min(c->stage_bytes, h->total_bytes - off);
+    cudaError_t e = cudaMemcpy(c->stage, h->record() + off, nb, cudaMemcpyDefault);
+    if (e != cudaSuccess || std::fwrite(c->stage, 1, nb, f) != nb) {
+      std::fclose(f);
+      std::remove(tmp.c_str());
+      if (e != cudaSuccess) return cuda_fail(e, "snapshot read-back");
+      return fail(PCS_E_IO, "write to %s failed", tmp.c_str());
+    }
+  }
+  if (std::fflush(f) != 0 || fsync(fileno(f)) != 0) {
+    std::fclose(f);
+    std::remove(tmp.c_str());
+    return fail(PCS_E_IO, "flush of %s failed", tmp.c_str());
+  }
+  std::fclose(f);
+  if (std::rename(tmp.c_str(), path) != 0) {
+    std::remove(tmp.c_str());
+    return fail(PCS_E_IO, "rename to %s failed: %s", path, std::strerror(errno));
+  }
+  return PCS_OK;
+}
+
+pcs_status pcs_snapshot_read_file(pcs_ctx* c, const char* path, uint32_t placement,
+                                  pcs_snapshot** out) {
+  if (!c || !path || !out) return fail(PCS_E_INVAL, "null argument");
+  if (placement != PCS_PLACE_DEVICE && placement != PCS_PLACE_PINNED_HOST)
+    return fail(PCS_E_INVAL, "unknown placement %u", placement);
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  FILE* f = std::fopen(path, "rb");
+  if (!f) return fail(PCS_E_IO, "cannot open %s: %s", path, std::strerror(errno));
+  auto close_fail = [&](pcs_status s) {
+    std::fclose(f);
+    return s;
+  };
+  if (std::fseek(f, 0, SEEK_END) != 0) return close_fail(fail(PCS_E_IO, "seek failed"));
+  const long fsize = std::ftell(f);
+  std::rewind(f);
+  uint8_t hdr[64];
+  if (fsize < 64 || std::fread(hdr, 1, 64, f) != 64)
+    return close_fail(fail(PCS_E_CORRUPT, "%s: too short for a record header", path));
+  uint32_t magic, vn, sid, kind;
+  uint64_t total;
+  std::memcpy(&magic, hdr, 4);
+  std::memcpy(&vn, hdr + 4, 4);
+  std::memcpy(&sid, hdr + 8, 4);
+  std::memcpy(&kind, hdr + 12, 4);
+  std::memcpy(&total, hdr + 16, 8);
+  const uint32_t nsec = vn >> 16;
+  if (magic != kMagic || (vn & 0xFFFFu) != kVersion)
+    return close_fail(fail(PCS_E_CORRUPT, "%s: not a PCS1 record", path));
+  const uint64_t pstart = round_up(kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * nsec, kRecordAlign);
+  if (nsec < 1 || total != static_cast<uint64_t>(fsize) || total % kRecordAlign != 0 || pstart > total)
+    return close_fail(fail(PCS_E_CORRUPT, "%s: header sizes do not match the file", path));
+  std::vector<Entry> table(nsec);
+  if (std::fread(table.data(), sizeof(Entry), nsec, f) != nsec)
+    return close_fail(fail(PCS_E_CORRUPT, "%s: truncated section table", path));
+  uint64_t expect = pstart;
+  for (uint32_t i = 0; i < nsec; ++i) {
+    const Entry& e = table[i];
+    if (e.offset != expect || e.bytes > total - e.offset || e.layout > PCS_LAYOUT_RING)
+      return close_fail(fail(PCS_E_CORRUPT, "%s: section %u has an impossible offset or size", path, i));
+    expect = round_up(e.offset + e.bytes, kRecordAlign);
+  }
+  if (expect != total) return close_fail(fail(PCS_E_CORRUPT, "%s: record size mismatch", path));
+  Block* blk = nullptr;
+  st = arena_of(c, placement)->alloc(total, nullptr, &blk);
+  if (st) return close_fail(st);
+  // Anything that reused this range must be done before the host writes it.
+  PCS_CUDA(cudaDeviceSynchronize());
+  std::rewind(f);
+  if (placement == PCS_PLACE_PINNED_HOST) {
+    if (std::fread(blk->ptr, 1, total, f) != total) {
+      arena_of(c, placement)->free(blk);
+      return close_fail(fail(PCS_E_IO, "%s: read failed", path));
+    }
+  } else {
+    st = ensure_stage(c);
+    if (st) {
+      arena_of(c, placement)->free(blk);
+      return close_fail(st);
+    }
+    for (uint64_t off = 0; off < total; off += c->stage_bytes) {
+      const uint64_t nb = std::min(c->stage_bytes, total - off);
+      if (std::fread(c->stage, 1, nb, f) != nb ||
+          cudaMemcpy(blk->ptr + off, c->stage, nb, cudaMemcpyHostToDevice) != cudaSuccess) {
+        arena_of(c, placement)->free(blk);
+        return close_fail(fail(PCS_E_IO, "%s: read failed", path));
+      }
+    }
+  }
+  std::fclose(f);
+  blk->refs = 1;
+  auto h = std::make_unique<pcs_snapshot>();
+  h->block = blk;
+  h->offset = 0;
+  h->total_bytes = total;
+  h->payload_start = pstart;
+  h->session_id = sid;
+  h->kind = kind;
+  h->table = table;
+  for (auto& e : h->table) e.fp = 0;
+  *out = h.release();
+  c->live.insert(*out);
+  return PCS_OK;
+}
+
+}  // extern "C"

@@ -25,3 +25,20 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+@pytest.fixture(scope="session")
+def ctx():
+    import torch
+    from paper_2607_21686_gb300 import build, pcs
+    build.build()
+    torch.cuda.set_device(0)
+    c = pcs.Context(0)
+    yield c
+    c.close()
+
+
+@pytest.fixture(scope="session")
+def dev():
+    import torch
+    return torch.device("cuda:0")
