@@ -29,8 +29,10 @@
  *   - Pointers marked "device" must be device (or mapped pinned host) memory
  *     reachable from the GPU of the context; the caller owns every buffer it
  *     passes.  Buffers are read or written only by work enqueued on `stream`.
- *   - Alignment: every contiguous buffer, row base and row size must be a
- *     multiple of 16 bytes (else PCS_E_ALIGN).  Byte counts may be any size.
+ *   - Alignment: row bases and row sizes (ROWS / RING layouts) and bank
+ *     keys / queries must be multiples of 16 bytes (else PCS_E_ALIGN).
+ *     Contiguous buffers and sections may have any address and byte count;
+ *     16-byte aligned ones take the 128-bit vector path.
  *   - Snapshots are owned by the library (device or pinned host arenas) and
  *     are immutable after checkpoint; a handle is valid until pcs_delete.
  *   - A context may be used from several host threads; calls are serialised
@@ -114,7 +116,7 @@ typedef struct pcs_snapshot pcs_snapshot;
 
 /* A runtime buffer to fingerprint: `bytes` bytes at device pointer `ptr`. */
 typedef struct pcs_buf {
-    const void *ptr;   /* device, 16-byte aligned (may be NULL if bytes==0) */
+    const void *ptr;   /* device, any alignment (may be NULL if bytes==0)   */
     uint64_t bytes;
     uint32_t dtype;    /* PCS_DT_* (informational)                          */
     uint32_t flags;    /* reserved, 0                                       */
@@ -130,7 +132,8 @@ typedef struct pcs_buf {
  *           every page id must lie in [0, base_rows); window must be a
  *           multiple of page_rows; ring_start < window (restore targets may
  *           pass PCS_RING_START_FROM_SNAPSHOT).
- * row_bytes and base must be multiples of 16; `index` is device int32.
+ * ROWS / RING: row_bytes and base must be multiples of 16; `index` is
+ * device int32.  CONTIG: any address.
  */
 typedef struct pcs_section {
     uint32_t type;        /* PCS_SEC_*                                      */

@@ -50,7 +50,8 @@ struct alignas(16) SecDesc {
   uint32_t task_begin;     // first warp task (= node slot) of this stream
   uint32_t n_tasks;
   uint64_t n_chunks;
-  uint64_t pad0;
+  uint32_t align;          // CONTIG layout side: 16, 4 or 1 (largest that divides lbase)
+  uint32_t pad0;
 };
 static_assert(sizeof(SecDesc) == 96, "SecDesc layout");
 

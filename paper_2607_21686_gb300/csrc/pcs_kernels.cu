@@ -108,20 +108,35 @@ __device__ __forceinline__ void st_stream(uint8_t* p, uint4 v) {
   __stcs(reinterpret_cast<uint4*>(p), v);
 }
 
-// Bytes [0, n) of a segment, n < 16; the rest read as zero.
-__device__ __forceinline__ uint4 ld_partial(const uint8_t* p, int n) {
+// Bytes [0, n) of a segment (n <= 16) at an address that may not be 16-byte
+// aligned; whole 32-bit words when `a4` (4-byte aligned).  The rest read as 0.
+__device__ __forceinline__ uint4 ld_small(const uint8_t* p, int n, bool a4) {
   uint32_t w[4] = {0, 0, 0, 0};
 #pragma unroll
-  for (int i = 0; i < 16; ++i)
-    if (i < n) w[i >> 2] |= static_cast<uint32_t>(p[i]) << (8 * (i & 3));
+  for (int j = 0; j < 4; ++j) {
+    if (a4 && 4 * j + 4 <= n) {
+      w[j] = *reinterpret_cast<const uint32_t*>(p + 4 * j);
+    } else {
+#pragma unroll
+      for (int b = 0; b < 4; ++b)
+        if (4 * j + b < n) w[j] |= static_cast<uint32_t>(p[4 * j + b]) << (8 * b);
+    }
+  }
   return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-__device__ __forceinline__ void st_partial(uint8_t* p, uint4 v, int n) {
+__device__ __forceinline__ void st_small(uint8_t* p, uint4 v, int n, bool a4) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-  for (int i = 0; i < 16; ++i)
-    if (i < n) p[i] = static_cast<uint8_t>(w[i >> 2] >> (8 * (i & 3)));
+  for (int j = 0; j < 4; ++j) {
+    if (a4 && 4 * j + 4 <= n) {
+      *reinterpret_cast<uint32_t*>(p + 4 * j) = w[j];
+    } else {
+#pragma unroll
+      for (int b = 0; b < 4; ++b)
+        if (4 * j + b < n) p[4 * j + b] = static_cast<uint8_t>(w[j] >> (8 * b));
+    }
+  }
 }
 
 // Zero the bytes of a segment at or past `n` (n in [1, 16)).
@@ -185,8 +200,8 @@ __device__ __forceinline__ uint4 load_seg(const SecDesc& s, uint64_t off, uint32
   if (ModeTraits<MODE>::kLoadLayout) {
     if (s.layout == kContig) {
       const uint64_t left = s.bytes - off;
-      if (left >= 16) return ld_stream(s.lbase + off);
-      return ld_partial(s.lbase + off, static_cast<int>(left));
+      if (left >= 16 && s.align == 16) return ld_stream(s.lbase + off);
+      return ld_small(s.lbase + off, left < 16 ? static_cast<int>(left) : 16, s.align >= 4);
     }
     const uint8_t* p = row_addr(s, off, err);
     return p ? ld_stream(p) : z;
@@ -211,8 +226,8 @@ __device__ __forceinline__ void store_seg(const SecDesc& s, uint64_t off, uint4 
     if (off >= s.bytes) return;
     if (s.layout == kContig) {
       const uint64_t left = s.bytes - off;
-      if (left >= 16) st_stream(s.lbase + off, v);
-      else st_partial(s.lbase + off, v, static_cast<int>(left));
+      if (left >= 16 && s.align == 16) st_stream(s.lbase + off, v);
+      else st_small(s.lbase + off, v, left < 16 ? static_cast<int>(left) : 16, s.align >= 4);
       return;
     }
     uint8_t* p = row_addr(s, off, err);

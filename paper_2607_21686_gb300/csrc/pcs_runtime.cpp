@@ -482,8 +482,6 @@ pcs_status check_section(const pcs_section& s, int sess, int i, bool target) {
   if (s.layout == PCS_LAYOUT_CONTIG) {
     if (s.bytes > 0 && !s.base)
       return fail(PCS_E_INVAL, "session %d section %d: null base", sess, i);
-    if (s.bytes > 0 && !aligned16(s.base))
-      return fail(PCS_E_ALIGN, "session %d section %d: base not 16-byte aligned", sess, i);
     return PCS_OK;
   }
   if (s.row_bytes == 0 || s.row_bytes % 16 != 0)
@@ -531,6 +529,8 @@ SecDesc make_desc(const pcs_section& s, uint8_t* payload, uint32_t ring_start) {
   d.page_rows = s.page_rows;
   d.pr_shift = s.layout == PCS_LAYOUT_RING ? log2_exact(s.page_rows) : 0;
   d.n_chunks = n_chunks_of(s.bytes);
+  const uintptr_t a = reinterpret_cast<uintptr_t>(s.base);
+  d.align = (a & 15u) == 0 ? 16u : ((a & 3u) == 0 ? 4u : 1u);
   return d;
 }
 
@@ -560,8 +560,6 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   uint64_t chunks = 0;
   for (int i = 0; i < n; ++i) {
     if (bufs[i].bytes > 0 && !bufs[i].ptr) return fail(PCS_E_INVAL, "buffer %d: null pointer", i);
-    if (bufs[i].bytes > 0 && !aligned16(bufs[i].ptr))
-      return fail(PCS_E_ALIGN, "buffer %d: pointer not 16-byte aligned", i);
     pcs_section s{};
     s.layout = PCS_LAYOUT_CONTIG;
     s.base = const_cast<void*>(bufs[i].ptr);

@@ -79,11 +79,12 @@ def test_rng_single_bit_flip(ctx, dev):
         assert u64(ctx.fingerprint([r2]))[0] != base
 
 
-def test_unaligned_pointer_rejected(ctx, dev):
-    t = torch.zeros(64, dtype=torch.uint8, device=dev)
-    with pytest.raises(pcs.PcsError) as e:
-        ctx.fingerprint([t[1:]])
-    assert e.value.status == pcs.PCS_E_ALIGN
+def test_unaligned_views(ctx, dev):
+    # Views at every offset mod 16 (byte and 4-byte aligned paths).
+    base = _rand_bytes(3 * 4096 + 200, 9, dev)
+    views = [base[o:o + n] for o in [1, 2, 3, 4, 5, 8, 12, 15] for n in [0, 1, 5, 17, 4100]]
+    got = u64(ctx.fingerprint(views))
+    assert got == [oracle.fingerprint(np_bytes(v)) for v in views]
 
 
 def test_empty_list(ctx, dev):

@@ -326,7 +326,7 @@ def test_bad_handle_and_shape_errors(ctx, dev):
     obs, rng = m.obs.to(dev), m.rng.to(dev)
     snap = ctx.checkpoint([pcs.markov_session(1, obs, rng)])[0]
     with pytest.raises(pcs.PcsError) as e:
-        ctx.restore([snap], [pcs.markov_session(1, obs[:, :4], rng)])
+        ctx.restore([snap], [pcs.markov_session(1, obs.reshape(-1)[:100], rng)])
     assert e.value.status == pcs.PCS_E_INVAL
     handle = snap.handle
     ctx.delete(snap)
