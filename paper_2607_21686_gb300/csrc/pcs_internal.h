@@ -19,6 +19,7 @@ constexpr int kMaxGroupLog2 = 5;         // at most 32 chunks per warp task
 
 // Errors a kernel records (OR-ed into the context's device error word).
 constexpr uint32_t kDevErrIndex = 1u;    // a row / page id out of range
+constexpr uint32_t kDevErrTimeout = 2u;  // a bounded wait inside a kernel gave up
 
 enum Layout : uint32_t { kContig = 0, kRows = 1, kRing = 2 };
 
@@ -87,16 +88,34 @@ struct alignas(16) BankDesc {
 };
 static_assert(sizeof(BankDesc) == 48, "BankDesc layout");
 
-// Kernel launchers (pcs_kernels.cu).  All enqueue on `stream`, return the
-// CUDA error of the launch.
-struct LaunchShape {
-  int blocks;
-  int threads;
+// The streams one streaming kernel processes: item j is stream secs[ids[j]],
+// owning this kernel's tasks [begin[j], begin[j+1]) (the last up to n_tasks).
+// Task t of item j writes node secs[ids[j]].task_begin + (t - begin[j]).
+struct WorkList {
+  const uint32_t* ids;
+  const uint32_t* begin;
+  int n_items;
+  uint32_t n_tasks;
 };
 
-cudaError_t launch_stream(int mode, const SecDesc* secs, int n_secs, uint32_t n_tasks,
-                          int group_log2, uint64_t* nodes, uint32_t* dev_err, int sm_count,
-                          int blocks_per_sm, cudaStream_t stream);
+// Chunks per task of the TMA-staged kernel (a 16 KiB tile).
+constexpr int kBulkTileChunks = 4;
+// Smallest row size the TMA-staged kernel takes for ROWS / RING streams.
+constexpr uint64_t kBulkMinRowBytes = 512;
+
+// Kernel launchers (pcs_kernels.cu).  All enqueue on `stream`, return the
+// CUDA error of the launch.
+
+// Register kernel: warp tasks of 2^group_log2 chunks, 128-bit loads/stores.
+cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_log2,
+                          uint64_t* nodes, uint32_t* dev_err, int sm_count, int blocks_per_sm,
+                          cudaStream_t stream);
+
+// TMA-staged kernel: tasks of kBulkTileChunks chunks staged through shared
+// memory with cp.async.bulk; one persistent block per SM.
+cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* nodes,
+                        uint32_t* dev_err, int sm_count, cudaStream_t stream);
+size_t bulk_shared_bytes();
 
 // Section fps from the warp-task nodes (in place), then per mode:
 //   kModeHash: fp_out[i] = fp; if fp_before: flags[i] = fp != fp_before[i]

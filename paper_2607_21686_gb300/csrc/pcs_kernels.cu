@@ -235,9 +235,21 @@ __device__ __forceinline__ void store_seg(const SecDesc& s, uint64_t off, uint4 
   }
 }
 
+// Section of warp task `task` in a work list: last j with begin[j] <= task.
+__device__ __forceinline__ int find_item(const uint32_t* __restrict__ begin, int n_items,
+                                        uint32_t task) {
+  int lo = 0, hi = n_items - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (__ldg(begin + mid) <= task) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 2)
-    k_stream(const SecDesc* __restrict__ secs, int n_secs, uint32_t n_tasks, int glog2,
+    k_stream(const SecDesc* __restrict__ secs, WorkList wl, int glog2,
              uint64_t* __restrict__ nodes, uint32_t* err) {
   using T = ModeTraits<MODE>;
   __shared__ SecDesc sdesc[kWarps];
@@ -245,24 +257,19 @@ __global__ void __launch_bounds__(kThreads, 2)
   const int wib = threadIdx.x >> 5;
   const uint32_t nw = gridDim.x * kWarps;
   int cur = -1;
-  for (uint32_t task = blockIdx.x * kWarps + wib; task < n_tasks; task += nw) {
-    // The stream owning this task: last i with task_begin <= task.
-    int lo = 0, hi = n_secs - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (__ldg(&secs[mid].task_begin) <= task) lo = mid;
-      else hi = mid - 1;
-    }
-    if (lo != cur) {
+  for (uint32_t task = blockIdx.x * kWarps + wib; task < wl.n_tasks; task += nw) {
+    const int j = find_item(wl.begin, wl.n_items, task);
+    if (j != cur) {
       __syncwarp();
+      const SecDesc* src = &secs[__ldg(wl.ids + j)];
       if (lane < static_cast<int>(sizeof(SecDesc) / 16))
-        reinterpret_cast<uint4*>(&sdesc[wib])[lane] =
-            __ldg(reinterpret_cast<const uint4*>(&secs[lo]) + lane);
+        reinterpret_cast<uint4*>(&sdesc[wib])[lane] = __ldg(reinterpret_cast<const uint4*>(src) + lane);
       __syncwarp();
-      cur = lo;
+      cur = j;
     }
     const SecDesc& s = sdesc[wib];
-    const uint64_t c0 = static_cast<uint64_t>(task - s.task_begin) << glog2;
+    const uint32_t local = task - __ldg(wl.begin + j);
+    const uint64_t c0 = static_cast<uint64_t>(local) << glog2;
     const uint64_t c1 = min(c0 + (1ull << glog2), static_cast<unsigned long long>(s.n_chunks));
     uint64_t mine = 0;  // lane j keeps the hash of chunk c0 + j
     for (uint64_t c = c0; c < c1; c += 2) {
@@ -285,27 +292,483 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
       if (T::kHash) {
         uint64_t ha = fmix(kSeed ^ (c * 32u + lane));
-        uint64_t hb = fmix(kSeed ^ ((c + 1) * 32u + lane));
 #pragma unroll
         for (int k = 0; k < kSegs; ++k) ha = absorb(ha, va[k]);
+        ha = __shfl_sync(kFull, warp_tree(fmix(ha), 32, lane), 0);
+        const int jj = static_cast<int>(c - c0);
+        if (lane == jj) mine = ha;
         if (two) {
+          uint64_t hb = fmix(kSeed ^ ((c + 1) * 32u + lane));
 #pragma unroll
           for (int k = 0; k < kSegs; ++k) hb = absorb(hb, vb[k]);
+          hb = __shfl_sync(kFull, warp_tree(fmix(hb), 32, lane), 0);
+          if (lane == jj + 1) mine = hb;
         }
-        ha = warp_tree(fmix(ha), 32, lane);
-        hb = warp_tree(fmix(hb), 32, lane);
-        ha = __shfl_sync(kFull, ha, 0);
-        hb = __shfl_sync(kFull, hb, 0);
-        const int j = static_cast<int>(c - c0);
-        if (lane == j) mine = ha;
-        if (two && lane == j + 1) mine = hb;
       }
     }
     if (T::kHash) {
       const uint64_t root = warp_tree(mine, static_cast<int>(c1 - c0), lane);
-      if (lane == 0) nodes[task] = root;
+      if (lane == 0) nodes[s.task_begin + local] = root;
     }
   }
+}
+
+// ---------------------------------------------------------------------------
+// TMA-staged streaming kernel
+//
+// One block per SM: warp 0 produces, warps 1..8 consume.  A tile is 4 chunks
+// (16 KiB) of one stream in payload order.  The producer stages each tile in
+// shared memory with cp.async.bulk copies (one per contiguous run of rows of
+// the layout side, or one for the contiguous payload), completing on the
+// stage's mbarrier; consumer warp w owns stage w: it hashes the 4 chunks from
+// shared memory (4 interleaved lane chains), issues the bulk store of the
+// tile (payload, or the runs of the layout side), and frees the stage once
+// the store has read it.  Every wait is bounded in time; a wait that gives
+// up records kDevErrTimeout and the block stops.
+// ---------------------------------------------------------------------------
+
+constexpr int kBulkConsumers = 8;
+constexpr int kBulkStages = kBulkConsumers;
+constexpr int kTileChunks = kBulkTileChunks;
+constexpr uint32_t kTileBytes = kTileChunks * kChunkBytes;
+constexpr int kBulkThreads = 32 * (1 + kBulkConsumers);
+constexpr int kTileRows = 64;  // rows of >= 512 bytes in a tile, plus one
+constexpr uint64_t kWaitNs = 2000000000ull;  // give up a wait after 2 s
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait for the phase of `bar` with the given parity to complete.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (global_ns() - t0 > kWaitNs) return false;
+  return true;
+}
+
+__device__ __forceinline__ void bulk_g2s(void* sdst, const void* gsrc, uint32_t bytes,
+                                         uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(sdst)),
+      "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void bulk_s2g(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst),
+               "r"(smem_u32(ssrc)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Per-stage description of the tile in flight (written by the producer
+// before it arrives on the stage's barrier).
+struct StageMeta {
+  uint32_t sec;         // section index
+  uint32_t node;        // node slot of the tile
+  uint64_t p0, p1;      // payload bytes of the tile: [p0, p1)
+  uint64_t r0;          // first row of the tile (ROWS / RING)
+  uint32_t n_rows;      // rows touching [p0, p1)
+  uint32_t live;        // 1 = a tile, 0 = no more work
+  uint8_t* rowp[kTileRows];  // restore: layout-side address of each row
+};
+
+struct BulkShared {
+  alignas(128) uint8_t stage[kBulkStages][kTileBytes];
+  alignas(8) uint64_t full[kBulkStages];
+  uint64_t empty[kBulkStages];
+  StageMeta meta[kBulkStages];
+  // Producer scratch: the next batch's tiles, prepared before waiting.
+  StageMeta next[kBulkStages];
+  int32_t armed[kBulkStages];  // last use of each stage whose copies were issued
+  uint32_t abort;
+};
+
+// Layout-side address of row r of a ROWS / RING stream (null if out of range).
+__device__ __forceinline__ uint8_t* row_ptr(const SecDesc& s, uint64_t r, uint32_t* err) {
+  uint64_t id, row;
+  if (s.layout == kRows) {
+    id = static_cast<uint32_t>(__ldg(s.index + r));
+    row = id;
+  } else {
+    uint64_t slot = s.ring_start + r;
+    if (slot >= s.window) slot -= s.window;
+    const uint64_t pg = div_rows(slot, s.page_rows, s.pr_shift);
+    id = static_cast<uint32_t>(__ldg(s.index + pg));
+    row = id * s.page_rows + (slot - pg * s.page_rows);
+  }
+  if (id >= s.base_rows) {
+    atomicOr(err, kDevErrIndex);
+    return nullptr;
+  }
+  return s.lbase + row * s.row_bytes;
+}
+
+// End of the bytes of tile [p0, p1) that bulk copies stage: the layout side
+// up to its last whole 16-byte segment; the payload (padded to 256 bytes in
+// the record) up to its 16-byte-rounded end.
+template <int MODE>
+__device__ __forceinline__ uint64_t staged_end(const SecDesc& s, uint64_t p1) {
+  const uint64_t end =
+      ModeTraits<MODE>::kLoadLayout ? (s.bytes & ~15ull) : ((s.bytes + 15) & ~15ull);
+  return p1 < end ? p1 : end;
+}
+
+// Issue bulk copies between a tile's shared buffer and the layout side, one
+// per run of rows that are contiguous in memory, covering payload bytes
+// [m.p0, pe).  Lane i owns rows i and i + 32 (addresses rp0, rp1; null =
+// skipped).  Returns the bytes this lane copied.
+template <bool kLoad>
+__device__ __forceinline__ uint32_t issue_runs(const SecDesc& s, const StageMeta& m,
+                                               uint8_t* rp0, uint8_t* rp1, uint64_t pe,
+                                               uint8_t* tile, uint64_t* bar, int lane) {
+  const uint64_t rb = s.row_bytes;
+  const int n = static_cast<int>(m.n_rows);
+  const uintptr_t u0 = reinterpret_cast<uintptr_t>(rp0), u1 = reinterpret_cast<uintptr_t>(rp1);
+  uintptr_t prev0 = __shfl_up_sync(kFull, u0, 1);
+  uintptr_t prev1 = __shfl_up_sync(kFull, u1, 1);
+  const uintptr_t last0 = __shfl_sync(kFull, u0, 31);
+  if (lane == 0) prev1 = last0;
+  const bool v0 = lane < n, v1 = lane + 32 < n;
+  const bool st0 = v0 && (lane == 0 || u0 == 0 || prev0 == 0 || u0 != prev0 + rb);
+  const bool st1 = v1 && (u1 == 0 || prev1 == 0 || u1 != prev1 + rb);
+  const uint64_t starts = static_cast<uint64_t>(__ballot_sync(kFull, st0)) |
+                          (static_cast<uint64_t>(__ballot_sync(kFull, st1)) << 32);
+  uint32_t copied = 0;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int i = lane + 32 * h;
+    const bool st = h == 0 ? st0 : st1;
+    uint8_t* rp = h == 0 ? rp0 : rp1;
+    if (!st || rp == nullptr) continue;
+    const uint64_t later = i + 1 < 64 ? (starts >> (i + 1)) : 0;
+    const int next = later ? i + __ffsll(static_cast<long long>(later)) : n;
+    const uint64_t row_lo = (m.r0 + i) * rb, row_hi = (m.r0 + next) * rb;
+    const uint64_t a = row_lo > m.p0 ? row_lo : m.p0;
+    const uint64_t b = row_hi < pe ? row_hi : pe;
+    if (a >= b) continue;
+    uint8_t* g = rp + (a - row_lo);
+    uint8_t* sp = tile + (a - m.p0);
+    if (kLoad) bulk_g2s(sp, g, static_cast<uint32_t>(b - a), bar);
+    else bulk_s2g(g, sp, static_cast<uint32_t>(b - a));
+    copied += static_cast<uint32_t>(b - a);
+  }
+  return copied;
+}
+
+// Bytes of tile [p0, pe) that row i (owned by the calling lane) covers.
+__device__ __forceinline__ uint32_t row_share(const StageMeta& m, uint64_t rb, int i,
+                                              uint64_t pe) {
+  const uint64_t lo = (m.r0 + i) * rb, hi = lo + rb;
+  const uint64_t a = lo > m.p0 ? lo : m.p0, b = hi < pe ? hi : pe;
+  return b > a ? static_cast<uint32_t>(b - a) : 0u;
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kBulkThreads, 1)
+    k_bulk(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
+           uint32_t* err) {
+  using T = ModeTraits<MODE>;
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  BulkShared& sh = *reinterpret_cast<BulkShared*>(smem_raw);
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  if (threadIdx.x < kBulkStages) {
+    mbar_init(&sh.full[threadIdx.x], 1);
+    mbar_init(&sh.empty[threadIdx.x], 1);
+    sh.armed[threadIdx.x] = -1;
+  }
+  if (threadIdx.x == 0) sh.abort = 0;
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncthreads();
+
+  if (warp == 0) {
+    // ------------------------------ producer ------------------------------
+    bool stop = false;
+    for (uint32_t use = 0; !stop; ++use) {
+      // Batch `use`: tile m = use * kBulkStages + j goes to stage j; its
+      // global index is blockIdx.x + m * gridDim.x.
+      uint32_t sec_j = 0, loc_j = 0, node_j = 0;
+      bool have_j = false;
+      if (lane < kBulkStages) {
+        const uint64_t t = blockIdx.x + (static_cast<uint64_t>(use) * kBulkStages + lane) * gridDim.x;
+        if (t < wl.n_tasks) {
+          const int it = find_item(wl.begin, wl.n_items, static_cast<uint32_t>(t));
+          sec_j = __ldg(wl.ids + it);
+          loc_j = static_cast<uint32_t>(t) - __ldg(wl.begin + it);
+          node_j = __ldg(&secs[sec_j].task_begin) + loc_j;
+          have_j = true;
+        }
+      }
+      const unsigned have = __ballot_sync(kFull, have_j);
+      // Describe every tile of the batch and fetch its row addresses (all
+      // index loads of the batch in flight together).
+#pragma unroll
+      for (int j = 0; j < kBulkStages; ++j) {
+        if (!((have >> j) & 1u)) continue;
+        const uint32_t sec = __shfl_sync(kFull, sec_j, j);
+        const uint32_t loc = __shfl_sync(kFull, loc_j, j);
+        const uint32_t node = __shfl_sync(kFull, node_j, j);
+        const SecDesc& s = secs[sec];
+        const uint64_t L = s.bytes;
+        const uint64_t p0 = static_cast<uint64_t>(loc) * kTileBytes;
+        const uint64_t cend = s.n_chunks * kChunkBytes;
+        const uint64_t p1 = p0 + kTileBytes < cend ? p0 + kTileBytes : cend;
+        uint64_t r0 = 0;
+        uint32_t n_rows = 0;
+        StageMeta& nx = sh.next[j];
+        if (s.layout != kContig) {
+          r0 = div_rows(p0, s.row_bytes, s.rb_shift);
+          const uint64_t lim = L < p1 ? L : p1;
+          if (lim > p0) n_rows = static_cast<uint32_t>(div_rows(lim - 1, s.row_bytes, s.rb_shift) + 1 - r0);
+          nx.rowp[lane] = lane < static_cast<int>(n_rows) ? row_ptr(s, r0 + lane, err) : nullptr;
+          nx.rowp[lane + 32] = lane + 32 < static_cast<int>(n_rows) ? row_ptr(s, r0 + lane + 32, err) : nullptr;
+        }
+        if (lane == 0) {
+          nx.sec = sec;
+          nx.node = node;
+          nx.p0 = p0;
+          nx.p1 = p1;
+          nx.r0 = r0;
+          nx.n_rows = n_rows;
+          nx.live = 1;
+        }
+      }
+      __syncwarp();
+      for (int j = 0; j < kBulkStages; ++j) {
+        // Wait until consumer j has released stage j.
+        bool ok = true;
+        if (use > 0 && lane == 0) ok = mbar_wait(&sh.empty[j], (use - 1) & 1);
+        ok = __shfl_sync(kFull, ok, 0);
+        if (!ok || *reinterpret_cast<volatile uint32_t*>(&sh.abort)) {
+          if (lane == 0) {
+            atomicOr(err, kDevErrTimeout);
+            sh.abort = 1;
+          }
+          stop = true;
+          break;
+        }
+        StageMeta& m = sh.meta[j];
+        if (!((have >> j) & 1u)) {
+          // No tile: the consumer of stage j stops.
+          if (lane == 0) {
+            m.live = 0;
+            mbar_arrive_expect_tx(&sh.full[j], 0);
+          }
+          stop = true;
+          continue;
+        }
+        const StageMeta& nx = sh.next[j];
+        const SecDesc& s = secs[nx.sec];
+        const uint64_t p0 = nx.p0;
+        const uint64_t pe = staged_end<MODE>(s, nx.p1);
+        uint8_t* rp0 = nullptr;
+        uint8_t* rp1 = nullptr;
+        if (s.layout != kContig) {
+          rp0 = nx.rowp[lane];
+          rp1 = nx.rowp[lane + 32];
+          m.rowp[lane] = rp0;
+          m.rowp[lane + 32] = rp1;
+        }
+        if (lane == 0) {
+          m.sec = nx.sec;
+          m.node = nx.node;
+          m.p0 = nx.p0;
+          m.p1 = nx.p1;
+          m.r0 = nx.r0;
+          m.n_rows = nx.n_rows;
+          m.live = 1;
+          sh.armed[j] = static_cast<int32_t>(use);
+        }
+        uint8_t* tile = sh.stage[j];
+        if (!T::kLoadLayout || s.layout == kContig) {
+          // One contiguous piece: the record payload, or a contiguous buffer.
+          const uint32_t bytes = pe > p0 ? static_cast<uint32_t>(pe - p0) : 0u;
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive_expect_tx(&sh.full[j], bytes);
+            if (bytes) bulk_g2s(tile, T::kLoadLayout ? s.lbase + p0 : s.payload + p0, bytes, &sh.full[j]);
+          }
+        } else {
+          // Rows: zero the share of rows whose ids were out of range, count
+          // the bytes the copies will bring, arm the barrier, issue runs.
+          const uint64_t rb = s.row_bytes;
+          uint32_t mine = 0;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int i = lane + 32 * h;
+            if (i >= static_cast<int>(nx.n_rows)) continue;
+            const uint32_t share = row_share(nx, rb, i, pe);
+            if ((h == 0 ? rp0 : rp1) == nullptr) {
+              const uint64_t a = (nx.r0 + i) * rb > p0 ? (nx.r0 + i) * rb : p0;
+              for (uint32_t o = 0; o < share; o += 16)
+                *reinterpret_cast<uint4*>(tile + (a - p0) + o) = make_uint4(0, 0, 0, 0);
+            } else {
+              mine += share;
+            }
+          }
+          fence_async_smem();
+#pragma unroll
+          for (int d = 16; d > 0; d >>= 1) mine += __shfl_xor_sync(kFull, mine, d);
+          __syncwarp();
+          if (lane == 0) mbar_arrive_expect_tx(&sh.full[j], mine);
+          __syncwarp();
+          issue_runs<true>(s, nx, rp0, rp1, pe, tile, &sh.full[j], lane);
+        }
+        __syncwarp();
+      }
+      if (have != (1u << kBulkStages) - 1u) stop = true;
+    }
+    if (*reinterpret_cast<volatile uint32_t*>(&sh.abort) && lane == 0) {
+      // Let copies already issued land before the block leaves.
+      for (int j = 0; j < kBulkStages; ++j)
+        if (sh.armed[j] >= 0) mbar_wait(&sh.full[j], static_cast<uint32_t>(sh.armed[j]) & 1);
+    }
+    return;
+  }
+
+  // ------------------------------ consumers ------------------------------
+  const int w = warp - 1;  // owns stage w
+  uint64_t* full = &sh.full[w];
+  uint64_t* empty = &sh.empty[w];
+  uint8_t* tile = sh.stage[w];
+  const uint4 zero = make_uint4(0, 0, 0, 0);
+  for (uint32_t use = 0;; ++use) {
+    bool ok = true;
+    if (lane == 0) ok = mbar_wait(full, use & 1);
+    ok = __shfl_sync(kFull, ok, 0);
+    if (!ok || *reinterpret_cast<volatile uint32_t*>(&sh.abort)) {
+      if (lane == 0) {
+        atomicOr(err, kDevErrTimeout);
+        sh.abort = 1;
+      }
+      break;
+    }
+    const StageMeta& m = sh.meta[w];
+    if (!m.live) break;
+    const SecDesc& s = secs[m.sec];
+    const uint64_t L = s.bytes, p0 = m.p0, p1 = m.p1;
+    const uint64_t pe = staged_end<MODE>(s, p1);
+    // Complete the tile in shared memory: [pe, p1) holds the stream's
+    // unaligned tail (layout side) and zeros past its end.
+    for (uint64_t o = pe + 16u * lane; o < p1; o += 512u) {
+      uint4 v = zero;
+      if (T::kLoadLayout && o < L) {
+        const uint64_t left = L - o;
+        v = ld_small(s.lbase + o, left < 16 ? static_cast<int>(left) : 16, true);
+      }
+      *reinterpret_cast<uint4*>(tile + (o - p0)) = v;
+    }
+    if (!T::kLoadLayout && (L & 15u) && L >= p0 && L < p1 && lane == 0) {
+      // Restore: payload bytes past the logical end read as zero.
+      const uint64_t o = L & ~15ull;
+      uint4* q = reinterpret_cast<uint4*>(tile + (o - p0));
+      *q = mask_tail(*q, static_cast<int>(L - o));
+    }
+    fence_async_smem();
+    __syncwarp();
+    bool issued = false;
+    if (MODE == kModePack) {
+      // Contiguous payload, through the record's 256-byte padding.
+      const uint64_t padded = (L + kRecordAlign - 1) / kRecordAlign * kRecordAlign;
+      const uint64_t se = p1 < padded ? p1 : padded;
+      if (lane == 0 && se > p0) {
+        bulk_s2g(s.payload + p0, tile, static_cast<uint32_t>(se - p0));
+        bulk_commit();
+        issued = true;
+      }
+    } else if (MODE == kModeRestore || MODE == kModeRestoreV) {
+      const uint64_t lim = L < p1 ? L : p1;
+      if (s.layout == kContig) {
+        const uint64_t vend = lim & ~15ull;  // whole segments by bulk copy
+        if (lane == 0 && vend > p0) {
+          bulk_s2g(s.lbase + p0, tile, static_cast<uint32_t>(vend - p0));
+          bulk_commit();
+          issued = true;
+        }
+        for (uint64_t o = (vend > p0 ? vend : p0) + lane; o < lim; o += 32) s.lbase[o] = tile[o - p0];
+      } else {
+        uint8_t* rp0 = m.rowp[lane];
+        uint8_t* rp1 = m.rowp[lane + 32];
+        if (issue_runs<false>(s, m, rp0, rp1, lim, tile, nullptr, lane)) {
+          bulk_commit();
+          issued = true;
+        }
+      }
+    }
+    if (T::kHash) {
+      // The tile's chunks, 4 interleaved lane chains, read from shared memory.
+      const uint64_t c0 = p0 / kChunkBytes;
+      const int nc = static_cast<int>((p1 - p0) / kChunkBytes);
+      uint64_t h[kTileChunks];
+#pragma unroll
+      for (int q = 0; q < kTileChunks; ++q) h[q] = fmix(kSeed ^ ((c0 + q) * 32u + lane));
+#pragma unroll
+      for (int k = 0; k < kSegs; ++k) {
+#pragma unroll
+        for (int q = 0; q < kTileChunks; ++q) {
+          const uint4 v = q < nc ? *reinterpret_cast<const uint4*>(tile + q * kChunkBytes + 512 * k + 16 * lane)
+                                 : zero;
+          h[q] = absorb(h[q], v);
+        }
+      }
+      uint64_t mine = 0;
+#pragma unroll
+      for (int q = 0; q < kTileChunks; ++q) {
+        const uint64_t x = __shfl_sync(kFull, warp_tree(fmix(h[q]), 32, lane), 0);
+        if (lane == q) mine = x;
+      }
+      const uint64_t root = warp_tree(mine, nc, lane);
+      if (lane == 0) nodes[m.node] = root;
+    }
+    if (issued) bulk_wait_read();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty);
+  }
+  bulk_wait_all();
 }
 
 // ---------------------------------------------------------------------------
@@ -621,35 +1084,71 @@ int occupancy() {
   return b > 0 ? b : 1;
 }
 
+template <int MODE>
+cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, uint32_t* err,
+                             int sm_count, cudaStream_t stream) {
+  const size_t smem = sizeof(BulkShared);
+  static uint64_t configured = 0;  // one bit per device (callers hold the context lock)
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (!(configured & bit)) {
+    e = cudaFuncSetAttribute(k_bulk<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    configured |= bit;
+  }
+  const uint64_t want = wl.n_tasks;
+  const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
+  k_bulk<MODE><<<blocks, kBulkThreads, smem, stream>>>(secs, wl, nodes, err);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 int stream_blocks_per_sm() { return occupancy<kModePack>(); }
 
-cudaError_t launch_stream(int mode, const SecDesc* secs, int n_secs, uint32_t n_tasks,
-                          int group_log2, uint64_t* nodes, uint32_t* dev_err, int sm_count,
-                          int blocks_per_sm, cudaStream_t stream) {
-  if (n_tasks == 0) return cudaSuccess;
-  const uint64_t want = (static_cast<uint64_t>(n_tasks) + kWarps - 1) / kWarps;
-  const int blocks = static_cast<int>(
-      want < static_cast<uint64_t>(sm_count) * blocks_per_sm ? want
-                                                            : static_cast<uint64_t>(sm_count) * blocks_per_sm);
+size_t bulk_shared_bytes() { return sizeof(BulkShared); }
+
+cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_log2,
+                          uint64_t* nodes, uint32_t* dev_err, int sm_count, int blocks_per_sm,
+                          cudaStream_t stream) {
+  if (wl.n_tasks == 0) return cudaSuccess;
+  const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + kWarps - 1) / kWarps;
+  const uint64_t cap = static_cast<uint64_t>(sm_count) * blocks_per_sm;
+  const int blocks = static_cast<int>(want < cap ? want : cap);
   switch (mode) {
     case kModeHash:
-      k_stream<kModeHash><<<blocks, kThreads, 0, stream>>>(secs, n_secs, n_tasks, group_log2, nodes, dev_err);
+      k_stream<kModeHash><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
       break;
     case kModePack:
-      k_stream<kModePack><<<blocks, kThreads, 0, stream>>>(secs, n_secs, n_tasks, group_log2, nodes, dev_err);
+      k_stream<kModePack><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
       break;
     case kModeRestore:
-      k_stream<kModeRestore><<<blocks, kThreads, 0, stream>>>(secs, n_secs, n_tasks, group_log2, nodes, dev_err);
+      k_stream<kModeRestore><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
       break;
     case kModeRestoreV:
-      k_stream<kModeRestoreV><<<blocks, kThreads, 0, stream>>>(secs, n_secs, n_tasks, group_log2, nodes, dev_err);
+      k_stream<kModeRestoreV><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
       break;
     default:
       return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
+}
+
+cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* nodes,
+                        uint32_t* dev_err, int sm_count, cudaStream_t stream) {
+  if (wl.n_tasks == 0) return cudaSuccess;
+  switch (mode) {
+    case kModeHash: return launch_bulk_mode<kModeHash>(secs, wl, nodes, dev_err, sm_count, stream);
+    case kModePack: return launch_bulk_mode<kModePack>(secs, wl, nodes, dev_err, sm_count, stream);
+    case kModeRestore:
+      return launch_bulk_mode<kModeRestore>(secs, wl, nodes, dev_err, sm_count, stream);
+    case kModeRestoreV:
+      return launch_bulk_mode<kModeRestoreV>(secs, wl, nodes, dev_err, sm_count, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess, int n_sess,

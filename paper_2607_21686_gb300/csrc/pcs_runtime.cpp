@@ -15,7 +15,9 @@
 #include <cerrno>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
+#include <unordered_map>
 #include <map>
 #include <memory>
 #include <mutex>
@@ -315,6 +317,7 @@ struct pcs_ctx {
   int device = 0;
   int sm_count = 0;
   int stream_bps = 1;          // resident blocks per SM of the streaming kernel
+  bool use_bulk = true;        // TMA-staged kernel for eligible streams
   std::mutex mu;
   std::shared_ptr<EventPool> events = std::make_shared<EventPool>();
   std::unique_ptr<Arena> dev_arena, host_arena;
@@ -353,12 +356,13 @@ pcs_status set_device(pcs_ctx* c) {
 // Kernels the context launches, for counting and timing.
 enum KernelKind {
   kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
-  kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKCopy, kKernelKinds
+  kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKCopy, kKBulkHash, kKBulkPack,
+  kKBulkRestore, kKBulkRestoreV, kKernelKinds
 };
 const char* kKernelNames[kKernelKinds] = {
     "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
-    "k_copy"};
+    "k_copy", "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>"};
 
 cudaEvent_t timing_event(pcs_ctx* c) {
   if (!c->timing_events.empty()) {
@@ -400,6 +404,15 @@ int stream_kind(int mode) {
     case kModePack: return kKStreamPack;
     case kModeRestore: return kKStreamRestore;
     default: return kKStreamRestoreV;
+  }
+}
+
+int bulk_kind(int mode) {
+  switch (mode) {
+    case kModeHash: return kKBulkHash;
+    case kModePack: return kKBulkPack;
+    case kModeRestore: return kKBulkRestore;
+    default: return kKBulkRestoreV;
   }
 }
 
@@ -534,21 +547,100 @@ SecDesc make_desc(const pcs_section& s, uint8_t* payload, uint32_t ring_start) {
   return d;
 }
 
-// Assign warp tasks to descriptors for a given group size.
-uint64_t assign_tasks(std::vector<SecDesc>& d, int glog2) {
-  uint64_t t = 0;
-  for (auto& x : d) {
-    x.task_begin = static_cast<uint32_t>(t);
-    x.n_tasks = static_cast<uint32_t>((x.n_chunks + (1ull << glog2) - 1) >> glog2);
-    t += x.n_tasks;
+// Is `p` device memory of the current device (not host, managed or unknown)?
+bool is_device_ptr(const void* p, std::unordered_map<const void*, bool>& cache) {
+  if (!p) return true;
+  auto it = cache.find(p);
+  if (it != cache.end()) return it->second;
+  cudaPointerAttributes a{};
+  bool dev = false;
+  if (cudaPointerGetAttributes(&a, p) == cudaSuccess) dev = a.type == cudaMemoryTypeDevice;
+  else cudaGetLastError();
+  cache.emplace(p, dev);
+  return dev;
+}
+
+// How the streams of one call are split between the two kernels.
+struct StreamPlan {
+  std::vector<uint32_t> bulk_ids, bulk_begin, reg_ids, reg_begin;
+  uint32_t bulk_tasks = 0, reg_tasks = 0;
+  uint64_t nodes = 0;
+  int glog2 = 0;
+};
+
+// The TMA-staged kernel takes a stream whose bytes on both sides live in
+// device memory and can be moved as whole 16-byte pieces: a 16-byte aligned
+// contiguous buffer, or rows of at least 512 bytes.
+bool bulk_eligible(const pcs_ctx* c, const SecDesc& d, bool payload_device,
+                   std::unordered_map<const void*, bool>& cache) {
+  if (!c->use_bulk || !payload_device) return false;
+  if (!is_device_ptr(d.lbase, cache)) return false;
+  if (d.layout == kContig) return d.align == 16 || d.bytes == 0;
+  return d.row_bytes >= kBulkMinRowBytes && d.row_bytes % 16 == 0;
+}
+
+// Give every stream its node slots and its kernel.  bulk[i] says which.
+bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<char>& bulk,
+                  StreamPlan& P) {
+  uint64_t reg_chunks = 0;
+  for (size_t i = 0; i < d.size(); ++i)
+    if (!bulk[i]) reg_chunks += d[i].n_chunks;
+  P.glog2 = choose_group_log2(c, reg_chunks);
+  uint64_t node = 0, tb = 0, tr = 0;
+  for (size_t i = 0; i < d.size(); ++i) {
+    uint64_t n;
+    if (bulk[i]) {
+      n = (d[i].n_chunks + kBulkTileChunks - 1) / kBulkTileChunks;
+      P.bulk_ids.push_back(static_cast<uint32_t>(i));
+      P.bulk_begin.push_back(static_cast<uint32_t>(tb));
+      tb += n;
+    } else {
+      n = (d[i].n_chunks + (1ull << P.glog2) - 1) >> P.glog2;
+      P.reg_ids.push_back(static_cast<uint32_t>(i));
+      P.reg_begin.push_back(static_cast<uint32_t>(tr));
+      tr += n;
+    }
+    d[i].task_begin = static_cast<uint32_t>(node);
+    d[i].n_tasks = static_cast<uint32_t>(n);
+    node += n;
   }
-  return t;
+  P.bulk_tasks = static_cast<uint32_t>(tb);
+  P.reg_tasks = static_cast<uint32_t>(tr);
+  P.nodes = node;
+  return node < (1ull << 32);
+}
+
+// Workspace offsets of a stream plan's lists, after `base` bytes.
+struct ListLayout {
+  uint64_t bulk_ids, bulk_begin, reg_ids, reg_begin, end;
+};
+
+ListLayout list_layout(const StreamPlan& P, uint64_t base) {
+  ListLayout L;
+  L.bulk_ids = round_up(base, kRecordAlign);
+  L.bulk_begin = L.bulk_ids + 4 * P.bulk_ids.size();
+  L.reg_ids = L.bulk_begin + 4 * P.bulk_begin.size();
+  L.reg_begin = L.reg_ids + 4 * P.reg_ids.size();
+  L.end = L.reg_begin + 4 * P.reg_begin.size();
+  return L;
 }
 
 template <class T>
 void put(std::vector<uint8_t>& plan, uint64_t off, const std::vector<T>& v) {
   if (!v.empty()) std::memcpy(plan.data() + off, v.data(), v.size() * sizeof(T));
 }
+
+void put_lists(std::vector<uint8_t>& plan, const StreamPlan& P, const ListLayout& L) {
+  put(plan, L.bulk_ids, P.bulk_ids);
+  put(plan, L.bulk_begin, P.bulk_begin);
+  put(plan, L.reg_ids, P.reg_ids);
+  put(plan, L.reg_begin, P.reg_begin);
+}
+
+// Launch both streaming kernels of a plan (TMA-staged first).
+cudaError_t launch_streams(pcs_ctx* c, int mode, const SecDesc* dsecs, const StreamPlan& P,
+                           const ListLayout& L, uint8_t* ws, uint64_t* nodes,
+                           cudaStream_t stream);
 
 // Fingerprint (and optionally classify) contiguous buffers.
 pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t* fp_out,
@@ -567,32 +659,56 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
     d[i] = make_desc(s, nullptr, 0);
     chunks += d[i].n_chunks;
   }
-  const int g = choose_group_log2(c, chunks);
-  const uint64_t tasks = assign_tasks(d, g);
-  if (tasks >= (1ull << 32)) return fail(PCS_E_INVAL, "too much data in one call");
+  (void)chunks;
+  std::unordered_map<const void*, bool> cache;
+  std::vector<char> bulk(n);
+  for (int i = 0; i < n; ++i) bulk[i] = bulk_eligible(c, d[i], true, cache);
+  StreamPlan P;
+  if (!plan_streams(c, d, bulk, P)) return fail(PCS_E_INVAL, "too much data in one call");
   WsLayout L;
   L.secs = 0;
-  L.nodes = round_up(L.secs + sizeof(SecDesc) * n, kRecordAlign);
-  L.total = L.nodes + 8 * tasks;
+  const ListLayout LL = list_layout(P, sizeof(SecDesc) * n);
+  L.nodes = round_up(LL.end, kRecordAlign);
+  L.total = L.nodes + 8 * P.nodes;
   uint8_t* ws = nullptr;
   pcs_status st = ws_acquire(c, L.total, stream, &ws);
   if (st) return st;
   c->plan.resize(L.nodes);
   put(c->plan, L.secs, d);
+  put_lists(c->plan, P, LL);
   PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
-  {
-    LaunchScope ls(c, kKStreamHash, stream);
-    PCS_CUDA(launch_stream(kModeHash, dsecs, n, static_cast<uint32_t>(tasks), g, nodes, c->words,
-                           c->sm_count, c->stream_bps, stream));
-  }
+  PCS_CUDA(launch_streams(c, kModeHash, dsecs, P, LL, ws, nodes, stream));
   {
     LaunchScope ls(c, kKFinalizeHash, stream);
     PCS_CUDA(launch_finalize(kModeHash, dsecs, nullptr, n, nullptr, nodes, fp_out, fp_before,
                              flags, nullptr, stream));
   }
   return ws_release(c, stream);
+}
+
+cudaError_t launch_streams(pcs_ctx* c, int mode, const SecDesc* dsecs, const StreamPlan& P,
+                           const ListLayout& L, uint8_t* ws, uint64_t* nodes,
+                           cudaStream_t stream) {
+  cudaError_t e = cudaSuccess;
+  if (P.bulk_tasks) {
+    WorkList wl{reinterpret_cast<const uint32_t*>(ws + L.bulk_ids),
+                reinterpret_cast<const uint32_t*>(ws + L.bulk_begin),
+                static_cast<int>(P.bulk_ids.size()), P.bulk_tasks};
+    LaunchScope ls(c, bulk_kind(mode), stream);
+    e = launch_bulk(mode, dsecs, wl, nodes, c->words, c->sm_count, stream);
+    if (e != cudaSuccess) return e;
+  }
+  if (P.reg_tasks) {
+    WorkList wl{reinterpret_cast<const uint32_t*>(ws + L.reg_ids),
+                reinterpret_cast<const uint32_t*>(ws + L.reg_begin),
+                static_cast<int>(P.reg_ids.size()), P.reg_tasks};
+    LaunchScope ls(c, stream_kind(mode), stream);
+    e = launch_stream(mode, dsecs, wl, P.glog2, nodes, c->words, c->sm_count, c->stream_bps,
+                      stream);
+  }
+  return e;
 }
 
 pcs_snapshot* check_handle(pcs_ctx* c, const pcs_snapshot* h) {
@@ -642,6 +758,8 @@ pcs_status pcs_create(int32_t device, pcs_ctx** out) {
   PCS_CUDA(cudaSetDevice(device));
   PCS_CUDA(cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, device));
   c->stream_bps = stream_blocks_per_sm();
+  const char* no_tma = std::getenv("PCS_DISABLE_TMA");
+  c->use_bulk = !(no_tma && no_tma[0] == '1');
   c->dev_arena = std::make_unique<Arena>(PCS_PLACE_DEVICE, c->events);
   c->host_arena = std::make_unique<Arena>(PCS_PLACE_PINNED_HOST, c->events);
   PCS_CUDA(cudaMalloc(&c->words, 256));
@@ -742,6 +860,8 @@ pcs_status pcs_sync(pcs_ctx* c, void* stream) {
   PCS_CUDA(cudaMemcpy(&w, c->words, 4, cudaMemcpyDeviceToHost));
   if (w != 0) {
     PCS_CUDA(cudaMemset(c->words, 0, 4));
+    if (w & kDevErrTimeout)
+      return fail(PCS_E_TIMEOUT, "a bounded wait inside a kernel gave up (error bits 0x%x)", w);
     return fail(PCS_E_RANGE, "a kernel met a row or page id out of range (error bits 0x%x)", w);
   }
   return PCS_OK;
@@ -963,19 +1083,25 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
     }
     handles[s] = std::move(h);
   }
-  const int g = choose_group_log2(c, chunks);
-  const uint64_t tasks = assign_tasks(d, g);
+  (void)chunks;
+  std::unordered_map<const void*, bool> cache;
+  std::vector<char> bulk(d.size());
+  for (size_t i = 0; i < d.size(); ++i)
+    bulk[i] = bulk_eligible(c, d[i], placement == PCS_PLACE_DEVICE, cache);
+  StreamPlan P;
+  const bool fits = plan_streams(c, d, bulk, P);
   WsLayout L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
   L.entries = round_up(L.sess + sizeof(SessDesc) * n, kRecordAlign);
-  L.nodes = round_up(L.entries + sizeof(Entry) * ent.size(), kRecordAlign);
-  L.total = L.nodes + 8 * tasks;
+  const ListLayout LL = list_layout(P, L.entries + sizeof(Entry) * ent.size());
+  L.nodes = round_up(LL.end, kRecordAlign);
+  L.total = L.nodes + 8 * P.nodes;
   auto undo = [&](pcs_status s) {
     arena_of(c, placement)->free(blk);
     return s;
   };
-  if (tasks >= (1ull << 32)) return undo(fail(PCS_E_INVAL, "too much data in one call"));
+  if (!fits) return undo(fail(PCS_E_INVAL, "too much data in one call"));
   uint8_t* ws = nullptr;
   st = ws_acquire(c, L.total, stream, &ws);
   if (st) return undo(st);
@@ -983,16 +1109,13 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   put(c->plan, L.secs, d);
   put(c->plan, L.sess, sd);
   put(c->plan, L.entries, ent);
+  put_lists(c->plan, P, LL);
   cudaError_t e = cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream);
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
   auto* dent = reinterpret_cast<const Entry*>(ws + L.entries);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
-  if (e == cudaSuccess) {
-    LaunchScope ls(c, kKStreamPack, stream);
-    e = launch_stream(kModePack, dsecs, static_cast<int>(d.size()), static_cast<uint32_t>(tasks), g,
-                      nodes, c->words, c->sm_count, c->stream_bps, stream);
-  }
+  if (e == cudaSuccess) e = launch_streams(c, kModePack, dsecs, P, LL, ws, nodes, stream);
   if (e == cudaSuccess) {
     LaunchScope ls(c, kKFinalizePack, stream);
     e = launch_finalize(kModePack, dsecs, dsess, n, dent, nodes, nullptr, nullptr, nullptr, nullptr,
@@ -1057,6 +1180,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   if (st) return st;
   std::vector<SecDesc> d;
   std::vector<SessDesc> sd(n);
+  std::vector<char> payload_dev;
   uint64_t chunks = 0;
   for (int s = 0; s < n; ++s) {
     pcs_snapshot* h = check_handle(c, snaps[s]);
@@ -1089,37 +1213,39 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
       SecDesc desc = make_desc(x, h->record() + e.offset, rs);
       chunks += desc.n_chunks;
       d.push_back(desc);
+      payload_dev.push_back(h->block->placement == PCS_PLACE_DEVICE);
     }
   }
   for (int s = 0; s < n; ++s) {
     st = wait_written(snaps[s]->block, stream);
     if (st) return st;
   }
-  const int g = choose_group_log2(c, chunks);
-  const uint64_t tasks = assign_tasks(d, g);
-  if (tasks >= (1ull << 32)) return fail(PCS_E_INVAL, "too much data in one call");
+  (void)chunks;
+  std::unordered_map<const void*, bool> cache;
+  std::vector<char> bulk(d.size());
+  for (size_t i = 0; i < d.size(); ++i) bulk[i] = bulk_eligible(c, d[i], payload_dev[i], cache);
+  StreamPlan P;
+  if (!plan_streams(c, d, bulk, P)) return fail(PCS_E_INVAL, "too much data in one call");
   WsLayout L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
-  L.nodes = round_up(L.sess + sizeof(SessDesc) * n, kRecordAlign);
-  L.total = L.nodes + (verify ? 8 * tasks : 0);
+  const ListLayout LL = list_layout(P, L.sess + sizeof(SessDesc) * n);
+  L.nodes = round_up(LL.end, kRecordAlign);
+  L.total = L.nodes + (verify ? 8 * P.nodes : 0);
   uint8_t* ws = nullptr;
   st = ws_acquire(c, L.total, stream, &ws);
   if (st) return st;
   c->plan.resize(L.nodes);
   put(c->plan, L.secs, d);
   put(c->plan, L.sess, sd);
+  put_lists(c->plan, P, LL);
   PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
   if (verify) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
-  {
-    const int mode = verify ? kModeRestoreV : kModeRestore;
-    LaunchScope ls(c, stream_kind(mode), stream);
-    PCS_CUDA(launch_stream(mode, dsecs, static_cast<int>(d.size()), static_cast<uint32_t>(tasks), g,
-                           nodes, c->words, c->sm_count, c->stream_bps, stream));
-  }
+  PCS_CUDA(launch_streams(c, verify ? kModeRestoreV : kModeRestore, dsecs, P, LL, ws,
+                          verify ? nodes : nullptr, stream));
   if (verify) {
     LaunchScope ls(c, kKFinalizeRestoreV, stream);
     PCS_CUDA(launch_finalize(kModeRestoreV, dsecs, dsess, n, nullptr, nodes, nullptr, nullptr,
