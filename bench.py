@@ -348,8 +348,9 @@ def main():
         sps = a.sessions * world / (ms_step / 1e3)
         # Roofline of the dominant kernel: pack or restore stream pass.
         kt = r["ktimes"]
-        cand = {k: v for k, v in kt.items() if k.startswith("k_stream")}
+        cand = {k: v for k, v in kt.items() if k.startswith(("k_stream", "k_bulk"))}
         top = max(cand, key=lambda k: cand[k][1]) if cand else None
+        # One pass moves every payload byte once in and once out.
         roof = None
         if top:
             n_l, tot = cand[top]

@@ -98,8 +98,8 @@ struct WorkList {
   uint32_t n_tasks;
 };
 
-// Chunks per task of the TMA-staged kernel (a 16 KiB tile).
-constexpr int kBulkTileChunks = 4;
+// Chunks per task of the TMA-staged kernel (an 8 KiB tile).
+constexpr int kBulkTileChunks = 2;
 // Smallest row size the TMA-staged kernel takes for ROWS / RING streams.
 constexpr uint64_t kBulkMinRowBytes = 512;
 

@@ -316,33 +316,29 @@ __global__ void __launch_bounds__(kThreads, 2)
 // ---------------------------------------------------------------------------
 // TMA-staged streaming kernel
 //
-// One block per SM: warp 0 produces, warps 1..8 consume.  A tile is 4 chunks
-// (16 KiB) of one stream in payload order.  The producer stages each tile in
-// shared memory with cp.async.bulk copies (one per contiguous run of rows of
-// the layout side, or one for the contiguous payload), completing on the
-// stage's mbarrier; consumer warp w owns stage w: it hashes the 4 chunks from
-// shared memory (4 interleaved lane chains), issues the bulk store of the
-// tile (payload, or the runs of the layout side), and frees the stage once
-// the store has read it.  Every wait is bounded in time; a wait that gives
-// up records kDevErrTimeout and the block stops.
+// Every warp runs its own pipeline over a contiguous range of tiles; a tile
+// is 2 chunks (8 KiB) of one stream in payload order.  A warp owns
+// kWarpStages shared-memory stages: it stages tile i + kWarpStages while it
+// works on tile i.  Staging is one cp.async.bulk copy per run of rows that
+// are contiguous in memory (or one copy of the contiguous payload), all
+// completing on the stage's mbarrier; working on a tile = hash its chunks
+// from shared memory, issue the bulk store of the tile (to the payload, or
+// one per row run of the layout side), and wait until the store has read
+// the stage.  Warps never wait on each other.  Every wait is bounded; a wait
+// that gives up records kDevErrTimeout and the warp stops.
 // ---------------------------------------------------------------------------
 
-constexpr int kBulkConsumers = 8;
-constexpr int kBulkStages = kBulkConsumers;
+constexpr int kBulkWarps = 8;
+constexpr int kWarpStages = 3;
 constexpr int kTileChunks = kBulkTileChunks;
 constexpr uint32_t kTileBytes = kTileChunks * kChunkBytes;
-constexpr int kBulkThreads = 32 * (1 + kBulkConsumers);
-constexpr int kTileRows = 64;  // rows of >= 512 bytes in a tile, plus one
-constexpr uint64_t kWaitNs = 2000000000ull;  // give up a wait after 2 s
+constexpr int kBulkThreads = 32 * kBulkWarps;
+constexpr int kTileRows = 32;  // rows >= 512 bytes touching an 8 KiB tile: at most 17
+constexpr long long kWaitCycles = 4000000000ll;  // give up a wait after ~2 s of SM clock
+static_assert(kTileBytes / kBulkMinRowBytes + 1 <= kTileRows, "tile rows");
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ uint64_t global_ns() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
 }
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
@@ -355,18 +351,14 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(20000u)
       : "memory");
   return ok != 0;
 }
@@ -374,9 +366,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // Bounded wait for the phase of `bar` with the given parity to complete.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = global_ns();
+  const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity))
-    if (global_ns() - t0 > kWaitNs) return false;
+    if (clock64() - t0 > kWaitCycles) return false;
   return true;
 }
 
@@ -404,27 +396,20 @@ __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Per-stage description of the tile in flight (written by the producer
-// before it arrives on the stage's barrier).
-struct StageMeta {
-  uint32_t sec;         // section index
-  uint32_t node;        // node slot of the tile
-  uint64_t p0, p1;      // payload bytes of the tile: [p0, p1)
-  uint64_t r0;          // first row of the tile (ROWS / RING)
-  uint32_t n_rows;      // rows touching [p0, p1)
-  uint32_t live;        // 1 = a tile, 0 = no more work
-  uint8_t* rowp[kTileRows];  // restore: layout-side address of each row
+// What a stage holds (written by the warp when it stages the tile).
+struct WarpStage {
+  SecDesc d;                // the tile's stream
+  uint64_t p0, p1;          // payload bytes of the tile: [p0, p1)
+  uint64_t r0;              // first row touching the tile (ROWS / RING)
+  uint32_t node;            // node slot of the tile
+  uint32_t n_rows;          // rows touching [p0, min(p1, L))
+  uint8_t* rowp[kTileRows]; // layout-side address of each row (null = out of range)
 };
 
 struct BulkShared {
-  alignas(128) uint8_t stage[kBulkStages][kTileBytes];
-  alignas(8) uint64_t full[kBulkStages];
-  uint64_t empty[kBulkStages];
-  StageMeta meta[kBulkStages];
-  // Producer scratch: the next batch's tiles, prepared before waiting.
-  StageMeta next[kBulkStages];
-  int32_t armed[kBulkStages];  // last use of each stage whose copies were issued
-  uint32_t abort;
+  alignas(128) uint8_t buf[kBulkWarps][kWarpStages][kTileBytes];
+  alignas(8) uint64_t bar[kBulkWarps][kWarpStages];
+  WarpStage st[kBulkWarps][kWarpStages];
 };
 
 // Layout-side address of row r of a ROWS / RING stream (null if out of range).
@@ -457,54 +442,103 @@ __device__ __forceinline__ uint64_t staged_end(const SecDesc& s, uint64_t p1) {
   return p1 < end ? p1 : end;
 }
 
-// Issue bulk copies between a tile's shared buffer and the layout side, one
-// per run of rows that are contiguous in memory, covering payload bytes
-// [m.p0, pe).  Lane i owns rows i and i + 32 (addresses rp0, rp1; null =
-// skipped).  Returns the bytes this lane copied.
-template <bool kLoad>
-__device__ __forceinline__ uint32_t issue_runs(const SecDesc& s, const StageMeta& m,
-                                               uint8_t* rp0, uint8_t* rp1, uint64_t pe,
-                                               uint8_t* tile, uint64_t* bar, int lane) {
-  const uint64_t rb = s.row_bytes;
-  const int n = static_cast<int>(m.n_rows);
-  const uintptr_t u0 = reinterpret_cast<uintptr_t>(rp0), u1 = reinterpret_cast<uintptr_t>(rp1);
-  uintptr_t prev0 = __shfl_up_sync(kFull, u0, 1);
-  uintptr_t prev1 = __shfl_up_sync(kFull, u1, 1);
-  const uintptr_t last0 = __shfl_sync(kFull, u0, 31);
-  if (lane == 0) prev1 = last0;
-  const bool v0 = lane < n, v1 = lane + 32 < n;
-  const bool st0 = v0 && (lane == 0 || u0 == 0 || prev0 == 0 || u0 != prev0 + rb);
-  const bool st1 = v1 && (u1 == 0 || prev1 == 0 || u1 != prev1 + rb);
-  const uint64_t starts = static_cast<uint64_t>(__ballot_sync(kFull, st0)) |
-                          (static_cast<uint64_t>(__ballot_sync(kFull, st1)) << 32);
-  uint32_t copied = 0;
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int i = lane + 32 * h;
-    const bool st = h == 0 ? st0 : st1;
-    uint8_t* rp = h == 0 ? rp0 : rp1;
-    if (!st || rp == nullptr) continue;
-    const uint64_t later = i + 1 < 64 ? (starts >> (i + 1)) : 0;
-    const int next = later ? i + __ffsll(static_cast<long long>(later)) : n;
-    const uint64_t row_lo = (m.r0 + i) * rb, row_hi = (m.r0 + next) * rb;
-    const uint64_t a = row_lo > m.p0 ? row_lo : m.p0;
-    const uint64_t b = row_hi < pe ? row_hi : pe;
-    if (a >= b) continue;
-    uint8_t* g = rp + (a - row_lo);
-    uint8_t* sp = tile + (a - m.p0);
-    if (kLoad) bulk_g2s(sp, g, static_cast<uint32_t>(b - a), bar);
-    else bulk_s2g(g, sp, static_cast<uint32_t>(b - a));
-    copied += static_cast<uint32_t>(b - a);
-  }
-  return copied;
-}
-
-// Bytes of tile [p0, pe) that row i (owned by the calling lane) covers.
-__device__ __forceinline__ uint32_t row_share(const StageMeta& m, uint64_t rb, int i,
-                                              uint64_t pe) {
+// Bytes of [p0, pe) that row i of a stage covers.
+__device__ __forceinline__ uint32_t row_share(const WarpStage& m, uint64_t rb, int i, uint64_t pe) {
   const uint64_t lo = (m.r0 + i) * rb, hi = lo + rb;
   const uint64_t a = lo > m.p0 ? lo : m.p0, b = hi < pe ? hi : pe;
   return b > a ? static_cast<uint32_t>(b - a) : 0u;
+}
+
+// Bulk copies between a stage's buffer and the layout side, one per run of
+// rows contiguous in memory, covering payload bytes [m.p0, pe).  Lane i owns
+// row i (address rp; null = skipped).  Returns the bytes this lane copied.
+template <bool kLoad>
+__device__ __forceinline__ uint32_t issue_runs(const WarpStage& m, uint8_t* rp, uint64_t pe,
+                                               uint8_t* tile, uint64_t* bar, int lane) {
+  const uint64_t rb = m.d.row_bytes;
+  const int n = static_cast<int>(m.n_rows);
+  const uintptr_t u = reinterpret_cast<uintptr_t>(rp);
+  const uintptr_t prev = __shfl_up_sync(kFull, u, 1);
+  const bool start = lane < n && (lane == 0 || u == 0 || prev == 0 || u != prev + rb);
+  const unsigned starts = __ballot_sync(kFull, start);
+  if (!start || rp == nullptr) return 0;
+  const unsigned later = lane < 31 ? (starts >> (lane + 1)) : 0u;
+  const int next = later ? lane + __ffs(later) : n;
+  const uint64_t row_lo = (m.r0 + lane) * rb, row_hi = (m.r0 + next) * rb;
+  const uint64_t a = row_lo > m.p0 ? row_lo : m.p0;
+  const uint64_t b = row_hi < pe ? row_hi : pe;
+  if (a >= b) return 0;
+  uint8_t* g = rp + (a - row_lo);
+  uint8_t* sp = tile + (a - m.p0);
+  if (kLoad) bulk_g2s(sp, g, static_cast<uint32_t>(b - a), bar);
+  else bulk_s2g(g, sp, static_cast<uint32_t>(b - a));
+  return static_cast<uint32_t>(b - a);
+}
+
+// Stage tile t (of work list item `item`) into stage `st` / barrier `bar`.
+template <int MODE>
+__device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, const WorkList& wl,
+                                           int item, uint32_t t, WarpStage& st, uint8_t* tile,
+                                           uint64_t* bar, uint32_t* err, int lane) {
+  using T = ModeTraits<MODE>;
+  const uint32_t sec = __ldg(wl.ids + item);
+  const uint32_t loc = t - __ldg(wl.begin + item);
+  if (lane < static_cast<int>(sizeof(SecDesc) / 16))
+    reinterpret_cast<uint4*>(&st.d)[lane] = __ldg(reinterpret_cast<const uint4*>(secs + sec) + lane);
+  __syncwarp();
+  const SecDesc& s = st.d;
+  const uint64_t L = s.bytes;
+  const uint64_t p0 = static_cast<uint64_t>(loc) * kTileBytes;
+  const uint64_t cend = s.n_chunks * kChunkBytes;
+  const uint64_t p1 = p0 + kTileBytes < cend ? p0 + kTileBytes : cend;
+  const uint64_t pe = staged_end<MODE>(s, p1);
+  uint64_t r0 = 0;
+  uint32_t n_rows = 0;
+  uint8_t* rp = nullptr;
+  if (s.layout != kContig) {
+    r0 = div_rows(p0, s.row_bytes, s.rb_shift);
+    const uint64_t lim = L < p1 ? L : p1;
+    if (lim > p0) n_rows = static_cast<uint32_t>(div_rows(lim - 1, s.row_bytes, s.rb_shift) + 1 - r0);
+    if (lane < static_cast<int>(n_rows)) rp = row_ptr(s, r0 + lane, err);
+    st.rowp[lane] = rp;
+  }
+  if (lane == 0) {
+    st.p0 = p0;
+    st.p1 = p1;
+    st.r0 = r0;
+    st.node = s.task_begin + loc;
+    st.n_rows = n_rows;
+  }
+  __syncwarp();
+  if (!T::kLoadLayout || s.layout == kContig) {
+    // One contiguous piece: the record payload, or a contiguous buffer.
+    if (lane == 0) {
+      const uint32_t bytes = pe > p0 ? static_cast<uint32_t>(pe - p0) : 0u;
+      mbar_arrive_expect_tx(bar, bytes);
+      if (bytes) bulk_g2s(tile, T::kLoadLayout ? s.lbase + p0 : s.payload + p0, bytes, bar);
+    }
+    return;
+  }
+  // Rows: zero the share of rows whose id was out of range, arm the barrier
+  // with the bytes the copies will bring, then one bulk copy per run.
+  uint32_t mine = 0;
+  if (lane < static_cast<int>(n_rows)) {
+    const uint32_t share = row_share(st, s.row_bytes, lane, pe);
+    if (rp == nullptr) {
+      const uint64_t lo = (r0 + lane) * s.row_bytes;
+      const uint64_t a = lo > p0 ? lo : p0;
+      for (uint32_t o = 0; o < share; o += 16)
+        *reinterpret_cast<uint4*>(tile + (a - p0) + o) = make_uint4(0, 0, 0, 0);
+      fence_async_smem();
+    } else {
+      mine = share;
+    }
+  }
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) mine += __shfl_xor_sync(kFull, mine, d);
+  if (lane == 0) mbar_arrive_expect_tx(bar, mine);
+  __syncwarp();
+  issue_runs<true>(st, rp, pe, tile, bar, lane);
 }
 
 template <int MODE>
@@ -516,184 +550,46 @@ __global__ void __launch_bounds__(kBulkThreads, 1)
   BulkShared& sh = *reinterpret_cast<BulkShared*>(smem_raw);
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  if (threadIdx.x < kBulkStages) {
-    mbar_init(&sh.full[threadIdx.x], 1);
-    mbar_init(&sh.empty[threadIdx.x], 1);
-    sh.armed[threadIdx.x] = -1;
-  }
-  if (threadIdx.x == 0) sh.abort = 0;
+  if (lane < kWarpStages) mbar_init(&sh.bar[warp][lane], 1);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  __syncthreads();
+  __syncwarp();
 
-  if (warp == 0) {
-    // ------------------------------ producer ------------------------------
-    bool stop = false;
-    for (uint32_t use = 0; !stop; ++use) {
-      // Batch `use`: tile m = use * kBulkStages + j goes to stage j; its
-      // global index is blockIdx.x + m * gridDim.x.
-      uint32_t sec_j = 0, loc_j = 0, node_j = 0;
-      bool have_j = false;
-      if (lane < kBulkStages) {
-        const uint64_t t = blockIdx.x + (static_cast<uint64_t>(use) * kBulkStages + lane) * gridDim.x;
-        if (t < wl.n_tasks) {
-          const int it = find_item(wl.begin, wl.n_items, static_cast<uint32_t>(t));
-          sec_j = __ldg(wl.ids + it);
-          loc_j = static_cast<uint32_t>(t) - __ldg(wl.begin + it);
-          node_j = __ldg(&secs[sec_j].task_begin) + loc_j;
-          have_j = true;
-        }
-      }
-      const unsigned have = __ballot_sync(kFull, have_j);
-      // Describe every tile of the batch and fetch its row addresses (all
-      // index loads of the batch in flight together).
-#pragma unroll
-      for (int j = 0; j < kBulkStages; ++j) {
-        if (!((have >> j) & 1u)) continue;
-        const uint32_t sec = __shfl_sync(kFull, sec_j, j);
-        const uint32_t loc = __shfl_sync(kFull, loc_j, j);
-        const uint32_t node = __shfl_sync(kFull, node_j, j);
-        const SecDesc& s = secs[sec];
-        const uint64_t L = s.bytes;
-        const uint64_t p0 = static_cast<uint64_t>(loc) * kTileBytes;
-        const uint64_t cend = s.n_chunks * kChunkBytes;
-        const uint64_t p1 = p0 + kTileBytes < cend ? p0 + kTileBytes : cend;
-        uint64_t r0 = 0;
-        uint32_t n_rows = 0;
-        StageMeta& nx = sh.next[j];
-        if (s.layout != kContig) {
-          r0 = div_rows(p0, s.row_bytes, s.rb_shift);
-          const uint64_t lim = L < p1 ? L : p1;
-          if (lim > p0) n_rows = static_cast<uint32_t>(div_rows(lim - 1, s.row_bytes, s.rb_shift) + 1 - r0);
-          nx.rowp[lane] = lane < static_cast<int>(n_rows) ? row_ptr(s, r0 + lane, err) : nullptr;
-          nx.rowp[lane + 32] = lane + 32 < static_cast<int>(n_rows) ? row_ptr(s, r0 + lane + 32, err) : nullptr;
-        }
-        if (lane == 0) {
-          nx.sec = sec;
-          nx.node = node;
-          nx.p0 = p0;
-          nx.p1 = p1;
-          nx.r0 = r0;
-          nx.n_rows = n_rows;
-          nx.live = 1;
-        }
-      }
-      __syncwarp();
-      for (int j = 0; j < kBulkStages; ++j) {
-        // Wait until consumer j has released stage j.
-        bool ok = true;
-        if (use > 0 && lane == 0) ok = mbar_wait(&sh.empty[j], (use - 1) & 1);
-        ok = __shfl_sync(kFull, ok, 0);
-        if (!ok || *reinterpret_cast<volatile uint32_t*>(&sh.abort)) {
-          if (lane == 0) {
-            atomicOr(err, kDevErrTimeout);
-            sh.abort = 1;
-          }
-          stop = true;
-          break;
-        }
-        StageMeta& m = sh.meta[j];
-        if (!((have >> j) & 1u)) {
-          // No tile: the consumer of stage j stops.
-          if (lane == 0) {
-            m.live = 0;
-            mbar_arrive_expect_tx(&sh.full[j], 0);
-          }
-          stop = true;
-          continue;
-        }
-        const StageMeta& nx = sh.next[j];
-        const SecDesc& s = secs[nx.sec];
-        const uint64_t p0 = nx.p0;
-        const uint64_t pe = staged_end<MODE>(s, nx.p1);
-        uint8_t* rp0 = nullptr;
-        uint8_t* rp1 = nullptr;
-        if (s.layout != kContig) {
-          rp0 = nx.rowp[lane];
-          rp1 = nx.rowp[lane + 32];
-          m.rowp[lane] = rp0;
-          m.rowp[lane + 32] = rp1;
-        }
-        if (lane == 0) {
-          m.sec = nx.sec;
-          m.node = nx.node;
-          m.p0 = nx.p0;
-          m.p1 = nx.p1;
-          m.r0 = nx.r0;
-          m.n_rows = nx.n_rows;
-          m.live = 1;
-          sh.armed[j] = static_cast<int32_t>(use);
-        }
-        uint8_t* tile = sh.stage[j];
-        if (!T::kLoadLayout || s.layout == kContig) {
-          // One contiguous piece: the record payload, or a contiguous buffer.
-          const uint32_t bytes = pe > p0 ? static_cast<uint32_t>(pe - p0) : 0u;
-          __syncwarp();
-          if (lane == 0) {
-            mbar_arrive_expect_tx(&sh.full[j], bytes);
-            if (bytes) bulk_g2s(tile, T::kLoadLayout ? s.lbase + p0 : s.payload + p0, bytes, &sh.full[j]);
-          }
-        } else {
-          // Rows: zero the share of rows whose ids were out of range, count
-          // the bytes the copies will bring, arm the barrier, issue runs.
-          const uint64_t rb = s.row_bytes;
-          uint32_t mine = 0;
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int i = lane + 32 * h;
-            if (i >= static_cast<int>(nx.n_rows)) continue;
-            const uint32_t share = row_share(nx, rb, i, pe);
-            if ((h == 0 ? rp0 : rp1) == nullptr) {
-              const uint64_t a = (nx.r0 + i) * rb > p0 ? (nx.r0 + i) * rb : p0;
-              for (uint32_t o = 0; o < share; o += 16)
-                *reinterpret_cast<uint4*>(tile + (a - p0) + o) = make_uint4(0, 0, 0, 0);
-            } else {
-              mine += share;
-            }
-          }
-          fence_async_smem();
-#pragma unroll
-          for (int d = 16; d > 0; d >>= 1) mine += __shfl_xor_sync(kFull, mine, d);
-          __syncwarp();
-          if (lane == 0) mbar_arrive_expect_tx(&sh.full[j], mine);
-          __syncwarp();
-          issue_runs<true>(s, nx, rp0, rp1, pe, tile, &sh.full[j], lane);
-        }
-        __syncwarp();
-      }
-      if (have != (1u << kBulkStages) - 1u) stop = true;
-    }
-    if (*reinterpret_cast<volatile uint32_t*>(&sh.abort) && lane == 0) {
-      // Let copies already issued land before the block leaves.
-      for (int j = 0; j < kBulkStages; ++j)
-        if (sh.armed[j] >= 0) mbar_wait(&sh.full[j], static_cast<uint32_t>(sh.armed[j]) & 1);
-    }
-    return;
-  }
-
-  // ------------------------------ consumers ------------------------------
-  const int w = warp - 1;  // owns stage w
-  uint64_t* full = &sh.full[w];
-  uint64_t* empty = &sh.empty[w];
-  uint8_t* tile = sh.stage[w];
+  // This warp's tiles: a contiguous, balanced range [t0, t1).
+  const uint64_t T_all = wl.n_tasks;
+  const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kBulkWarps + warp;
+  const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kBulkWarps;
+  const uint32_t t0 = static_cast<uint32_t>(T_all * gw / nw);
+  const uint32_t t1 = static_cast<uint32_t>(T_all * (gw + 1) / nw);
+  if (t0 >= t1) return;
+  int item = find_item(wl.begin, wl.n_items, t0);  // item of the next tile to stage
+  auto item_of = [&](uint32_t t) {
+    while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= t) ++item;
+    return item;
+  };
+  const int pre = static_cast<int>(t1 - t0 < static_cast<uint32_t>(kWarpStages) ? t1 - t0 : kWarpStages);
+  for (int k = 0; k < pre; ++k)
+    stage_tile<MODE>(secs, wl, item_of(t0 + k), t0 + k, sh.st[warp][k], sh.buf[warp][k],
+                     &sh.bar[warp][k], err, lane);
   const uint4 zero = make_uint4(0, 0, 0, 0);
-  for (uint32_t use = 0;; ++use) {
+  bool any_issued = false;
+  for (uint32_t i = 0; t0 + i < t1; ++i) {
+    const int sidx = static_cast<int>(i % kWarpStages);
+    const uint32_t use = i / kWarpStages;
+    uint64_t* bar = &sh.bar[warp][sidx];
+    uint8_t* tile = sh.buf[warp][sidx];
+    WarpStage& m = sh.st[warp][sidx];
     bool ok = true;
-    if (lane == 0) ok = mbar_wait(full, use & 1);
+    if (lane == 0) ok = mbar_wait(bar, use & 1);
     ok = __shfl_sync(kFull, ok, 0);
-    if (!ok || *reinterpret_cast<volatile uint32_t*>(&sh.abort)) {
-      if (lane == 0) {
-        atomicOr(err, kDevErrTimeout);
-        sh.abort = 1;
-      }
+    if (!ok) {
+      if (lane == 0) atomicOr(err, kDevErrTimeout);
       break;
     }
-    const StageMeta& m = sh.meta[w];
-    if (!m.live) break;
-    const SecDesc& s = secs[m.sec];
+    const SecDesc& s = m.d;
     const uint64_t L = s.bytes, p0 = m.p0, p1 = m.p1;
     const uint64_t pe = staged_end<MODE>(s, p1);
-    // Complete the tile in shared memory: [pe, p1) holds the stream's
-    // unaligned tail (layout side) and zeros past its end.
+    // Complete the tile: [pe, p1) holds the stream's unaligned tail (layout
+    // side) and zeros past its end.
     for (uint64_t o = pe + 16u * lane; o < p1; o += 512u) {
       uint4 v = zero;
       if (T::kLoadLayout && o < L) {
@@ -731,16 +627,15 @@ __global__ void __launch_bounds__(kBulkThreads, 1)
         }
         for (uint64_t o = (vend > p0 ? vend : p0) + lane; o < lim; o += 32) s.lbase[o] = tile[o - p0];
       } else {
-        uint8_t* rp0 = m.rowp[lane];
-        uint8_t* rp1 = m.rowp[lane + 32];
-        if (issue_runs<false>(s, m, rp0, rp1, lim, tile, nullptr, lane)) {
+        uint8_t* rp = m.rowp[lane];
+        if (issue_runs<false>(m, rp, lim, tile, nullptr, lane)) {
           bulk_commit();
           issued = true;
         }
       }
     }
     if (T::kHash) {
-      // The tile's chunks, 4 interleaved lane chains, read from shared memory.
+      // The tile's chunks, interleaved lane chains, read from shared memory.
       const uint64_t c0 = p0 / kChunkBytes;
       const int nc = static_cast<int>((p1 - p0) / kChunkBytes);
       uint64_t h[kTileChunks];
@@ -764,11 +659,16 @@ __global__ void __launch_bounds__(kBulkThreads, 1)
       const uint64_t root = warp_tree(mine, nc, lane);
       if (lane == 0) nodes[m.node] = root;
     }
-    if (issued) bulk_wait_read();
+    if (issued) {
+      bulk_wait_read();
+      any_issued = true;
+    }
     __syncwarp();
-    if (lane == 0) mbar_arrive(empty);
+    // Reuse the stage for tile i + kWarpStages.
+    const uint32_t tn = t0 + i + kWarpStages;
+    if (tn < t1) stage_tile<MODE>(secs, wl, item_of(tn), tn, m, tile, bar, err, lane);
   }
-  bulk_wait_all();
+  if (any_issued) bulk_wait_all();
 }
 
 // ---------------------------------------------------------------------------
@@ -1099,7 +999,7 @@ cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, 
     if (e != cudaSuccess) return e;
     configured |= bit;
   }
-  const uint64_t want = wl.n_tasks;
+  const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + kBulkWarps - 1) / kBulkWarps;
   const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
   k_bulk<MODE><<<blocks, kBulkThreads, smem, stream>>>(secs, wl, nodes, err);
   return cudaGetLastError();

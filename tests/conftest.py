@@ -42,3 +42,13 @@ def ctx():
 def dev():
     import torch
     return torch.device("cuda:0")
+
+
+@pytest.fixture(autouse=True)
+def _device_errors_are_failures(request):
+    """After every GPU test, errors recorded by kernels (an index out of
+    range, a bounded wait that gave up) surface through pcs_sync."""
+    yield
+    for name in ("ctx", "ctx_reg"):
+        if name in request.fixturenames:
+            request.getfixturevalue(name).sync()

@@ -94,7 +94,7 @@ def test_bank_rows_paths_agree(ctx, ctx_reg, dev):
         sm = small[lo:hi].to(dev)
         kd = kept.to(dev)
         sess = pcs.Session(s, pcs.PCS_KIND_BANK, [
-            pcs.contig_section(pcs.PCS_SEC_KEPT_IDX, kd),
+            pcs.contig_section(pcs.PCS_SEC_KEPT_IDX, kd, dim0=kd.numel()),
             pcs.rows_section(pcs.PCS_SEC_KEYS, keys, kd),
             pcs.rows_section(pcs.PCS_SEC_VALUES, vals.reshape(vals.shape[0], -1), kd),
             pcs.rows_section(9, sm, kd)], keep=[keys, vals, sm, kd])
