@@ -350,6 +350,38 @@ pcs_status pcs_snapshot_write_file(pcs_ctx *ctx, const pcs_snapshot *snap, const
 pcs_status pcs_snapshot_read_file(pcs_ctx *ctx, const char *path, uint32_t placement,
                                   pcs_snapshot **out);
 
+/*
+ * Fingerprints without any allocation.  The paper has no counterpart: this is
+ * a service of this library for callers that cannot allocate device memory,
+ * for example a serving process that has already carved nearly all of HBM
+ * into its own page pools (a cudaMalloc would fail or upset its accounting),
+ * or a latency-critical loop that cannot afford the device-wide
+ * synchronisation that cudaMalloc / cudaFree bring.
+ *
+ * Same result as pcs_fingerprint (PCSFP64-v1 of each buffer), but no context
+ * is needed and nothing is allocated: the plan travels as a kernel
+ * parameter, and the only working memory is one fixed array of
+ * PCS_STATIC_MAX_NODES tree nodes (512 KiB) that the library's GPU code
+ * defines.  Every GPU that runs this call holds that array until the process
+ * exits.
+ *   bufs    host array of n buffer descriptions (device pointers, any
+ *           alignment); n <= PCS_STATIC_MAX_BUFFERS
+ *   fp_out  device uint64[n]
+ * Limits: each buffer needs ceil(bytes / 131072) nodes (at least 1) and one
+ * call may use at most PCS_STATIC_MAX_NODES of them: about 8 GiB per call.
+ * A call beyond a limit returns PCS_E_INVAL before anything is enqueued.
+ * The first call on a device looks up the array's device address with that
+ * device current (this may load the library's GPU code on that device); make
+ * that first call before any stream capture.  All calls share the array: two
+ * calls whose work overlaps on the GPU (unordered streams) corrupt each
+ * other's results, so order them.  No part of the array needs to start at
+ * zero; each call writes every node it later reads.  On success the call
+ * allocates neither device nor host memory.
+ */
+#define PCS_STATIC_MAX_BUFFERS 64
+#define PCS_STATIC_MAX_NODES 65536
+pcs_status pcs_fingerprint_static(const pcs_buf *bufs, int32_t n, uint64_t *fp_out, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -140,4 +140,33 @@ cudaError_t launch_copy(const void* src, void* dst, uint64_t bytes, int sm_count
 // Occupancy of the streaming kernel (blocks per SM) for the launch shape.
 int stream_blocks_per_sm();
 
+// ---- Fingerprints with no allocation (pcs_fingerprint_static) -------------
+constexpr int kStaticMaxBufs = 64;         // buffers per call
+constexpr uint32_t kStaticMaxNodes = 65536;  // tree nodes per call (512 KiB)
+
+struct StaticBuf {
+  const uint8_t* ptr;
+  uint64_t bytes;
+  uint64_t n_chunks;
+  uint32_t task_begin;  // first node slot of this buffer
+  uint32_t n_tasks;
+  uint32_t align;       // 16, 4 or 1
+  uint32_t pad;
+};
+
+// Passed by value as a kernel parameter (no device copy of the plan).
+struct StaticPlan {
+  StaticBuf b[kStaticMaxBufs];
+  int32_t n;
+  uint32_t n_tasks;
+  int32_t glog2;
+  int32_t pad;
+};
+
+// Device address of the fixed node scratch on the current device; the first
+// call on a device looks it up (cudaGetSymbolAddress) with that device current.
+cudaError_t static_scratch(uint64_t** nodes);
+cudaError_t launch_fingerprint_static(const StaticPlan& plan, uint64_t* nodes, uint64_t* fp_out,
+                                      cudaStream_t stream);
+
 }  // namespace pcs

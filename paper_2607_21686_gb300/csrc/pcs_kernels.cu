@@ -23,6 +23,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <mutex>
 
 #include "pcs_internal.h"
 
@@ -1099,6 +1100,103 @@ cudaError_t launch_copy(const void* src, void* dst, uint64_t bytes, int sm_count
   const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
   const int blocks = static_cast<int>(want < cap ? want : cap);
   k_copy<<<blocks, kThreads, 0, stream>>>(static_cast<const uint4*>(src), static_cast<uint4*>(dst), n16);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Fingerprints with no allocation
+//
+// For callers that cannot allocate device memory, pcs_fingerprint_static runs
+// the fingerprint with its whole working set in one fixed array owned by this
+// file: the tree nodes of one call.  The plan (at most kStaticMaxBufs buffers)
+// travels as a kernel parameter.  The array is created with the module on
+// every GPU that runs the call and stays there until the process exits; all
+// calls share it, so calls that overlap on the GPU race on it.  No slot needs
+// to start at zero: a call writes every node it later reads.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+static __device__ __align__(256) uint64_t g_static_nodes[kStaticMaxNodes];
+
+__global__ void __launch_bounds__(kThreads)
+    k_fp_static(const StaticPlan plan, uint64_t* __restrict__ nodes) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t nw = gridDim.x * kWarps;
+  const int g = plan.glog2;
+  for (uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5); task < plan.n_tasks; task += nw) {
+    int j = 0;
+    while (j + 1 < plan.n && plan.b[j + 1].task_begin <= task) ++j;
+    const StaticBuf& b = plan.b[j];
+    const uint32_t local = task - b.task_begin;
+    const uint64_t c0 = static_cast<uint64_t>(local) << g;
+    const uint64_t c1 = min(c0 + (1ull << g), static_cast<unsigned long long>(b.n_chunks));
+    uint64_t mine = 0;  // lane j keeps the hash of chunk c0 + j
+    for (uint64_t c = c0; c < c1; ++c) {
+      uint64_t h = fmix(kSeed ^ (c * 32u + lane));
+#pragma unroll
+      for (int k = 0; k < kSegs; ++k) {
+        const uint64_t off = c * kChunkBytes + 512u * k + 16u * lane;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (off < b.bytes) {
+          const uint64_t left = b.bytes - off;
+          if (left >= 16 && b.align == 16) v = ld_stream(b.ptr + off);
+          else v = ld_small(b.ptr + off, left < 16 ? static_cast<int>(left) : 16, b.align >= 4);
+        }
+        h = absorb(h, v);
+      }
+      const uint64_t x = __shfl_sync(kFull, warp_tree(fmix(h), 32, lane), 0);
+      if (lane == static_cast<int>(c - c0)) mine = x;
+    }
+    const uint64_t root = warp_tree(mine, static_cast<int>(c1 - c0), lane);
+    if (lane == 0) nodes[b.task_begin + local] = root;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+    k_fp_static_final(const StaticPlan plan, uint64_t* nodes, uint64_t* __restrict__ fp_out) {
+  const int lane = threadIdx.x & 31;
+  const int i = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (i >= plan.n) return;
+  const StaticBuf& b = plan.b[i];
+  const uint64_t root = warp_tree_inplace(nodes + b.task_begin, b.n_tasks, lane);
+  if (lane == 0) fp_out[i] = fmix(root ^ (b.bytes * kP));
+}
+
+}  // namespace
+
+cudaError_t static_scratch(uint64_t** nodes) {
+  static std::mutex mu;
+  static uint64_t* addr[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_static_nodes);
+    if (e != cudaSuccess) return e;
+    addr[dev] = static_cast<uint64_t*>(p);
+  }
+  *nodes = addr[dev];
+  return cudaSuccess;
+}
+
+cudaError_t launch_fingerprint_static(const StaticPlan& plan, uint64_t* nodes, uint64_t* fp_out,
+                                      cudaStream_t stream) {
+  if (plan.n <= 0) return cudaSuccess;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t want = (static_cast<uint64_t>(plan.n_tasks) + kWarps - 1) / kWarps;
+  const uint64_t cap = static_cast<uint64_t>(sms) * 4;
+  const int blocks = static_cast<int>(want < cap ? (want ? want : 1) : cap);
+  k_fp_static<<<blocks, kThreads, 0, stream>>>(plan, nodes);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_fp_static_final<<<(plan.n + kWarps - 1) / kWarps, kThreads, 0, stream>>>(plan, nodes, fp_out);
   return cudaGetLastError();
 }
 

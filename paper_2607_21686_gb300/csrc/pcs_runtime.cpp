@@ -1480,4 +1480,56 @@ pcs_status pcs_snapshot_read_file(pcs_ctx* c, const char* path, uint32_t placeme
   return PCS_OK;
 }
 
+pcs_status pcs_fingerprint_static(const pcs_buf* bufs, int32_t n, uint64_t* fp_out,
+                                  void* stream) {
+  static_assert(kStaticMaxBufs == PCS_STATIC_MAX_BUFFERS, "limit");
+  static_assert(kStaticMaxNodes == PCS_STATIC_MAX_NODES, "limit");
+  if (n < 0 || n > kStaticMaxBufs)
+    return fail(PCS_E_INVAL, "pcs_fingerprint_static takes 0..%d buffers, got %d", kStaticMaxBufs, n);
+  if (n == 0) return PCS_OK;
+  if (!bufs || !fp_out) return fail(PCS_E_INVAL, "null argument");
+  StaticPlan plan{};  // on the stack; passed to the kernels by value
+  plan.n = n;
+  uint64_t chunks = 0;
+  for (int i = 0; i < n; ++i) {
+    if (bufs[i].bytes > 0 && !bufs[i].ptr) return fail(PCS_E_INVAL, "buffer %d: null pointer", i);
+    StaticBuf& b = plan.b[i];
+    b.ptr = static_cast<const uint8_t*>(bufs[i].ptr);
+    b.bytes = bufs[i].bytes;
+    b.n_chunks = n_chunks_of(b.bytes);
+    const uintptr_t a = reinterpret_cast<uintptr_t>(b.ptr);
+    b.align = (a & 15u) == 0 ? 16u : ((a & 3u) == 0 ? 4u : 1u);
+    chunks += b.n_chunks;
+  }
+  // Smallest warp task (2^g chunks) that keeps every warp busy and fits the
+  // fixed node array.
+  auto tasks_for = [&](int g) {
+    uint64_t t = 0;
+    for (int i = 0; i < n; ++i) t += (plan.b[i].n_chunks + (1ull << g) - 1) >> g;
+    return t;
+  };
+  int g = 0;
+  while (g < kMaxGroupLog2 && (tasks_for(g) > kStaticMaxNodes || (chunks >> (g + 1)) >= 8192)) ++g;
+  const uint64_t tasks = tasks_for(g);
+  if (tasks > kStaticMaxNodes)
+    return fail(PCS_E_INVAL,
+                "pcs_fingerprint_static: these buffers need %llu scratch nodes, the fixed limit "
+                "is %u (about 8 GiB per call)",
+                static_cast<unsigned long long>(tasks), kStaticMaxNodes);
+  uint32_t t = 0;
+  for (int i = 0; i < n; ++i) {
+    plan.b[i].task_begin = t;
+    plan.b[i].n_tasks = static_cast<uint32_t>((plan.b[i].n_chunks + (1ull << g) - 1) >> g);
+    t += plan.b[i].n_tasks;
+  }
+  plan.n_tasks = t;
+  plan.glog2 = g;
+  uint64_t* nodes = nullptr;
+  cudaError_t e = static_scratch(&nodes);
+  if (e != cudaSuccess) return cuda_fail(e, "looking up the fixed scratch");
+  e = launch_fingerprint_static(plan, nodes, fp_out, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "pcs_fingerprint_static launch");
+  return PCS_OK;
+}
+
 }  // extern "C"

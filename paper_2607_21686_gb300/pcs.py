@@ -138,7 +138,10 @@ SIGNATURES = {
     "pcs_snapshot_copy_out": (_st, [_vp, _vp, _u64, _u64, _vp, _vp]),
     "pcs_snapshot_write_file": (_st, [_vp, _vp, ctypes.c_char_p]),
     "pcs_snapshot_read_file": (_st, [_vp, ctypes.c_char_p, _u32, ctypes.POINTER(_vp)]),
+    "pcs_fingerprint_static": (_st, [ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
 }
+PCS_STATIC_MAX_BUFFERS = 64
+PCS_STATIC_MAX_NODES = 65536
 
 _lib = None
 _lock = threading.Lock()
