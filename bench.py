@@ -36,11 +36,21 @@ sys.path.insert(0, ROOT)
 
 METRIC = "snapshot+restore GB/s and sessions/s on 1 GB300; % of HBM (PCIe) roofline"
 
+# DRAM bytes (read + write) per launch of the streaming kernels, from the ncu
+# capture summarised in profiles/k_bulk_kv8x24_full.md (8 sessions, scaled by
+# sessions / 8), valid only for the kernel source it was taken on.
+NCU_TRAFFIC = {
+    "source_sha256_prefix": "d4fc58b0b1d3d65b",
+    "sessions": 8,
+    "k_bulk<pack>": (805.718272 + 754.997504) * 1e6,
+    "k_bulk<restore_verify>": (805.773824 + 754.557184) * 1e6,
+}
+
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=60)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="pcs", choices=["pcs", "reference"])
     ap.add_argument("--sessions", type=int, default=256)
@@ -67,6 +77,20 @@ def step_bytes(a) -> int:
     meta = 32
     payload = a.sessions * (2 * a.layers * sec + meta)
     return 4 * payload
+
+
+def kernel_source_sha() -> str:
+    import hashlib
+    p = os.path.join(ROOT, "paper_2607_21686_gb300", "csrc", "pcs_kernels.cu")
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def ncu_traffic(kernel: str, sessions: int):
+    """Measured DRAM traffic per launch scaled to `sessions`, or None."""
+    if kernel not in NCU_TRAFFIC or kernel_source_sha() != NCU_TRAFFIC["source_sha256_prefix"]:
+        return None
+    return round(NCU_TRAFFIC[kernel] * sessions / NCU_TRAFFIC["sessions"])
 
 
 def load_peaks() -> dict:
@@ -361,7 +385,7 @@ def main():
                     "peak": peaks["hbm_gbs"], "peak_source": peaks["source"], "unit": "GB/s",
                     "frac": round(achieved / peaks["hbm_gbs"], 4),
                     "bytes_per_launch": algo, "ms_per_launch": round(per_launch_ms, 4),
-                    "traffic": None}
+                    "traffic": ncu_traffic(top, a.sessions)}
         cpu = None
         if not a.no_cpu_baseline:
             cpu = cpu_oracle_rate(a, a.cpu_seconds)

@@ -1,0 +1,129 @@
+"""GPU parity at the full workload sizes, in the launch shape bench.py times.
+
+The oracle is too slow for every byte, so each test checks sampled outputs
+against the oracle one by one (whole records of sampled sessions, scores and
+kept sets of sampled banks) and checks properties that hold at any size on
+every output (every restored row equals its source row; every section's
+stored fingerprint is re-verified by the restore).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_21686_gb300 import pcs, synth
+from helpers import np_view
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+def _session_pages(pool, pt):
+    """The pages a session uses, compacted, with the page table renumbered."""
+    flat = pt.reshape(-1).long()
+    pages = pool[flat].cpu()
+    return pages, torch.arange(flat.numel(), dtype=torch.int32).view(pt.shape)
+
+
+def test_kv_full_size(ctx, dev):
+    # 256 sessions x 24 layers x 16 heads x 64, window 1024, 16-token pages.
+    kv = synth.kv(device=dev)
+    S, Lyr, W, P = kv.sessions, kv.layers, kv.window, kv.page_rows
+    sess = [pcs.kv_session(s, kv.meta[s], kv.k_pool, kv.v_pool, kv.page_table[s], kv.ring_start[s], W)
+            for s in range(S)]
+    snaps = ctx.checkpoint(sess)
+    pt2 = synth.page_permutation(synth.seed_for(3) + 7, S, Lyr, W // P, device=dev)
+    k2, v2 = torch.empty_like(kv.k_pool), torch.empty_like(kv.v_pool)
+    meta2 = torch.empty_like(kv.meta)
+    tg = [pcs.kv_session(s, meta2[s], k2, v2, pt2[s], pcs.PCS_RING_START_FROM_SNAPSHOT, W)
+          for s in range(S)]
+    ctx.restore(snaps, tg, verify=True)
+    torch.cuda.synchronize()
+    # Every restored row of every session equals its source row.
+    j = torch.arange(W, device=dev)
+    for s in range(S):
+        slot = (kv.ring_start[s] + j) % W
+        a = kv.page_table[s].long()[:, slot // P]
+        b = pt2[s].long()[:, slot // P]
+        r = slot % P
+        assert torch.equal(kv.k_pool[a, r], k2[b, r]), s
+        assert torch.equal(kv.v_pool[a, r], v2[b, r]), s
+    assert torch.equal(meta2, kv.meta)
+    # Sampled whole records against the oracle.
+    for s in (0, 127, S - 1):
+        kp, ptc = _session_pages(kv.k_pool, kv.page_table[s])
+        vp, _ = _session_pages(kv.v_pool, kv.page_table[s])
+        ref = oracle.pack(oracle.kv_session(s, kv.meta[s].cpu().numpy(), np_view(kp), np_view(vp),
+                                            ptc.numpy(), kv.ring_start[s], W, P, kv.row_bytes))
+        assert np.array_equal(ctx.record(snaps[s]).numpy(), ref), s
+    for x in snaps:
+        ctx.delete(x)
+
+
+def test_mass_banks_full_size(ctx, dev):
+    # 2048 sessions, n ~ U[256,4096], key bf16[512], value u8[2048], query
+    # bf16[512]; host budget 8 GiB; pack to pinned host, restore to HBM.
+    b = synth.banks_config5(device=dev)
+    S = b.sessions
+    E = 1024 + 2048
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    vals = [b.values[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    qs = [b.queries[s] for s in range(S)]
+    banks = ctx.banks_array(keys, qs, E)
+    params = ctx.params(pcs.PCS_K_BUDGET, budget=8 << 30)
+    ks = ctx.prune_counts(banks, S, params)
+    assert sum(ks) * E <= 8 << 30
+    kept = torch.empty(sum(ks), dtype=torch.int32, device=dev)
+    koff = torch.empty(S + 1, dtype=torch.int32, device=dev)
+    scores = torch.empty(b.keys.shape[0], dtype=torch.float32, device=dev)
+    ctx.prune(banks, S, params, kept, koff, scores)
+    koff_h = koff.cpu().tolist()
+    sess = [pcs.bank_session(s, keys[s], vals[s], kept[koff_h[s]:koff_h[s + 1]]) for s in range(S)]
+    snaps = ctx.checkpoint(sess, placement=pcs.PCS_PLACE_PINNED_HOST)
+    outs = [(torch.empty(ks[s], dtype=torch.int32, device=dev),
+             torch.empty(ks[s], 512, dtype=torch.bfloat16, device=dev),
+             torch.empty(ks[s], 2048, dtype=torch.uint8, device=dev)) for s in range(S)]
+    ctx.restore(snaps, [pcs.bank_targets(s, *outs[s]) for s in range(S)], verify=True)
+    torch.cuda.synchronize()
+    # Every restored bank equals the kept rows of the live bank.
+    for s in range(S):
+        ki = kept[koff_h[s]:koff_h[s + 1]]
+        assert torch.equal(outs[s][0], ki), s
+        assert torch.equal(outs[s][1], keys[s][ki.long()]), s
+        assert torch.equal(outs[s][2], vals[s][ki.long()]), s
+        assert bool((ki[1:] > ki[:-1]).all()), s
+    # Sampled banks against the oracle: scores (bit-exact fp32, 1e-3 vs fp64),
+    # kept sets, whole records.
+    sc = scores.cpu().numpy()
+    kept_h = kept.cpu().numpy()
+    for s in (0, 1, 1000, S - 1):
+        lo, hi = b.entry_off[s], b.entry_off[s + 1]
+        kh, vh = np_view(keys[s]), vals[s].cpu().numpy()
+        s32, s64 = oracle.scores(np_view(qs[s]), kh, want64=True)
+        assert np.array_equal(sc[lo:hi].view(np.uint32), s32.view(np.uint32)), s
+        np.testing.assert_allclose(sc[lo:hi], s64, rtol=1e-3, atol=1e-6)
+        want = oracle.topk(s32, ks[s])
+        assert kept_h[koff_h[s]:koff_h[s + 1]].tolist() == want.tolist(), s
+        ref = oracle.pack(oracle.bank_session(s, kh, vh, want, oracle.DT_BF16, oracle.DT_U8))
+        assert np.array_equal(ctx.record(snaps[s]).numpy(), ref), s
+    for x in snaps:
+        ctx.delete(x)
+
+
+def test_markov_batch_full_size(ctx, dev):
+    # 4096 Markovian sessions of [3,256,256] uint8 + 16-byte RNG in one call.
+    S = 4096
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(1))
+    obs = torch.randint(0, 256, (S, 3, 256, 256), generator=g, device=dev, dtype=torch.uint8)
+    rng = torch.randint(-2**62, 2**62, (S, 2), generator=g, device=dev, dtype=torch.int64)
+    sess = [pcs.markov_session(s, obs[s], rng[s]) for s in range(S)]
+    snaps = ctx.checkpoint(sess)
+    o2, r2 = torch.zeros_like(obs), torch.zeros_like(rng)
+    ctx.restore(snaps, [pcs.markov_session(s, o2[s], r2[s]) for s in range(S)], verify=True)
+    torch.cuda.synchronize()
+    assert torch.equal(o2, obs) and torch.equal(r2, rng)
+    for s in (0, S // 2, S - 1):
+        ref = oracle.pack(oracle.markov_session(s, obs[s].cpu().numpy(),
+                                                rng[s].cpu().numpy().view(np.uint64)))
+        assert np.array_equal(ctx.record(snaps[s]).numpy(), ref), s
+    for x in snaps:
+        ctx.delete(x)
