@@ -93,6 +93,18 @@ def ncu_traffic(kernel: str, sessions: int):
     return round(NCU_TRAFFIC[kernel] * sessions / NCU_TRAFFIC["sessions"])
 
 
+def max_over_ranks(x: float) -> float:
+    """The largest of one float across the ranks of the default process group."""
+    if not torch.distributed.is_initialized() or torch.distributed.get_world_size() == 1:
+        return x
+    dev = "cpu"
+    if torch.distributed.get_backend() == "nccl":
+        dev = torch.device("cuda", torch.cuda.current_device())
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
 def load_peaks() -> dict:
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -285,10 +297,7 @@ def run_pcs(a, rank, world, local_rank):
     ktimes = ctx.kernel_times()
     ctx.timing(False)
     launches = ctx.stats().kernel_launches - launches0
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms)
 
     # End to end through the public API with the state coming from host memory.
     e2e = None

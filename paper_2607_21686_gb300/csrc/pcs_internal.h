@@ -52,9 +52,11 @@ struct alignas(16) SecDesc {
   uint32_t n_tasks;
   uint64_t n_chunks;
   uint32_t align;          // CONTIG layout side: 16, 4 or 1 (largest that divides lbase)
-  uint32_t pad0;
+  uint32_t fin_count;      // nodes the finaliser trees: [fin_begin, fin_begin + fin_count)
+  uint32_t fin_begin;      // (the task nodes, or their 32-to-1 reduction)
+  uint32_t pad[3];
 };
-static_assert(sizeof(SecDesc) == 96, "SecDesc layout");
+static_assert(sizeof(SecDesc) == 112, "SecDesc layout");
 
 // One session: a record and the contiguous range of its sections.
 struct alignas(16) SessDesc {
@@ -117,7 +119,13 @@ cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* no
                         uint32_t* dev_err, int sm_count, cudaStream_t stream);
 size_t bulk_shared_bytes();
 
-// Section fps from the warp-task nodes (in place), then per mode:
+// Streams with many task nodes: reduce each aligned group of 32 nodes of
+// stream i (nodes[task_begin_i ...]) to one node at nodes[fin_begin_i + g].
+// Groups of all streams are numbered by fin_begin - base (monotone).
+cudaError_t launch_reduce_nodes(const SecDesc* secs, int n_secs, uint64_t* nodes, uint32_t base,
+                                uint32_t n_groups, int sm_count, cudaStream_t stream);
+
+// Section fps from the nodes [fin_begin, fin_begin + fin_count) (in place), then per mode:
 //   kModeHash: fp_out[i] = fp; if fp_before: flags[i] = fp != fp_before[i]
 //   kModePack: header + section table of each session's record
 //   kModeRestoreV: compare with the record's stored fps; corrupt[s] = 1 and
@@ -127,9 +135,8 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
                             const uint64_t* fp_before, uint8_t* flags, uint32_t* bad,
                             cudaStream_t stream);
 
-cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
-                         const uint64_t* entry_begin_sorted, float* scores, int sm_count,
-                         cudaStream_t stream);
+cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
+                         float* scores, int sm_count, cudaStream_t stream);
 
 cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
                         int32_t* kept_idx, cudaStream_t stream);

@@ -677,8 +677,30 @@ __global__ void __launch_bounds__(kBulkThreads, 1)
 // ---------------------------------------------------------------------------
 
 __device__ __forceinline__ uint64_t stream_fp(const SecDesc& s, uint64_t* nodes, int lane) {
-  const uint64_t root = warp_tree_inplace(nodes + s.task_begin, s.n_tasks, lane);
+  const uint64_t root = warp_tree_inplace(nodes + s.fin_begin, s.fin_count, lane);
   return fmix(root ^ (s.bytes * kP));
+}
+
+// One warp per aligned group of 32 task nodes of one stream.
+__global__ void __launch_bounds__(kThreads)
+    k_reduce_nodes(const SecDesc* __restrict__ secs, int n_secs, uint64_t* nodes, uint32_t base,
+                   uint32_t n_groups) {
+  const int lane = threadIdx.x & 31;
+  const uint32_t nw = gridDim.x * kWarps;
+  for (uint32_t g = blockIdx.x * kWarps + (threadIdx.x >> 5); g < n_groups; g += nw) {
+    int lo = 0, hi = n_secs - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (__ldg(&secs[mid].fin_begin) - base <= g) lo = mid;
+      else hi = mid - 1;
+    }
+    const SecDesc& s = secs[lo];
+    const uint32_t local = g - (s.fin_begin - base);
+    const uint32_t n = min(32u, s.n_tasks - 32u * local);
+    const uint64_t v = lane < static_cast<int>(n) ? nodes[s.task_begin + 32u * local + lane] : 0;
+    const uint64_t r = warp_tree(v, static_cast<int>(n), lane);
+    if (lane == 0) nodes[s.fin_begin + local] = r;
+  }
 }
 
 // Fingerprints of independent buffers (pcs_fingerprint / pcs_classify).
@@ -785,10 +807,10 @@ __device__ __forceinline__ float elem(uint32_t bits16, bool bf16) {
               : __half2float(__ushort_as_half(static_cast<unsigned short>(bits16)));
 }
 
-// Accumulate the 8 elements of one 16-byte segment, ascending element order,
-// with separately rounded products and sums.
-__device__ __forceinline__ void accum8(uint4 q, uint4 k, bool bf16, float& sd, float& sq,
-                                       float& sk) {
+// Accumulate the key terms (q.k and k.k) of the 8 elements of one 16-byte
+// segment, ascending element order, with separately rounded products and
+// sums.  (q.q is the same for every key of a bank: accum8_query.)
+__device__ __forceinline__ void accum8_key(uint4 q, uint4 k, bool bf16, float& sd, float& sk) {
   const uint32_t qw[4] = {q.x, q.y, q.z, q.w};
   const uint32_t kw[4] = {k.x, k.y, k.z, k.w};
 #pragma unroll
@@ -797,8 +819,17 @@ __device__ __forceinline__ void accum8(uint4 q, uint4 k, bool bf16, float& sd, f
     const uint32_t kb = (kw[i >> 1] >> (16 * (i & 1))) & 0xFFFFu;
     const float qe = elem(qb, bf16), ke = elem(kb, bf16);
     sd = __fadd_rn(sd, __fmul_rn(qe, ke));
-    sq = __fadd_rn(sq, __fmul_rn(qe, qe));
     sk = __fadd_rn(sk, __fmul_rn(ke, ke));
+  }
+}
+
+// The query's own term, accumulated in the same lane order.
+__device__ __forceinline__ void accum8_query(uint4 q, bool bf16, float& sq) {
+  const uint32_t qw[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float qe = elem((qw[i >> 1] >> (16 * (i & 1))) & 0xFFFFu, bf16);
+    sq = __fadd_rn(sq, __fmul_rn(qe, qe));
   }
 }
 
@@ -808,42 +839,100 @@ __device__ __forceinline__ float lane_tree_sum(float v) {
   return v;
 }
 
+constexpr int kScoreIlp = 4;  // entries a warp scores at once
+
+// Each warp scores a contiguous, balanced range of entries, kScoreIlp at a
+// time, following a cursor over the banks (one search per warp).  SPL = 16-byte
+// key segments per lane (D <= 256 * SPL); every key load of the kScoreIlp
+// entries is issued before any arithmetic.  SPL = 0: any D, loop per segment.
+template <int SPL>
 __global__ void __launch_bounds__(kThreads)
     k_score(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
             float* __restrict__ scores) {
   const int lane = threadIdx.x & 31;
+  const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
   const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kWarps;
-  int cur = -1;
-  BankDesc B{};
-  for (uint64_t e = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5); e < n_entries;
-       e += nw) {
+  const uint64_t e_begin = n_entries * gw / nw, e_end = n_entries * (gw + 1) / nw;
+  if (e_begin >= e_end) return;
+  int b = 0;
+  {
     int lo = 0, hi = n_banks - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (__ldg(&banks[mid].entry_begin) <= e) lo = mid;
+      if (__ldg(&banks[mid].entry_begin) <= e_begin) lo = mid;
       else hi = mid - 1;
     }
-    if (lo != cur) {
-      B = banks[lo];
-      cur = lo;
+    b = lo;
+  }
+  // |q| of the current bank: the same fixed-order sum for every one of its keys.
+  int qbank = -1;
+  float qnorm = 0.f;
+  for (uint64_t e0 = e_begin; e0 < e_end; e0 += kScoreIlp) {
+    float sd[kScoreIlp], sk[kScoreIlp];
+    int bank[kScoreIlp];
+    const uint8_t* krow[kScoreIlp];
+#pragma unroll
+    for (int q = 0; q < kScoreIlp; ++q) {
+      sd[q] = sk[q] = 0.f;
+      bank[q] = -1;
+      krow[q] = nullptr;
+      const uint64_t e = e0 + q;
+      if (e >= e_end) continue;
+      while (b + 1 < n_banks && __ldg(&banks[b + 1].entry_begin) <= e) ++b;
+      bank[q] = b;
+      const BankDesc& B = banks[b];
+      krow[q] = reinterpret_cast<const uint8_t*>(B.keys) +
+                (e - B.entry_begin) * static_cast<uint64_t>(B.D) * 2;
     }
-    const uint64_t i = e - B.entry_begin;
-    const bool bf16 = B.is_bf16 != 0;
-    const int segs = B.D / 8;
-    const uint8_t* krow = reinterpret_cast<const uint8_t*>(B.keys) + i * static_cast<uint64_t>(B.D) * 2;
-    const uint8_t* qrow = reinterpret_cast<const uint8_t*>(B.query);
-    float sd = 0.f, sq = 0.f, sk = 0.f;
-    for (int t = lane; t < segs; t += 32) {
-      const uint4 kv = ld_stream(krow + 16 * t);
-      const uint4 qv = __ldg(reinterpret_cast<const uint4*>(qrow) + t);
-      accum8(qv, kv, bf16, sd, sq, sk);
+    if (SPL > 0) {
+      uint4 kv[kScoreIlp][SPL > 0 ? SPL : 1];
+#pragma unroll
+      for (int q = 0; q < kScoreIlp; ++q) {
+        const int segs = bank[q] >= 0 ? banks[bank[q]].D / 8 : 0;
+#pragma unroll
+        for (int j = 0; j < SPL; ++j) {
+          const int t = lane + 32 * j;
+          kv[q][j] = t < segs ? ld_stream(krow[q] + 16 * t) : make_uint4(0, 0, 0, 0);
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kScoreIlp; ++q) {
+        if (bank[q] < 0) continue;
+        const BankDesc& B = banks[bank[q]];
+        const int segs = B.D / 8;
+        const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
+#pragma unroll
+        for (int j = 0; j < SPL; ++j) {
+          const int t = lane + 32 * j;
+          if (t < segs) accum8_key(__ldg(qrow + t), kv[q][j], B.is_bf16 != 0, sd[q], sk[q]);
+        }
+      }
+    } else {
+#pragma unroll
+      for (int q = 0; q < kScoreIlp; ++q) {
+        if (bank[q] < 0) continue;
+        const BankDesc& B = banks[bank[q]];
+        const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
+        for (int t = lane; t < B.D / 8; t += 32)
+          accum8_key(__ldg(qrow + t), ld_stream(krow[q] + 16 * t), B.is_bf16 != 0, sd[q], sk[q]);
+      }
     }
-    sd = lane_tree_sum(sd);
-    sq = lane_tree_sum(sq);
-    sk = lane_tree_sum(sk);
-    if (lane == 0) {
-      const float den = __fmul_rn(__fsqrt_rn(sq), __fsqrt_rn(sk));
-      scores[e] = den == 0.f ? 0.f : __fdiv_rn(sd, den);
+#pragma unroll
+    for (int q = 0; q < kScoreIlp; ++q) {
+      if (bank[q] >= 0 && bank[q] != qbank) {  // warp-uniform
+        const BankDesc& B = banks[bank[q]];
+        const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
+        float sq = 0.f;
+        for (int t = lane; t < B.D / 8; t += 32) accum8_query(__ldg(qrow + t), B.is_bf16 != 0, sq);
+        qnorm = __fsqrt_rn(lane_tree_sum(sq));
+        qbank = bank[q];
+      }
+      const float d = lane_tree_sum(sd[q]);
+      const float kk = lane_tree_sum(sk[q]);
+      if (lane == 0 && bank[q] >= 0) {
+        const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
+        scores[e0 + q] = den == 0.f ? 0.f : __fdiv_rn(d, den);
+      }
     }
   }
 }
@@ -1073,14 +1162,26 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
   return cudaGetLastError();
 }
 
-cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
-                         const uint64_t* /*entry_begin_sorted*/, float* scores, int sm_count,
-                         cudaStream_t stream) {
-  if (n_entries == 0) return cudaSuccess;
-  const uint64_t want = (n_entries + kWarps - 1) / kWarps;
+cudaError_t launch_reduce_nodes(const SecDesc* secs, int n_secs, uint64_t* nodes, uint32_t base,
+                                uint32_t n_groups, int sm_count, cudaStream_t stream) {
+  if (n_groups == 0) return cudaSuccess;
+  const uint64_t want = (static_cast<uint64_t>(n_groups) + kWarps - 1) / kWarps;
   const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
   const int blocks = static_cast<int>(want < cap ? want : cap);
-  k_score<<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  k_reduce_nodes<<<blocks, kThreads, 0, stream>>>(secs, n_secs, nodes, base, n_groups);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
+                         float* scores, int sm_count, cudaStream_t stream) {
+  if (n_entries == 0) return cudaSuccess;
+  const uint64_t want = (n_entries + kWarps * kScoreIlp * 8 - 1) / (kWarps * kScoreIlp * 8);
+  const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
+  const int blocks = static_cast<int>(want < cap ? want : cap);
+  if (max_dim <= 256) k_score<1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  else if (max_dim <= 512) k_score<2><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  else if (max_dim <= 1024) k_score<4><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  else k_score<0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
   return cudaGetLastError();
 }
 

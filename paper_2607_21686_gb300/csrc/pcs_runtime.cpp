@@ -357,12 +357,13 @@ pcs_status set_device(pcs_ctx* c) {
 enum KernelKind {
   kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
   kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKCopy, kKBulkHash, kKBulkPack,
-  kKBulkRestore, kKBulkRestoreV, kKernelKinds
+  kKBulkRestore, kKBulkRestoreV, kKReduce, kKernelKinds
 };
 const char* kKernelNames[kKernelKinds] = {
     "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
-    "k_copy", "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>"};
+    "k_copy", "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
+    "k_reduce_nodes"};
 
 cudaEvent_t timing_event(pcs_ctx* c) {
   if (!c->timing_events.empty()) {
@@ -564,7 +565,9 @@ bool is_device_ptr(const void* p, std::unordered_map<const void*, bool>& cache) 
 struct StreamPlan {
   std::vector<uint32_t> bulk_ids, bulk_begin, reg_ids, reg_begin;
   uint32_t bulk_tasks = 0, reg_tasks = 0;
-  uint64_t nodes = 0;
+  uint64_t nodes = 0;          // task nodes
+  uint32_t reduce_groups = 0;  // 32-to-1 groups reduced before finalising (0 = none)
+  uint64_t nodes_total = 0;    // task nodes + reduced nodes
   int glog2 = 0;
 };
 
@@ -607,7 +610,24 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   P.bulk_tasks = static_cast<uint32_t>(tb);
   P.reg_tasks = static_cast<uint32_t>(tr);
   P.nodes = node;
-  return node < (1ull << 32);
+  // A stream with many task nodes would leave one finalising warp a long
+  // serial tree: reduce aligned groups of 32 nodes across the GPU first.
+  uint64_t max_tasks = 0;
+  for (const auto& x : d) max_tasks = std::max<uint64_t>(max_tasks, x.n_tasks);
+  uint64_t groups = 0;
+  for (auto& x : d) {
+    if (max_tasks > 64) {
+      x.fin_begin = static_cast<uint32_t>(node + groups);
+      x.fin_count = (x.n_tasks + 31) / 32;
+      groups += x.fin_count;
+    } else {
+      x.fin_begin = x.task_begin;
+      x.fin_count = x.n_tasks;
+    }
+  }
+  P.reduce_groups = static_cast<uint32_t>(groups);
+  P.nodes_total = node + groups;
+  return P.nodes_total < (1ull << 32);
 }
 
 // Workspace offsets of a stream plan's lists, after `base` bytes.
@@ -669,7 +689,7 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   L.secs = 0;
   const ListLayout LL = list_layout(P, sizeof(SecDesc) * n);
   L.nodes = round_up(LL.end, kRecordAlign);
-  L.total = L.nodes + 8 * P.nodes;
+  L.total = L.nodes + 8 * P.nodes_total;
   uint8_t* ws = nullptr;
   pcs_status st = ws_acquire(c, L.total, stream, &ws);
   if (st) return st;
@@ -707,6 +727,12 @@ cudaError_t launch_streams(pcs_ctx* c, int mode, const SecDesc* dsecs, const Str
     LaunchScope ls(c, stream_kind(mode), stream);
     e = launch_stream(mode, dsecs, wl, P.glog2, nodes, c->words, c->sm_count, c->stream_bps,
                       stream);
+    if (e != cudaSuccess) return e;
+  }
+  if (nodes && P.reduce_groups) {
+    LaunchScope ls(c, kKReduce, stream);
+    e = launch_reduce_nodes(dsecs, static_cast<int>(P.bulk_ids.size() + P.reg_ids.size()), nodes,
+                            static_cast<uint32_t>(P.nodes), P.reduce_groups, c->sm_count, stream);
   }
   return e;
 }
@@ -987,7 +1013,9 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
   auto* dbanks = reinterpret_cast<const BankDesc*>(ws + L.banks);
   {
     LaunchScope ls(c, kKScore, stream);
-    PCS_CUDA(launch_score(dbanks, n, entries, nullptr, sc, c->sm_count, stream));
+    int max_dim = 0;
+    for (int s = 0; s < n; ++s) max_dim = std::max(max_dim, banks[s].key_dim);
+    PCS_CUDA(launch_score(dbanks, n, entries, max_dim, sc, c->sm_count, stream));
   }
   {
     LaunchScope ls(c, kKTopk, stream);
@@ -1096,7 +1124,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   L.entries = round_up(L.sess + sizeof(SessDesc) * n, kRecordAlign);
   const ListLayout LL = list_layout(P, L.entries + sizeof(Entry) * ent.size());
   L.nodes = round_up(LL.end, kRecordAlign);
-  L.total = L.nodes + 8 * P.nodes;
+  L.total = L.nodes + 8 * P.nodes_total;
   auto undo = [&](pcs_status s) {
     arena_of(c, placement)->free(blk);
     return s;
@@ -1231,7 +1259,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
   const ListLayout LL = list_layout(P, L.sess + sizeof(SessDesc) * n);
   L.nodes = round_up(LL.end, kRecordAlign);
-  L.total = L.nodes + (verify ? 8 * P.nodes : 0);
+  L.total = L.nodes + (verify ? 8 * P.nodes_total : 0);
   uint8_t* ws = nullptr;
   st = ws_acquire(c, L.total, stream, &ws);
   if (st) return st;

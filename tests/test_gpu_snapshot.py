@@ -367,3 +367,13 @@ def test_mixed_kinds_one_call(ctx, dev):
     for s, r in zip(snaps, refs):
         assert np.array_equal(ctx.record(s).numpy(), r)
         ctx.delete(s)
+
+
+@pytest.mark.parametrize("D,dtype", [(8, torch.float16), (264, torch.bfloat16),
+                                     (1024, torch.float16), (1536, torch.bfloat16)])
+def test_prune_key_dims(ctx, dev, D, dtype):
+    # Every code path of the score kernel: 1, 2, 4 segments per lane and the
+    # generic loop for D > 1024.
+    b = synth.banks(70 + D, 9, 1, 70, D, dtype, (8,), torch.uint8)
+    keys, vals, qs = _bank_views(b, dev)
+    _check_prune(ctx, b, keys, qs, ctx.params(pcs.PCS_K_FRACTION, fraction=0.3), dev)
