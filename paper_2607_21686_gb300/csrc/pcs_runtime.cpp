@@ -97,7 +97,7 @@ struct Event {
   ~Event() {
     if (ev) pool->put(ev);
   }
-  bool done() const { return cudaEventQuery(ev) == cudaSuccess; }
+  bool done() const { return ev && cudaEventQuery(ev) == cudaSuccess; }
 };
 using Ev = std::shared_ptr<Event>;
 
@@ -329,6 +329,11 @@ struct pcs_ctx {
   // Small device words: [0] kernel error bits, [1] verification failures.
   uint32_t* words = nullptr;
   std::vector<uint8_t> plan;   // host staging of the descriptors
+  // Pinned ring for small plans: a true async copy, no driver-side staging.
+  uint8_t* plan_ring = nullptr;
+  Ev plan_slot_busy[8];
+  int plan_slot = 0;
+  int plan_slot_used = -1;     // slot of the call in progress, or -1
   uint8_t* stage = nullptr;    // pinned staging for file I/O
   uint64_t stage_bytes = 0;
   uint64_t launches = 0;       // kernels launched by this context
@@ -445,9 +450,45 @@ pcs_status ws_acquire(pcs_ctx* c, uint64_t bytes, cudaStream_t stream, uint8_t**
   return PCS_OK;
 }
 
-pcs_status ws_release(pcs_ctx* c, cudaStream_t stream) {
-  c->ws_busy = record_event(c->events, stream);
+constexpr uint64_t kPlanSlotBytes = 64 << 10;
+constexpr int kPlanSlots = 8;
+
+// Copy the call's descriptors (c->plan, `bytes`) into the workspace.  Small
+// plans go through a slot of a pinned ring, reusable once the call that last
+// used it has passed its end event; larger ones are copied from pageable memory.
+cudaError_t plan_copy(pcs_ctx* c, uint8_t* ws, uint64_t bytes, cudaStream_t stream) {
+  if (bytes <= kPlanSlotBytes) {
+    if (!c->plan_ring &&
+        cudaHostAlloc(&c->plan_ring, kPlanSlotBytes * kPlanSlots, cudaHostAllocDefault) != cudaSuccess) {
+      cudaGetLastError();
+      c->plan_ring = nullptr;
+    }
+    if (c->plan_ring) {
+      const int i = c->plan_slot;
+      Ev& busy = c->plan_slot_busy[i];
+      if (!busy || busy->done()) {
+        uint8_t* slot = c->plan_ring + kPlanSlotBytes * i;
+        std::memcpy(slot, c->plan.data(), bytes);
+        c->plan_slot = (i + 1) % kPlanSlots;
+        // Held until ws_release records the call's end; a call that fails
+        // before then leaves the slot held for good (never reused early).
+        busy = std::make_shared<Event>();
+        c->plan_slot_used = i;
+        return cudaMemcpyAsync(ws, slot, bytes, cudaMemcpyHostToDevice, stream);
+      }
+    }
+  }
+  c->plan_slot_used = -1;
+  return cudaMemcpyAsync(ws, c->plan.data(), bytes, cudaMemcpyHostToDevice, stream);
+}
+
+// End of a call's use of the workspace (and of its plan slot): `done`, if
+// given, is an event already recorded at this point of the stream.
+pcs_status ws_release(pcs_ctx* c, cudaStream_t stream, Ev done = nullptr) {
+  c->ws_busy = done ? done : record_event(c->events, stream);
   if (!c->ws_busy) return fail(PCS_E_CUDA, "cudaEventRecord failed");
+  if (c->plan_slot_used >= 0) c->plan_slot_busy[c->plan_slot_used] = c->ws_busy;
+  c->plan_slot_used = -1;
   return PCS_OK;
 }
 
@@ -574,12 +615,22 @@ struct StreamPlan {
 // The TMA-staged kernel takes a stream whose bytes on both sides live in
 // device memory and can be moved as whole 16-byte pieces: a 16-byte aligned
 // contiguous buffer, or rows of at least 512 bytes.
-bool bulk_eligible(const pcs_ctx* c, const SecDesc& d, bool payload_device,
+bool bulk_eligible(const pcs_ctx* c, const SecDesc& d, bool payload_device, bool small_call,
                    std::unordered_map<const void*, bool>& cache) {
-  if (!c->use_bulk || !payload_device) return false;
+  if (!c->use_bulk || !payload_device || small_call) return false;
   if (!is_device_ptr(d.lbase, cache)) return false;
   if (d.layout == kContig) return d.align == 16 || d.bytes == 0;
   return d.row_bytes >= kBulkMinRowBytes && d.row_bytes % 16 == 0;
+}
+
+// Calls moving at most this many bytes take the register kernel: their time
+// is launch latency, which the shared-memory pipeline does not shorten.
+constexpr uint64_t kSmallCallBytes = 1ull << 20;
+
+uint64_t total_bytes(const std::vector<SecDesc>& d) {
+  uint64_t t = 0;
+  for (const auto& x : d) t += x.bytes;
+  return t;
 }
 
 // Give every stream its node slots and its kernel.  bulk[i] says which.
@@ -682,7 +733,8 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   (void)chunks;
   std::unordered_map<const void*, bool> cache;
   std::vector<char> bulk(n);
-  for (int i = 0; i < n; ++i) bulk[i] = bulk_eligible(c, d[i], true, cache);
+  const bool small = total_bytes(d) <= kSmallCallBytes;
+  for (int i = 0; i < n; ++i) bulk[i] = bulk_eligible(c, d[i], true, small, cache);
   StreamPlan P;
   if (!plan_streams(c, d, bulk, P)) return fail(PCS_E_INVAL, "too much data in one call");
   WsLayout L;
@@ -696,7 +748,7 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   c->plan.resize(L.nodes);
   put(c->plan, L.secs, d);
   put_lists(c->plan, P, LL);
-  PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
+  PCS_CUDA(plan_copy(c, ws, L.nodes, stream));
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
   PCS_CUDA(launch_streams(c, kModeHash, dsecs, P, LL, ws, nodes, stream));
@@ -809,6 +861,8 @@ pcs_status pcs_destroy(pcs_ctx* c) {
     if (c->ws) cudaFree(c->ws);
     if (c->words) cudaFree(c->words);
     if (c->stage) cudaFreeHost(c->stage);
+    for (auto& e : c->plan_slot_busy) e.reset();
+    if (c->plan_ring) cudaFreeHost(c->plan_ring);
     for (auto& t : c->timed) {
       cudaEventDestroy(t.start);
       cudaEventDestroy(t.stop);
@@ -1006,7 +1060,7 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
   c->plan.resize(L.nodes);
   put(c->plan, L.banks, d);
   put(c->plan, L.secs, koff);
-  PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
+  PCS_CUDA(plan_copy(c, ws, L.nodes, stream));
   if (kept_off)
     PCS_CUDA(cudaMemcpyAsync(kept_off, ws + L.secs, 4ull * (n + 1), cudaMemcpyDeviceToDevice, stream));
   float* sc = scores ? scores : reinterpret_cast<float*>(ws + L.nodes);
@@ -1114,8 +1168,9 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   (void)chunks;
   std::unordered_map<const void*, bool> cache;
   std::vector<char> bulk(d.size());
+  const bool small = total_bytes(d) <= kSmallCallBytes;
   for (size_t i = 0; i < d.size(); ++i)
-    bulk[i] = bulk_eligible(c, d[i], placement == PCS_PLACE_DEVICE, cache);
+    bulk[i] = bulk_eligible(c, d[i], placement == PCS_PLACE_DEVICE, small, cache);
   StreamPlan P;
   const bool fits = plan_streams(c, d, bulk, P);
   WsLayout L;
@@ -1138,7 +1193,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   put(c->plan, L.sess, sd);
   put(c->plan, L.entries, ent);
   put_lists(c->plan, P, LL);
-  cudaError_t e = cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream);
+  cudaError_t e = plan_copy(c, ws, L.nodes, stream);
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
   auto* dent = reinterpret_cast<const Entry*>(ws + L.entries);
@@ -1151,7 +1206,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   }
   if (e != cudaSuccess) return undo(cuda_fail(e, "checkpoint launch"));
   blk->written = record_event(c->events, stream);
-  st = ws_release(c, stream);
+  st = ws_release(c, stream, blk->written);
   if (st) return undo(st);
   blk->refs = n;
   for (int s = 0; s < n; ++s) {
@@ -1251,7 +1306,8 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   (void)chunks;
   std::unordered_map<const void*, bool> cache;
   std::vector<char> bulk(d.size());
-  for (size_t i = 0; i < d.size(); ++i) bulk[i] = bulk_eligible(c, d[i], payload_dev[i], cache);
+  const bool small = total_bytes(d) <= kSmallCallBytes;
+  for (size_t i = 0; i < d.size(); ++i) bulk[i] = bulk_eligible(c, d[i], payload_dev[i], small, cache);
   StreamPlan P;
   if (!plan_streams(c, d, bulk, P)) return fail(PCS_E_INVAL, "too much data in one call");
   WsLayout L;
@@ -1267,7 +1323,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   put(c->plan, L.secs, d);
   put(c->plan, L.sess, sd);
   put_lists(c->plan, P, LL);
-  PCS_CUDA(cudaMemcpyAsync(ws, c->plan.data(), L.nodes, cudaMemcpyHostToDevice, stream));
+  PCS_CUDA(plan_copy(c, ws, L.nodes, stream));
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
