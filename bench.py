@@ -63,6 +63,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-rows", action="store_true",
+                    help="skip the per-row measurements on the other populations")
     return ap.parse_args()
 
 
@@ -257,13 +259,16 @@ def run_pcs(a, rank, world, local_rank):
                           a.window) for s in range(a.sessions)]
     dst = [pcs.kv_session(s, meta2[s], k2, v2, pt2[s], pcs.PCS_RING_START_FROM_SNAPSHOT,
                           a.window) for s in range(a.sessions)]
-    verify = not a.no_verify
+    src_arr, dst_arr = ctx.session_array(src), ctx.session_array(dst)
+    # Verification runs on the device inside the restore kernels; mismatches
+    # are reported by the pcs_sync after the timed region (verify mode 2).
+    verify = 0 if a.no_verify else 2
+    S = a.sessions
 
     def step():
-        snaps = ctx.checkpoint(src)
-        ctx.restore(snaps, dst, verify=verify)
-        for s in snaps:
-            ctx.delete(s)
+        hs = ctx.checkpoint_raw(src_arr, S)
+        ctx.restore_raw(hs, S, dst_arr, verify=verify)
+        ctx.delete_raw(hs, S)
 
     for _ in range(a.warmup):
         step()
@@ -293,6 +298,7 @@ def run_pcs(a, rank, world, local_rank):
     if world > 1:
         torch.distributed.barrier()
     clk = clocks.stop()
+    ctx.sync()  # raises if any verified restore of the timed steps failed
     ms = e0.elapsed_time(e1)
     ktimes = ctx.kernel_times()
     ctx.timing(False)
@@ -304,9 +310,169 @@ def run_pcs(a, rank, world, local_rank):
     if not a.no_e2e:
         e2e = run_e2e(a, ctx, kv, src, dst, stream, dev)
 
-    res = {"ms": ms, "ktimes": ktimes, "launches": launches, "clocks": clk, "e2e": e2e}
+    rows = None
+    if not a.no_rows and rank == 0:
+        rows = {"fork": measure_fork(ctx, src, stream)}
+        del src, dst, kv, k2, v2, meta2
+        torch.cuda.empty_cache()
+        rows.update(run_rows(ctx, dev, stream))
+
+    res = {"ms": ms, "ktimes": ktimes, "launches": launches, "clocks": clk, "e2e": e2e,
+           "rows": rows}
     ctx.close()
     return res
+
+
+# ---------------------------------------------------------------------------
+# The other rows of the path, each on its own population (informational;
+# the headline `value` above is the KV checkpoint + restore step)
+# ---------------------------------------------------------------------------
+
+def _events_ms(fn, stream, reps=5, warm=2):
+    """Best and median device time of fn() over reps, CUDA events on `stream`."""
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    ts.sort()
+    return ts[0], ts[len(ts) // 2]
+
+
+def measure_fork(ctx, src, stream):
+    """a9: fork every snapshot of the KV step (independent byte copies)."""
+    snaps = ctx.checkpoint(src)
+    nbytes = sum(ctx.info(s).total_bytes for s in snaps)
+
+    def fork_all():
+        for s in snaps:
+            ctx.delete(ctx.fork(s))
+    best, med = _events_ms(fork_all, stream, reps=3, warm=1)
+    for s in snaps:
+        ctx.delete(s)
+    peak = load_peaks()["hbm_gbs"]
+    gbs = 2 * nbytes / (med / 1e3) / 1e9
+    return {"population": "256 KV snapshots (96 MiB each)", "bytes_rw": 2 * nbytes,
+            "ms": round(med, 3), "GBs": round(gbs, 1), "frac_of_hbm": round(gbs / peak, 4)}
+
+
+def run_rows(ctx, dev, stream):
+    from paper_2607_21686_gb300 import pcs, synth
+
+    peak = load_peaks()["hbm_gbs"]
+    out = {}
+    # Host link (pinned cudaMemcpyAsync, 1 GiB, best of 5): the roofline of
+    # host placement.
+    x = torch.empty(1 << 30, dtype=torch.uint8, pin_memory=True)
+    y = torch.empty(1 << 30, dtype=torch.uint8, device=dev)
+    h2d = (1 << 30) / (_events_ms(lambda: y.copy_(x, non_blocking=True), stream)[0] / 1e3) / 1e9
+    d2h = (1 << 30) / (_events_ms(lambda: x.copy_(y, non_blocking=True), stream)[0] / 1e3) / 1e9
+    del x, y
+    out["host_link"] = {"h2d_GBs": round(h2d, 1), "d2h_GBs": round(d2h, 1),
+                        "how": "pinned cudaMemcpyAsync 1 GiB, best of 5"}
+
+    # a1-a3: classification sweep, 200 buffers of 64 B .. 256 MiB.
+    sw = synth.sweep(device=dev)
+    tot = sum(sw.sizes)
+    fp0 = ctx.fingerprint(sw.before)
+    best, med = _events_ms(lambda: ctx.classify(sw.after, fp0), stream)
+    must, _ = ctx.classify(sw.after, fp0)
+    flips_ok = must.cpu().tolist() == [1 if f else 0 for f in sw.flipped]
+    gbs = tot / (med / 1e3) / 1e9
+    out["classify"] = {"population": "200 buffers, log-uniform 64 B..256 MiB, 60 flipped",
+                       "bytes_read": tot, "ms": round(med, 3), "GBs": round(gbs, 1),
+                       "frac_of_hbm": round(gbs / peak, 4), "flags_match_ground_truth": flips_ok}
+    del sw, fp0, must
+
+    # a4-a5, a7, a10: 2048 banks, relevance top-k under an 8 GiB host budget,
+    # pack to pinned host, verified restore to HBM.
+    b = synth.banks_config5(device=dev)
+    S = b.sessions
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    vals = [b.values[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    qs = [b.queries[s] for s in range(S)]
+    banks = ctx.banks_array(keys, qs, 1024 + 2048)
+    params = ctx.params(pcs.PCS_K_BUDGET, budget=8 << 30)
+    ks = ctx.prune_counts(banks, S, params)
+    kept = torch.empty(sum(ks), dtype=torch.int32, device=dev)
+    koff = torch.empty(S + 1, dtype=torch.int32, device=dev)
+    kb = b.keys.numel() * b.keys.element_size()
+    best, med = _events_ms(lambda: ctx.prune(banks, S, params, kept, koff), stream)
+    gbs = kb / (med / 1e3) / 1e9
+    out["prune"] = {"population": "2048 banks, n ~ U[256,4096], key bf16[512]",
+                    "key_bytes_read": kb, "ms": round(med, 3), "GBs": round(gbs, 1),
+                    "frac_of_hbm": round(gbs / peak, 4), "kept_fraction": round(sum(ks) / sum(b.n), 4)}
+    koff_h = koff.cpu().tolist()
+    sess = [pcs.bank_session(s, keys[s], vals[s], kept[koff_h[s]:koff_h[s + 1]]) for s in range(S)]
+    kept_bytes = sum(ks) * (1024 + 2048)
+    outs = [(torch.empty(ks[s], dtype=torch.int32, device=dev),
+             torch.empty(ks[s], 512, dtype=torch.bfloat16, device=dev),
+             torch.empty(ks[s], 2048, dtype=torch.uint8, device=dev)) for s in range(S)]
+    tg = [pcs.bank_targets(s, *outs[s]) for s in range(S)]
+
+    def ckpt_del():
+        for x_ in ctx.checkpoint(sess, placement=pcs.PCS_PLACE_PINNED_HOST):
+            ctx.delete(x_)
+    best, med = _events_ms(ckpt_del, stream, reps=3, warm=1)
+    snaps = ctx.checkpoint(sess, placement=pcs.PCS_PLACE_PINNED_HOST)
+    bestr, medr = _events_ms(lambda: ctx.restore(snaps, tg, verify=True), stream, reps=3, warm=1)
+    for x_ in snaps:
+        ctx.delete(x_)
+    out["suspend_to_host"] = {
+        "population": "the 2048 pruned banks, %.2f GB kept" % (kept_bytes / 1e9),
+        "ms": round(med, 3), "GBs": round(kept_bytes / (med / 1e3) / 1e9, 1),
+        "frac_of_d2h_link": round(kept_bytes / (med / 1e3) / 1e9 / d2h, 4)}
+    out["resume_from_host"] = {
+        "population": "the same records, verified restore into HBM",
+        "ms": round(medr, 3), "GBs": round(kept_bytes / (medr / 1e3) / 1e9, 1),
+        "frac_of_h2d_link": round(kept_bytes / (medr / 1e3) / 1e9 / h2d, 4)}
+    del b, keys, vals, outs, tg, sess, kept
+
+    # Markovian sessions: one-session latency and a 4096-session batch.
+    mk = synth.markov(device=dev)
+    one = [pcs.markov_session(0, mk.obs, mk.rng)]
+    oarr = ctx.session_array(one)
+    for _ in range(20):
+        ctx.delete_raw(ctx.checkpoint_raw(oarr, 1), 1)
+    torch.cuda.synchronize()
+    n = 1000
+    t0 = time.perf_counter()
+    for _ in range(n):
+        ctx.delete_raw(ctx.checkpoint_raw(oarr, 1), 1)
+    torch.cuda.synchronize()
+    ck_us = (time.perf_counter() - t0) / n * 1e6
+    h0 = ctx.checkpoint_raw(oarr, 1)
+    t0 = time.perf_counter()
+    for _ in range(n):
+        ctx.restore_raw(h0, 1, oarr)
+    torch.cuda.synchronize()
+    rs_us = (time.perf_counter() - t0) / n * 1e6
+    ctx.delete_raw(h0, 1)
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(1))
+    obs = torch.randint(0, 256, (4096, 3, 256, 256), generator=g, device=dev, dtype=torch.uint8)
+    rng = torch.randint(-2**62, 2**62, (4096, 2), generator=g, device=dev, dtype=torch.int64)
+    batch = [pcs.markov_session(s, obs[s], rng[s]) for s in range(4096)]
+    barr = ctx.session_array(batch)
+
+    def batch_step():
+        hs = ctx.checkpoint_raw(barr, 4096)
+        ctx.restore_raw(hs, 4096, barr)
+        ctx.delete_raw(hs, 4096)
+    best, med = _events_ms(batch_step, stream, reps=3, warm=1)
+    out["markov"] = {"one_session_checkpoint_us": round(ck_us, 2),
+                     "one_session_restore_us": round(rs_us, 2),
+                     "how": "wall clock per call (checkpoint incl. delete) through the ctypes "
+                            "binding with a prebuilt session array, 1000 calls",
+                     "paper_context_us": 12.0,
+                     "batch_4096_sessions_per_s": round(4096 / (med / 1e3), 1),
+                     "batch_GBs": round(4 * 4096 * (196608 + 16) / (med / 1e3) / 1e9, 1)}
+    return out
 
 
 def run_e2e(a, ctx, kv, src, dst, stream, dev):
@@ -325,16 +491,18 @@ def run_e2e(a, ctx, kv, src, dst, stream, dev):
     fps_d = torch.empty(a.sessions, dtype=torch.int64, device=dev)
     steps = max(2, min(a.steps, 5))
 
+    src_arr, dst_arr = ctx.session_array(src), ctx.session_array(dst)
+    S = a.sessions
+
     def one():
         kv.k_pool.copy_(kh, non_blocking=True)
         kv.v_pool.copy_(vh, non_blocking=True)
-        snaps = ctx.checkpoint(src)
-        ctx.restore(snaps, dst, verify=not a.no_verify)
-        for i, s in enumerate(snaps):
-            ctx.copy_out(s, 24, 8, fps_d[i:i + 1])
+        hs = ctx.checkpoint_raw(src_arr, S)
+        ctx.restore_raw(hs, S, dst_arr, verify=0 if a.no_verify else 2)
+        for i in range(S):
+            ctx.copy_out(pcs.Snapshot(ctx, hs[i]), 24, 8, fps_d[i:i + 1])
         fps_h.copy_(fps_d, non_blocking=True)
-        for s in snaps:
-            ctx.delete(s)
+        ctx.delete_raw(hs, S)
 
     one()
     torch.cuda.synchronize()
@@ -344,6 +512,7 @@ def run_e2e(a, ctx, kv, src, dst, stream, dev):
         one()
     e1.record(stream)
     torch.cuda.synchronize()
+    ctx.sync()
     ms = e0.elapsed_time(e1) / steps
     h2d = kh.numel() * kh.element_size() * 2
     d2h = fps_h.numel() * 8
@@ -408,7 +577,7 @@ def main():
                 "sessions_per_s": round(sps, 2),
                 "frac_of_nominal_8tbs": round(gbs / 8000.0, 4),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": r["e2e"],
-                "gpu_launches": r["launches"], "clocks": r["clocks"],
+                "gpu_launches": r["launches"], "clocks": r["clocks"], "rows": r["rows"],
                 "kernel_ms": {k: [v[0], round(v[1], 3)] for k, v in r["ktimes"].items()}}
         print(json.dumps(line), flush=True)
     if world > 1:

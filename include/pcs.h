@@ -243,8 +243,10 @@ pcs_status pcs_timing_enable(pcs_ctx *ctx, int32_t on);
 pcs_status pcs_timing_read(pcs_ctx *ctx, pcs_kernel_time *out, int32_t max, int32_t *n);
 
 /*
- * Wait for `stream`, then report errors recorded by kernels since the last
- * pcs_sync (PCS_E_RANGE) or by CUDA (PCS_E_CUDA).  Clears them.
+ * Wait for `stream`, then report what kernels recorded since the last
+ * pcs_sync -- failed asynchronous verifications (PCS_E_CORRUPT), a bounded
+ * wait that gave up (PCS_E_TIMEOUT), an out-of-range index (PCS_E_RANGE) --
+ * or a CUDA error (PCS_E_CUDA).  Clears them.
  */
 pcs_status pcs_sync(pcs_ctx *ctx, void *stream);
 
@@ -321,9 +323,11 @@ pcs_status pcs_fork(pcs_ctx *ctx, const pcs_snapshot *parent, pcs_snapshot **chi
 /*
  * restore(c) for n snapshots (I1): scatter each section payload to the
  * target section of targets[i] (same section count and byte counts; any
- * layout).  verify != 0 also recomputes every section fingerprint and the
+ * layout).  verify = 1 also recomputes every section fingerprint and the
  * session fp, waits for `stream`, and returns PCS_E_CORRUPT if any differs
- * from the record (the bytes have been written by then).
+ * from the record (the bytes have been written by then).  verify = 2 does
+ * the same checks without waiting: failures are counted on the device and
+ * the next pcs_sync returns PCS_E_CORRUPT.  verify = 0: no check.
  */
 pcs_status pcs_restore(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n,
                        const pcs_session *targets, int32_t verify, void *stream);
@@ -331,6 +335,10 @@ pcs_status pcs_restore(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n,
 /* delete(c): release a snapshot (its memory is reused once pending work
  * that reads it has finished). */
 pcs_status pcs_delete(pcs_ctx *ctx, pcs_snapshot *snap);
+
+/* delete(c) for n snapshots at once; PCS_E_HANDLE (and nothing deleted)
+ * if any handle is unknown. */
+pcs_status pcs_delete_many(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n);
 
 /* Header fields of a snapshot; waits for the work that wrote it. */
 pcs_status pcs_snapshot_get_info(pcs_ctx *ctx, const pcs_snapshot *snap, pcs_snapshot_info *out);

@@ -1,0 +1,102 @@
+"""Run one workload of the PCS hot path once (for profiling a single kernel).
+
+    python -m paper_2607_21686_gb300.cases kv --sessions 8
+    python -m paper_2607_21686_gb300.cases classify --n 200 --hi-mib 32
+    python -m paper_2607_21686_gb300.cases prune --sessions 256
+    python -m paper_2607_21686_gb300.cases markov --sessions 4096
+
+Each case builds its seeded synthetic population on cuda:0, runs the step
+`--warmup` times, then once more, and prints the device time of that last
+run.  Intended to be run under a profiler with the launch count of the
+warm-up runs skipped.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import torch
+
+from . import build, pcs, synth
+
+
+def _timed(fn, warmup):
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1)
+
+
+def case_kv(ctx, a, dev):
+    kv = synth.kv(sessions=a.sessions, device=dev)
+    pt2 = synth.page_permutation(7, kv.sessions, kv.layers, kv.window // kv.page_rows, device=dev)
+    k2, v2, m2 = torch.empty_like(kv.k_pool), torch.empty_like(kv.v_pool), torch.empty_like(kv.meta)
+    src = ctx.session_array([pcs.kv_session(s, kv.meta[s], kv.k_pool, kv.v_pool, kv.page_table[s],
+                                            kv.ring_start[s], kv.window) for s in range(kv.sessions)])
+    dst = ctx.session_array([pcs.kv_session(s, m2[s], k2, v2, pt2[s],
+                                            pcs.PCS_RING_START_FROM_SNAPSHOT, kv.window)
+                             for s in range(kv.sessions)])
+
+    def step():
+        hs = ctx.checkpoint_raw(src, kv.sessions)
+        ctx.restore_raw(hs, kv.sessions, dst, verify=2)
+        ctx.delete_raw(hs, kv.sessions)
+    return _timed(step, a.warmup)
+
+
+def case_classify(ctx, a, dev):
+    sw = synth.sweep(n=a.n, hi=a.hi_mib << 20, device=dev)
+    fp0 = ctx.fingerprint(sw.before)
+    return _timed(lambda: ctx.classify(sw.after, fp0), a.warmup)
+
+
+def case_prune(ctx, a, dev):
+    b = synth.banks_config5(sessions=a.sessions, device=dev)
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(b.sessions)]
+    banks = ctx.banks_array(keys, [b.queries[s] for s in range(b.sessions)], 1024 + 2048)
+    params = ctx.params(pcs.PCS_K_BUDGET, budget=int(sum(b.n) * 3072 * 0.627))
+    ks = ctx.prune_counts(banks, b.sessions, params)
+    kept = torch.empty(sum(ks), dtype=torch.int32, device=dev)
+    return _timed(lambda: ctx.prune(banks, b.sessions, params, kept), a.warmup)
+
+
+def case_markov(ctx, a, dev):
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(1))
+    obs = torch.randint(0, 256, (a.sessions, 3, 256, 256), generator=g, device=dev, dtype=torch.uint8)
+    rng = torch.randint(-2**62, 2**62, (a.sessions, 2), generator=g, device=dev, dtype=torch.int64)
+    arr = ctx.session_array([pcs.markov_session(s, obs[s], rng[s]) for s in range(a.sessions)])
+
+    def step():
+        hs = ctx.checkpoint_raw(arr, a.sessions)
+        ctx.restore_raw(hs, a.sessions, arr)
+        ctx.delete_raw(hs, a.sessions)
+    return _timed(step, a.warmup)
+
+
+CASES = {"kv": case_kv, "classify": case_classify, "prune": case_prune, "markov": case_markov}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("case", choices=sorted(CASES))
+    ap.add_argument("--sessions", type=int, default=8)
+    ap.add_argument("--n", type=int, default=200)
+    ap.add_argument("--hi-mib", type=int, default=32)
+    ap.add_argument("--warmup", type=int, default=1)
+    a = ap.parse_args()
+    build.build()
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    with pcs.Context(0) as ctx:
+        ms = CASES[a.case](ctx, a, dev)
+        ctx.sync()
+    print(json.dumps({"case": a.case, "ms": round(ms, 4)}))
+
+
+if __name__ == "__main__":
+    main()

@@ -589,16 +589,51 @@ SecDesc make_desc(const pcs_section& s, uint8_t* payload, uint32_t ring_start) {
   return d;
 }
 
+// Device allocations known to one call, as [lo, hi) address ranges, and the
+// verdict for pointers outside them.
+struct PtrCache {
+  std::vector<std::pair<uintptr_t, uintptr_t>> dev;
+  std::unordered_map<const void*, bool> other;
+};
+
+// cuMemGetAddressRange, looked up once through the runtime (no libcuda link).
+using AddrRangeFn = int (*)(unsigned long long*, size_t*, unsigned long long);
+AddrRangeFn addr_range_fn() {
+  static AddrRangeFn fn = [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuMemGetAddressRange", &f, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      f = nullptr;
+    }
+    return reinterpret_cast<AddrRangeFn>(f);
+  }();
+  return fn;
+}
+
 // Is `p` device memory of the current device (not host, managed or unknown)?
-bool is_device_ptr(const void* p, std::unordered_map<const void*, bool>& cache) {
+// One query per device allocation: its whole address range is remembered.
+bool is_device_ptr(const void* p, PtrCache& cache) {
   if (!p) return true;
-  auto it = cache.find(p);
-  if (it != cache.end()) return it->second;
+  const uintptr_t u = reinterpret_cast<uintptr_t>(p);
+  for (const auto& r : cache.dev)
+    if (u >= r.first && u < r.second) return true;
+  auto it = cache.other.find(p);
+  if (it != cache.other.end()) return it->second;
   cudaPointerAttributes a{};
   bool dev = false;
   if (cudaPointerGetAttributes(&a, p) == cudaSuccess) dev = a.type == cudaMemoryTypeDevice;
   else cudaGetLastError();
-  cache.emplace(p, dev);
+  unsigned long long base = 0;
+  size_t size = 0;
+  AddrRangeFn fn = addr_range_fn();
+  if (dev && fn && fn(&base, &size, u) == 0 && size > 0) {
+    cache.dev.emplace_back(static_cast<uintptr_t>(base), static_cast<uintptr_t>(base + size));
+  } else {
+    cache.other.emplace(p, dev);
+  }
   return dev;
 }
 
@@ -616,7 +651,7 @@ struct StreamPlan {
 // device memory and can be moved as whole 16-byte pieces: a 16-byte aligned
 // contiguous buffer, or rows of at least 512 bytes.
 bool bulk_eligible(const pcs_ctx* c, const SecDesc& d, bool payload_device, bool small_call,
-                   std::unordered_map<const void*, bool>& cache) {
+                   PtrCache& cache) {
   if (!c->use_bulk || !payload_device || small_call) return false;
   if (!is_device_ptr(d.lbase, cache)) return false;
   if (d.layout == kContig) return d.align == 16 || d.bytes == 0;
@@ -731,7 +766,7 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
     chunks += d[i].n_chunks;
   }
   (void)chunks;
-  std::unordered_map<const void*, bool> cache;
+  PtrCache cache;
   std::vector<char> bulk(n);
   const bool small = total_bytes(d) <= kSmallCallBytes;
   for (int i = 0; i < n; ++i) bulk[i] = bulk_eligible(c, d[i], true, small, cache);
@@ -936,8 +971,14 @@ pcs_status pcs_sync(pcs_ctx* c, void* stream) {
   pcs_status st = set_device(c);
   if (st) return st;
   PCS_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
-  uint32_t w = 0;
-  PCS_CUDA(cudaMemcpy(&w, c->words, 4, cudaMemcpyDeviceToHost));
+  uint32_t w3[3] = {0, 0, 0};
+  PCS_CUDA(cudaMemcpy(w3, c->words, sizeof w3, cudaMemcpyDeviceToHost));
+  const uint32_t w = w3[0];
+  if (w3[2] != 0) {
+    PCS_CUDA(cudaMemset(c->words + 2, 0, 4));
+    if (w) PCS_CUDA(cudaMemset(c->words, 0, 4));
+    return fail(PCS_E_CORRUPT, "%u restored sessions failed asynchronous verification", w3[2]);
+  }
   if (w != 0) {
     PCS_CUDA(cudaMemset(c->words, 0, 4));
     if (w & kDevErrTimeout)
@@ -1166,7 +1207,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
     handles[s] = std::move(h);
   }
   (void)chunks;
-  std::unordered_map<const void*, bool> cache;
+  PtrCache cache;
   std::vector<char> bulk(d.size());
   const bool small = total_bytes(d) <= kSmallCallBytes;
   for (size_t i = 0; i < d.size(); ++i)
@@ -1257,6 +1298,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   if (n < 0 || (n > 0 && (!snaps || !targets))) return fail(PCS_E_INVAL, "bad arguments");
+  if (verify < 0 || verify > 2) return fail(PCS_E_INVAL, "verify must be 0, 1 or 2");
   if (n == 0) return PCS_OK;
   std::lock_guard<std::mutex> lk(c->mu);
   pcs_status st = set_device(c);
@@ -1304,7 +1346,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
     if (st) return st;
   }
   (void)chunks;
-  std::unordered_map<const void*, bool> cache;
+  PtrCache cache;
   std::vector<char> bulk(d.size());
   const bool small = total_bytes(d) <= kSmallCallBytes;
   for (size_t i = 0; i < d.size(); ++i) bulk[i] = bulk_eligible(c, d[i], payload_dev[i], small, cache);
@@ -1327,13 +1369,15 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
-  if (verify) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
+  // verify == 1: count failures of this call in words[1] and wait for them;
+  // verify == 2: accumulate them in words[2] for the next pcs_sync.
+  if (verify == 1) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
   PCS_CUDA(launch_streams(c, verify ? kModeRestoreV : kModeRestore, dsecs, P, LL, ws,
                           verify ? nodes : nullptr, stream));
   if (verify) {
     LaunchScope ls(c, kKFinalizeRestoreV, stream);
     PCS_CUDA(launch_finalize(kModeRestoreV, dsecs, dsess, n, nullptr, nodes, nullptr, nullptr,
-                             nullptr, c->words + 1, stream));
+                             nullptr, c->words + (verify == 1 ? 1 : 2), stream));
   }
   for (int s = 0; s < n; ++s) {
     st = note_use(c, snaps[s]->block, stream);
@@ -1341,7 +1385,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   }
   st = ws_release(c, stream);
   if (st) return st;
-  if (verify) {
+  if (verify == 1) {
     uint32_t bad = 0;
     PCS_CUDA(cudaMemcpyAsync(&bad, c->words + 1, 4, cudaMemcpyDeviceToHost, stream));
     PCS_CUDA(cudaStreamSynchronize(stream));
@@ -1357,6 +1401,20 @@ pcs_status pcs_delete(pcs_ctx* c, pcs_snapshot* h) {
   c->live.erase(h);
   release_block(c, h->block);
   delete h;
+  return PCS_OK;
+}
+
+pcs_status pcs_delete_many(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n) {
+  if (!c || n < 0 || (n > 0 && !snaps)) return fail(PCS_E_INVAL, "bad arguments");
+  std::lock_guard<std::mutex> lk(c->mu);
+  for (int i = 0; i < n; ++i)
+    if (!check_handle(c, snaps[i])) return fail(PCS_E_HANDLE, "snapshot %d: unknown handle", i);
+  for (int i = 0; i < n; ++i) {
+    pcs_snapshot* h = snaps[i];
+    if (!c->live.erase(h)) return fail(PCS_E_HANDLE, "snapshot %d: listed twice", i);
+    release_block(c, h->block);
+    delete h;
+  }
   return PCS_OK;
 }
 

@@ -133,6 +133,7 @@ SIGNATURES = {
     "pcs_restore": (_st, [_vp, ctypes.POINTER(_vp), _i32, ctypes.POINTER(pcs_session), _i32,
                           _vp]),
     "pcs_delete": (_st, [_vp, _vp]),
+    "pcs_delete_many": (_st, [_vp, ctypes.POINTER(_vp), _i32]),
     "pcs_snapshot_get_info": (_st, [_vp, _vp, ctypes.POINTER(pcs_snapshot_info)]),
     "pcs_snapshot_get_section": (_st, [_vp, _vp, _i32, ctypes.POINTER(pcs_section_info)]),
     "pcs_snapshot_copy_out": (_st, [_vp, _vp, _u64, _u64, _vp, _vp]),
@@ -416,17 +417,40 @@ class Context:
               "pcs_checkpoint")
         return [Snapshot(self, out[i]) for i in range(n)]
 
+    # -- batch forms: prebuilt struct arrays, raw handle arrays ------------------
+    @staticmethod
+    def session_array(sessions):
+        """A ctypes pcs_session array for repeated batch calls (keeps `sessions`)."""
+        arr = (pcs_session * max(len(sessions), 1))(*[s.struct() for s in sessions])
+        arr._keep = list(sessions)
+        return arr
+
+    def checkpoint_raw(self, arr, n: int, placement: int = PCS_PLACE_DEVICE, stream=None):
+        """checkpoint of a prebuilt session array; returns a ctypes handle array."""
+        out = (ctypes.c_void_p * max(n, 1))()
+        check(self.lib.pcs_checkpoint(self.h, arr, n, placement, out, _stream_ptr(stream)),
+              "pcs_checkpoint")
+        return out
+
+    def restore_raw(self, handles, n: int, arr, verify: int = 0, stream=None) -> None:
+        check(self.lib.pcs_restore(self.h, handles, n, arr, verify, _stream_ptr(stream)),
+              "pcs_restore")
+
+    def delete_raw(self, handles, n: int) -> None:
+        check(self.lib.pcs_delete_many(self.h, handles, n), "pcs_delete_many")
+
     def fork(self, snap: Snapshot, stream=None) -> Snapshot:
         out = ctypes.c_void_p()
         check(self.lib.pcs_fork(self.h, snap.handle, ctypes.byref(out), _stream_ptr(stream)),
               "pcs_fork")
         return Snapshot(self, out.value)
 
-    def restore(self, snaps, targets, verify: bool = False, stream=None) -> None:
+    def restore(self, snaps, targets, verify=False, stream=None) -> None:
+        """verify: False/0 none, True/1 check and wait, 2 check, report at sync."""
         n = len(snaps)
         hs = (ctypes.c_void_p * max(n, 1))(*[s.handle for s in snaps])
         arr = (pcs_session * max(n, 1))(*[t.struct() for t in targets])
-        check(self.lib.pcs_restore(self.h, hs, n, arr, 1 if verify else 0, _stream_ptr(stream)),
+        check(self.lib.pcs_restore(self.h, hs, n, arr, int(verify), _stream_ptr(stream)),
               "pcs_restore")
 
     def restore_status(self, snaps, targets, verify: bool = True, stream=None) -> int:

@@ -377,3 +377,42 @@ def test_prune_key_dims(ctx, dev, D, dtype):
     b = synth.banks(70 + D, 9, 1, 70, D, dtype, (8,), torch.uint8)
     keys, vals, qs = _bank_views(b, dev)
     _check_prune(ctx, b, keys, qs, ctx.params(pcs.PCS_K_FRACTION, fraction=0.3), dev)
+
+
+def test_async_verify_and_batch_forms(ctx, dev, tmp_path):
+    # verify = 2 checks on the device and reports at the next pcs_sync.
+    ms = [synth.markov(seed=300 + i, shape=(3, 20, 20)) for i in range(5)]
+    sess = [pcs.markov_session(i, m.obs.to(dev), m.rng.to(dev)) for i, m in enumerate(ms)]
+    arr = ctx.session_array(sess)
+    hs = ctx.checkpoint_raw(arr, 5)
+    outs = [pcs.markov_session(i, torch.zeros_like(m.obs, device=dev),
+                               torch.zeros_like(m.rng, device=dev)) for i, m in enumerate(ms)]
+    oarr = ctx.session_array(outs)
+    ctx.restore_raw(hs, 5, oarr, verify=2)
+    ctx.sync()
+    for m, o in zip(ms, outs):
+        assert torch.equal(o.keep[0].cpu(), m.obs) and torch.equal(o.keep[1].cpu(), m.rng)
+    # A corrupted record read from a file: no error at restore, one at sync.
+    snap = pcs.Snapshot(ctx, hs[2])
+    path = str(tmp_path / "c.pcs")
+    ctx.write_file(snap, path)
+    raw = np.fromfile(path, dtype=np.uint8)
+    raw[ctx.section(snap, 0).offset + 5] ^= 0x20
+    raw.tofile(path)
+    bad = ctx.read_file(path)
+    ctx.restore([bad], [outs[2]], verify=2)
+    with pytest.raises(pcs.PcsError) as e:
+        ctx.sync()
+    assert e.value.status == pcs.PCS_E_CORRUPT
+    ctx.sync()  # cleared
+    ctx.delete(bad)
+    # delete_many: all or nothing.
+    import ctypes
+    junk = (ctypes.c_void_p * 2)(hs[0], 12345)
+    with pytest.raises(pcs.PcsError) as e:
+        ctx.delete_raw(junk, 2)
+    assert e.value.status == pcs.PCS_E_HANDLE
+    assert ctx.stats().live_snapshots >= 5
+    ctx.delete_raw(hs, 5)
+    with pytest.raises(pcs.PcsError):
+        ctx.delete_raw(hs, 1)
