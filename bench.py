@@ -82,10 +82,14 @@ def step_bytes(a) -> int:
 
 
 def kernel_source_sha() -> str:
+    """sha256 prefix of the streaming kernels' source: pcs_kernels.cu up to the
+    finalisation kernels (helpers, the register kernel, the TMA kernel)."""
     import hashlib
     p = os.path.join(ROOT, "paper_2607_21686_gb300", "csrc", "pcs_kernels.cu")
     with open(p, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+        text = f.read()
+    cut = text.find(b"// Finalisation: stream fps")
+    return hashlib.sha256(text[:cut if cut > 0 else len(text)]).hexdigest()[:16]
 
 
 def ncu_traffic(kernel: str, sessions: int):

@@ -136,7 +136,7 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
                             cudaStream_t stream);
 
 cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
-                         float* scores, int sm_count, cudaStream_t stream);
+                         int key_types, float* scores, int sm_count, cudaStream_t stream);
 
 cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
                         int32_t* kept_idx, cudaStream_t stream);

@@ -329,11 +329,18 @@ __global__ void __launch_bounds__(kThreads, 2)
 // that gives up records kDevErrTimeout and the warp stops.
 // ---------------------------------------------------------------------------
 
-constexpr int kBulkWarps = 8;
-constexpr int kWarpStages = 3;
 constexpr int kTileChunks = kBulkTileChunks;
 constexpr uint32_t kTileBytes = kTileChunks * kChunkBytes;
-constexpr int kBulkThreads = 32 * kBulkWarps;
+
+// Shape of the TMA kernel per mode: warps per block and stages per warp.
+// Moving modes keep 3 tiles per warp in flight; the read-only hash mode,
+// bound by the hash chains' latency, trades a stage for more warps.
+template <int MODE>
+struct BulkShape {
+  static constexpr int kWarps = MODE == kModeHash ? 12 : 8;
+  static constexpr int kStages = MODE == kModeHash ? 2 : 3;
+  static constexpr int kThreads = 32 * kWarps;
+};
 constexpr int kTileRows = 32;  // rows >= 512 bytes touching an 8 KiB tile: at most 17
 constexpr long long kWaitCycles = 4000000000ll;  // give up a wait after ~2 s of SM clock
 static_assert(kTileBytes / kBulkMinRowBytes + 1 <= kTileRows, "tile rows");
@@ -407,10 +414,11 @@ struct WarpStage {
   uint8_t* rowp[kTileRows]; // layout-side address of each row (null = out of range)
 };
 
+template <int W, int S>
 struct BulkShared {
-  alignas(128) uint8_t buf[kBulkWarps][kWarpStages][kTileBytes];
-  alignas(8) uint64_t bar[kBulkWarps][kWarpStages];
-  WarpStage st[kBulkWarps][kWarpStages];
+  alignas(128) uint8_t buf[W][S][kTileBytes];
+  alignas(8) uint64_t bar[W][S];
+  WarpStage st[W][S];
 };
 
 // Layout-side address of row r of a ROWS / RING stream (null if out of range).
@@ -543,12 +551,14 @@ __device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, con
 }
 
 template <int MODE>
-__global__ void __launch_bounds__(kBulkThreads, 1)
+__global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     k_bulk(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
            uint32_t* err) {
   using T = ModeTraits<MODE>;
+  constexpr int kBulkWarps = BulkShape<MODE>::kWarps;
+  constexpr int kWarpStages = BulkShape<MODE>::kStages;
   extern __shared__ __align__(128) uint8_t smem_raw[];
-  BulkShared& sh = *reinterpret_cast<BulkShared*>(smem_raw);
+  auto& sh = *reinterpret_cast<BulkShared<kBulkWarps, kWarpStages>*>(smem_raw);
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   if (lane < kWarpStages) mbar_init(&sh.bar[warp][lane], 1);
@@ -841,14 +851,24 @@ __device__ __forceinline__ float lane_tree_sum(float v) {
 
 constexpr int kScoreIlp = 4;  // entries a warp scores at once
 
+// Element i (0..7) of a 16-byte segment as fp32 (exact conversion).
+template <int DT>  // 1 = bf16, 0 = fp16
+__device__ __forceinline__ float seg_elem(const uint4& v, int i) {
+  const uint32_t w = (i >> 1) == 0 ? v.x : (i >> 1) == 1 ? v.y : (i >> 1) == 2 ? v.z : v.w;
+  if (DT == 1) return __uint_as_float((i & 1) ? (w & 0xFFFF0000u) : (w << 16));
+  return __half2float(__ushort_as_half(static_cast<unsigned short>((i & 1) ? (w >> 16) : (w & 0xFFFFu))));
+}
+
 // Each warp scores a contiguous, balanced range of entries, kScoreIlp at a
 // time, following a cursor over the banks (one search per warp).  SPL = 16-byte
-// key segments per lane (D <= 256 * SPL); every key load of the kScoreIlp
-// entries is issued before any arithmetic.  SPL = 0: any D, loop per segment.
-template <int SPL>
+// key segments per lane (D <= 256 * SPL); DT = key type (1 bf16, 0 fp16).
+// The bank's query is held in registers as fp32, with |q| computed once per
+// bank in the same fixed order; every key load of the kScoreIlp entries is
+// issued before any arithmetic.
+template <int SPL, int DT>
 __global__ void __launch_bounds__(kThreads)
-    k_score(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
-            float* __restrict__ scores) {
+    k_score_fixed(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
+                  float* __restrict__ scores) {
   const int lane = threadIdx.x & 31;
   const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
   const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kWarps;
@@ -864,75 +884,116 @@ __global__ void __launch_bounds__(kThreads)
     }
     b = lo;
   }
-  // |q| of the current bank: the same fixed-order sum for every one of its keys.
-  int qbank = -1;
+  int qbank = -1, segs = 0;
   float qnorm = 0.f;
+  float qf[SPL][8];
+#pragma unroll
+  for (int j = 0; j < SPL; ++j)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) qf[j][i] = 0.f;
   for (uint64_t e0 = e_begin; e0 < e_end; e0 += kScoreIlp) {
-    float sd[kScoreIlp], sk[kScoreIlp];
-    int bank[kScoreIlp];
-    const uint8_t* krow[kScoreIlp];
+    // Entries of this round must share one bank to use the cached query;
+    // a round stops early at a bank boundary.
+    while (b + 1 < n_banks && __ldg(&banks[b + 1].entry_begin) <= e0) ++b;
+    const BankDesc& B = banks[b];
+    if (b != qbank) {  // warp-uniform: load the query, compute |q|
+      segs = B.D / 8;
+      const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
+      float sq = 0.f;
 #pragma unroll
-    for (int q = 0; q < kScoreIlp; ++q) {
-      sd[q] = sk[q] = 0.f;
-      bank[q] = -1;
-      krow[q] = nullptr;
-      const uint64_t e = e0 + q;
-      if (e >= e_end) continue;
-      while (b + 1 < n_banks && __ldg(&banks[b + 1].entry_begin) <= e) ++b;
-      bank[q] = b;
-      const BankDesc& B = banks[b];
-      krow[q] = reinterpret_cast<const uint8_t*>(B.keys) +
-                (e - B.entry_begin) * static_cast<uint64_t>(B.D) * 2;
-    }
-    if (SPL > 0) {
-      uint4 kv[kScoreIlp][SPL > 0 ? SPL : 1];
+      for (int j = 0; j < SPL; ++j) {
+        const int t = lane + 32 * j;
+        const uint4 qv = t < segs ? __ldg(qrow + t) : make_uint4(0, 0, 0, 0);
 #pragma unroll
-      for (int q = 0; q < kScoreIlp; ++q) {
-        const int segs = bank[q] >= 0 ? banks[bank[q]].D / 8 : 0;
-#pragma unroll
-        for (int j = 0; j < SPL; ++j) {
-          const int t = lane + 32 * j;
-          kv[q][j] = t < segs ? ld_stream(krow[q] + 16 * t) : make_uint4(0, 0, 0, 0);
+        for (int i = 0; i < 8; ++i) {
+          qf[j][i] = seg_elem<DT>(qv, i);
+          if (t < segs) sq = __fadd_rn(sq, __fmul_rn(qf[j][i], qf[j][i]));
         }
       }
-#pragma unroll
-      for (int q = 0; q < kScoreIlp; ++q) {
-        if (bank[q] < 0) continue;
-        const BankDesc& B = banks[bank[q]];
-        const int segs = B.D / 8;
-        const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
-#pragma unroll
-        for (int j = 0; j < SPL; ++j) {
-          const int t = lane + 32 * j;
-          if (t < segs) accum8_key(__ldg(qrow + t), kv[q][j], B.is_bf16 != 0, sd[q], sk[q]);
-        }
-      }
-    } else {
-#pragma unroll
-      for (int q = 0; q < kScoreIlp; ++q) {
-        if (bank[q] < 0) continue;
-        const BankDesc& B = banks[bank[q]];
-        const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
-        for (int t = lane; t < B.D / 8; t += 32)
-          accum8_key(__ldg(qrow + t), ld_stream(krow[q] + 16 * t), B.is_bf16 != 0, sd[q], sk[q]);
-      }
+      qnorm = __fsqrt_rn(lane_tree_sum(sq));
+      qbank = b;
     }
+    const uint64_t bank_end = b + 1 < n_banks ? __ldg(&banks[b + 1].entry_begin) : n_entries;
+    const uint64_t lim = min(static_cast<unsigned long long>(e_end), static_cast<unsigned long long>(bank_end));
+    const int cnt = static_cast<int>(min(static_cast<uint64_t>(kScoreIlp), lim - e0));
+    const uint8_t* kbase = reinterpret_cast<const uint8_t*>(B.keys) +
+                           (e0 - B.entry_begin) * static_cast<uint64_t>(B.D) * 2;
+    uint4 kv[kScoreIlp][SPL];
+#pragma unroll
+    for (int q = 0; q < kScoreIlp; ++q)
+#pragma unroll
+      for (int j = 0; j < SPL; ++j) {
+        const int t = lane + 32 * j;
+        kv[q][j] = (q < cnt && t < segs) ? ld_stream(kbase + static_cast<uint64_t>(q) * B.D * 2 + 16 * t)
+                                         : make_uint4(0, 0, 0, 0);
+      }
 #pragma unroll
     for (int q = 0; q < kScoreIlp; ++q) {
-      if (bank[q] >= 0 && bank[q] != qbank) {  // warp-uniform
-        const BankDesc& B = banks[bank[q]];
-        const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
-        float sq = 0.f;
-        for (int t = lane; t < B.D / 8; t += 32) accum8_query(__ldg(qrow + t), B.is_bf16 != 0, sq);
-        qnorm = __fsqrt_rn(lane_tree_sum(sq));
-        qbank = bank[q];
+      float sd = 0.f, sk = 0.f;
+#pragma unroll
+      for (int j = 0; j < SPL; ++j) {
+        if (lane + 32 * j < segs) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float ke = seg_elem<DT>(kv[q][j], i);
+            sd = __fadd_rn(sd, __fmul_rn(qf[j][i], ke));
+            sk = __fadd_rn(sk, __fmul_rn(ke, ke));
+          }
+        }
       }
-      const float d = lane_tree_sum(sd[q]);
-      const float kk = lane_tree_sum(sk[q]);
-      if (lane == 0 && bank[q] >= 0) {
+      const float d = lane_tree_sum(sd);
+      const float kk = lane_tree_sum(sk);
+      if (lane == 0 && q < cnt) {
         const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
         scores[e0 + q] = den == 0.f ? 0.f : __fdiv_rn(d, den);
       }
+    }
+    e0 = e0 + cnt - kScoreIlp;  // the loop adds kScoreIlp: next round starts at e0 + cnt
+  }
+}
+
+// Any key width or a mix of key types: the query is re-read per entry.
+__global__ void __launch_bounds__(kThreads)
+    k_score_any(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
+                float* __restrict__ scores) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+  const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kWarps;
+  const uint64_t e_begin = n_entries * gw / nw, e_end = n_entries * (gw + 1) / nw;
+  if (e_begin >= e_end) return;
+  int b = 0;
+  {
+    int lo = 0, hi = n_banks - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (__ldg(&banks[mid].entry_begin) <= e_begin) lo = mid;
+      else hi = mid - 1;
+    }
+    b = lo;
+  }
+  int qbank = -1;
+  float qnorm = 0.f;
+  for (uint64_t e = e_begin; e < e_end; ++e) {
+    while (b + 1 < n_banks && __ldg(&banks[b + 1].entry_begin) <= e) ++b;
+    const BankDesc& B = banks[b];
+    const bool bf16 = B.is_bf16 != 0;
+    const uint4* qrow = reinterpret_cast<const uint4*>(B.query);
+    if (b != qbank) {
+      float sq = 0.f;
+      for (int t = lane; t < B.D / 8; t += 32) accum8_query(__ldg(qrow + t), bf16, sq);
+      qnorm = __fsqrt_rn(lane_tree_sum(sq));
+      qbank = b;
+    }
+    const uint8_t* krow = reinterpret_cast<const uint8_t*>(B.keys) +
+                          (e - B.entry_begin) * static_cast<uint64_t>(B.D) * 2;
+    float sd = 0.f, sk = 0.f;
+    for (int t = lane; t < B.D / 8; t += 32)
+      accum8_key(__ldg(qrow + t), ld_stream(krow + 16 * t), bf16, sd, sk);
+    const float d = lane_tree_sum(sd);
+    const float kk = lane_tree_sum(sk);
+    if (lane == 0) {
+      const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
+      scores[e] = den == 0.f ? 0.f : __fdiv_rn(d, den);
     }
   }
 }
@@ -1077,7 +1138,8 @@ int occupancy() {
 template <int MODE>
 cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, uint32_t* err,
                              int sm_count, cudaStream_t stream) {
-  const size_t smem = sizeof(BulkShared);
+  using Shape = BulkShape<MODE>;
+  const size_t smem = sizeof(BulkShared<Shape::kWarps, Shape::kStages>);
   static uint64_t configured = 0;  // one bit per device (callers hold the context lock)
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -1089,9 +1151,9 @@ cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, 
     if (e != cudaSuccess) return e;
     configured |= bit;
   }
-  const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + kBulkWarps - 1) / kBulkWarps;
+  const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + Shape::kWarps - 1) / Shape::kWarps;
   const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
-  k_bulk<MODE><<<blocks, kBulkThreads, smem, stream>>>(secs, wl, nodes, err);
+  k_bulk<MODE><<<blocks, Shape::kThreads, smem, stream>>>(secs, wl, nodes, err);
   return cudaGetLastError();
 }
 
@@ -1099,7 +1161,7 @@ cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, 
 
 int stream_blocks_per_sm() { return occupancy<kModePack>(); }
 
-size_t bulk_shared_bytes() { return sizeof(BulkShared); }
+size_t bulk_shared_bytes() { return sizeof(BulkShared<BulkShape<kModePack>::kWarps, BulkShape<kModePack>::kStages>); }
 
 cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_log2,
                           uint64_t* nodes, uint32_t* dev_err, int sm_count, int blocks_per_sm,
@@ -1173,15 +1235,23 @@ cudaError_t launch_reduce_nodes(const SecDesc* secs, int n_secs, uint64_t* nodes
 }
 
 cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
-                         float* scores, int sm_count, cudaStream_t stream) {
+                         int key_types, float* scores, int sm_count, cudaStream_t stream) {
   if (n_entries == 0) return cudaSuccess;
   const uint64_t want = (n_entries + kWarps * kScoreIlp * 8 - 1) / (kWarps * kScoreIlp * 8);
   const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
   const int blocks = static_cast<int>(want < cap ? want : cap);
-  if (max_dim <= 256) k_score<1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-  else if (max_dim <= 512) k_score<2><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-  else if (max_dim <= 1024) k_score<4><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-  else k_score<0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  // key_types: 0 = all fp16, 1 = all bf16, 2 = mixed.
+  if (key_types == 2 || max_dim > 1024) {
+    k_score_any<<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  } else if (key_types == 1) {
+    if (max_dim <= 256) k_score_fixed<1, 1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+    else if (max_dim <= 512) k_score_fixed<2, 1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+    else k_score_fixed<4, 1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  } else {
+    if (max_dim <= 256) k_score_fixed<1, 0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+    else if (max_dim <= 512) k_score_fixed<2, 0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+    else k_score_fixed<4, 0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+  }
   return cudaGetLastError();
 }
 

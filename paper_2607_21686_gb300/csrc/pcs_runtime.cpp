@@ -1108,9 +1108,13 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
   auto* dbanks = reinterpret_cast<const BankDesc*>(ws + L.banks);
   {
     LaunchScope ls(c, kKScore, stream);
-    int max_dim = 0;
-    for (int s = 0; s < n; ++s) max_dim = std::max(max_dim, banks[s].key_dim);
-    PCS_CUDA(launch_score(dbanks, n, entries, max_dim, sc, c->sm_count, stream));
+    int max_dim = 0, n_bf16 = 0;
+    for (int s = 0; s < n; ++s) {
+      max_dim = std::max(max_dim, banks[s].key_dim);
+      n_bf16 += banks[s].key_dtype == PCS_DT_BF16;
+    }
+    const int key_types = n_bf16 == 0 ? 0 : (n_bf16 == n ? 1 : 2);
+    PCS_CUDA(launch_score(dbanks, n, entries, max_dim, key_types, sc, c->sm_count, stream));
   }
   {
     LaunchScope ls(c, kKTopk, stream);

@@ -416,3 +416,27 @@ def test_async_verify_and_batch_forms(ctx, dev, tmp_path):
     ctx.delete_raw(hs, 5)
     with pytest.raises(pcs.PcsError):
         ctx.delete_raw(hs, 1)
+
+
+def test_prune_mixed_key_types(ctx, dev):
+    # fp16 and bf16 banks in one call take the general score kernel.
+    b1 = synth.banks(80, 3, 5, 60, 128, torch.float16, (8,), torch.uint8)
+    b2 = synth.banks(81, 3, 5, 60, 128, torch.bfloat16, (8,), torch.uint8)
+    keys = [x.to(dev) for x in _bank_views(b1, "cpu")[0] + _bank_views(b2, "cpu")[0]]
+    qs = [x.to(dev) for x in _bank_views(b1, "cpu")[2] + _bank_views(b2, "cpu")[2]]
+    banks = ctx.banks_array(keys, qs, 272)
+    p = ctx.params(pcs.PCS_K_FIXED, k_max=7)
+    ks = ctx.prune_counts(banks, 6, p)
+    kept = torch.empty(sum(ks), dtype=torch.int32, device=dev)
+    scores = torch.empty(sum(k.shape[0] for k in keys), dtype=torch.float32, device=dev)
+    ctx.prune(banks, 6, p, kept, None, scores)
+    ctx.sync()
+    sc, kh = scores.cpu().numpy(), kept.cpu().numpy()
+    off = eo = 0
+    for k, q, kk in zip(keys, qs, ks):
+        s32 = oracle.scores(np_view(q), np_view(k))
+        n = k.shape[0]
+        assert np.array_equal(sc[eo:eo + n].view(np.uint32), s32.view(np.uint32))
+        assert kh[off:off + kk].tolist() == oracle.topk(s32, kk).tolist()
+        off += kk
+        eo += n
