@@ -38,12 +38,12 @@ METRIC = "snapshot+restore GB/s and sessions/s on 1 GB300; % of HBM (PCIe) roofl
 
 # DRAM bytes (read + write) per launch of the streaming kernels, from the ncu
 # capture summarised in profiles/k_bulk_kv8x24_full.md (8 sessions, scaled by
-# sessions / 8), valid only for the kernel source it was taken on.
+# sessions / 8), valid only for the streaming-kernel source it was taken on.
 NCU_TRAFFIC = {
-    "source_sha256_prefix": "d4fc58b0b1d3d65b",
+    "source_sha256_prefix": "a26b1f42260b6bcc",
     "sessions": 8,
-    "k_bulk<pack>": (805.718272 + 754.997504) * 1e6,
-    "k_bulk<restore_verify>": (805.773824 + 754.557184) * 1e6,
+    "k_bulk<pack>": (805.724160 + 754.243840) * 1e6,
+    "k_bulk<restore_verify>": (805.782016 + 754.359808) * 1e6,
 }
 
 
