@@ -297,6 +297,33 @@ pcs_status pcs_prune(pcs_ctx *ctx, const pcs_bank *banks, int32_t n,
                      int32_t *kept_off, void *stream);
 
 /*
+ * Keep-k by caller-supplied rank keys, for the recency-keyed policies the
+ * paper compares against relevance (Sec. 7.5, Table tab:evict: lru ranks a
+ * frame by its last use, fifo by its insertion order): per bank, keep the k_b
+ * entries with the largest (key, -index) -- ties to the lower index, NaN
+ * lowest -- and write their indices ascending.
+ *   keys:     device float[sum n] (CSR by bank, bank b = n[b] entries)
+ *   n, k:     host int32[n_banks]; k_b > n_b keeps the whole bank
+ *   kept_idx: device int32[sum min(k, n)]; kept_off: device int32[n+1] or NULL
+ */
+pcs_status pcs_topk(pcs_ctx *ctx, const float *keys, const int32_t *n, const int32_t *k,
+                    int32_t n_banks, int32_t *kept_idx, int32_t *kept_off, void *stream);
+
+/*
+ * Host only: the reactive shrink-then-drop plan of a host budget (Sec. 7.10:
+ * the runtime escalates shrink -> nothing left to shrink -> drop, and acts
+ * only when the budget binds).  Sessions are visited in ascending priority
+ * (ties: lower index first; priority NULL = session index).  While the kept
+ * bytes sum(k_s * entry_bytes_s) exceed `budget`, the next bank is shrunk to
+ * round-half-even(fraction * n_s); once every bank is shrunk, sessions are
+ * dropped (k_s = 0) in the same order.  k_out: host int32[count]; shrinks /
+ * drops: host int32 counts (may be NULL).
+ */
+pcs_status pcs_budget_plan(const int32_t *n, const uint64_t *entry_bytes, const double *priority,
+                           int32_t count, uint64_t budget, double fraction, int32_t *k_out,
+                           int32_t *shrinks, int32_t *drops);
+
+/*
  * Host only: bytes of the PCS1 record a session of these sections packs to:
  * 256-byte aligned header + 64-byte entries, then each payload at a
  * 256-byte aligned offset.

@@ -102,6 +102,7 @@ def lib():
             "pcso_record_header": (i32, [vp, vp, vp, vp, vp, vp]),
             "pcso_record_section": (None, [vp, i32, vp, vp, vp, vp]),
             "pcso_restore": (i32, [vp, vp, i32, i32]),
+            "pcso_budget_plan": (i32, [vp, vp, vp, i32, u64, ctypes.c_double, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -237,6 +238,19 @@ def k_fraction(n, frac: float) -> np.ndarray:
     out = np.zeros_like(a)
     lib().pcso_k_fraction(_ptr(a), a.size, frac, _ptr(out))
     return out
+
+
+def budget_plan(n, entry_bytes, budget: int, frac: float, priority=None):
+    """Reactive shrink-then-drop plan: (k per bank, shrinks, drops)."""
+    a = np.ascontiguousarray(n, dtype=np.int32)
+    e = np.ascontiguousarray(np.broadcast_to(np.asarray(entry_bytes, dtype=np.uint64), a.shape))
+    pr = None if priority is None else np.ascontiguousarray(priority, dtype=np.float64)
+    k = np.zeros_like(a)
+    sh, dr = ctypes.c_int32(), ctypes.c_int32()
+    rc = lib().pcso_budget_plan(_ptr(a), _ptr(e), None if pr is None else _ptr(pr), a.size,
+                                budget, frac, _ptr(k), ctypes.byref(sh), ctypes.byref(dr))
+    assert rc == 0
+    return k, sh.value, dr.value
 
 
 # --------------------------------------------------------------------------

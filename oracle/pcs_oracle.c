@@ -595,3 +595,74 @@ int32_t pcso_restore(const uint8_t *rec, pcso_section *t, int32_t n, int32_t ver
     }
     return 0;
 }
+
+/* ------------------------------------------------------------------------ */
+/* Reactive host-budget plan: shrink, then drop (Sec. 7.10 "Predictive      */
+/* eviction": the runtime escalates shrink -> nothing left to shrink ->     */
+/* drop, and acts only when the budget binds; Sec. 7.5 "At 16 MB no policy  */
+/* evicts at all").  Reading: sessions are visited in ascending priority    */
+/* (ties: lower index first); each shrink takes a bank to the retention     */
+/* fraction (round-half-even of frac * n); shrinking stops as soon as the   */
+/* kept bytes fit; if every bank is shrunk and they still do not fit,       */
+/* sessions are dropped (k = 0) in the same order until they do.            */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+    double priority;
+    int32_t index;
+} pcso_order;
+
+static int cmp_order(const void *a, const void *b)
+{
+    const pcso_order *x = (const pcso_order *)a, *y = (const pcso_order *)b;
+    if (x->priority < y->priority) return -1;
+    if (x->priority > y->priority) return 1;
+    return (x->index > y->index) - (x->index < y->index);
+}
+
+int32_t pcso_budget_plan(const int32_t *n, const uint64_t *entry_bytes, const double *priority,
+                         int32_t count, uint64_t budget, double frac, int32_t *k,
+                         int32_t *shrinks, int32_t *drops)
+{
+    pcso_order *ord;
+    unsigned __int128 kept = 0;
+    int32_t s, i;
+    *shrinks = 0;
+    *drops = 0;
+    for (s = 0; s < count; s++) {
+        k[s] = n[s];
+        kept += (unsigned __int128)(uint64_t)n[s] * entry_bytes[s];
+    }
+    if (kept <= budget) return 0;
+    ord = (pcso_order *)malloc((size_t)(count > 0 ? count : 1) * sizeof(pcso_order));
+    if (!ord) return -1;
+    for (s = 0; s < count; s++) {
+        ord[s].priority = priority ? priority[s] : (double)s;
+        ord[s].index = s;
+    }
+    qsort(ord, (size_t)count, sizeof(pcso_order), cmp_order);
+    for (i = 0; i < count && kept > budget; i++) {
+        int32_t target;
+        double v;
+        s = ord[i].index;
+        v = nearbyint(frac * (double)n[s]);
+        if (v < 0) v = 0;
+        if (v > n[s]) v = n[s];
+        target = (int32_t)v;
+        if (target < k[s]) {
+            kept -= (unsigned __int128)(uint64_t)(k[s] - target) * entry_bytes[s];
+            k[s] = target;
+            (*shrinks)++;
+        }
+    }
+    for (i = 0; i < count && kept > budget; i++) {
+        s = ord[i].index;
+        if (k[s] > 0) {
+            kept -= (unsigned __int128)(uint64_t)k[s] * entry_bytes[s];
+            k[s] = 0;
+            (*drops)++;
+        }
+    }
+    free(ord);
+    return 0;
+}

@@ -1123,6 +1123,97 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
   return ws_release(c, stream);
 }
 
+pcs_status pcs_topk(pcs_ctx* c, const float* keys, const int32_t* n, const int32_t* k,
+                    int32_t n_banks, int32_t* kept_idx, int32_t* kept_off, void* stream_) {
+  if (!c || n_banks < 0 || (n_banks > 0 && (!n || !k))) return fail(PCS_E_INVAL, "bad arguments");
+  if (n_banks == 0) return PCS_OK;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::vector<BankDesc> d(n_banks);
+  std::vector<int32_t> koff(n_banks + 1, 0);
+  uint64_t entries = 0, kept = 0;
+  for (int b = 0; b < n_banks; ++b) {
+    if (n[b] < 0 || k[b] < 0) return fail(PCS_E_INVAL, "bank %d: negative n or k", b);
+    d[b].entry_begin = entries;
+    d[b].kept_begin = kept;
+    d[b].n = n[b];
+    d[b].k = std::min(k[b], n[b]);
+    entries += n[b];
+    kept += d[b].k;
+    koff[b + 1] = static_cast<int32_t>(kept);
+  }
+  if (entries > 0 && !keys) return fail(PCS_E_INVAL, "keys is null");
+  if (kept > 0 && !kept_idx) return fail(PCS_E_INVAL, "kept_idx is null");
+  if (entries > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many entries in one call");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  const uint64_t off_at = round_up(sizeof(BankDesc) * n_banks, kRecordAlign);
+  const uint64_t total = off_at + 4ull * (n_banks + 1);
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, total, stream, &ws);
+  if (st) return st;
+  c->plan.resize(total);
+  put(c->plan, 0, d);
+  put(c->plan, off_at, koff);
+  PCS_CUDA(plan_copy(c, ws, total, stream));
+  if (kept_off)
+    PCS_CUDA(cudaMemcpyAsync(kept_off, ws + off_at, 4ull * (n_banks + 1), cudaMemcpyDeviceToDevice,
+                             stream));
+  {
+    LaunchScope ls(c, kKTopk, stream);
+    PCS_CUDA(launch_topk(reinterpret_cast<const BankDesc*>(ws), n_banks, keys, kept_idx, stream));
+  }
+  return ws_release(c, stream);
+}
+
+pcs_status pcs_budget_plan(const int32_t* n, const uint64_t* entry_bytes, const double* priority,
+                           int32_t count, uint64_t budget, double fraction, int32_t* k_out,
+                           int32_t* shrinks, int32_t* drops) {
+  if (count < 0 || (count > 0 && (!n || !entry_bytes || !k_out)))
+    return fail(PCS_E_INVAL, "bad arguments");
+  if (!(fraction >= 0.0 && fraction <= 1.0)) return fail(PCS_E_INVAL, "fraction must lie in [0, 1]");
+  int32_t n_shrink = 0, n_drop = 0;
+  unsigned __int128 kept = 0;
+  for (int s = 0; s < count; ++s) {
+    if (n[s] < 0) return fail(PCS_E_INVAL, "session %d: negative n", s);
+    k_out[s] = n[s];
+    kept += static_cast<unsigned __int128>(static_cast<uint64_t>(n[s])) * entry_bytes[s];
+  }
+  if (kept > budget) {
+    std::vector<int32_t> order(count);
+    for (int s = 0; s < count; ++s) order[s] = s;
+    std::stable_sort(order.begin(), order.end(), [&](int32_t a, int32_t b) {
+      const double pa = priority ? priority[a] : a, pb = priority ? priority[b] : b;
+      return pa < pb;
+    });
+    auto bytes_of = [&](int32_t s, int32_t rows) {
+      return static_cast<unsigned __int128>(static_cast<uint64_t>(rows)) * entry_bytes[s];
+    };
+    for (int i = 0; i < count && kept > budget; ++i) {  // shrink
+      const int32_t s = order[i];
+      double v = __builtin_nearbyint(fraction * static_cast<double>(n[s]));
+      v = std::min<double>(std::max(v, 0.0), n[s]);
+      const int32_t target = static_cast<int32_t>(v);
+      if (target < k_out[s]) {
+        kept -= bytes_of(s, k_out[s] - target);
+        k_out[s] = target;
+        ++n_shrink;
+      }
+    }
+    for (int i = 0; i < count && kept > budget; ++i) {  // nothing left to shrink: drop
+      const int32_t s = order[i];
+      if (k_out[s] > 0) {
+        kept -= bytes_of(s, k_out[s]);
+        k_out[s] = 0;
+        ++n_drop;
+      }
+    }
+  }
+  if (shrinks) *shrinks = n_shrink;
+  if (drops) *drops = n_drop;
+  return PCS_OK;
+}
+
 pcs_status pcs_record_bytes(const pcs_section* sections, int32_t n, uint64_t* out) {
   if (!out || n < 1 || n > 65535 || !sections) return fail(PCS_E_INVAL, "bad section list");
   uint64_t off = round_up(kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * n, kRecordAlign);

@@ -127,6 +127,10 @@ SIGNATURES = {
     "pcs_prune": (_st, [_vp, ctypes.POINTER(pcs_bank), _i32, ctypes.POINTER(pcs_prune_params),
                         _vp, _vp, _vp, _vp]),
     "pcs_record_bytes": (_st, [ctypes.POINTER(pcs_section), _i32, ctypes.POINTER(_u64)]),
+    "pcs_topk": (_st, [_vp, _vp, ctypes.POINTER(_i32), ctypes.POINTER(_i32), _i32, _vp, _vp, _vp]),
+    "pcs_budget_plan": (_st, [ctypes.POINTER(_i32), ctypes.POINTER(_u64), ctypes.POINTER(ctypes.c_double),
+                              _i32, _u64, ctypes.c_double, ctypes.POINTER(_i32),
+                              ctypes.POINTER(_i32), ctypes.POINTER(_i32)]),
     "pcs_checkpoint": (_st, [_vp, ctypes.POINTER(pcs_session), _i32, _u32, ctypes.POINTER(_vp),
                              _vp]),
     "pcs_fork": (_st, [_vp, _vp, ctypes.POINTER(_vp), _vp]),
@@ -165,6 +169,21 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
             fn.argtypes = args
         _lib = lib
         return lib
+
+
+def budget_plan(n, entry_bytes, budget: int, fraction: float, priority=None):
+    """Host shrink-then-drop plan: (k per session, shrinks, drops)."""
+    lib = load_library()
+    c = len(n)
+    na = (ctypes.c_int32 * max(c, 1))(*n)
+    eb = entry_bytes if not isinstance(entry_bytes, int) else [entry_bytes] * c
+    ea = (ctypes.c_uint64 * max(c, 1))(*eb)
+    pa = None if priority is None else (ctypes.c_double * max(c, 1))(*priority)
+    ko = (ctypes.c_int32 * max(c, 1))()
+    sh, dr = ctypes.c_int32(), ctypes.c_int32()
+    check(lib.pcs_budget_plan(na, ea, pa, c, budget, fraction, ko, ctypes.byref(sh),
+                              ctypes.byref(dr)), "pcs_budget_plan")
+    return list(ko)[:c], sh.value, dr.value
 
 
 class PcsError(RuntimeError):
@@ -401,6 +420,14 @@ class Context:
         check(self.lib.pcs_prune(self.h, banks, n, ctypes.byref(params), _ptr(scores),
                                  _ptr(kept_idx), _ptr(kept_off), _stream_ptr(stream)),
               "pcs_prune")
+
+    def topk(self, keys: torch.Tensor, n, k, kept_idx: torch.Tensor, kept_off=None, stream=None):
+        """Keep-k per bank by caller rank keys (CSR float32 `keys`)."""
+        nb = len(n)
+        na = (ctypes.c_int32 * max(nb, 1))(*n)
+        ka = (ctypes.c_int32 * max(nb, 1))(*k)
+        check(self.lib.pcs_topk(self.h, _ptr(keys), na, ka, nb, _ptr(kept_idx), _ptr(kept_off),
+                                _stream_ptr(stream)), "pcs_topk")
 
     # -- snapshots -------------------------------------------------------------
     def record_bytes(self, session: Session) -> int:

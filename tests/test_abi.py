@@ -157,3 +157,18 @@ def test_record_bytes_match_oracle(lib):
         out = ctypes.c_uint64()
         assert lib.pcs_record_bytes(arr, ns, ctypes.byref(out)) == 0
         assert out.value == oracle.record_bytes(sp)
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_budget_plan_matches_oracle(lib, seed):
+    rnd = np.random.default_rng(100 + seed)
+    S = int(rnd.integers(1, 300))
+    n = rnd.integers(0, 500, S).tolist()
+    E = rnd.integers(1, 4096, S).tolist()
+    pr = rnd.normal(size=S).tolist() if seed % 2 else None
+    total = sum(a * b for a, b in zip(n, E))
+    for B in [total + 1, total, total * 3 // 4, total // 4, total // 50, 0]:
+        for frac in [0.0, 0.12, 0.5]:
+            got = pcs.budget_plan(n, E, B, frac, priority=pr)
+            k, sh, dr = oracle.budget_plan(n, E, B, frac, priority=pr)
+            assert got == (k.tolist(), sh, dr), (B, frac)

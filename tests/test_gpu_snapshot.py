@@ -440,3 +440,26 @@ def test_prune_mixed_key_types(ctx, dev):
         assert kh[off:off + kk].tolist() == oracle.topk(s32, kk).tolist()
         off += kk
         eo += n
+
+
+@pytest.mark.parametrize("policy", ["lru", "fifo"])
+def test_topk_by_recency_keys(ctx, dev, policy):
+    # Recency-keyed retention (Table tab:evict lru / fifo): rank keys supplied
+    # by the caller; ties by entry index.
+    rnd = np.random.default_rng(7)
+    n = rnd.integers(1, 300, 20).tolist()
+    k = [max(1, int(x * 0.12 + 0.5)) for x in n]
+    if policy == "lru":
+        keys = [rnd.integers(0, 50, x).astype(np.float32) for x in n]  # last-use step (ties)
+    else:
+        keys = [np.arange(x, dtype=np.float32) for x in n]             # insertion order
+    flat = torch.from_numpy(np.concatenate(keys)).to(dev)
+    kept = torch.empty(sum(min(a, b) for a, b in zip(n, k)), dtype=torch.int32, device=dev)
+    koff = torch.empty(len(n) + 1, dtype=torch.int32, device=dev)
+    ctx.topk(flat, n, k, kept, koff)
+    ctx.sync()
+    kh, oh = kept.cpu().numpy(), koff.cpu().numpy()
+    for b, (kk, x) in enumerate(zip(keys, k)):
+        assert kh[oh[b]:oh[b + 1]].tolist() == oracle.topk(kk, x).tolist(), b
+    if policy == "fifo":
+        assert kh[oh[0]:oh[1]].tolist() == list(range(n[0] - k[0], n[0]))

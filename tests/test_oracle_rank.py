@@ -150,3 +150,54 @@ def test_budget_rule_mixed_entry_sizes():
     T = sum(a * b for a, b in zip(n, E))
     assert k == [a * B // T for a in n]
     assert sum(a * b for a, b in zip(k, E)) <= B
+
+
+def _golden_kv(name):
+    g = {}
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                k, v = line.split()
+                g[k] = float(v)
+    return g
+
+
+def test_budget_plan_paper_boundary():
+    # Sec. 7.5: at 16 MB nothing is evicted; the footprint is 15.4 MB.
+    g = _golden_kv("evict_boundary.txt")
+    S, n, E = int(g["sessions"]), int(g["frames_per_session"]), int(g["frame_bytes"])
+    assert round(S * n * E / 1e6, 1) == g["unconstrained_mb"]
+    k, sh, dr = oracle.budget_plan([n] * S, E, int(g["budget_no_evict_mb"] * 1e6), g["keep_fraction"])
+    assert (sh, dr) == (0, 0) and k.tolist() == [n] * S
+    # Just below the footprint the plan must act, and only as much as needed.
+    k, sh, dr = oracle.budget_plan([n] * S, E, S * n * E - 1, g["keep_fraction"])
+    assert (sh, dr) == (1, 0) and k.tolist()[0] == 3 and k.tolist()[1:] == [n] * (S - 1)
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_budget_plan_properties(seed):
+    rnd = np.random.default_rng(seed)
+    S = int(rnd.integers(1, 40))
+    n = rnd.integers(0, 60, S)
+    E = rnd.integers(1, 5000, S).astype(np.uint64)
+    pr = rnd.permutation(S).astype(np.float64)
+    frac = float(rnd.choice([0.0, 0.12, 0.25, 0.5]))
+    total = int((n.astype(np.uint64) * E).sum())
+    prev = -1
+    # Budgets from loose to tight: the plan may only ever do more.
+    for B in sorted(set([0, total // 10, total // 3, total // 2, total - 1, total, total + 5]),
+                    reverse=True):
+        k, sh, dr = oracle.budget_plan(n, E, B, frac, priority=pr)
+        kept = int((k.astype(np.uint64) * E).sum())
+        target = np.array([min(max(int(np.round(frac * x)), 0), x) for x in n])  # half-even ok: frac*n rarely .5
+        assert kept <= B or B >= total
+        if B >= total:
+            assert (sh, dr) == (0, 0)
+        # Drops happen only once every bank that can shrink has been shrunk.
+        if dr:
+            assert sh == int((target < n).sum())
+        # Each bank is whole, at its retention target, or dropped.
+        assert all(kk in (nn, tt, 0) for kk, nn, tt in zip(k, n, target))
+        # Reactive: acting is monotone in the pressure (tighter budget, more actions).
+        assert sh + dr >= prev
+        prev = sh + dr
