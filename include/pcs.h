@@ -346,6 +346,9 @@ pcs_status pcs_checkpoint(pcs_ctx *ctx, const pcs_session *sessions, int32_t n,
  */
 pcs_status pcs_fork(pcs_ctx *ctx, const pcs_snapshot *parent, pcs_snapshot **child,
                     void *stream);
+/* fork(c) for n snapshots in one call; children: host array of n handles. */
+pcs_status pcs_fork_many(pcs_ctx *ctx, pcs_snapshot *const *parents, int32_t n,
+                         pcs_snapshot **children, void *stream);
 
 /*
  * restore(c) for n snapshots (I1): scatter each section payload to the

@@ -141,8 +141,6 @@ cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
 cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
                         int32_t* kept_idx, cudaStream_t stream);
 
-cudaError_t launch_copy(const void* src, void* dst, uint64_t bytes, int sm_count,
-                        cudaStream_t stream);
 
 // Occupancy of the streaming kernel (blocks per SM) for the launch shape.
 int stream_blocks_per_sm();

@@ -14,7 +14,6 @@
 // k_score         cos(query, key) per bank entry, fp32, fixed order (Sec. 5).
 // k_topk          per-bank radix select of the k largest (score, -index),
 //                 kept indices written in ascending order (Sec. 7.5).
-// k_copy          fork: independent copy of a record (I3).
 //
 // No kernel waits on another block: every pass is a plain data-parallel
 // sweep, so nothing here can spin.  Index values read from device memory are
@@ -1109,25 +1108,6 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-// ---------------------------------------------------------------------------
-// Fork copy
-// ---------------------------------------------------------------------------
-
-__global__ void __launch_bounds__(kThreads)
-    k_copy(const uint4* __restrict__ src, uint4* __restrict__ dst, uint64_t n16) {
-  const uint64_t stride = static_cast<uint64_t>(gridDim.x) * kThreads;
-  uint64_t i = static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x;
-  for (; i + 3 * stride < n16; i += 4 * stride) {
-    const uint4 a = __ldcs(src + i), b = __ldcs(src + i + stride);
-    const uint4 c = __ldcs(src + i + 2 * stride), d = __ldcs(src + i + 3 * stride);
-    __stcs(dst + i, a);
-    __stcs(dst + i + stride, b);
-    __stcs(dst + i + 2 * stride, c);
-    __stcs(dst + i + 3 * stride, d);
-  }
-  for (; i < n16; i += stride) __stcs(dst + i, __ldcs(src + i));
-}
-
 template <int MODE>
 int occupancy() {
   int b = 0;
@@ -1263,16 +1243,6 @@ cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
   return cudaGetLastError();
 }
 
-cudaError_t launch_copy(const void* src, void* dst, uint64_t bytes, int sm_count,
-                        cudaStream_t stream) {
-  const uint64_t n16 = bytes / 16;
-  if (n16 == 0) return cudaSuccess;
-  const uint64_t want = (n16 + kThreads - 1) / kThreads;
-  const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
-  const int blocks = static_cast<int>(want < cap ? want : cap);
-  k_copy<<<blocks, kThreads, 0, stream>>>(static_cast<const uint4*>(src), static_cast<uint4*>(dst), n16);
-  return cudaGetLastError();
-}
 
 // ---------------------------------------------------------------------------
 // Fingerprints with no allocation

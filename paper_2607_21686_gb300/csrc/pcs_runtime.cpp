@@ -361,13 +361,13 @@ pcs_status set_device(pcs_ctx* c) {
 // Kernels the context launches, for counting and timing.
 enum KernelKind {
   kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
-  kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKCopy, kKBulkHash, kKBulkPack,
+  kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKBulkHash, kKBulkPack,
   kKBulkRestore, kKBulkRestoreV, kKReduce, kKernelKinds
 };
 const char* kKernelNames[kKernelKinds] = {
     "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
-    "k_copy", "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
+    "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
     "k_reduce_nodes"};
 
 cudaEvent_t timing_event(pcs_ctx* c) {
@@ -1352,40 +1352,96 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   return PCS_OK;
 }
 
-pcs_status pcs_fork(pcs_ctx* c, const pcs_snapshot* parent, pcs_snapshot** child, void* stream_) {
-  if (!c || !child) return fail(PCS_E_INVAL, "null argument");
+pcs_status pcs_fork_many(pcs_ctx* c, pcs_snapshot* const* parents, int32_t n,
+                         pcs_snapshot** children, void* stream_) {
+  if (!c || n < 0 || (n > 0 && (!parents || !children))) return fail(PCS_E_INVAL, "bad arguments");
+  if (n == 0) return PCS_OK;
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   std::lock_guard<std::mutex> lk(c->mu);
-  pcs_snapshot* p = check_handle(c, parent);
-  if (!p) return fail(PCS_E_HANDLE, "unknown snapshot handle");
+  for (int i = 0; i < n; ++i)
+    if (!check_handle(c, parents[i])) return fail(PCS_E_HANDLE, "snapshot %d: unknown handle", i);
   pcs_status st = set_device(c);
   if (st) return st;
-  Block* blk = nullptr;
-  st = arena_of(c, p->block->placement)->alloc(p->total_bytes, stream, &blk);
-  if (st) return st;
-  st = wait_written(p->block, stream);
-  if (st) {
-    arena_of(c, blk->placement)->free(blk);
-    return st;
+  // One new block per placement holds the children of that placement.
+  uint64_t need[2] = {0, 0};
+  std::vector<uint64_t> off(n);
+  for (int i = 0; i < n; ++i) {
+    const uint32_t pl = parents[i]->block->placement;
+    off[i] = need[pl];
+    need[pl] += parents[i]->total_bytes;
   }
-  cudaError_t e;
-  {
-    LaunchScope ls(c, kKCopy, stream);
-    e = launch_copy(p->record(), blk->ptr, p->total_bytes, c->sm_count, stream);
+  Block* blk[2] = {nullptr, nullptr};
+  auto undo = [&](pcs_status s) {
+    for (int pl = 0; pl < 2; ++pl)
+      if (blk[pl]) arena_of(c, pl)->free(blk[pl]);
+    return s;
+  };
+  for (uint32_t pl = 0; pl < 2; ++pl) {
+    if (!need[pl]) continue;
+    st = arena_of(c, pl)->alloc(need[pl], stream, &blk[pl]);
+    if (st) return undo(st);
   }
-  if (e != cudaSuccess) {
-    arena_of(c, blk->placement)->free(blk);
-    return cuda_fail(e, "fork copy");
+  for (int i = 0; i < n; ++i) {
+    st = wait_written(parents[i]->block, stream);
+    if (st) return undo(st);
   }
-  note_use(c, p->block, stream);
-  blk->written = record_event(c->events, stream);
-  blk->refs = 1;
-  auto h = std::make_unique<pcs_snapshot>(*p);
-  h->block = blk;
-  h->offset = 0;
-  *child = h.release();
-  c->live.insert(*child);
+  // A fork is a restore of the whole record into a contiguous target: the
+  // streaming kernels copy it (no hashing), TMA-staged when both are in HBM.
+  std::vector<SecDesc> d(n);
+  std::vector<char> bulk(n);
+  PtrCache cache;
+  uint64_t bytes = 0;
+  for (int i = 0; i < n; ++i) {
+    pcs_section x{};
+    x.layout = PCS_LAYOUT_CONTIG;
+    x.base = blk[parents[i]->block->placement]->ptr + off[i];
+    x.bytes = parents[i]->total_bytes;
+    d[i] = make_desc(x, parents[i]->record(), 0);
+    bytes += x.bytes;
+  }
+  const bool small = bytes <= kSmallCallBytes;
+  for (int i = 0; i < n; ++i)
+    bulk[i] = c->use_bulk && !small && parents[i]->block->placement == PCS_PLACE_DEVICE;
+  StreamPlan P;
+  if (!plan_streams(c, d, bulk, P)) return undo(fail(PCS_E_INVAL, "too much data in one call"));
+  const ListLayout LL = list_layout(P, sizeof(SecDesc) * n);
+  const uint64_t total = round_up(LL.end, kRecordAlign);
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, total, stream, &ws);
+  if (st) return undo(st);
+  c->plan.resize(total);
+  put(c->plan, 0, d);
+  put_lists(c->plan, P, LL);
+  cudaError_t e = plan_copy(c, ws, total, stream);
+  if (e == cudaSuccess)
+    e = launch_streams(c, kModeRestore, reinterpret_cast<const SecDesc*>(ws), P, LL, ws, nullptr,
+                       stream);
+  if (e != cudaSuccess) return undo(cuda_fail(e, "fork copy"));
+  Ev done = record_event(c->events, stream);
+  st = ws_release(c, stream, done);
+  if (st) return undo(st);
+  for (int i = 0; i < n; ++i) note_use(c, parents[i]->block, stream);
+  for (int pl = 0; pl < 2; ++pl) {
+    if (!blk[pl]) continue;
+    blk[pl]->written = done;
+    blk[pl]->refs = 0;
+  }
+  for (int i = 0; i < n; ++i) {
+    Block* b = blk[parents[i]->block->placement];
+    auto h = std::make_unique<pcs_snapshot>(*parents[i]);
+    h->block = b;
+    h->offset = off[i];
+    b->refs += 1;
+    children[i] = h.release();
+    c->live.insert(children[i]);
+  }
   return PCS_OK;
+}
+
+pcs_status pcs_fork(pcs_ctx* c, const pcs_snapshot* parent, pcs_snapshot** child, void* stream) {
+  if (!c || !child) return fail(PCS_E_INVAL, "null argument");
+  pcs_snapshot* p = const_cast<pcs_snapshot*>(parent);
+  return pcs_fork_many(c, &p, 1, child, stream);
 }
 
 pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const pcs_session* targets,

@@ -134,6 +134,7 @@ SIGNATURES = {
     "pcs_checkpoint": (_st, [_vp, ctypes.POINTER(pcs_session), _i32, _u32, ctypes.POINTER(_vp),
                              _vp]),
     "pcs_fork": (_st, [_vp, _vp, ctypes.POINTER(_vp), _vp]),
+    "pcs_fork_many": (_st, [_vp, ctypes.POINTER(_vp), _i32, ctypes.POINTER(_vp), _vp]),
     "pcs_restore": (_st, [_vp, ctypes.POINTER(_vp), _i32, ctypes.POINTER(pcs_session), _i32,
                           _vp]),
     "pcs_delete": (_st, [_vp, _vp]),
@@ -457,6 +458,12 @@ class Context:
         out = (ctypes.c_void_p * max(n, 1))()
         check(self.lib.pcs_checkpoint(self.h, arr, n, placement, out, _stream_ptr(stream)),
               "pcs_checkpoint")
+        return out
+
+    def fork_raw(self, handles, n: int, stream=None):
+        """fork of n snapshots in one call; returns a ctypes handle array."""
+        out = (ctypes.c_void_p * max(n, 1))()
+        check(self.lib.pcs_fork_many(self.h, handles, n, out, _stream_ptr(stream)), "pcs_fork_many")
         return out
 
     def restore_raw(self, handles, n: int, arr, verify: int = 0, stream=None) -> None:

@@ -463,3 +463,23 @@ def test_topk_by_recency_keys(ctx, dev, policy):
         assert kh[oh[b]:oh[b + 1]].tolist() == oracle.topk(kk, x).tolist(), b
     if policy == "fifo":
         assert kh[oh[0]:oh[1]].tolist() == list(range(n[0] - k[0], n[0]))
+
+
+def test_fork_many_mixed_placements(ctx, dev):
+    # Device records over 1 MiB take the TMA copy; pinned-host ones the register copy.
+    kv = synth.kv(seed=90, sessions=3, layers=2, heads=16, head_dim=64, window=256, page_rows=16)
+    kp, vp, pt, meta = kv.k_pool.to(dev), kv.v_pool.to(dev), kv.page_table.to(dev), kv.meta.to(dev)
+    sess = [pcs.kv_session(s, meta[s], kp, vp, pt[s], kv.ring_start[s], kv.window) for s in range(3)]
+    dev_snaps = ctx.checkpoint(sess)
+    host_snaps = ctx.checkpoint(sess, placement=pcs.PCS_PLACE_PINNED_HOST)
+    import ctypes
+    parents = dev_snaps + host_snaps
+    hs = (ctypes.c_void_p * 6)(*[x.handle for x in parents])
+    kids = ctx.fork_raw(hs, 6)
+    for i, p in enumerate(parents):
+        child = pcs.Snapshot(ctx, kids[i])
+        assert ctx.info(child).placement == ctx.info(p).placement
+        assert np.array_equal(ctx.record(child).numpy(), ctx.record(p).numpy()), i
+    ctx.delete_raw(kids, 6)
+    for x in parents:
+        ctx.delete(x)
