@@ -119,6 +119,16 @@ cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* no
                         uint32_t* dev_err, int sm_count, cudaStream_t stream);
 size_t bulk_shared_bytes();
 
+// One launch for a small call: the register streaming pass over wl (no
+// node reduction), then the finaliser of `mode` run by the last block to
+// finish (hash: n_items buffers; pack / restore_verify: n_items sessions).
+// `ticket` must be zero; the last block resets it.
+cudaError_t launch_small(int mode, const SecDesc* secs, WorkList wl, int group_log2,
+                         uint64_t* nodes, uint32_t* dev_err, uint32_t* ticket, int n_items,
+                         const SessDesc* sess, const Entry* entries, uint64_t* fp_out,
+                         const uint64_t* fp_before, uint8_t* flags, uint32_t* bad, int sm_count,
+                         int blocks_per_sm, cudaStream_t stream);
+
 // Streams with many task nodes: reduce each aligned group of 32 nodes of
 // stream i (nodes[task_begin_i ...]) to one node at nodes[fin_begin_i + g].
 // Groups of all streams are numbered by fin_begin - base (monotone).

@@ -247,12 +247,12 @@ __device__ __forceinline__ int find_item(const uint32_t* __restrict__ begin, int
   return lo;
 }
 
+// The warp tasks of one streaming pass (body of k_stream and k_small).
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, 2)
-    k_stream(const SecDesc* __restrict__ secs, WorkList wl, int glog2,
-             uint64_t* __restrict__ nodes, uint32_t* err) {
+__device__ __forceinline__ void run_stream_tasks(const SecDesc* __restrict__ secs, const WorkList& wl,
+                                                 int glog2, uint64_t* __restrict__ nodes,
+                                                 uint32_t* err, SecDesc* sdesc) {
   using T = ModeTraits<MODE>;
-  __shared__ SecDesc sdesc[kWarps];
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
   const uint32_t nw = gridDim.x * kWarps;
@@ -311,6 +311,14 @@ __global__ void __launch_bounds__(kThreads, 2)
       if (lane == 0) nodes[s.task_begin + local] = root;
     }
   }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 2)
+    k_stream(const SecDesc* __restrict__ secs, WorkList wl, int glog2,
+             uint64_t* __restrict__ nodes, uint32_t* err) {
+  __shared__ SecDesc sdesc[kWarps];
+  run_stream_tasks<MODE>(secs, wl, glog2, nodes, err, sdesc);
 }
 
 // ---------------------------------------------------------------------------
@@ -712,13 +720,14 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-// Fingerprints of independent buffers (pcs_fingerprint / pcs_classify).
-__global__ void __launch_bounds__(kThreads)
-    k_finalize_hash(const SecDesc* __restrict__ secs, int n_secs, uint64_t* nodes,
-                    uint64_t* fp_out, const uint64_t* fp_before, uint8_t* flags) {
+// Fingerprints of independent buffers (pcs_fingerprint / pcs_classify):
+// warps w0, w0 + nw, ... take buffer after buffer.
+__device__ __forceinline__ void finalize_hash_warps(const SecDesc* __restrict__ secs, int n_secs,
+                                                    uint64_t* nodes, uint64_t* fp_out,
+                                                    const uint64_t* fp_before, uint8_t* flags,
+                                                    int w0, int nw) {
   const int lane = threadIdx.x & 31;
-  const int nw = gridDim.x * kWarps;
-  for (int i = blockIdx.x * kWarps + (threadIdx.x >> 5); i < n_secs; i += nw) {
+  for (int i = w0; i < n_secs; i += nw) {
     const SecDesc s = secs[i];
     const uint64_t fp = stream_fp(s, nodes, lane);
     if (lane == 0) {
@@ -726,6 +735,13 @@ __global__ void __launch_bounds__(kThreads)
       if (fp_before) flags[i] = fp != fp_before[i] ? 1 : 0;
     }
   }
+}
+
+__global__ void __launch_bounds__(kThreads)
+    k_finalize_hash(const SecDesc* __restrict__ secs, int n_secs, uint64_t* nodes,
+                    uint64_t* fp_out, const uint64_t* fp_before, uint8_t* flags) {
+  finalize_hash_warps(secs, n_secs, nodes, fp_out, fp_before, flags,
+                      blockIdx.x * kWarps + (threadIdx.x >> 5), gridDim.x * kWarps);
 }
 
 constexpr uint32_t kMaxSmemFps = 2048;  // level-1 nodes of up to 65535 fps
@@ -748,19 +764,19 @@ __device__ uint64_t session_fp(const uint64_t* fps, uint32_t stride, uint32_t n,
 
 // Checkpoint: fps into the section table, then header and session fp.
 // Restore with verification: compare recomputed fps with the record.
+// The whole block handles sessions b0, b0 + stride, ...
 template <int MODE>
-__global__ void __launch_bounds__(kThreads)
-    k_finalize_sessions(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
-                        int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
-                        uint8_t* corrupt, uint32_t* bad) {
-  __shared__ uint64_t smem[kMaxSmemFps];
-  __shared__ uint32_t s_bad;
+__device__ void finalize_sessions_block(const SecDesc* __restrict__ secs,
+                                        const SessDesc* __restrict__ sess, int n_sess,
+                                        const Entry* __restrict__ entries, uint64_t* nodes,
+                                        uint8_t* corrupt, uint32_t* bad, int b0, int stride,
+                                        uint64_t* smem, uint32_t* s_bad) {
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
-  for (int b = blockIdx.x; b < n_sess; b += gridDim.x) {
+  for (int b = b0; b < n_sess; b += stride) {
     const SessDesc S = sess[b];
     Entry* table = reinterpret_cast<Entry*>(S.record + kHeaderBytes);
-    if (threadIdx.x == 0) s_bad = 0;
+    if (threadIdx.x == 0) *s_bad = 0;
     __syncthreads();
     for (uint32_t j = wib; j < S.n_sections; j += kWarps) {
       const SecDesc s = secs[S.sec_begin + j];
@@ -773,7 +789,7 @@ __global__ void __launch_bounds__(kThreads)
           reinterpret_cast<uint4*>(&table[j])[lane] = reinterpret_cast<const uint4*>(&e)[lane];
         }
       } else {
-        if (lane == 0 && table[j].fp != fp) atomicOr(&s_bad, 1u);
+        if (lane == 0 && table[j].fp != fp) atomicOr(s_bad, 1u);
       }
     }
     __syncthreads();
@@ -791,7 +807,7 @@ __global__ void __launch_bounds__(kThreads)
           h[3] = make_uint4(0, 0, 0, 0);
         } else {
           const uint64_t stored = *reinterpret_cast<const uint64_t*>(S.record + 24);
-          const bool broken = s_bad != 0 || stored != sfp;
+          const bool broken = *s_bad != 0 || stored != sfp;
           if (corrupt) corrupt[b] = broken ? 1 : 0;
           if (broken) atomicAdd(bad, 1u);
         }
@@ -805,6 +821,46 @@ __global__ void __launch_bounds__(kThreads)
     }
     __syncthreads();
   }
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(kThreads)
+    k_finalize_sessions(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
+                        int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
+                        uint8_t* corrupt, uint32_t* bad) {
+  __shared__ uint64_t smem[kMaxSmemFps];
+  __shared__ uint32_t s_bad;
+  finalize_sessions_block<MODE>(secs, sess, n_sess, entries, nodes, corrupt, bad, blockIdx.x,
+                                gridDim.x, smem, &s_bad);
+}
+
+// Small calls in one launch: the streaming pass, then the finalisation by
+// the last block to finish (an atomic ticket; no block waits for another).
+// `ticket` is zero on entry and reset by the last block.
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, 2)
+    k_small(const SecDesc* __restrict__ secs, WorkList wl, int glog2, uint64_t* nodes,
+            uint32_t* err, uint32_t* ticket, int n_items, const SessDesc* __restrict__ sess,
+            const Entry* __restrict__ entries, uint64_t* fp_out, const uint64_t* fp_before,
+            uint8_t* flags, uint32_t* bad) {
+  __shared__ SecDesc sdesc[kWarps];
+  __shared__ uint64_t smem[64];  // up to 2048 sections per session
+  __shared__ uint32_t s_bad;
+  __shared__ bool s_last;
+  run_stream_tasks<MODE>(secs, wl, glog2, nodes, err, sdesc);
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (MODE == kModeHash) {
+    finalize_hash_warps(secs, n_items, nodes, fp_out, fp_before, flags, threadIdx.x >> 5, kWarps);
+  } else {
+    finalize_sessions_block<MODE>(secs, sess, n_items, entries, nodes, nullptr, bad, 0, 1, smem,
+                                  &s_bad);
+  }
+  if (threadIdx.x == 0) *ticket = 0;
 }
 
 // ---------------------------------------------------------------------------
@@ -1181,6 +1237,37 @@ cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* no
       return launch_bulk_mode<kModeRestoreV>(secs, wl, nodes, dev_err, sm_count, stream);
     default: return cudaErrorInvalidValue;
   }
+}
+
+cudaError_t launch_small(int mode, const SecDesc* secs, WorkList wl, int group_log2,
+                         uint64_t* nodes, uint32_t* dev_err, uint32_t* ticket, int n_items,
+                         const SessDesc* sess, const Entry* entries, uint64_t* fp_out,
+                         const uint64_t* fp_before, uint8_t* flags, uint32_t* bad, int sm_count,
+                         int blocks_per_sm, cudaStream_t stream) {
+  if (wl.n_tasks == 0) return cudaErrorInvalidValue;
+  const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + kWarps - 1) / kWarps;
+  const uint64_t cap = static_cast<uint64_t>(sm_count) * blocks_per_sm;
+  const int blocks = static_cast<int>(want < cap ? want : cap);
+  switch (mode) {
+    case kModeHash:
+      k_small<kModeHash><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err, ticket,
+                                                          n_items, sess, entries, fp_out, fp_before,
+                                                          flags, bad);
+      break;
+    case kModePack:
+      k_small<kModePack><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err, ticket,
+                                                          n_items, sess, entries, fp_out, fp_before,
+                                                          flags, bad);
+      break;
+    case kModeRestoreV:
+      k_small<kModeRestoreV><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err,
+                                                              ticket, n_items, sess, entries, fp_out,
+                                                              fp_before, flags, bad);
+      break;
+    default:
+      return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess, int n_sess,

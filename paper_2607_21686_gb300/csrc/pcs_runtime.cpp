@@ -670,7 +670,7 @@ uint64_t total_bytes(const std::vector<SecDesc>& d) {
 
 // Give every stream its node slots and its kernel.  bulk[i] says which.
 bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<char>& bulk,
-                  StreamPlan& P) {
+                  StreamPlan& P, bool allow_reduce = true) {
   uint64_t reg_chunks = 0;
   for (size_t i = 0; i < d.size(); ++i)
     if (!bulk[i]) reg_chunks += d[i].n_chunks;
@@ -702,7 +702,7 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   for (const auto& x : d) max_tasks = std::max<uint64_t>(max_tasks, x.n_tasks);
   uint64_t groups = 0;
   for (auto& x : d) {
-    if (max_tasks > 64) {
+    if (allow_reduce && max_tasks > 64) {
       x.fin_begin = static_cast<uint32_t>(node + groups);
       x.fin_count = (x.n_tasks + 31) / 32;
       groups += x.fin_count;
@@ -714,6 +714,17 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   P.reduce_groups = static_cast<uint32_t>(groups);
   P.nodes_total = node + groups;
   return P.nodes_total < (1ull << 32);
+}
+
+// A small call whose streams all take the register kernel runs in one
+// launch (k_small): the streaming pass and its finalisation.
+constexpr int kSmallMaxItems = 64;
+
+bool fused_ok(const std::vector<char>& bulk, bool small, int n_items) {
+  if (!small || n_items > kSmallMaxItems) return false;
+  for (char b : bulk)
+    if (b) return false;
+  return true;
 }
 
 // Workspace offsets of a stream plan's lists, after `base` bytes.
@@ -770,8 +781,9 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   std::vector<char> bulk(n);
   const bool small = total_bytes(d) <= kSmallCallBytes;
   for (int i = 0; i < n; ++i) bulk[i] = bulk_eligible(c, d[i], true, small, cache);
+  const bool fused = fused_ok(bulk, small, n);
   StreamPlan P;
-  if (!plan_streams(c, d, bulk, P)) return fail(PCS_E_INVAL, "too much data in one call");
+  if (!plan_streams(c, d, bulk, P, !fused)) return fail(PCS_E_INVAL, "too much data in one call");
   WsLayout L;
   L.secs = 0;
   const ListLayout LL = list_layout(P, sizeof(SecDesc) * n);
@@ -786,6 +798,16 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   PCS_CUDA(plan_copy(c, ws, L.nodes, stream));
   auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
+  if (fused) {
+    WorkList wl{reinterpret_cast<const uint32_t*>(ws + LL.reg_ids),
+                reinterpret_cast<const uint32_t*>(ws + LL.reg_begin),
+                static_cast<int>(P.reg_ids.size()), P.reg_tasks};
+    LaunchScope ls(c, kKStreamHash, stream);
+    PCS_CUDA(launch_small(kModeHash, dsecs, wl, P.glog2, nodes, c->words, c->words + 3, n, nullptr,
+                          nullptr, fp_out, fp_before, flags, nullptr, c->sm_count, c->stream_bps,
+                          stream));
+    return ws_release(c, stream);
+  }
   PCS_CUDA(launch_streams(c, kModeHash, dsecs, P, LL, ws, nodes, stream));
   {
     LaunchScope ls(c, kKFinalizeHash, stream);
@@ -1307,8 +1329,11 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   const bool small = total_bytes(d) <= kSmallCallBytes;
   for (size_t i = 0; i < d.size(); ++i)
     bulk[i] = bulk_eligible(c, d[i], placement == PCS_PLACE_DEVICE, small, cache);
+  uint32_t max_secs = 0;
+  for (int s = 0; s < n; ++s) max_secs = std::max<uint32_t>(max_secs, sd[s].n_sections);
+  const bool fused = fused_ok(bulk, small, n) && max_secs <= 2048;
   StreamPlan P;
-  const bool fits = plan_streams(c, d, bulk, P);
+  const bool fits = plan_streams(c, d, bulk, P, !fused);
   WsLayout L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
@@ -1334,11 +1359,20 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
   auto* dent = reinterpret_cast<const Entry*>(ws + L.entries);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
-  if (e == cudaSuccess) e = launch_streams(c, kModePack, dsecs, P, LL, ws, nodes, stream);
-  if (e == cudaSuccess) {
-    LaunchScope ls(c, kKFinalizePack, stream);
-    e = launch_finalize(kModePack, dsecs, dsess, n, dent, nodes, nullptr, nullptr, nullptr, nullptr,
-                        stream);
+  if (fused && e == cudaSuccess) {
+    WorkList wl{reinterpret_cast<const uint32_t*>(ws + LL.reg_ids),
+                reinterpret_cast<const uint32_t*>(ws + LL.reg_begin),
+                static_cast<int>(P.reg_ids.size()), P.reg_tasks};
+    LaunchScope ls(c, kKStreamPack, stream);
+    e = launch_small(kModePack, dsecs, wl, P.glog2, nodes, c->words, c->words + 3, n, dsess, dent,
+                     nullptr, nullptr, nullptr, nullptr, c->sm_count, c->stream_bps, stream);
+  } else {
+    if (e == cudaSuccess) e = launch_streams(c, kModePack, dsecs, P, LL, ws, nodes, stream);
+    if (e == cudaSuccess) {
+      LaunchScope ls(c, kKFinalizePack, stream);
+      e = launch_finalize(kModePack, dsecs, dsess, n, dent, nodes, nullptr, nullptr, nullptr,
+                          nullptr, stream);
+    }
   }
   if (e != cudaSuccess) return undo(cuda_fail(e, "checkpoint launch"));
   blk->written = record_event(c->events, stream);
@@ -1501,8 +1535,11 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   std::vector<char> bulk(d.size());
   const bool small = total_bytes(d) <= kSmallCallBytes;
   for (size_t i = 0; i < d.size(); ++i) bulk[i] = bulk_eligible(c, d[i], payload_dev[i], small, cache);
+  uint32_t max_secs = 0;
+  for (int s = 0; s < n; ++s) max_secs = std::max<uint32_t>(max_secs, sd[s].n_sections);
+  const bool fused = verify && fused_ok(bulk, small, n) && max_secs <= 2048;
   StreamPlan P;
-  if (!plan_streams(c, d, bulk, P)) return fail(PCS_E_INVAL, "too much data in one call");
+  if (!plan_streams(c, d, bulk, P, !fused)) return fail(PCS_E_INVAL, "too much data in one call");
   WsLayout L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
@@ -1523,12 +1560,22 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   // verify == 1: count failures of this call in words[1] and wait for them;
   // verify == 2: accumulate them in words[2] for the next pcs_sync.
   if (verify == 1) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
-  PCS_CUDA(launch_streams(c, verify ? kModeRestoreV : kModeRestore, dsecs, P, LL, ws,
-                          verify ? nodes : nullptr, stream));
-  if (verify) {
-    LaunchScope ls(c, kKFinalizeRestoreV, stream);
-    PCS_CUDA(launch_finalize(kModeRestoreV, dsecs, dsess, n, nullptr, nodes, nullptr, nullptr,
-                             nullptr, c->words + (verify == 1 ? 1 : 2), stream));
+  if (fused) {
+    WorkList wl{reinterpret_cast<const uint32_t*>(ws + LL.reg_ids),
+                reinterpret_cast<const uint32_t*>(ws + LL.reg_begin),
+                static_cast<int>(P.reg_ids.size()), P.reg_tasks};
+    LaunchScope ls(c, kKStreamRestoreV, stream);
+    PCS_CUDA(launch_small(kModeRestoreV, dsecs, wl, P.glog2, nodes, c->words, c->words + 3, n,
+                          dsess, nullptr, nullptr, nullptr, nullptr,
+                          c->words + (verify == 1 ? 1 : 2), c->sm_count, c->stream_bps, stream));
+  } else {
+    PCS_CUDA(launch_streams(c, verify ? kModeRestoreV : kModeRestore, dsecs, P, LL, ws,
+                            verify ? nodes : nullptr, stream));
+    if (verify) {
+      LaunchScope ls(c, kKFinalizeRestoreV, stream);
+      PCS_CUDA(launch_finalize(kModeRestoreV, dsecs, dsess, n, nullptr, nodes, nullptr, nullptr,
+                               nullptr, c->words + (verify == 1 ? 1 : 2), stream));
+    }
   }
   for (int s = 0; s < n; ++s) {
     st = note_use(c, snaps[s]->block, stream);
