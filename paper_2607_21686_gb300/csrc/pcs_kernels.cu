@@ -96,6 +96,29 @@ __device__ uint64_t warp_tree_inplace(uint64_t* a, uint32_t n, int lane) {
   return a[0];
 }
 
+// Tree of a 2-chunk tile, both chunks at once.  Lane l holds a0 = lane value
+// l of chunk 0 and a1 = lane value l of chunk 1.  Level 1 puts chunk q's pair
+// (2i, 2i+1) in lane 16q + i; from then on the pair of every level is in lanes
+// (2L, 2L+1), so each level is one comb across the warp.  After five levels
+// lane q holds chunk q's hash; with nc == 2 one more level gives the tile's
+// node comb(x0, x1) (the pairwise tree over its chunks).  Result in lane 0.
+__device__ __forceinline__ uint64_t tile_tree2(uint64_t a0, uint64_t a1, int nc, int lane) {
+  const int i = lane & 15;
+  const uint64_t l0 = __shfl_sync(kFull, a0, 2 * i), r0 = __shfl_sync(kFull, a0, 2 * i + 1);
+  const uint64_t l1 = __shfl_sync(kFull, a1, 2 * i), r1 = __shfl_sync(kFull, a1, 2 * i + 1);
+  uint64_t v = lane < 16 ? comb(l0, r0) : comb(l1, r1);
+  const int levels = nc == 2 ? 5 : 4;
+#pragma unroll
+  for (int k = 0; k < 5; ++k) {
+    if (k < levels) {
+      const uint64_t l = __shfl_sync(kFull, v, (2 * lane) & 31);
+      const uint64_t r = __shfl_sync(kFull, v, (2 * lane + 1) & 31);
+      v = comb(l, r);
+    }
+  }
+  return v;
+}
+
 // ---------------------------------------------------------------------------
 // Memory helpers
 // ---------------------------------------------------------------------------
@@ -414,6 +437,7 @@ __device__ __forceinline__ void fence_async_smem() {
 // What a stage holds (written by the warp when it stages the tile).
 struct WarpStage {
   SecDesc d;                // the tile's stream
+  uint32_t sec;             // its index (0xFFFFFFFF: none yet)
   uint64_t p0, p1;          // payload bytes of the tile: [p0, p1)
   uint64_t r0;              // first row touching the tile (ROWS / RING)
   uint32_t node;            // node slot of the tile
@@ -499,8 +523,12 @@ __device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, con
   using T = ModeTraits<MODE>;
   const uint32_t sec = __ldg(wl.ids + item);
   const uint32_t loc = t - __ldg(wl.begin + item);
-  if (lane < static_cast<int>(sizeof(SecDesc) / 16))
-    reinterpret_cast<uint4*>(&st.d)[lane] = __ldg(reinterpret_cast<const uint4*>(secs + sec) + lane);
+  if (st.sec != sec) {  // warp-uniform
+    __syncwarp();
+    if (lane < static_cast<int>(sizeof(SecDesc) / 16))
+      reinterpret_cast<uint4*>(&st.d)[lane] = __ldg(reinterpret_cast<const uint4*>(secs + sec) + lane);
+    if (lane == 0) st.sec = sec;
+  }
   __syncwarp();
   const SecDesc& s = st.d;
   const uint64_t L = s.bytes;
@@ -568,7 +596,10 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
   auto& sh = *reinterpret_cast<BulkShared<kBulkWarps, kWarpStages>*>(smem_raw);
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  if (lane < kWarpStages) mbar_init(&sh.bar[warp][lane], 1);
+  if (lane < kWarpStages) {
+    mbar_init(&sh.bar[warp][lane], 1);
+    sh.st[warp][lane].sec = 0xFFFFFFFFu;
+  }
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncwarp();
 
@@ -668,13 +699,24 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
           h[q] = absorb(h[q], v);
         }
       }
-      uint64_t mine = 0;
+      uint64_t root;
+      if (MODE == kModeHash) {
+        // Read-only pass: bound by the warps' work, so both chunks share
+        // each level of the tree.
+        static_assert(kTileChunks == 2, "tile_tree2 reduces two chunks");
+        root = tile_tree2(fmix(h[0]), fmix(h[1]), nc, lane);
+      } else {
+        // Moving passes are bound by DRAM; one tree per chunk paces the
+        // warps so that loads and stores interleave best (measured: the
+        // shared tree makes pack and restore slower).
+        uint64_t mine = 0;
 #pragma unroll
-      for (int q = 0; q < kTileChunks; ++q) {
-        const uint64_t x = __shfl_sync(kFull, warp_tree(fmix(h[q]), 32, lane), 0);
-        if (lane == q) mine = x;
+        for (int q = 0; q < kTileChunks; ++q) {
+          const uint64_t x = __shfl_sync(kFull, warp_tree(fmix(h[q]), 32, lane), 0);
+          if (lane == q) mine = x;
+        }
+        root = warp_tree(mine, nc, lane);
       }
-      const uint64_t root = warp_tree(mine, nc, lane);
       if (lane == 0) nodes[m.node] = root;
     }
     if (issued) {

@@ -25,7 +25,7 @@
 #include <unordered_set>
 #include <vector>
 
-#include "../../include/pcs.h"
+#include "pcs.h"
 #include "pcs_internal.h"
 
 using namespace pcs;
