@@ -103,6 +103,7 @@ def lib():
             "pcso_record_section": (None, [vp, i32, vp, vp, vp, vp]),
             "pcso_restore": (i32, [vp, vp, i32, i32]),
             "pcso_budget_plan": (i32, [vp, vp, vp, i32, u64, ctypes.c_double, vp, vp, vp]),
+            "pcso_prune_global": (ctypes.c_int64, [vp, vp, vp, i32, u64, vp, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -251,6 +252,22 @@ def budget_plan(n, entry_bytes, budget: int, frac: float, priority=None):
                                 budget, frac, _ptr(k), ctypes.byref(sh), ctypes.byref(dr))
     assert rc == 0
     return k, sh.value, dr.value
+
+
+def prune_global(scores32, n, entry_bytes, budget: int):
+    """One relevance threshold across all banks under a byte budget.
+
+    Returns (kept indices per bank concatenated, offsets int32[len(n)+1]).
+    """
+    a = np.ascontiguousarray(n, dtype=np.int32)
+    e = np.ascontiguousarray(np.broadcast_to(np.asarray(entry_bytes, dtype=np.uint64), a.shape))
+    s = np.ascontiguousarray(scores32, dtype=np.float32)
+    assert s.size == int(a.astype(np.int64).sum())
+    kept = np.zeros(max(s.size, 1), dtype=np.int32)
+    off = np.zeros(a.size + 1, dtype=np.int32)
+    m = lib().pcso_prune_global(_ptr(s), _ptr(a), _ptr(e), a.size, budget, _ptr(kept), _ptr(off))
+    assert m >= 0 and m == off[-1]
+    return kept[:m].copy(), off
 
 
 # --------------------------------------------------------------------------

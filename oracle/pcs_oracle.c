@@ -373,6 +373,70 @@ void pcso_k_fraction(const int32_t *n, int32_t count, double frac, int32_t *k)
     }
 }
 
+/*
+ * Global relevance threshold under one host byte budget (a variant of the
+ * budgeted pruning of Sec. 7.5: instead of pruning every bank to the same
+ * fraction, one score threshold is drawn across all banks, so a session with
+ * more relevant frames keeps more of them).  All entries of all banks are
+ * ranked together by (score desc, bank asc, index asc) -- the ranking key of
+ * the entry's position in the bank-major concatenation -- and the longest
+ * prefix of that order whose entry bytes sum to at most `budget` is kept.
+ * scores: float[sum n] bank-major; kept: int32[sum n] capacity, written per
+ * bank in ascending entry index; kept_off: int32[count + 1] offsets into kept.
+ * Returns the number kept, -1 on allocation failure.
+ */
+int64_t pcso_prune_global(const float *scores, const int32_t *n, const uint64_t *entry_bytes,
+                          int32_t count, uint64_t budget, int32_t *kept, int32_t *kept_off)
+{
+    uint64_t total = 0, *keys, j, m;
+    uint8_t *keep;
+    unsigned __int128 used = 0;
+    int64_t written = 0;
+    int32_t s, *bank_of;
+    uint64_t pos;
+    for (s = 0; s < count; s++) total += (uint64_t)n[s];
+    keys = (uint64_t *)malloc((size_t)(total ? total : 1) * sizeof(uint64_t));
+    keep = (uint8_t *)calloc((size_t)(total ? total : 1), 1);
+    bank_of = (int32_t *)malloc((size_t)(total ? total : 1) * sizeof(int32_t));
+    if (!keys || !keep || !bank_of) {
+        free(keys);
+        free(keep);
+        free(bank_of);
+        return -1;
+    }
+    pos = 0;
+    for (s = 0; s < count; s++) {
+        int32_t i;
+        for (i = 0; i < n[s]; i++, pos++) {
+            keys[pos] = pcso_key64(scores[pos], (uint32_t)pos);
+            bank_of[pos] = s;
+        }
+    }
+    qsort(keys, (size_t)total, sizeof(uint64_t), cmp_u64_desc);
+    /* Walk the global order; stop at the first entry that does not fit. */
+    m = 0;
+    for (j = 0; j < total; j++) {
+        uint64_t p = 0xFFFFFFFFu - (uint32_t)(keys[j] & 0xFFFFFFFFu);
+        used += entry_bytes[bank_of[p]];
+        if (used > budget) break;
+        keep[p] = 1;
+        m++;
+    }
+    /* Emit per bank, ascending entry index. */
+    pos = 0;
+    for (s = 0; s < count; s++) {
+        int32_t i;
+        kept_off[s] = (int32_t)written;
+        for (i = 0; i < n[s]; i++, pos++)
+            if (keep[pos]) kept[written++] = i;
+    }
+    kept_off[count] = (int32_t)written;
+    free(keys);
+    free(keep);
+    free(bank_of);
+    return (int64_t)m;
+}
+
 /* ------------------------------------------------------------------------ */
 /* Snapshot record "PCS1": the storage format of one checkpointed session   */
 /* (Sec. 3 "Boundary": storage owns serialisation; the layout is a frozen   */

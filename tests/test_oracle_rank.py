@@ -201,3 +201,73 @@ def test_budget_plan_properties(seed):
         # Reactive: acting is monotone in the pressure (tighter budget, more actions).
         assert sh + dr >= prev
         prev = sh + dr
+
+
+def _global_order(scores):
+    # Independent of the oracle: Python's sort on (NaN last, -score, position).
+    def rank_key(p):
+        s = float(scores[p])
+        return (1, 0.0, p) if np.isnan(s) else (0, -s, p)
+    return sorted(range(len(scores)), key=rank_key)
+
+
+def _check_global(scores, n, E, B):
+    kept, off = oracle.prune_global(scores, n, E, B)
+    starts = np.concatenate([[0], np.cumsum(n)]).astype(np.int64)
+    Eb = np.repeat(np.asarray(E, dtype=np.int64), n)
+    assert off[0] == 0 and np.all(np.diff(off) >= 0) and off[-1] == kept.size
+    chosen = set()
+    for b in range(len(n)):
+        part = kept[off[b]:off[b + 1]]
+        assert np.all(np.diff(part) > 0) and np.all(part >= 0) and np.all(part < n[b])
+        chosen.update((starts[b] + part).tolist())
+    total = int(Eb.sum())
+    used = int(sum(Eb[p] for p in chosen))
+    # The kept set is exactly a prefix of the global order ...
+    order = _global_order(scores)
+    m = len(chosen)
+    assert set(order[:m]) == chosen
+    # ... within the budget, and the next entry of the order does not fit.
+    assert used <= B
+    if m < len(order):
+        assert used + int(Eb[order[m]]) > B
+    else:
+        assert total <= B
+    return kept, off
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_prune_global_is_the_longest_fitting_prefix(seed):
+    rnd = np.random.default_rng(seed)
+    nb = int(rnd.integers(1, 7))
+    n = rnd.integers(0, 9, nb).astype(np.int32)
+    E = rnd.integers(0, 40, nb).astype(np.uint64)
+    pool = np.array([0.5, -0.25, 0.0, -0.0, 1.0, np.nan, 0.5, 0.125], dtype=np.float32)
+    s = pool[rnd.integers(0, pool.size, int(n.sum()))]
+    total = int((n.astype(np.int64) * E.astype(np.int64)).sum())
+    for B in sorted({0, 1, total // 3, total // 2, max(total - 1, 0), total, total + 7}):
+        _check_global(s, n, E, B)
+
+
+def test_prune_global_special_cases():
+    rnd = np.random.default_rng(5)
+    s = rnd.standard_normal(50).astype(np.float32)
+    # One bank, uniform entry bytes: a global threshold is the bank's top-k.
+    for k in (0, 1, 7, 49, 50):
+        kept, off = oracle.prune_global(s, [50], [3072], k * 3072 + 100)
+        assert kept.tolist() == oracle.topk(s, k).tolist()
+    # Budget that does not bind keeps everything; zero budget keeps nothing.
+    kept, off = oracle.prune_global(s, [20, 0, 30], [8, 8, 8], 50 * 8)
+    assert off.tolist() == [0, 20, 20, 50] and kept.tolist() == list(range(20)) + list(range(30))
+    kept, off = oracle.prune_global(s, [20, 0, 30], [8, 8, 8], 0)
+    assert kept.size == 0 and off.tolist() == [0, 0, 0, 0]
+    # Equal scores everywhere: ties go to the lower bank, then the lower index.
+    eq = np.full(12, 0.25, dtype=np.float32)
+    kept, off = oracle.prune_global(eq, [4, 4, 4], [1, 1, 1], 6)
+    assert off.tolist() == [0, 4, 6, 6] and kept.tolist() == [0, 1, 2, 3, 0, 1]
+    # A bank of more relevant entries keeps more than the same-fraction rule gives it.
+    hi = np.linspace(0.9, 0.8, 10).astype(np.float32)
+    lo = np.linspace(0.1, 0.0, 10).astype(np.float32)
+    kept, off = oracle.prune_global(np.concatenate([lo, hi]), [10, 10], [5, 5], 50)
+    assert off.tolist() == [0, 0, 10]
+    assert oracle.k_budget([10, 10], 5, 50).tolist() == [5, 5]
