@@ -418,6 +418,18 @@ def run_rows(ctx, dev, stream):
     out["prune"] = {"population": "2048 banks, n ~ U[256,4096], key bf16[512]",
                     "key_bytes_read": kb, "ms": round(med, 3), "GBs": round(gbs, 1),
                     "frac_of_hbm": round(gbs / peak, 4), "kept_fraction": round(sum(ks) / sum(b.n), 4)}
+    # The same banks under one relevance threshold across all of them.
+    gkept = torch.empty(sum(b.n), dtype=torch.int32, device=dev)
+    gkoff = torch.empty(S + 1, dtype=torch.int32, device=dev)
+    bestg, medg = _events_ms(lambda: ctx.prune_global(banks, S, 8 << 30, gkept, gkoff), stream)
+    gk = int(gkoff[-1].item())
+    out["prune_global"] = {
+        "population": "the same 2048 banks, one threshold across all under 8 GiB",
+        "key_bytes_read": kb, "ms": round(medg, 3), "GBs": round(kb / (medg / 1e3) / 1e9, 1),
+        "frac_of_hbm": round(kb / (medg / 1e3) / 1e9 / peak, 4),
+        "kept_fraction": round(gk / sum(b.n), 4),
+        "kept_bytes": gk * (1024 + 2048)}
+    del gkept, gkoff
     koff_h = koff.cpu().tolist()
     sess = [pcs.bank_session(s, keys[s], vals[s], kept[koff_h[s]:koff_h[s + 1]]) for s in range(S)]
     kept_bytes = sum(ks) * (1024 + 2048)

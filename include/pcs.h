@@ -169,7 +169,8 @@ typedef struct pcs_bank {
     int32_t key_dim;       /* multiple of 8                                 */
     uint32_t key_dtype;    /* PCS_DT_F16 or PCS_DT_BF16                     */
     uint32_t reserved;     /* 0                                             */
-    uint64_t entry_bytes;  /* bytes one kept entry costs (PCS_K_BUDGET)     */
+    uint64_t entry_bytes;  /* bytes one kept entry costs (PCS_K_BUDGET,     */
+                           /* pcs_prune_global)                             */
 } pcs_bank;
 
 typedef struct pcs_prune_params {
@@ -308,6 +309,24 @@ pcs_status pcs_prune(pcs_ctx *ctx, const pcs_bank *banks, int32_t n,
  */
 pcs_status pcs_topk(pcs_ctx *ctx, const float *keys, const int32_t *n, const int32_t *k,
                     int32_t n_banks, int32_t *kept_idx, int32_t *kept_off, void *stream);
+
+/*
+ * One relevance threshold across all banks under a host byte budget: the
+ * budgeted pruning of Sec. 7.5 with a cross-session threshold instead of the
+ * same fraction per bank, so a session with more relevant frames keeps more
+ * of them.  Every entry is scored as by pcs_prune; all entries of all banks
+ * are ranked together by (score desc, bank asc, index asc) and the longest
+ * prefix of that order whose entry_bytes sum to at most `budget` is kept (a
+ * budget that does not bind keeps everything).
+ *   scores:   device float[sum n] (CSR by bank) or NULL
+ *   kept_idx: device int32[sum n] (capacity); kept entries of bank b, in
+ *             ascending index, at kept_idx[kept_off[b] .. kept_off[b+1])
+ *   kept_off: device int32[n + 1], required; kept_off[n] = entries kept
+ * PCS_E_INVAL if the total entry bytes exceed 2^64 - 1; bank errors as for
+ * pcs_prune.
+ */
+pcs_status pcs_prune_global(pcs_ctx *ctx, const pcs_bank *banks, int32_t n, uint64_t budget,
+                            float *scores, int32_t *kept_idx, int32_t *kept_off, void *stream);
 
 /*
  * Host only: the reactive shrink-then-drop plan of a host budget (Sec. 7.10:

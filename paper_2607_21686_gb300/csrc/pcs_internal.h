@@ -152,6 +152,45 @@ cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
                         int32_t* kept_idx, cudaStream_t stream);
 
 
+// ---- One relevance threshold across all banks (pcs_prune_global) ---------
+constexpr int kGTile = 4096;  // entries per tile of the global passes
+
+// Select state: the kept set is every entry whose ranking key exceeds
+// `threshold`.  Set by the host, advanced by the last block of each pass.
+struct alignas(16) GState {
+  uint64_t prefix, mask;  // key bits fixed so far
+  uint64_t remaining;     // budget left for keys inside the prefix
+  uint64_t threshold;
+  uint32_t done, ticket, total_kept, pad;
+  uint64_t whist[256];    // entry bytes per digit (mixed entry sizes)
+  uint32_t chist[256];    // entries per digit
+};
+
+// Passed by value as a kernel parameter.
+struct GPlan {
+  const float* scores;        // [entries], bank-major
+  const uint64_t* ebeg;       // [n_banks + 1]: first entry of each bank; ebeg[n_banks] = entries
+  const uint64_t* ebytes;     // [n_banks]: bytes one entry of the bank costs
+  const uint32_t* tile_bank;  // [tiles + 1]: bank of entry min(t * kGTile, entries - 1)
+  uint32_t* tile_cnt;         // [tiles]: kept per tile, then its exclusive scan
+  GState* st;
+  int32_t* kept_idx;          // [<= entries], CSR by bank
+  int32_t* kept_off;          // [n_banks + 1]
+  uint64_t entries;
+  uint64_t uniform_bytes;     // entry bytes when every bank costs the same
+  int32_t n_banks;
+  int32_t tiles;
+  int32_t uniform;
+  int32_t pad;
+};
+
+// Pass `pass` (0..7) of the byte-weighted radix select; a no-op once the
+// threshold is known.
+cudaError_t launch_gselect(const GPlan& p, int pass, int sm_count, cudaStream_t stream);
+// Count per tile and scan (first launch), then write kept indices and bank
+// offsets (second launch).
+cudaError_t launch_gcompact(const GPlan& p, int sm_count, cudaStream_t stream);
+
 // Occupancy of the streaming kernel (blocks per SM) for the launch shape.
 int stream_blocks_per_sm();
 

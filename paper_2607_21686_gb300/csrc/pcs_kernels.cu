@@ -1206,6 +1206,239 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// ---------------------------------------------------------------------------
+// One relevance threshold across all banks under a byte budget
+//
+// The entry at bank-major position i ranks by
+//   key(i) = ord32(score_i) << 32 | (0xFFFFFFFF - i)
+// (score descending, then bank, then index ascending; unique keys).  The kept
+// set is the longest prefix of the descending key order whose entry bytes
+// fit the budget: every key above the key of the first entry that does not
+// fit.  That key is found most significant byte first, each pass summing the
+// bytes (not the count) of the candidate keys per digit; the last block of a
+// pass (atomic ticket, no block waits for another) picks the digit where the
+// budget runs out.
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint64_t gkey(const float* sc, uint64_t i) {
+  return (static_cast<uint64_t>(ord32(__ldg(sc + i))) << 32) | (0xFFFFFFFFull - i);
+}
+
+// The bank holding entry i: the last bank in [lo, hi] whose first entry is
+// <= i (empty banks share their successor's first entry and come before it).
+__device__ __forceinline__ int gbank(const uint64_t* __restrict__ ebeg, int lo, int hi,
+                                     uint64_t i) {
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (__ldg(ebeg + mid) <= i) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+template <bool UNIFORM>
+__global__ void __launch_bounds__(kThreads) k_gselect(GPlan p, int pass) {
+  __shared__ uint64_t wh[256];
+  __shared__ uint32_t ch[256];
+  __shared__ bool s_last;
+  GState* st = p.st;
+  if (__ldcg(&st->done)) return;  // the same for every block of the launch
+  const int shift = 56 - 8 * pass;
+  const uint64_t prefix = __ldcg(&st->prefix), mask = __ldcg(&st->mask);
+  for (int i = threadIdx.x; i < 256; i += kThreads) {
+    wh[i] = 0;
+    ch[i] = 0;
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
+    const uint64_t start = static_cast<uint64_t>(t) * kGTile;
+    const uint64_t end = start + kGTile < p.entries ? start + kGTile : p.entries;
+    int b = p.tile_bank[t];
+    const int hi = p.tile_bank[t + 1];
+#pragma unroll 4
+    for (int j = 0; j < kGTile / kThreads; ++j) {
+      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
+      uint32_t d = 256;  // not a candidate
+      if (i < end) {
+        const uint64_t key = gkey(p.scores, i);
+        if ((key & mask) == prefix) d = static_cast<uint32_t>(key >> shift) & 255u;
+      }
+      if (UNIFORM) {
+        // Lanes with the same digit add once (the hot digits are few).
+        const unsigned same = __match_any_sync(kFull, d);
+        if (d < 256 && lane == __ffs(same) - 1) atomicAdd(&ch[d], __popc(same));
+      } else if (d < 256) {
+        b = gbank(p.ebeg, b, hi, i);
+        atomicAdd(&ch[d], 1u);
+        atomicAdd(reinterpret_cast<unsigned long long*>(&wh[d]),
+                  static_cast<unsigned long long>(__ldg(p.ebytes + b)));
+      }
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < 256; i += kThreads) {
+    if (ch[i]) atomicAdd(&st->chist[i], ch[i]);
+    if (!UNIFORM && wh[i])
+      atomicAdd(reinterpret_cast<unsigned long long*>(&st->whist[i]),
+                static_cast<unsigned long long>(wh[i]));
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(&st->ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (threadIdx.x < 32) {
+    // Lane l covers digits 255-8l .. 248-8l (descending).
+    uint64_t w[8], local = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int bin = 255 - 8 * lane - j;
+      w[j] = UNIFORM ? static_cast<uint64_t>(__ldcg(&st->chist[bin])) * p.uniform_bytes
+                     : __ldcg(&st->whist[bin]);
+      local += w[j];
+    }
+    uint64_t incl = local;
+#pragma unroll
+    for (int dd = 1; dd < 32; dd <<= 1) {
+      const uint64_t o = __shfl_up_sync(kFull, incl, dd);
+      if (lane >= dd) incl += o;
+    }
+    const uint64_t R = __ldcg(&st->remaining);
+    const unsigned hit = __ballot_sync(kFull, incl > R);
+    if (hit == 0) {
+      // Every candidate fits (only when the whole population does).
+      if (lane == 0) {
+        st->threshold = 0;
+        st->done = 1;
+      }
+    } else if (lane == __ffs(hit) - 1) {
+      uint64_t cum = incl - local;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (cum + w[j] > R) {
+          const int bin = 255 - 8 * lane - j;
+          const uint64_t np = prefix | (static_cast<uint64_t>(bin) << shift);
+          const uint64_t nm = mask | (0xFFull << shift);
+          st->prefix = np;
+          st->mask = nm;
+          st->remaining = R - cum;
+          // One key left in the digit, or the last digit: that key is the
+          // first that does not fit.
+          if (__ldcg(&st->chist[bin]) == 1u || shift == 0) {
+            st->threshold = np | ~nm;
+            st->done = 1;
+          }
+          break;
+        }
+        cum += w[j];
+      }
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < 256; i += kThreads) {
+    st->chist[i] = 0;
+    st->whist[i] = 0;
+  }
+  if (threadIdx.x == 0) st->ticket = 0;
+}
+
+// Exclusive block scan of one uint32 per thread; *total = block sum.
+__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_sum,
+                                                    uint32_t* total) {
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  uint32_t incl = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint32_t o = __shfl_up_sync(kFull, incl, d);
+    if (lane >= d) incl += o;
+  }
+  if (lane == 31) warp_sum[wib] = incl;
+  __syncthreads();
+  uint32_t before = 0, sum = 0;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) {
+    const uint32_t c = warp_sum[w];
+    if (w < wib) before += c;
+    sum += c;
+  }
+  __syncthreads();
+  *total = sum;
+  return before + incl - v;
+}
+
+// Kept entries per tile; the last block scans the tile counts into offsets
+// and closes the bank offsets of trailing empty banks.
+__global__ void __launch_bounds__(kThreads) k_gcount(GPlan p) {
+  __shared__ uint32_t warp_sum[kWarps];
+  __shared__ bool s_last;
+  const uint64_t T = __ldcg(&p.st->threshold);
+  for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
+    const uint64_t start = static_cast<uint64_t>(t) * kGTile;
+    const uint64_t end = start + kGTile < p.entries ? start + kGTile : p.entries;
+    uint32_t c = 0;
+    for (uint64_t i = start + threadIdx.x; i < end; i += kThreads) c += gkey(p.scores, i) > T;
+    uint32_t total;
+    block_excl_scan(c, warp_sum, &total);
+    if (threadIdx.x == 0) p.tile_cnt[t] = total;
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(&p.st->ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  uint32_t run = 0;
+  for (int base = 0; base < p.tiles; base += kThreads) {
+    const int t = base + threadIdx.x;
+    const uint32_t v = t < p.tiles ? __ldcg(&p.tile_cnt[t]) : 0u;
+    uint32_t total;
+    const uint32_t ex = block_excl_scan(v, warp_sum, &total);
+    if (t < p.tiles) p.tile_cnt[t] = run + ex;
+    run += total;
+  }
+  if (threadIdx.x == 0) {
+    p.st->total_kept = run;
+    p.kept_off[p.n_banks] = static_cast<int32_t>(run);
+    for (int b = p.n_banks - 1; b >= 0 && p.ebeg[b] == p.entries; --b)
+      p.kept_off[b] = static_cast<int32_t>(run);
+    p.st->ticket = 0;
+  }
+}
+
+// Kept indices (bank-local, ascending) at their global rank, and the offset
+// of every bank at the rank of its first entry.
+__global__ void __launch_bounds__(kThreads) k_gwrite(GPlan p) {
+  __shared__ uint32_t warp_cnt[kWarps];
+  const uint64_t T = __ldcg(&p.st->threshold);
+  for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
+    const uint64_t start = static_cast<uint64_t>(t) * kGTile;
+    const uint64_t end = start + kGTile < p.entries ? start + kGTile : p.entries;
+    uint32_t base = p.tile_cnt[t];
+    int b = p.tile_bank[t];
+    const int hi = p.tile_bank[t + 1];
+    for (int j = 0; j < kGTile / kThreads; ++j) {
+      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
+      const bool valid = i < end;
+      const bool keep = valid && gkey(p.scores, i) > T;
+      uint32_t total;
+      const uint32_t r = block_rank(keep, warp_cnt, &total);
+      if (valid) {
+        b = gbank(p.ebeg, b, hi, i);
+        const uint64_t first = __ldg(p.ebeg + b);
+        if (keep) p.kept_idx[base + r] = static_cast<int32_t>(i - first);
+        if (i == first) {
+          p.kept_off[b] = static_cast<int32_t>(base + r);
+          for (int e = b - 1; e >= 0 && __ldg(p.ebeg + e) == i; --e)
+            p.kept_off[e] = static_cast<int32_t>(base + r);
+        }
+      }
+      base += total;
+    }
+  }
+}
+
 template <int MODE>
 int occupancy() {
   int b = 0;
@@ -1369,6 +1602,27 @@ cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
   if (n_banks <= 0) return cudaSuccess;
   k_topk<<<n_banks < 65535 ? n_banks : 65535, kThreads, 0, stream>>>(banks, n_banks, scores,
                                                                      kept_idx);
+  return cudaGetLastError();
+}
+
+static int gblocks(const GPlan& p, int sm_count) {
+  const int cap = 4 * sm_count;
+  return p.tiles < cap ? p.tiles : cap;
+}
+
+cudaError_t launch_gselect(const GPlan& p, int pass, int sm_count, cudaStream_t stream) {
+  if (p.tiles <= 0) return cudaSuccess;
+  if (p.uniform) k_gselect<true><<<gblocks(p, sm_count), kThreads, 0, stream>>>(p, pass);
+  else k_gselect<false><<<gblocks(p, sm_count), kThreads, 0, stream>>>(p, pass);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gcompact(const GPlan& p, int sm_count, cudaStream_t stream) {
+  if (p.tiles <= 0) return cudaSuccess;
+  k_gcount<<<gblocks(p, sm_count), kThreads, 0, stream>>>(p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_gwrite<<<gblocks(p, sm_count), kThreads, 0, stream>>>(p);
   return cudaGetLastError();
 }
 

@@ -362,13 +362,13 @@ pcs_status set_device(pcs_ctx* c) {
 enum KernelKind {
   kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
   kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKBulkHash, kKBulkPack,
-  kKBulkRestore, kKBulkRestoreV, kKReduce, kKernelKinds
+  kKBulkRestore, kKBulkRestoreV, kKReduce, kKGSelect, kKGCompact, kKernelKinds
 };
 const char* kKernelNames[kKernelKinds] = {
     "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
     "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
-    "k_reduce_nodes"};
+    "k_reduce_nodes", "k_gselect", "k_gcompact"};
 
 cudaEvent_t timing_event(pcs_ctx* c) {
   if (!c->timing_events.empty()) {
@@ -1074,6 +1074,54 @@ pcs_status pcs_prune_counts(const pcs_bank* banks, int32_t n, const pcs_prune_pa
   }
 }
 
+// Validated scoring descriptors of n banks (k per bank, or all 0 if k is
+// NULL), entry offsets bank-major; *entries = total entries.
+pcs_status bank_descs(const pcs_bank* banks, int32_t n, const int32_t* k,
+                      std::vector<BankDesc>* d, uint64_t* entries_out) {
+  d->assign(std::max(n, 0), BankDesc{});
+  uint64_t entries = 0, kept = 0;
+  for (int s = 0; s < n; ++s) {
+    const pcs_bank& b = banks[s];
+    if (b.key_dtype != PCS_DT_F16 && b.key_dtype != PCS_DT_BF16)
+      return fail(PCS_E_INVAL, "bank %d: key_dtype must be F16 or BF16", s);
+    if (b.key_dim <= 0 || b.key_dim % 8 != 0)
+      return fail(PCS_E_ALIGN, "bank %d: key_dim must be a positive multiple of 8", s);
+    if (b.n_entries < 0) return fail(PCS_E_INVAL, "bank %d: negative n_entries", s);
+    if (b.n_entries > 0 && (!b.keys || !b.query))
+      return fail(PCS_E_INVAL, "bank %d: null keys or query", s);
+    if (b.n_entries > 0 && (!aligned16(b.keys) || !aligned16(b.query)))
+      return fail(PCS_E_ALIGN, "bank %d: keys / query not 16-byte aligned", s);
+    BankDesc& x = (*d)[s];
+    x.keys = static_cast<const uint16_t*>(b.keys);
+    x.query = static_cast<const uint16_t*>(b.query);
+    x.entry_begin = entries;
+    x.kept_begin = kept;
+    x.n = b.n_entries;
+    x.D = b.key_dim;
+    x.k = k ? k[s] : 0;
+    x.is_bf16 = b.key_dtype == PCS_DT_BF16;
+    entries += b.n_entries;
+    kept += x.k;
+  }
+  if (entries > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many entries in one call");
+  *entries_out = entries;
+  return PCS_OK;
+}
+
+// The relevance score of every entry (descriptors already on the device).
+cudaError_t launch_bank_scores(pcs_ctx* c, const pcs_bank* banks, int32_t n,
+                               const BankDesc* dbanks, uint64_t entries, float* sc,
+                               cudaStream_t stream) {
+  LaunchScope ls(c, kKScore, stream);
+  int max_dim = 0, n_bf16 = 0;
+  for (int s = 0; s < n; ++s) {
+    max_dim = std::max(max_dim, banks[s].key_dim);
+    n_bf16 += banks[s].key_dtype == PCS_DT_BF16;
+  }
+  const int key_types = n_bf16 == 0 ? 0 : (n_bf16 == n ? 1 : 2);
+  return launch_score(dbanks, n, entries, max_dim, key_types, sc, c->sm_count, stream);
+}
+
 pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_prune_params* p,
                      float* scores, int32_t* kept_idx, int32_t* kept_off, void* stream_) {
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
@@ -1082,33 +1130,17 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
   pcs_status st = pcs_prune_counts(banks, n, p, k.data());
   if (st) return st;
   if (n == 0) return PCS_OK;
-  std::vector<BankDesc> d(n);
+  std::vector<BankDesc> d;
+  uint64_t entries = 0;
+  st = bank_descs(banks, n, k.data(), &d, &entries);
+  if (st) return st;
   std::vector<int32_t> koff(n + 1, 0);
-  uint64_t entries = 0, kept = 0;
+  uint64_t kept = 0;
   for (int s = 0; s < n; ++s) {
-    const pcs_bank& b = banks[s];
-    if (b.key_dtype != PCS_DT_F16 && b.key_dtype != PCS_DT_BF16)
-      return fail(PCS_E_INVAL, "bank %d: key_dtype must be F16 or BF16", s);
-    if (b.key_dim <= 0 || b.key_dim % 8 != 0)
-      return fail(PCS_E_ALIGN, "bank %d: key_dim must be a positive multiple of 8", s);
-    if (b.n_entries > 0 && (!b.keys || !b.query))
-      return fail(PCS_E_INVAL, "bank %d: null keys or query", s);
-    if (b.n_entries > 0 && (!aligned16(b.keys) || !aligned16(b.query)))
-      return fail(PCS_E_ALIGN, "bank %d: keys / query not 16-byte aligned", s);
-    d[s].keys = static_cast<const uint16_t*>(b.keys);
-    d[s].query = static_cast<const uint16_t*>(b.query);
-    d[s].entry_begin = entries;
-    d[s].kept_begin = kept;
-    d[s].n = b.n_entries;
-    d[s].D = b.key_dim;
-    d[s].k = k[s];
-    d[s].is_bf16 = b.key_dtype == PCS_DT_BF16;
-    entries += b.n_entries;
     kept += k[s];
     koff[s + 1] = static_cast<int32_t>(kept);
   }
   if (kept > 0 && !kept_idx) return fail(PCS_E_INVAL, "kept_idx is null");
-  if (entries > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many entries in one call");
   std::lock_guard<std::mutex> lk(c->mu);
   st = set_device(c);
   if (st) return st;
@@ -1128,16 +1160,7 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
     PCS_CUDA(cudaMemcpyAsync(kept_off, ws + L.secs, 4ull * (n + 1), cudaMemcpyDeviceToDevice, stream));
   float* sc = scores ? scores : reinterpret_cast<float*>(ws + L.nodes);
   auto* dbanks = reinterpret_cast<const BankDesc*>(ws + L.banks);
-  {
-    LaunchScope ls(c, kKScore, stream);
-    int max_dim = 0, n_bf16 = 0;
-    for (int s = 0; s < n; ++s) {
-      max_dim = std::max(max_dim, banks[s].key_dim);
-      n_bf16 += banks[s].key_dtype == PCS_DT_BF16;
-    }
-    const int key_types = n_bf16 == 0 ? 0 : (n_bf16 == n ? 1 : 2);
-    PCS_CUDA(launch_score(dbanks, n, entries, max_dim, key_types, sc, c->sm_count, stream));
-  }
+  PCS_CUDA(launch_bank_scores(c, banks, n, dbanks, entries, sc, stream));
   {
     LaunchScope ls(c, kKTopk, stream);
     PCS_CUDA(launch_topk(dbanks, n, sc, kept_idx, stream));
@@ -1184,6 +1207,106 @@ pcs_status pcs_topk(pcs_ctx* c, const float* keys, const int32_t* n, const int32
   {
     LaunchScope ls(c, kKTopk, stream);
     PCS_CUDA(launch_topk(reinterpret_cast<const BankDesc*>(ws), n_banks, keys, kept_idx, stream));
+  }
+  return ws_release(c, stream);
+}
+
+pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64_t budget,
+                            float* scores, int32_t* kept_idx, int32_t* kept_off, void* stream_) {
+  if (!c || n < 0 || (n > 0 && !banks)) return fail(PCS_E_INVAL, "bad arguments");
+  if (!kept_off) return fail(PCS_E_INVAL, "kept_off is null");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::vector<BankDesc> d;
+  uint64_t entries = 0;
+  pcs_status st = bank_descs(banks, n, nullptr, &d, &entries);
+  if (st) return st;
+  if (entries > 0 && !kept_idx) return fail(PCS_E_INVAL, "kept_idx is null");
+  std::vector<uint64_t> ebeg(n + 1), ebytes(n);
+  unsigned __int128 total = 0;
+  bool uniform = true;
+  for (int s = 0; s < n; ++s) {
+    ebeg[s] = d[s].entry_begin;
+    ebytes[s] = banks[s].entry_bytes;
+    total += static_cast<unsigned __int128>(banks[s].n_entries) * banks[s].entry_bytes;
+    uniform = uniform && banks[s].entry_bytes == banks[0].entry_bytes;
+  }
+  ebeg[n] = entries;
+  if (total > static_cast<unsigned __int128>(~0ull))
+    return fail(PCS_E_INVAL, "total entry bytes exceed 2^64");
+  std::lock_guard<std::mutex> lk(c->mu);
+  st = set_device(c);
+  if (st) return st;
+  if (entries == 0) {
+    // Nothing to rank: every bank keeps nothing.
+    PCS_CUDA(cudaMemsetAsync(kept_off, 0, 4ull * (n + 1), stream));
+    return PCS_OK;
+  }
+  const uint64_t tiles = (entries + kGTile - 1) / kGTile;
+  // Bank of entry min(t * kGTile, entries - 1), t = 0..tiles.
+  std::vector<uint32_t> tile_bank(tiles + 1);
+  {
+    int b = 0;
+    for (uint64_t t = 0; t <= tiles; ++t) {
+      const uint64_t i = std::min<uint64_t>(t * kGTile, entries - 1);
+      while (b + 1 < n && ebeg[b + 1] <= i) ++b;
+      tile_bank[t] = static_cast<uint32_t>(b);
+    }
+  }
+  GState g0{};
+  g0.remaining = budget;
+  g0.done = total <= budget;  // the budget does not bind: threshold 0 keeps all
+  uint64_t at = round_up(sizeof(BankDesc) * n, kRecordAlign);
+  const uint64_t o_ebeg = at;
+  at = round_up(at + 8ull * (n + 1), 16);
+  const uint64_t o_ebytes = at;
+  at = round_up(at + 8ull * n, 16);
+  const uint64_t o_tb = at;
+  at = round_up(at + 4ull * (tiles + 1), kRecordAlign);
+  const uint64_t o_st = at;
+  at = round_up(at + sizeof(GState), kRecordAlign);
+  const uint64_t plan_bytes = at;
+  const uint64_t o_tc = at;
+  at = round_up(at + 4ull * tiles, kRecordAlign);
+  const uint64_t o_sc = at;
+  const uint64_t ws_bytes = at + (scores ? 0 : 4ull * entries);
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, ws_bytes, stream, &ws);
+  if (st) return st;
+  c->plan.assign(plan_bytes, 0);
+  put(c->plan, 0, d);
+  put(c->plan, o_ebeg, ebeg);
+  put(c->plan, o_ebytes, ebytes);
+  put(c->plan, o_tb, tile_bank);
+  std::memcpy(c->plan.data() + o_st, &g0, sizeof g0);
+  PCS_CUDA(plan_copy(c, ws, plan_bytes, stream));
+  float* sc = scores ? scores : reinterpret_cast<float*>(ws + o_sc);
+  PCS_CUDA(launch_bank_scores(c, banks, n, reinterpret_cast<const BankDesc*>(ws), entries, sc,
+                              stream));
+  GPlan gp{};
+  gp.scores = sc;
+  gp.ebeg = reinterpret_cast<const uint64_t*>(ws + o_ebeg);
+  gp.ebytes = reinterpret_cast<const uint64_t*>(ws + o_ebytes);
+  gp.tile_bank = reinterpret_cast<const uint32_t*>(ws + o_tb);
+  gp.tile_cnt = reinterpret_cast<uint32_t*>(ws + o_tc);
+  gp.st = reinterpret_cast<GState*>(ws + o_st);
+  gp.kept_idx = kept_idx;
+  gp.kept_off = kept_off;
+  gp.entries = entries;
+  gp.uniform_bytes = n > 0 ? banks[0].entry_bytes : 0;
+  gp.n_banks = n;
+  gp.tiles = static_cast<int32_t>(tiles);
+  gp.uniform = uniform ? 1 : 0;
+  if (!g0.done) {
+    // Eight digit passes at most; each is a no-op once the threshold is known.
+    for (int pass = 0; pass < 8; ++pass) {
+      LaunchScope ls(c, kKGSelect, stream);
+      PCS_CUDA(launch_gselect(gp, pass, c->sm_count, stream));
+    }
+  }
+  {
+    LaunchScope ls(c, kKGCompact, stream);
+    c->launches += 1;  // count and write
+    PCS_CUDA(launch_gcompact(gp, c->sm_count, stream));
   }
   return ws_release(c, stream);
 }

@@ -128,6 +128,7 @@ SIGNATURES = {
                         _vp, _vp, _vp, _vp]),
     "pcs_record_bytes": (_st, [ctypes.POINTER(pcs_section), _i32, ctypes.POINTER(_u64)]),
     "pcs_topk": (_st, [_vp, _vp, ctypes.POINTER(_i32), ctypes.POINTER(_i32), _i32, _vp, _vp, _vp]),
+    "pcs_prune_global": (_st, [_vp, ctypes.POINTER(pcs_bank), _i32, _u64, _vp, _vp, _vp, _vp]),
     "pcs_budget_plan": (_st, [ctypes.POINTER(_i32), ctypes.POINTER(_u64), ctypes.POINTER(ctypes.c_double),
                               _i32, _u64, ctypes.c_double, ctypes.POINTER(_i32),
                               ctypes.POINTER(_i32), ctypes.POINTER(_i32)]),
@@ -429,6 +430,12 @@ class Context:
         ka = (ctypes.c_int32 * max(nb, 1))(*k)
         check(self.lib.pcs_topk(self.h, _ptr(keys), na, ka, nb, _ptr(kept_idx), _ptr(kept_off),
                                 _stream_ptr(stream)), "pcs_topk")
+
+    def prune_global(self, banks, n: int, budget: int, kept_idx: torch.Tensor,
+                     kept_off: torch.Tensor, scores=None, stream=None):
+        """One relevance threshold across all banks under a byte budget."""
+        check(self.lib.pcs_prune_global(self.h, banks, n, budget, _ptr(scores), _ptr(kept_idx),
+                                        _ptr(kept_off), _stream_ptr(stream)), "pcs_prune_global")
 
     # -- snapshots -------------------------------------------------------------
     def record_bytes(self, session: Session) -> int:

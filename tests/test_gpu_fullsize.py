@@ -109,6 +109,46 @@ def test_mass_banks_full_size(ctx, dev):
         ctx.delete(x)
 
 
+def _ord32_np(s):
+    u = s.view(np.uint32).astype(np.uint64)
+    out = np.where(u & 0x80000000, (~u) & 0xFFFFFFFF, u | 0x80000000)
+    out[s == 0] = 0x80000000
+    out[np.isnan(s)] = 0
+    return out
+
+
+def test_global_threshold_full_size(ctx, dev):
+    # The same 2048 banks under one relevance threshold across all of them:
+    # sampled scores against the oracle, then the defining property at full
+    # size -- the kept set is the longest prefix of the (score desc, bank,
+    # index) order whose bytes fit 8 GiB.
+    b = synth.banks_config5(device=dev)
+    S, E, B = b.sessions, 1024 + 2048, 8 << 30
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    qs = [b.queries[s] for s in range(S)]
+    banks = ctx.banks_array(keys, qs, E)
+    total = b.keys.shape[0]
+    kept = torch.empty(total, dtype=torch.int32, device=dev)
+    koff = torch.empty(S + 1, dtype=torch.int32, device=dev)
+    scores = torch.empty(total, dtype=torch.float32, device=dev)
+    ctx.prune_global(banks, S, B, kept, koff, scores)
+    sc = scores.cpu().numpy()
+    koff_h = koff.cpu().numpy().astype(np.int64)
+    kept_h = kept.cpu().numpy()[:koff_h[-1]]
+    for s in (0, 777, S - 1):
+        lo, hi = b.entry_off[s], b.entry_off[s + 1]
+        s32 = oracle.scores(np_view(qs[s]), np_view(keys[s]))
+        assert np.array_equal(sc[lo:hi].view(np.uint32), s32.view(np.uint32)), s
+    m = min(B // E, total)
+    assert koff_h[-1] == m and koff_h[0] == 0 and np.all(np.diff(koff_h) >= 0)
+    pos = np.arange(total, dtype=np.uint64)
+    key = (_ord32_np(sc) << np.uint64(32)) | (np.uint64(0xFFFFFFFF) - pos)
+    top = np.sort(np.argsort(key)[::-1][:m])
+    starts = np.asarray(b.entry_off[:-1], dtype=np.int64)
+    got = np.concatenate([starts[s] + kept_h[koff_h[s]:koff_h[s + 1]] for s in range(S)])
+    assert np.array_equal(got, top)
+
+
 def test_markov_batch_full_size(ctx, dev):
     # 4096 Markovian sessions of [3,256,256] uint8 + 16-byte RNG in one call.
     S = 4096

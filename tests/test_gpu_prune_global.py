@@ -1,0 +1,125 @@
+"""GPU parity: one relevance threshold across all banks under a byte budget.
+
+pcs_prune_global through the C ABI against the oracle on the same seeded
+banks: scores bit-equal to the oracle's fixed-order fp32 score, kept sets and
+bank offsets identical, across several 4096-entry tiles with a ragged tail,
+with uniform and mixed entry sizes (the two select paths), empty banks at
+either end and in the middle, exact ties across banks, and budgets that keep
+nothing, one entry, a fraction, all but one, and all.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_21686_gb300 import pcs, synth
+from helpers import np_view
+
+pytestmark = pytest.mark.gpu
+
+
+def _oracle_scores(keys, qs):
+    return np.concatenate([oracle.scores(np_view(q), np_view(k)) if k.shape[0] else
+                           np.zeros(0, np.float32) for k, q in zip(keys, qs)])
+
+
+def _run(ctx, dev, keys, qs, E, budget, want_scores=True):
+    n = len(keys)
+    banks = ctx.banks_array(keys, qs, E)
+    total = sum(k.shape[0] for k in keys)
+    kept = torch.full((max(total, 1),), -7, dtype=torch.int32, device=dev)
+    koff = torch.full((n + 1,), -7, dtype=torch.int32, device=dev)
+    scores = torch.empty(max(total, 1), dtype=torch.float32, device=dev) if want_scores else None
+    ctx.prune_global(banks, n, budget, kept, koff, scores)
+    ctx.sync()
+    koff_h = koff.cpu().numpy()
+    kept_h = kept.cpu().numpy()[:koff_h[-1]]
+    return kept_h, koff_h, (scores.cpu().numpy()[:total] if want_scores else None)
+
+
+def _check(ctx, dev, keys, qs, E, budgets):
+    s32 = _oracle_scores(keys, qs)
+    n = [k.shape[0] for k in keys]
+    Eb = [E] * len(n) if isinstance(E, int) else E
+    for B in budgets:
+        kept, koff, sc = _run(ctx, dev, keys, qs, E, B)
+        assert np.array_equal(sc.view(np.uint32), s32.view(np.uint32))
+        want, woff = oracle.prune_global(s32, n, Eb, B)
+        assert koff.tolist() == woff.tolist(), B
+        assert kept.tolist() == want.tolist(), B
+
+
+def _views(b, dev):
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]].to(dev) for s in range(b.sessions)]
+    qs = [b.queries[s].to(dev) for s in range(b.sessions)]
+    return keys, qs
+
+
+def test_global_threshold_uniform_bytes(ctx, dev):
+    # ~6,000 entries: two 4096-entry tiles, the second ragged.
+    b = synth.banks(301, 40, 1, 300, 256, torch.float16, (8,), torch.uint8)
+    keys, qs = _views(b, dev)
+    E = 512 + 8
+    T = sum(b.n) * E
+    _check(ctx, dev, keys, qs, E, [0, E - 1, E, 7 * E + 3, T // 10, T // 2, T - E, T - 1, T,
+                                   T + 1, 2 * T])
+
+
+def test_global_threshold_mixed_bytes_and_empty_banks(ctx, dev):
+    b = synth.banks(302, 30, 0, 700, 128, torch.bfloat16, (8,), torch.uint8)
+    keys, qs = _views(b, dev)
+    # Empty banks first, in the middle and last.
+    D = keys[0].shape[1]
+    empty = torch.empty(0, D, dtype=keys[0].dtype, device=dev)
+    keys = [empty, empty] + keys[:10] + [empty] + keys[10:] + [empty, empty]
+    qs = [qs[0], qs[1]] + qs[:10] + [qs[2]] + qs[10:] + [qs[3], qs[4]]
+    rnd = np.random.default_rng(3)
+    E = [int(x) for x in rnd.integers(0, 5000, len(keys))]
+    E[5] = 0  # free entries still take their place in the order
+    T = sum(k.shape[0] * e for k, e in zip(keys, E))
+    _check(ctx, dev, keys, qs, E, [0, 1, T // 7, T // 3, T // 2, T - 1, T])
+
+
+def test_global_threshold_ties_across_banks(ctx, dev):
+    # Zero keys score 0 everywhere and duplicated keys tie exactly: the order
+    # falls through to bank, then index -- the low digit passes decide.
+    D = 64
+    g = torch.Generator().manual_seed(8)
+    q = torch.randn(D, generator=g).half()
+    base = torch.randn(3, D, generator=g).half()
+    banks_k = []
+    for s in range(9):
+        parts = [torch.zeros(500 + 37 * s, D).half(), base, base[:1].repeat(4, 1)]
+        banks_k.append(torch.cat(parts).to(dev))
+    qs = [q.to(dev)] * 9
+    E = 96
+    T = sum(k.shape[0] for k in banks_k) * E
+    _check(ctx, dev, banks_k, qs, E, [0, E, 5 * E, 30 * E + 5, T // 2 + 17 * E, T - E, T])
+    _check(ctx, dev, banks_k, qs, [96, 1, 300, 96, 7, 96, 1000, 2, 96],
+           [0, 1000, 12345, 200000, 10**9])
+
+
+def test_global_threshold_scores_optional_and_no_entries(ctx, dev):
+    b = synth.banks(303, 7, 1, 50, 64, torch.float16, (8,), torch.uint8)
+    keys, qs = _views(b, dev)
+    s32 = _oracle_scores(keys, qs)
+    kept, koff, _ = _run(ctx, dev, keys, qs, 100, sum(b.n) * 40, want_scores=False)
+    want, woff = oracle.prune_global(s32, b.n, 100, sum(b.n) * 40)
+    assert koff.tolist() == woff.tolist() and kept.tolist() == want.tolist()
+    empty = torch.empty(0, 64, dtype=torch.float16, device=dev)
+    kept, koff, _ = _run(ctx, dev, [empty] * 3, qs[:3], 100, 10, want_scores=False)
+    assert koff.tolist() == [0, 0, 0, 0]
+
+
+def test_global_threshold_keeps_relevant_sessions(ctx, dev):
+    # Against the same-fraction rule: a bank aligned with its query keeps
+    # more under the global threshold.
+    D = 128
+    g = torch.Generator().manual_seed(12)
+    q = torch.randn(D, generator=g)
+    near = (q[None] + 0.3 * torch.randn(200, D, generator=g)).half()
+    far = torch.randn(200, D, generator=g).half()
+    keys = [near.to(dev), far.to(dev)]
+    qs = [q.half().to(dev)] * 2
+    kept, koff, _ = _run(ctx, dev, keys, qs, 10, 2000)
+    assert koff.tolist() == [0, 200, 200]
