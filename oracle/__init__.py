@@ -418,3 +418,80 @@ def kv_session(session_id: int, meta: np.ndarray, k_pool: np.ndarray, v_pool: np
         sp.ring(SEC_V, DT_BF16, v_pool, row_bytes, pt, rs, window, page_rows, layer=l,
                 dim0=window, dim1=row_bytes)
     return sp
+
+
+# --------------------------------------------------------------------------
+# Copy-on-write page pool (Sec. 3, I3: the mechanism realises fork
+# independence by copy-on-write; Sec. 3 "Boundary": the runtime owns
+# allocation and copy-on-write; Sec. 7.3: ref-counted blocks whose copy leg
+# fires on the first write).  Sequential reference model.
+# --------------------------------------------------------------------------
+
+class PoolError(Exception):
+    pass
+
+
+class PagePool:
+    """n_pages pages of page_bytes; a reference count per page; free stack.
+
+    alloc(n)               -> n fresh pages, count 1 each (lowest ids first)
+    share(ids)             -> the same ids, every valid page count + 1 (a fork
+                              of the tables that hold them: no bytes move)
+    prepare_write(t, e)    -> before writing table entries t[e]: an entry whose
+                              page is held elsewhere (count > 1) gets a fresh
+                              copy of it and gives up its hold; a page held by
+                              this entry alone is kept as it is
+    release(ids)           -> every valid page count - 1; pages at 0 are free
+    Page id -1 marks an empty table slot and is skipped everywhere.
+    """
+
+    def __init__(self, n_pages: int, page_bytes: int):
+        self.data = np.zeros((n_pages, page_bytes), dtype=np.uint8)
+        self.rc = np.zeros(n_pages, dtype=np.int64)
+        self.free = list(range(n_pages - 1, -1, -1))  # pop() gives the lowest id
+        self.copies = 0
+
+    def _pop(self) -> int:
+        if not self.free:
+            raise PoolError("no free page")
+        q = self.free.pop()
+        self.rc[q] = 1
+        return q
+
+    def alloc(self, n: int) -> np.ndarray:
+        return np.array([self._pop() for _ in range(n)], dtype=np.int32)
+
+    def share(self, ids) -> np.ndarray:
+        ids = np.asarray(ids, dtype=np.int32)
+        for p in ids.reshape(-1).tolist():
+            if p >= 0:
+                self.rc[p] += 1
+        return ids.copy()
+
+    def prepare_write(self, table: np.ndarray, entries=None) -> None:
+        flat = table.reshape(-1)
+        todo = range(flat.size) if entries is None else np.asarray(entries).reshape(-1).tolist()
+        for e in todo:
+            p = int(flat[e])
+            if p < 0 or self.rc[p] == 1:
+                continue
+            q = self._pop()
+            self.data[q] = self.data[p]
+            self.rc[p] -= 1
+            flat[e] = q
+            self.copies += 1
+
+    def release(self, ids) -> None:
+        for p in np.asarray(ids).reshape(-1).tolist():
+            if p < 0:
+                continue
+            if self.rc[p] <= 0:
+                raise PoolError("page %d released more often than held" % p)
+            self.rc[p] -= 1
+            if self.rc[p] == 0:
+                self.free.append(p)
+
+    def gather(self, table) -> np.ndarray:
+        """The bytes a table addresses, in table order (empty slots skipped)."""
+        ids = [p for p in np.asarray(table).reshape(-1).tolist() if p >= 0]
+        return self.data[ids].reshape(-1).copy()
