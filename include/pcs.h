@@ -113,6 +113,7 @@ typedef int32_t pcs_status;
 
 typedef struct pcs_ctx pcs_ctx;
 typedef struct pcs_snapshot pcs_snapshot;
+typedef struct pcs_pool pcs_pool;
 
 /* A runtime buffer to fingerprint: `bytes` bytes at device pointer `ptr`. */
 typedef struct pcs_buf {
@@ -341,6 +342,61 @@ pcs_status pcs_prune_global(pcs_ctx *ctx, const pcs_bank *banks, int32_t n, uint
 pcs_status pcs_budget_plan(const int32_t *n, const uint64_t *entry_bytes, const double *priority,
                            int32_t count, uint64_t budget, double fraction, int32_t *k_out,
                            int32_t *shrinks, int32_t *drops);
+
+/*
+ * Copy-on-write page pool (Sec. 3, I3: fork independence, which the
+ * mechanism realises by copy-on-write; Sec. 3 "Boundary": the runtime owns
+ * allocation and copy-on-write; Sec. 7.3: reference-counted blocks whose copy
+ * leg fires on the first write).  The pool manages n_pages pages of
+ * page_bytes in caller device memory at `base` (the caller keeps owning the
+ * bytes; sessions address the pages through int32 page tables, e.g. RING
+ * sections).  Each page carries the number of table slots that hold it; free
+ * pages sit on a device stack.  Page id -1 marks an empty slot and is skipped
+ * by every call.  Work is enqueued on `stream`; calls on one pool must be
+ * ordered (one stream, or events).  Device-side failures are sticky on the
+ * context and returned by pcs_sync: no free page -> PCS_E_NOMEM (the slot
+ * keeps its shared page, or an alloc slot gets -1); an id outside the pool
+ * -> PCS_E_RANGE (skipped); a page shared, written or released while held
+ * by nobody -> PCS_E_INVAL (skipped).  Pools die with their context.
+ *   base: device, 16-byte aligned; page_bytes: multiple of 16.
+ */
+pcs_status pcs_pool_create(pcs_ctx *ctx, void *base, uint64_t page_bytes, int32_t n_pages,
+                           pcs_pool **out);
+pcs_status pcs_pool_destroy(pcs_ctx *ctx, pcs_pool *pool);
+
+/* n free pages, each held once: ids: device int32[n]. */
+pcs_status pcs_pool_alloc(pcs_ctx *ctx, pcs_pool *pool, int32_t *ids, int32_t n, void *stream);
+
+/*
+ * Fork of the tables holding src: every page of src gains one holder and,
+ * if dst is not NULL, src is copied to dst (the child's table).  No page
+ * bytes move.  src, dst: device int32[n].
+ */
+pcs_status pcs_pool_share(pcs_ctx *ctx, pcs_pool *pool, const int32_t *src, int32_t *dst,
+                          int32_t n, void *stream);
+
+/*
+ * The copy leg, before the caller writes the pages at table[entries[j]]
+ * (j < n; entries NULL: table[0 .. n)): a slot whose page is also held
+ * elsewhere gets a fresh page holding a copy of it and gives up its hold on
+ * the old one; a page held by that slot alone stays.  Of several holders of
+ * one page in one call, all but one copy.  Entries must be distinct.
+ *   table: device int32[n_table] (updated in place); entries: device int32[n].
+ */
+pcs_status pcs_pool_prepare_write(pcs_ctx *ctx, pcs_pool *pool, int32_t *table, int64_t n_table,
+                                  const int32_t *entries, int32_t n, void *stream);
+
+/* Every page of ids loses one holder; pages held by nobody become free. */
+pcs_status pcs_pool_release(pcs_ctx *ctx, pcs_pool *pool, const int32_t *ids, int32_t n,
+                            void *stream);
+
+/*
+ * Synchronises `stream`, then reads the pool's state: free page count; the
+ * holder count of every page (host uint32[n_pages] or NULL); the free pages
+ * (host int32[n_pages] or NULL; the first *free_pages entries are valid).
+ */
+pcs_status pcs_pool_query(pcs_ctx *ctx, pcs_pool *pool, int32_t *free_pages, uint32_t *counts,
+                          int32_t *free_ids, void *stream);
 
 /*
  * Host only: bytes of the PCS1 record a session of these sections packs to:

@@ -405,17 +405,21 @@ def bank_targets(session_id: int, kept_out: np.ndarray, keys_out: np.ndarray,
 
 def kv_session(session_id: int, meta: np.ndarray, k_pool: np.ndarray, v_pool: np.ndarray,
                page_table: np.ndarray, ring_start: int, window: int, page_rows: int,
-               row_bytes: int, ring_start_override: int | None = None) -> SessionSpec:
-    """{META, then K_l, V_l for each layer l}; page_table is int32 [layers][pages]."""
+               row_bytes: int, ring_start_override: int | None = None,
+               v_page_table: np.ndarray | None = None) -> SessionSpec:
+    """{META, then K_l, V_l for each layer l}; page_table is int32 [layers][pages]
+    (of K, and of V unless v_page_table is given)."""
     layers = page_table.shape[0]
+    vt = page_table if v_page_table is None else v_page_table
     sp = SessionSpec(session_id, KIND_KV)
     sp.contig(SEC_META, DT_I64, meta, dim0=meta.size)
     rs = ring_start if ring_start_override is None else ring_start_override
     for l in range(layers):
         pt = np.ascontiguousarray(page_table[l], dtype=np.int32)
+        pv = np.ascontiguousarray(vt[l], dtype=np.int32)
         sp.ring(SEC_K, DT_BF16, k_pool, row_bytes, pt, rs, window, page_rows, layer=l,
                 dim0=window, dim1=row_bytes)
-        sp.ring(SEC_V, DT_BF16, v_pool, row_bytes, pt, rs, window, page_rows, layer=l,
+        sp.ring(SEC_V, DT_BF16, v_pool, row_bytes, pv, rs, window, page_rows, layer=l,
                 dim0=window, dim1=row_bytes)
     return sp
 

@@ -20,6 +20,8 @@ constexpr int kMaxGroupLog2 = 5;         // at most 32 chunks per warp task
 // Errors a kernel records (OR-ed into the context's device error word).
 constexpr uint32_t kDevErrIndex = 1u;    // a row / page id out of range
 constexpr uint32_t kDevErrTimeout = 2u;  // a bounded wait inside a kernel gave up
+constexpr uint32_t kDevErrNoPage = 4u;   // a page pool had no free page
+constexpr uint32_t kDevErrRefcount = 8u; // a page released, shared or written while held by nobody
 
 enum Layout : uint32_t { kContig = 0, kRows = 1, kRing = 2 };
 
@@ -190,6 +192,30 @@ cudaError_t launch_gselect(const GPlan& p, int pass, int sm_count, cudaStream_t 
 // Count per tile and scan (first launch), then write kept indices and bank
 // offsets (second launch).
 cudaError_t launch_gcompact(const GPlan& p, int sm_count, cudaStream_t stream);
+
+// ---- Copy-on-write page pool (pcs_pool_*) ---------------------------------
+// Reference counts and a free stack over caller memory.  A kernel either only
+// takes pages off the stack (alloc, copy leg) or only puts pages back
+// (release), never both, so the stack needs no lock.
+struct PoolDev {
+  uint8_t* base;       // n_pages * page_bytes, caller memory
+  uint32_t* rc;        // [n_pages] table slots holding each page
+  int32_t* free_ids;   // [n_pages] stack of free pages; [0, *top) valid
+  int32_t* top;
+  uint32_t* err;       // the context's error word
+  uint64_t page_bytes; // multiple of 16
+  int32_t n_pages;
+  int32_t pad;
+};
+
+cudaError_t launch_pool_alloc(const PoolDev& p, int32_t* ids, int32_t n, cudaStream_t stream);
+cudaError_t launch_pool_share(const PoolDev& p, const int32_t* src, int32_t* dst, int32_t n,
+                              cudaStream_t stream);
+// The copy leg before a write of table[entries[j]] (j < n; entries NULL: j).
+cudaError_t launch_pool_cow(const PoolDev& p, int32_t* table, int64_t n_table,
+                            const int32_t* entries, int32_t n, int sm_count, cudaStream_t stream);
+cudaError_t launch_pool_release(const PoolDev& p, const int32_t* ids, int32_t n,
+                                cudaStream_t stream);
 
 // Occupancy of the streaming kernel (blocks per SM) for the launch shape.
 int stream_blocks_per_sm();

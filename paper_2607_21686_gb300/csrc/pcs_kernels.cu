@@ -1439,6 +1439,131 @@ __global__ void __launch_bounds__(kThreads) k_gwrite(GPlan p) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// Copy-on-write page pool
+//
+// A page's count is the number of table slots that hold it.  A fork shares
+// pages (count + 1, no bytes move); before a slot's page is written, the copy
+// leg gives the slot a private copy if anybody else still holds the page.
+// Of several holders writing in one launch, the last one to give up its hold
+// finds the count at 1 and keeps the page, so exactly holders - 1 copies are
+// made and no page is lost.  Ids are checked against the pool; -1 is an empty
+// slot and is skipped.
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ bool pool_id_ok(const PoolDev& P, int32_t p) {
+  if (p < 0) return false;
+  if (p >= P.n_pages) {
+    atomicOr(P.err, kDevErrIndex);
+    return false;
+  }
+  return true;
+}
+
+// Take one free page (count 1), or -1 with the error recorded.
+__device__ __forceinline__ int32_t pool_pop(const PoolDev& P) {
+  const int32_t i = atomicSub(P.top, 1);
+  if (i <= 0) {
+    atomicAdd(P.top, 1);
+    atomicOr(P.err, kDevErrNoPage);
+    return -1;
+  }
+  const int32_t q = P.free_ids[i - 1];
+  P.rc[q] = 1;
+  return q;
+}
+
+__global__ void __launch_bounds__(kThreads) k_pool_alloc(PoolDev P, int32_t* ids, int32_t n) {
+  const int32_t j = blockIdx.x * kThreads + threadIdx.x;
+  if (j < n) ids[j] = pool_pop(P);
+}
+
+__global__ void __launch_bounds__(kThreads)
+    k_pool_share(PoolDev P, const int32_t* src, int32_t* dst, int32_t n) {
+  const int32_t j = blockIdx.x * kThreads + threadIdx.x;
+  if (j >= n) return;
+  const int32_t p = src[j];
+  if (dst) dst[j] = p;
+  if (!pool_id_ok(P, p)) return;
+  if (atomicAdd(&P.rc[p], 1u) == 0u) {
+    atomicSub(&P.rc[p], 1u);
+    atomicOr(P.err, kDevErrRefcount);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+    k_pool_release(PoolDev P, const int32_t* ids, int32_t n) {
+  const int32_t j = blockIdx.x * kThreads + threadIdx.x;
+  if (j >= n) return;
+  const int32_t p = ids[j];
+  if (!pool_id_ok(P, p)) return;
+  const uint32_t old = atomicSub(&P.rc[p], 1u);
+  if (old == 1u) {
+    const int32_t i = atomicAdd(P.top, 1);
+    if (i < P.n_pages) {
+      P.free_ids[i] = p;
+    } else {  // counts were inconsistent: never write past the stack
+      atomicSub(P.top, 1);
+      atomicOr(P.err, kDevErrRefcount);
+    }
+  } else if (old == 0u) {
+    atomicAdd(&P.rc[p], 1u);
+    atomicOr(P.err, kDevErrRefcount);
+  }
+}
+
+// One warp per table slot: lane 0 settles the hold, the warp copies the page.
+__global__ void __launch_bounds__(kThreads)
+    k_pool_cow(PoolDev P, int32_t* table, int64_t n_table, const int32_t* entries, int32_t n) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * kWarps;
+  for (int64_t j = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5); j < n;
+       j += warps) {
+    int32_t p = -1, q = -1;
+    int64_t e = 0;
+    if (lane == 0) {
+      e = entries ? static_cast<int64_t>(entries[j]) : j;
+      if (e < 0 || e >= n_table) {
+        atomicOr(P.err, kDevErrIndex);
+      } else {
+        p = table[e];
+        if (pool_id_ok(P, p)) {
+          const uint32_t old = atomicSub(&P.rc[p], 1u);
+          if (old == 1u) {
+            atomicAdd(&P.rc[p], 1u);  // held here alone: keep it
+          } else if (old == 0u) {
+            atomicAdd(&P.rc[p], 1u);
+            atomicOr(P.err, kDevErrRefcount);
+          } else {
+            q = pool_pop(P);
+            if (q < 0) atomicAdd(&P.rc[p], 1u);  // no page: keep the shared hold
+          }
+        }
+      }
+    }
+    q = __shfl_sync(kFull, q, 0);
+    if (q < 0) continue;
+    p = __shfl_sync(kFull, p, 0);
+    const uint4* src = reinterpret_cast<const uint4*>(P.base + static_cast<uint64_t>(p) * P.page_bytes);
+    uint4* dst = reinterpret_cast<uint4*>(P.base + static_cast<uint64_t>(q) * P.page_bytes);
+    const uint64_t words = P.page_bytes / 16;
+    for (uint64_t k0 = lane; k0 < words; k0 += 32 * 8) {
+      uint4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const uint64_t k = k0 + 32u * u;
+        if (k < words) v[u] = __ldcs(src + k);
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const uint64_t k = k0 + 32u * u;
+        if (k < words) dst[k] = v[u];
+      }
+    }
+    if (lane == 0) table[e] = q;
+  }
+}
+
 template <int MODE>
 int occupancy() {
   int b = 0;
@@ -1614,6 +1739,38 @@ cudaError_t launch_gselect(const GPlan& p, int pass, int sm_count, cudaStream_t 
   if (p.tiles <= 0) return cudaSuccess;
   if (p.uniform) k_gselect<true><<<gblocks(p, sm_count), kThreads, 0, stream>>>(p, pass);
   else k_gselect<false><<<gblocks(p, sm_count), kThreads, 0, stream>>>(p, pass);
+  return cudaGetLastError();
+}
+
+static unsigned grid_for(int64_t n) { return static_cast<unsigned>((n + kThreads - 1) / kThreads); }
+
+cudaError_t launch_pool_alloc(const PoolDev& p, int32_t* ids, int32_t n, cudaStream_t stream) {
+  if (n <= 0) return cudaSuccess;
+  k_pool_alloc<<<grid_for(n), kThreads, 0, stream>>>(p, ids, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pool_share(const PoolDev& p, const int32_t* src, int32_t* dst, int32_t n,
+                              cudaStream_t stream) {
+  if (n <= 0) return cudaSuccess;
+  k_pool_share<<<grid_for(n), kThreads, 0, stream>>>(p, src, dst, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pool_release(const PoolDev& p, const int32_t* ids, int32_t n,
+                                cudaStream_t stream) {
+  if (n <= 0) return cudaSuccess;
+  k_pool_release<<<grid_for(n), kThreads, 0, stream>>>(p, ids, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pool_cow(const PoolDev& p, int32_t* table, int64_t n_table,
+                            const int32_t* entries, int32_t n, int sm_count, cudaStream_t stream) {
+  if (n <= 0) return cudaSuccess;
+  const int64_t want = (static_cast<int64_t>(n) + kWarps - 1) / kWarps;
+  const int64_t cap = static_cast<int64_t>(sm_count) * 8;
+  k_pool_cow<<<static_cast<unsigned>(want < cap ? want : cap), kThreads, 0, stream>>>(
+      p, table, n_table, entries, n);
   return cudaGetLastError();
 }
 

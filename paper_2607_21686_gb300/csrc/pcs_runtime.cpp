@@ -313,6 +313,11 @@ struct pcs_snapshot {
   uint8_t* record() const { return block->ptr + offset; }
 };
 
+struct pcs_pool {
+  pcs::PoolDev d{};
+  void* meta = nullptr;  // counts, free stack and top in one allocation
+};
+
 struct pcs_ctx {
   int device = 0;
   int sm_count = 0;
@@ -345,8 +350,9 @@ struct pcs_ctx {
   };
   std::vector<Timed> timed;
   std::vector<cudaEvent_t> timing_events;  // free timing-capable events
-  double kernel_ms[16] = {};
-  uint64_t kernel_n[16] = {};
+  double kernel_ms[32] = {};
+  uint64_t kernel_n[32] = {};
+  std::unordered_set<pcs_pool*> pools;  // live page pools
 };
 
 namespace {
@@ -362,13 +368,16 @@ pcs_status set_device(pcs_ctx* c) {
 enum KernelKind {
   kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
   kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKBulkHash, kKBulkPack,
-  kKBulkRestore, kKBulkRestoreV, kKReduce, kKGSelect, kKGCompact, kKernelKinds
+  kKBulkRestore, kKBulkRestoreV, kKReduce, kKGSelect, kKGCompact, kKPoolAlloc, kKPoolShare,
+  kKPoolCow, kKPoolRelease, kKernelKinds
 };
+static_assert(kKernelKinds <= 32, "kernel timing table");
 const char* kKernelNames[kKernelKinds] = {
     "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
     "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
-    "k_reduce_nodes", "k_gselect", "k_gcompact"};
+    "k_reduce_nodes", "k_gselect", "k_gcompact", "k_pool_alloc", "k_pool_share", "k_pool_cow",
+    "k_pool_release"};
 
 cudaEvent_t timing_event(pcs_ctx* c) {
   if (!c->timing_events.empty()) {
@@ -914,6 +923,11 @@ pcs_status pcs_destroy(pcs_ctx* c) {
       delete h;
     }
     c->live.clear();
+    for (auto* pl : c->pools) {
+      cudaFree(pl->meta);
+      delete pl;
+    }
+    c->pools.clear();
     c->ws_busy.reset();
     if (c->ws) cudaFree(c->ws);
     if (c->words) cudaFree(c->words);
@@ -1005,6 +1019,12 @@ pcs_status pcs_sync(pcs_ctx* c, void* stream) {
     PCS_CUDA(cudaMemset(c->words, 0, 4));
     if (w & kDevErrTimeout)
       return fail(PCS_E_TIMEOUT, "a bounded wait inside a kernel gave up (error bits 0x%x)", w);
+    if (w & kDevErrNoPage)
+      return fail(PCS_E_NOMEM, "a page pool had no free page (error bits 0x%x)", w);
+    if (w & kDevErrRefcount)
+      return fail(PCS_E_INVAL,
+                  "a pool page was shared, written or released while held by nobody "
+                  "(error bits 0x%x)", w);
     return fail(PCS_E_RANGE, "a kernel met a row or page id out of range (error bits 0x%x)", w);
   }
   return PCS_OK;
@@ -1940,6 +1960,140 @@ pcs_status pcs_snapshot_read_file(pcs_ctx* c, const char* path, uint32_t placeme
   for (auto& e : h->table) e.fp = 0;
   *out = h.release();
   c->live.insert(*out);
+  return PCS_OK;
+}
+
+// ---- Copy-on-write page pool -------------------------------------------------
+
+pcs_status pcs_pool_create(pcs_ctx* c, void* base, uint64_t page_bytes, int32_t n_pages,
+                           pcs_pool** out) {
+  if (!c || !out) return fail(PCS_E_INVAL, "bad arguments");
+  *out = nullptr;
+  if (n_pages <= 0) return fail(PCS_E_INVAL, "n_pages must be positive");
+  if (!base) return fail(PCS_E_INVAL, "base is null");
+  if (page_bytes == 0 || page_bytes % 16 != 0 || !aligned16(base))
+    return fail(PCS_E_ALIGN, "page_bytes and base must be non-zero multiples of 16");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  auto pl = std::make_unique<pcs_pool>();
+  const uint64_t n = static_cast<uint64_t>(n_pages);
+  const uint64_t bytes = 8 * n + 256;
+  PCS_CUDA(cudaMalloc(&pl->meta, bytes));
+  auto* m = static_cast<uint8_t*>(pl->meta);
+  pl->d.base = static_cast<uint8_t*>(base);
+  pl->d.rc = reinterpret_cast<uint32_t*>(m);
+  pl->d.free_ids = reinterpret_cast<int32_t*>(m + 4 * n);
+  pl->d.top = reinterpret_cast<int32_t*>(m + 8 * n);
+  pl->d.err = c->words;
+  pl->d.page_bytes = page_bytes;
+  pl->d.n_pages = n_pages;
+  // All pages free; the stack hands out the lowest ids first.
+  std::vector<int32_t> init(n + 1);
+  for (uint64_t i = 0; i < n; ++i) init[i] = static_cast<int32_t>(n - 1 - i);
+  init[n] = n_pages;
+  cudaError_t e = cudaMemset(pl->d.rc, 0, 4 * n);
+  if (e == cudaSuccess) e = cudaMemcpy(pl->d.free_ids, init.data(), 4 * (n + 1), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    cudaFree(pl->meta);
+    return cuda_fail(e, "pcs_pool_create");
+  }
+  *out = pl.release();
+  c->pools.insert(*out);
+  return PCS_OK;
+}
+
+pcs_status pcs_pool_destroy(pcs_ctx* c, pcs_pool* pl) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  if (!pl) return PCS_OK;
+  std::lock_guard<std::mutex> lk(c->mu);
+  if (!c->pools.count(pl)) return fail(PCS_E_HANDLE, "not a live pool of this context");
+  pcs_status st = set_device(c);
+  if (st) return st;
+  c->pools.erase(pl);
+  PCS_CUDA(cudaDeviceSynchronize());
+  cudaFree(pl->meta);
+  delete pl;
+  return PCS_OK;
+}
+
+namespace {
+
+pcs_status pool_check(pcs_ctx* c, pcs_pool* pl) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  if (!pl || !c->pools.count(pl)) return fail(PCS_E_HANDLE, "not a live pool of this context");
+  return set_device(c);
+}
+
+}  // namespace
+
+pcs_status pcs_pool_alloc(pcs_ctx* c, pcs_pool* pl, int32_t* ids, int32_t n, void* stream) {
+  if (n < 0 || (n > 0 && !ids)) return fail(PCS_E_INVAL, "bad arguments");
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = pool_check(c, pl);
+  if (st) return st;
+  if (n == 0) return PCS_OK;
+  LaunchScope ls(c, kKPoolAlloc, static_cast<cudaStream_t>(stream));
+  PCS_CUDA(launch_pool_alloc(pl->d, ids, n, static_cast<cudaStream_t>(stream)));
+  return PCS_OK;
+}
+
+pcs_status pcs_pool_share(pcs_ctx* c, pcs_pool* pl, const int32_t* src, int32_t* dst, int32_t n,
+                          void* stream) {
+  if (n < 0 || (n > 0 && !src)) return fail(PCS_E_INVAL, "bad arguments");
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = pool_check(c, pl);
+  if (st) return st;
+  if (n == 0) return PCS_OK;
+  LaunchScope ls(c, kKPoolShare, static_cast<cudaStream_t>(stream));
+  PCS_CUDA(launch_pool_share(pl->d, src, dst, n, static_cast<cudaStream_t>(stream)));
+  return PCS_OK;
+}
+
+pcs_status pcs_pool_prepare_write(pcs_ctx* c, pcs_pool* pl, int32_t* table, int64_t n_table,
+                                  const int32_t* entries, int32_t n, void* stream) {
+  if (n < 0 || n_table < 0 || (n > 0 && !table)) return fail(PCS_E_INVAL, "bad arguments");
+  if (!entries && n > n_table) return fail(PCS_E_INVAL, "n exceeds the table");
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = pool_check(c, pl);
+  if (st) return st;
+  if (n == 0) return PCS_OK;
+  LaunchScope ls(c, kKPoolCow, static_cast<cudaStream_t>(stream));
+  PCS_CUDA(launch_pool_cow(pl->d, table, n_table, entries, n, c->sm_count,
+                           static_cast<cudaStream_t>(stream)));
+  return PCS_OK;
+}
+
+pcs_status pcs_pool_release(pcs_ctx* c, pcs_pool* pl, const int32_t* ids, int32_t n, void* stream) {
+  if (n < 0 || (n > 0 && !ids)) return fail(PCS_E_INVAL, "bad arguments");
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = pool_check(c, pl);
+  if (st) return st;
+  if (n == 0) return PCS_OK;
+  LaunchScope ls(c, kKPoolRelease, static_cast<cudaStream_t>(stream));
+  PCS_CUDA(launch_pool_release(pl->d, ids, n, static_cast<cudaStream_t>(stream)));
+  return PCS_OK;
+}
+
+pcs_status pcs_pool_query(pcs_ctx* c, pcs_pool* pl, int32_t* free_pages, uint32_t* counts,
+                          int32_t* free_ids, void* stream) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = pool_check(c, pl);
+  if (st) return st;
+  PCS_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  int32_t top = 0;
+  PCS_CUDA(cudaMemcpy(&top, pl->d.top, 4, cudaMemcpyDeviceToHost));
+  if (free_pages) *free_pages = top;
+  const uint64_t n = static_cast<uint64_t>(pl->d.n_pages);
+  if (counts) PCS_CUDA(cudaMemcpy(counts, pl->d.rc, 4 * n, cudaMemcpyDeviceToHost));
+  if (free_ids && top > 0)
+    PCS_CUDA(cudaMemcpy(free_ids, pl->d.free_ids, 4ull * std::min<uint64_t>(top, n),
+                        cudaMemcpyDeviceToHost));
   return PCS_OK;
 }
 

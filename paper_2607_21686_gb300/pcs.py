@@ -19,6 +19,7 @@ import ctypes
 import os
 import threading
 
+import numpy as np
 import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -145,6 +146,13 @@ SIGNATURES = {
     "pcs_snapshot_copy_out": (_st, [_vp, _vp, _u64, _u64, _vp, _vp]),
     "pcs_snapshot_write_file": (_st, [_vp, _vp, ctypes.c_char_p]),
     "pcs_snapshot_read_file": (_st, [_vp, ctypes.c_char_p, _u32, ctypes.POINTER(_vp)]),
+    "pcs_pool_create": (_st, [_vp, _vp, _u64, _i32, ctypes.POINTER(_vp)]),
+    "pcs_pool_destroy": (_st, [_vp, _vp]),
+    "pcs_pool_alloc": (_st, [_vp, _vp, _vp, _i32, _vp]),
+    "pcs_pool_share": (_st, [_vp, _vp, _vp, _vp, _i32, _vp]),
+    "pcs_pool_prepare_write": (_st, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _vp]),
+    "pcs_pool_release": (_st, [_vp, _vp, _vp, _i32, _vp]),
+    "pcs_pool_query": (_st, [_vp, _vp, ctypes.POINTER(_i32), _vp, _vp, _vp]),
     "pcs_fingerprint_static": (_st, [ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
 }
 PCS_STATIC_MAX_BUFFERS = 64
@@ -296,14 +304,16 @@ def bank_targets(session_id: int, kept_out: torch.Tensor, keys_out: torch.Tensor
 
 
 def kv_session(session_id: int, meta: torch.Tensor, k_pool: torch.Tensor, v_pool: torch.Tensor,
-               page_table: torch.Tensor, ring_start: int, window: int) -> Session:
-    """page_table: int32 [layers, window / page_rows] of pool page ids."""
+               page_table: torch.Tensor, ring_start: int, window: int,
+               v_page_table: torch.Tensor = None) -> Session:
+    """page_table: int32 [layers, window / page_rows] of pool page ids (of the
+    K pages, and of the V pages too unless v_page_table is given)."""
+    vt = page_table if v_page_table is None else v_page_table
     secs = [contig_section(PCS_SEC_META, meta, dim0=meta.numel())]
     for l in range(page_table.shape[0]):
-        pt = page_table[l]
-        secs.append(ring_section(PCS_SEC_K, k_pool, pt, ring_start, window, layer=l))
-        secs.append(ring_section(PCS_SEC_V, v_pool, pt, ring_start, window, layer=l))
-    return Session(session_id, PCS_KIND_KV, secs, keep=[meta, k_pool, v_pool, page_table])
+        secs.append(ring_section(PCS_SEC_K, k_pool, page_table[l], ring_start, window, layer=l))
+        secs.append(ring_section(PCS_SEC_V, v_pool, vt[l], ring_start, window, layer=l))
+    return Session(session_id, PCS_KIND_KV, secs, keep=[meta, k_pool, v_pool, page_table, vt])
 
 
 # --------------------------------------------------------------------------
@@ -322,6 +332,63 @@ class Snapshot:
 
     def delete(self) -> None:
         self.ctx.delete(self)
+
+
+class Pool:
+    """A copy-on-write page pool over the caller tensor `pages` ([n_pages, ...]).
+
+    Page ids index the first dimension of `pages`; -1 is an empty slot.
+    """
+
+    def __init__(self, ctx: "Context", pages: torch.Tensor):
+        assert pages.is_cuda and pages.is_contiguous() and pages.dim() >= 1
+        self.ctx = ctx
+        self.pages = pages
+        self.n_pages = pages.shape[0]
+        self.page_bytes = pages[0].numel() * pages.element_size()
+        h = ctypes.c_void_p()
+        check(ctx.lib.pcs_pool_create(ctx.h, pages.data_ptr(), self.page_bytes, self.n_pages,
+                                      ctypes.byref(h)), "pcs_pool_create")
+        self.h = h
+
+    def alloc(self, n: int, stream=None) -> torch.Tensor:
+        ids = torch.empty(n, dtype=torch.int32, device=self.pages.device)
+        check(self.ctx.lib.pcs_pool_alloc(self.ctx.h, self.h, _ptr(ids), n, _stream_ptr(stream)),
+              "pcs_pool_alloc")
+        return ids
+
+    def share(self, src: torch.Tensor, dst: torch.Tensor = None, stream=None) -> torch.Tensor:
+        """Fork: the pages of `src` gain a holder; returns the child's table."""
+        if dst is None:
+            dst = torch.empty_like(src)
+        check(self.ctx.lib.pcs_pool_share(self.ctx.h, self.h, _ptr(src), _ptr(dst), src.numel(),
+                                          _stream_ptr(stream)), "pcs_pool_share")
+        return dst
+
+    def prepare_write(self, table: torch.Tensor, entries: torch.Tensor = None, stream=None):
+        n = table.numel() if entries is None else entries.numel()
+        check(self.ctx.lib.pcs_pool_prepare_write(self.ctx.h, self.h, _ptr(table), table.numel(),
+                                                  _ptr(entries), n, _stream_ptr(stream)),
+              "pcs_pool_prepare_write")
+
+    def release(self, ids: torch.Tensor, stream=None):
+        check(self.ctx.lib.pcs_pool_release(self.ctx.h, self.h, _ptr(ids), ids.numel(),
+                                            _stream_ptr(stream)), "pcs_pool_release")
+
+    def query(self, stream=None):
+        """(free page count, holder counts uint32[n_pages], free page ids)."""
+        free = ctypes.c_int32()
+        counts = np.zeros(self.n_pages, dtype=np.uint32)
+        ids = np.zeros(self.n_pages, dtype=np.int32)
+        check(self.ctx.lib.pcs_pool_query(self.ctx.h, self.h, ctypes.byref(free),
+                                          counts.ctypes.data, ids.ctypes.data,
+                                          _stream_ptr(stream)), "pcs_pool_query")
+        return free.value, counts, ids[:free.value].copy()
+
+    def destroy(self):
+        if self.h:
+            check(self.ctx.lib.pcs_pool_destroy(self.ctx.h, self.h), "pcs_pool_destroy")
+            self.h = None
 
 
 class Context:
