@@ -494,7 +494,59 @@ def run_rows(ctx, dev, stream):
                      "paper_context_us": 12.0,
                      "batch_4096_sessions_per_s": round(4096 / (med / 1e3), 1),
                      "batch_GBs": round(4 * 4096 * (196608 + 16) / (med / 1e3) / 1e9, 1)}
+    del obs, rng, batch, barr
+    out["cow_fork"] = measure_cow_fork(ctx, dev, stream, peak)
     return out
+
+
+def measure_cow_fork(ctx, dev, stream, peak):
+    """Copy-on-write fork of the 256 KV sessions: share every K and V page
+    (no bytes move), then the copy leg of each child's first token append
+    (one page per layer and K/V: 12,288 page copies of 32 KiB)."""
+    from paper_2607_21686_gb300 import pcs
+
+    S, layers, per, page_rows = 256, 24, 64, 16
+    live = S * 2 * layers * per
+    spare = S * 2 * layers
+    pages = torch.empty(live + spare, page_rows, 16, 64, dtype=torch.bfloat16, device=dev)
+    pool = pcs.Pool(ctx, pages)
+    parent = pool.alloc(live).view(S, 2, layers, per)
+    g = torch.Generator().manual_seed(7)
+    ring = torch.randint(0, per * page_rows, (S,), generator=g)
+    # The ring page each child writes first, for every layer of K and V.
+    ent = (torch.arange(S)[:, None] * (2 * layers * per) + torch.arange(2 * layers)[None, :] * per
+           + (ring // page_rows)[:, None]).reshape(-1).to(torch.int32).to(dev)
+    child = torch.empty_like(parent)
+    page_bytes = pool.page_bytes
+
+    fork_ms, write_ms = [], []
+    for rep in range(7):
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        e[0].record(stream)
+        pool.share(parent, child)
+        e[1].record(stream)
+        pool.prepare_write(child, ent)
+        e[2].record(stream)
+        pool.release(child)
+        torch.cuda.synchronize()
+        if rep >= 2:
+            fork_ms.append(e[0].elapsed_time(e[1]))
+            write_ms.append(e[1].elapsed_time(e[2]))
+    ctx.sync()
+    free = pool.query()[0]
+    pool.destroy()
+    del pages
+    fork_ms.sort()
+    write_ms.sort()
+    fm, wm = fork_ms[len(fork_ms) // 2], write_ms[len(write_ms) // 2]
+    moved = 2 * ent.numel() * page_bytes
+    return {"population": "256 KV sessions (24 layers, K and V, 64 pages of 32 KiB each) "
+                          "in one page pool",
+            "fork_pages_shared": live, "fork_ms": round(fm, 4),
+            "first_write_pages_copied": int(ent.numel()), "first_write_ms": round(wm, 4),
+            "first_write_GBs": round(moved / (wm / 1e3) / 1e9, 1),
+            "first_write_frac_of_hbm": round(moved / (wm / 1e3) / 1e9 / peak, 4),
+            "pool_free_after": free, "pool_spare": spare}
 
 
 def run_e2e(a, ctx, kv, src, dst, stream, dev):
