@@ -499,3 +499,66 @@ class PagePool:
         """The bytes a table addresses, in table order (empty slots skipped)."""
         ids = [p for p in np.asarray(table).reshape(-1).tolist() if p >= 0]
         return self.data[ids].reshape(-1).copy()
+
+
+# --------------------------------------------------------------------------
+# State versus witness (Sec. 3, "A distinction the implementation forced"):
+# a buffer is PCS iff restore reads it.  Given the byte ranges a restore
+# read, a buffer is "read" iff some read of at least one byte overlaps it.
+# --------------------------------------------------------------------------
+
+def classify_reads(bufs, reads) -> np.ndarray:
+    """bufs, reads: sequences of (address, bytes); returns uint8 flags per buffer."""
+    flags = np.zeros(len(bufs), dtype=np.uint8)
+    for i, (b, nb) in enumerate(bufs):
+        for r, nr in reads:
+            if nb > 0 and nr > 0 and r < b + nb and b < r + nr:
+                flags[i] = 1
+                break
+    return flags
+
+
+# --------------------------------------------------------------------------
+# Discovering PCS by measurement (Sec. 4, procedure FINGERPRINT):
+#   1. necessity: for each component, snapshot all the others, run the probe,
+#      measure D; the component is necessary if D > eps;
+#   2. sufficiency: snapshot exactly the necessary set N; if D <= eps, PCS = N;
+#   3. redundancy fallback: otherwise greedily add the component that most
+#      reduces D until D <= eps;
+#   4. PCS and Derivable = the rest.
+# D here is a count of differing output bytes (eps = 0: byte identity).
+# --------------------------------------------------------------------------
+
+def mismatch(a, b) -> int:
+    """Bytes that differ between a and b, counting every byte past the shorter."""
+    a, b = _bytes_view(a), _bytes_view(b)
+    m = min(a.size, b.size)
+    return int(np.count_nonzero(a[:m] != b[:m])) + abs(a.size - b.size)
+
+
+def discover(k: int, probe, eps: int):
+    """probe(keep: list[bool]) -> D.  Returns (pcs flags, probes run, consistent)."""
+    probes = 0
+
+    def run(keep):
+        nonlocal probes
+        probes += 1
+        return probe(list(keep))
+
+    necessary = []
+    for i in range(k):
+        keep = [j != i for j in range(k)]
+        necessary.append(run(keep) > eps)
+    chosen = list(necessary)
+    d = run(chosen)
+    while d > eps and not all(chosen):
+        best_j, best_d = -1, None
+        for j in range(k):
+            if chosen[j]:
+                continue
+            dj = run([c or (x == j) for x, c in enumerate(chosen)])
+            if best_d is None or dj < best_d:
+                best_j, best_d = j, dj
+        chosen[best_j] = True
+        d = best_d
+    return np.array(chosen, dtype=np.uint8), probes, d <= eps
