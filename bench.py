@@ -398,6 +398,13 @@ def run_rows(ctx, dev, stream):
     out["classify"] = {"population": "200 buffers, log-uniform 64 B..256 MiB, 60 flipped",
                        "bytes_read": tot, "ms": round(med, 3), "GBs": round(gbs, 1),
                        "frac_of_hbm": round(gbs / peak, 4), "flags_match_ground_truth": flips_ok}
+    # The discovery distance on the same pairs: differing bytes of before / after.
+    best, med = _events_ms(lambda: ctx.mismatch(sw.before, sw.after), stream)
+    mm_ok = ctx.mismatch(sw.before, sw.after).cpu().tolist() == [1 if f else 0 for f in sw.flipped]
+    gbs = 2 * tot / (med / 1e3) / 1e9
+    out["mismatch"] = {"population": "the same 200 buffer pairs (before, after)",
+                       "bytes_read": 2 * tot, "ms": round(med, 3), "GBs": round(gbs, 1),
+                       "frac_of_hbm": round(gbs / peak, 4), "counts_match_ground_truth": mm_ok}
     del sw, fp0, must
 
     # a4-a5, a7, a10: 2048 banks, relevance top-k under an 8 GiB host budget,

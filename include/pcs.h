@@ -399,6 +399,50 @@ pcs_status pcs_pool_query(pcs_ctx *ctx, pcs_pool *pool, int32_t *free_pages, uin
                           int32_t *free_ids, void *stream);
 
 /*
+ * Distance for the discovery procedure (Sec. 4: a return-consistency metric
+ * D with tolerance eps; here D counts differing bytes, so eps = 0 is byte
+ * identity): counts[i] = number of byte positions below min(a[i].bytes,
+ * b[i].bytes) where the two buffers differ, plus the difference of their
+ * lengths.  a, b: host arrays of n device buffers (any alignment; 16-byte
+ * aligned pairs take the fast path); counts: device uint64[n].
+ */
+pcs_status pcs_mismatch(pcs_ctx *ctx, const pcs_buf *a, const pcs_buf *b, int32_t n,
+                        uint64_t *counts, void *stream);
+
+/*
+ * State versus witness (Sec. 3, "A distinction the implementation forced":
+ * a buffer is PCS iff restore reads it).  Given the byte ranges a restore
+ * read -- read j covers [addr[j], addr[j] + bytes[j]) -- flags[i] = 1 iff
+ * some read of at least one byte overlaps buffer i (a non-empty buffer).
+ * Buffers may overlap one another.  bufs: host array of n buffers (only ptr
+ * and bytes are used); addr, bytes: device uint64[m]; flags: device uint8[n].
+ */
+pcs_status pcs_classify_reads(pcs_ctx *ctx, const pcs_buf *bufs, int32_t n, const uint64_t *addr,
+                              const uint64_t *bytes, int64_t m, uint8_t *flags, void *stream);
+
+/*
+ * Probe of the discovery procedure: run the leave-and-return trajectory with
+ * exactly the components keep[i] != 0 restored from the snapshot (the others
+ * left to be re-derived), and write the distance D to *distance.  Returns 0,
+ * or non-zero to stop the procedure.
+ */
+typedef int32_t (*pcs_probe_fn)(void *user, const uint8_t *keep, uint64_t *distance);
+
+/*
+ * Host only: discovering PCS by measurement (Sec. 4, procedure
+ * FINGERPRINT) over k components: (1) necessity -- component i is necessary
+ * if D > eps with every component but i restored; (2) sufficiency -- if D <=
+ * eps with exactly the necessary set restored, that set is PCS; (3)
+ * redundancy fallback -- otherwise add, one at a time, the component whose
+ * addition gives the smallest D (ties: lowest index) until D <= eps.
+ *   pcs_out: host uint8[k] (1 = PCS, 0 = derivable); probes: probes run;
+ *   consistent: 1 if the returned set reaches D <= eps (0 if even every
+ *   component does not).  PCS_E_INVAL if the probe fails.
+ */
+pcs_status pcs_discover(int32_t k, pcs_probe_fn probe, void *user, uint64_t eps,
+                        uint8_t *pcs_out, int32_t *probes, int32_t *consistent);
+
+/*
  * Host only: bytes of the PCS1 record a session of these sections packs to:
  * 256-byte aligned header + 64-byte entries, then each payload at a
  * 256-byte aligned offset.

@@ -217,6 +217,34 @@ cudaError_t launch_pool_cow(const PoolDev& p, int32_t* table, int64_t n_table,
 cudaError_t launch_pool_release(const PoolDev& p, const int32_t* ids, int32_t n,
                                 cudaStream_t stream);
 
+// ---- Byte-mismatch distance (pcs_mismatch) --------------------------------
+constexpr uint32_t kMmTile = 16384;  // bytes of each pair per block iteration
+
+struct MmPair {
+  const uint8_t* a;
+  const uint8_t* b;
+  uint64_t bytes;       // bytes compared: min of the two lengths
+  uint32_t vec;         // both 16-byte aligned: 16-byte loads
+  uint32_t pad;
+};
+
+// Pair i owns tiles [tile_begin[i], tile_begin[i+1]); counts[i] += mismatches.
+cudaError_t launch_mismatch(const MmPair* pairs, const uint64_t* tile_begin, int32_t n,
+                            uint64_t tiles, uint64_t* counts, int sm_count, cudaStream_t stream);
+
+// ---- Reads against buffers (pcs_classify_reads) ---------------------------
+// Buffers sorted by start; maxend[i] = max(end[0..i]).
+struct ReadPlan {
+  const uint64_t* start;
+  const uint64_t* end;
+  const uint64_t* maxend;
+  const uint32_t* orig;   // caller index of each sorted buffer
+  int32_t n;
+  int32_t pad;
+};
+cudaError_t launch_classify_reads(const ReadPlan& p, const uint64_t* addr, const uint64_t* bytes,
+                                  int64_t m, uint8_t* flags, cudaStream_t stream);
+
 // Occupancy of the streaming kernel (blocks per SM) for the launch shape.
 int stream_blocks_per_sm();
 

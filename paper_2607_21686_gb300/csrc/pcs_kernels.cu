@@ -1564,6 +1564,103 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// ---------------------------------------------------------------------------
+// Byte-mismatch distance: the count of differing bytes of buffer pairs (the
+// distance D of the discovery procedure at the byte level).  Every block
+// takes 16 KiB tiles of the pairs in turn; 16-byte loads where both buffers
+// are 16-byte aligned, byte loads otherwise.
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t bytes_ne(uint32_t x, uint32_t y) {
+  return __popc(__vcmpne4(x, y)) >> 3;
+}
+
+__global__ void __launch_bounds__(kThreads)
+    k_mismatch(const MmPair* __restrict__ pairs, const uint64_t* __restrict__ tile_begin,
+               int32_t n, uint64_t tiles, uint64_t* counts) {
+  __shared__ uint32_t warp_sum[kWarps];
+  __shared__ int32_t s_pair;
+  for (uint64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
+    if (threadIdx.x == 0) {
+      int lo = 0, hi = n - 1;  // the last pair whose first tile is <= t
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (tile_begin[mid] <= t) lo = mid;
+        else hi = mid - 1;
+      }
+      s_pair = lo;
+    }
+    __syncthreads();
+    const MmPair P = pairs[s_pair];
+    const uint64_t off = (t - tile_begin[s_pair]) * kMmTile;
+    const uint64_t len = P.bytes - off < kMmTile ? P.bytes - off : kMmTile;
+    uint32_t c = 0;
+    if (P.vec) {
+      const uint4* a = reinterpret_cast<const uint4*>(P.a + off);
+      const uint4* b = reinterpret_cast<const uint4*>(P.b + off);
+      const uint32_t words = static_cast<uint32_t>(len / 16);
+      uint4 va[4], vb[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t k = threadIdx.x + u * kThreads;
+        if (k < words) {
+          va[u] = __ldcs(a + k);
+          vb[u] = __ldcs(b + k);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint32_t k = threadIdx.x + u * kThreads;
+        if (k < words)
+          c += bytes_ne(va[u].x, vb[u].x) + bytes_ne(va[u].y, vb[u].y) +
+               bytes_ne(va[u].z, vb[u].z) + bytes_ne(va[u].w, vb[u].w);
+      }
+      for (uint32_t k = words * 16 + threadIdx.x; k < len; k += kThreads)
+        c += P.a[off + k] != P.b[off + k];
+    } else {
+      for (uint32_t k = threadIdx.x; k < len; k += kThreads) c += P.a[off + k] != P.b[off + k];
+    }
+    uint32_t total;
+    block_excl_scan(c, warp_sum, &total);
+    if (threadIdx.x == 0 && total) atomicAdd(reinterpret_cast<unsigned long long*>(counts + s_pair),
+                                             static_cast<unsigned long long>(total));
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Reads against buffers: a buffer is read iff a read of at least one byte
+// overlaps it (state versus witness: restore reads state, not witness).
+// One thread per read; the candidates are the buffers starting before the
+// read ends and, among them, those from the first whose running maximum end
+// passes the read's start.
+// ---------------------------------------------------------------------------
+
+__global__ void __launch_bounds__(kThreads)
+    k_classify_reads(ReadPlan P, const uint64_t* __restrict__ addr,
+                     const uint64_t* __restrict__ bytes, int64_t m, uint8_t* flags) {
+  const int64_t j = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
+  if (j >= m) return;
+  const uint64_t a = addr[j], len = bytes[j];
+  if (len == 0) return;
+  const uint64_t e = a + len < a ? ~0ull : a + len;
+  int lo = 0, hi = P.n;  // hi: first buffer starting at or after e
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (P.start[mid] < e) lo = mid + 1;
+    else hi = mid;
+  }
+  const int end_i = lo;
+  lo = 0;
+  hi = end_i;  // first buffer whose running maximum end exceeds a
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (P.maxend[mid] > a) hi = mid;
+    else lo = mid + 1;
+  }
+  for (int i = lo; i < end_i; ++i)
+    if (P.end[i] > a && P.end[i] > P.start[i]) flags[P.orig[i]] = 1;
+}
+
 template <int MODE>
 int occupancy() {
   int b = 0;
@@ -1771,6 +1868,22 @@ cudaError_t launch_pool_cow(const PoolDev& p, int32_t* table, int64_t n_table,
   const int64_t cap = static_cast<int64_t>(sm_count) * 8;
   k_pool_cow<<<static_cast<unsigned>(want < cap ? want : cap), kThreads, 0, stream>>>(
       p, table, n_table, entries, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mismatch(const MmPair* pairs, const uint64_t* tile_begin, int32_t n,
+                            uint64_t tiles, uint64_t* counts, int sm_count, cudaStream_t stream) {
+  if (tiles == 0 || n <= 0) return cudaSuccess;
+  const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
+  k_mismatch<<<static_cast<unsigned>(tiles < cap ? tiles : cap), kThreads, 0, stream>>>(
+      pairs, tile_begin, n, tiles, counts);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_classify_reads(const ReadPlan& p, const uint64_t* addr, const uint64_t* bytes,
+                                  int64_t m, uint8_t* flags, cudaStream_t stream) {
+  if (m <= 0 || p.n <= 0) return cudaSuccess;
+  k_classify_reads<<<grid_for(m), kThreads, 0, stream>>>(p, addr, bytes, m, flags);
   return cudaGetLastError();
 }
 

@@ -369,7 +369,7 @@ enum KernelKind {
   kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
   kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKBulkHash, kKBulkPack,
   kKBulkRestore, kKBulkRestoreV, kKReduce, kKGSelect, kKGCompact, kKPoolAlloc, kKPoolShare,
-  kKPoolCow, kKPoolRelease, kKernelKinds
+  kKPoolCow, kKPoolRelease, kKMismatch, kKClassifyReads, kKernelKinds
 };
 static_assert(kKernelKinds <= 32, "kernel timing table");
 const char* kKernelNames[kKernelKinds] = {
@@ -377,7 +377,7 @@ const char* kKernelNames[kKernelKinds] = {
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
     "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
     "k_reduce_nodes", "k_gselect", "k_gcompact", "k_pool_alloc", "k_pool_share", "k_pool_cow",
-    "k_pool_release"};
+    "k_pool_release", "k_mismatch", "k_classify_reads"};
 
 cudaEvent_t timing_event(pcs_ctx* c) {
   if (!c->timing_events.empty()) {
@@ -2094,6 +2094,153 @@ pcs_status pcs_pool_query(pcs_ctx* c, pcs_pool* pl, int32_t* free_pages, uint32_
   if (free_ids && top > 0)
     PCS_CUDA(cudaMemcpy(free_ids, pl->d.free_ids, 4ull * std::min<uint64_t>(top, n),
                         cudaMemcpyDeviceToHost));
+  return PCS_OK;
+}
+
+// ---- Discovery: distance, reads, procedure -----------------------------------
+
+pcs_status pcs_mismatch(pcs_ctx* c, const pcs_buf* a, const pcs_buf* b, int32_t n,
+                        uint64_t* counts, void* stream_) {
+  if (!c || n < 0 || (n > 0 && (!a || !b || !counts))) return fail(PCS_E_INVAL, "bad arguments");
+  if (n == 0) return PCS_OK;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::vector<MmPair> pairs(n);
+  std::vector<uint64_t> tb(n + 1), extra(n);
+  uint64_t tiles = 0;
+  for (int i = 0; i < n; ++i) {
+    const uint64_t m = std::min(a[i].bytes, b[i].bytes);
+    if (m > 0 && (!a[i].ptr || !b[i].ptr)) return fail(PCS_E_INVAL, "pair %d: null buffer", i);
+    pairs[i].a = static_cast<const uint8_t*>(a[i].ptr);
+    pairs[i].b = static_cast<const uint8_t*>(b[i].ptr);
+    pairs[i].bytes = m;
+    pairs[i].vec = aligned16(a[i].ptr) && aligned16(b[i].ptr);
+    extra[i] = std::max(a[i].bytes, b[i].bytes) - m;
+    tb[i] = tiles;
+    tiles += (m + kMmTile - 1) / kMmTile;
+  }
+  tb[n] = tiles;
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  const uint64_t o_tb = round_up(sizeof(MmPair) * n, kRecordAlign);
+  const uint64_t o_ex = round_up(o_tb + 8ull * (n + 1), kRecordAlign);
+  const uint64_t total = o_ex + 8ull * n;
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, total, stream, &ws);
+  if (st) return st;
+  c->plan.assign(total, 0);
+  put(c->plan, 0, pairs);
+  put(c->plan, o_tb, tb);
+  put(c->plan, o_ex, extra);
+  PCS_CUDA(plan_copy(c, ws, total, stream));
+  // Counts start at the bytes only one buffer has.
+  PCS_CUDA(cudaMemcpyAsync(counts, ws + o_ex, 8ull * n, cudaMemcpyDeviceToDevice, stream));
+  {
+    LaunchScope ls(c, kKMismatch, stream);
+    PCS_CUDA(launch_mismatch(reinterpret_cast<const MmPair*>(ws),
+                             reinterpret_cast<const uint64_t*>(ws + o_tb), n, tiles, counts,
+                             c->sm_count, stream));
+  }
+  return ws_release(c, stream);
+}
+
+pcs_status pcs_classify_reads(pcs_ctx* c, const pcs_buf* bufs, int32_t n, const uint64_t* addr,
+                              const uint64_t* bytes, int64_t m, uint8_t* flags, void* stream_) {
+  if (!c || n < 0 || m < 0 || (n > 0 && (!bufs || !flags)) || (m > 0 && (!addr || !bytes)))
+    return fail(PCS_E_INVAL, "bad arguments");
+  if (n == 0) return PCS_OK;
+  if (n > 0x7FFFFFFF - 1) return fail(PCS_E_INVAL, "too many buffers");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::vector<uint32_t> ord(n);
+  for (int i = 0; i < n; ++i) ord[i] = static_cast<uint32_t>(i);
+  auto start_of = [&](uint32_t i) { return reinterpret_cast<uint64_t>(bufs[i].ptr); };
+  std::stable_sort(ord.begin(), ord.end(),
+                   [&](uint32_t x, uint32_t y) { return start_of(x) < start_of(y); });
+  std::vector<uint64_t> st_(n), en(n), mx(n);
+  uint64_t run = 0;
+  for (int k = 0; k < n; ++k) {
+    const uint64_t b0 = start_of(ord[k]);
+    const uint64_t len = bufs[ord[k]].bytes;
+    st_[k] = b0;
+    en[k] = b0 + len < b0 ? ~0ull : b0 + len;
+    run = std::max(run, en[k]);
+    mx[k] = run;
+  }
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  const uint64_t o_en = round_up(8ull * n, 256), o_mx = round_up(o_en + 8ull * n, 256);
+  const uint64_t o_or = round_up(o_mx + 8ull * n, 256), total = o_or + 4ull * n;
+  uint8_t* ws = nullptr;
+  st = ws_acquire(c, total, stream, &ws);
+  if (st) return st;
+  c->plan.assign(total, 0);
+  put(c->plan, 0, st_);
+  put(c->plan, o_en, en);
+  put(c->plan, o_mx, mx);
+  put(c->plan, o_or, ord);
+  PCS_CUDA(plan_copy(c, ws, total, stream));
+  PCS_CUDA(cudaMemsetAsync(flags, 0, n, stream));
+  ReadPlan rp{};
+  rp.start = reinterpret_cast<const uint64_t*>(ws);
+  rp.end = reinterpret_cast<const uint64_t*>(ws + o_en);
+  rp.maxend = reinterpret_cast<const uint64_t*>(ws + o_mx);
+  rp.orig = reinterpret_cast<const uint32_t*>(ws + o_or);
+  rp.n = n;
+  if (m > 0) {
+    LaunchScope ls(c, kKClassifyReads, stream);
+    PCS_CUDA(launch_classify_reads(rp, addr, bytes, m, flags, stream));
+  }
+  return ws_release(c, stream);
+}
+
+pcs_status pcs_discover(int32_t k, pcs_probe_fn probe, void* user, uint64_t eps,
+                        uint8_t* pcs_out, int32_t* probes_out, int32_t* consistent) {
+  if (k < 0 || !probe || (k > 0 && !pcs_out)) return fail(PCS_E_INVAL, "bad arguments");
+  int32_t probes = 0;
+  std::vector<uint8_t> keep(std::max(k, 1));
+  auto run = [&](const std::vector<uint8_t>& mask, uint64_t* d) -> pcs_status {
+    ++probes;
+    const int32_t rc = probe(user, mask.data(), d);
+    if (rc != 0) return fail(PCS_E_INVAL, "probe %d returned %d", probes, rc);
+    return PCS_OK;
+  };
+  // 1. necessity: leave one out.
+  std::vector<uint8_t> chosen(std::max(k, 1), 0);
+  for (int i = 0; i < k; ++i) {
+    for (int j = 0; j < k; ++j) keep[j] = j != i;
+    uint64_t d = 0;
+    pcs_status st = run(keep, &d);
+    if (st) return st;
+    chosen[i] = d > eps;
+  }
+  // 2. sufficiency of the necessary set.
+  uint64_t d = 0;
+  pcs_status st = run(chosen, &d);
+  if (st) return st;
+  // 3. redundancy fallback: add the component that most reduces D.
+  while (d > eps) {
+    int best = -1;
+    uint64_t best_d = 0;
+    for (int j = 0; j < k; ++j) {
+      if (chosen[j]) continue;
+      keep = chosen;
+      keep[j] = 1;
+      uint64_t dj = 0;
+      st = run(keep, &dj);
+      if (st) return st;
+      if (best < 0 || dj < best_d) {
+        best = j;
+        best_d = dj;
+      }
+    }
+    if (best < 0) break;  // everything is in and D still exceeds eps
+    chosen[best] = 1;
+    d = best_d;
+  }
+  for (int i = 0; i < k; ++i) pcs_out[i] = chosen[i];
+  if (probes_out) *probes_out = probes;
+  if (consistent) *consistent = d <= eps;
   return PCS_OK;
 }
 

@@ -153,8 +153,15 @@ SIGNATURES = {
     "pcs_pool_prepare_write": (_st, [_vp, _vp, _vp, ctypes.c_int64, _vp, _i32, _vp]),
     "pcs_pool_release": (_st, [_vp, _vp, _vp, _i32, _vp]),
     "pcs_pool_query": (_st, [_vp, _vp, ctypes.POINTER(_i32), _vp, _vp, _vp]),
+    "pcs_mismatch": (_st, [_vp, ctypes.POINTER(pcs_buf), ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
+    "pcs_classify_reads": (_st, [_vp, ctypes.POINTER(pcs_buf), _i32, _vp, _vp, ctypes.c_int64, _vp,
+                                 _vp]),
+    "pcs_discover": (_st, [_i32, _vp, _vp, _u64, ctypes.POINTER(ctypes.c_uint8),
+                           ctypes.POINTER(_i32), ctypes.POINTER(_i32)]),
     "pcs_fingerprint_static": (_st, [ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
 }
+# int32 probe(void* user, const uint8_t* keep, uint64_t* distance)
+PROBE_FN = ctypes.CFUNCTYPE(_i32, _vp, ctypes.POINTER(ctypes.c_uint8), ctypes.POINTER(_u64))
 PCS_STATIC_MAX_BUFFERS = 64
 PCS_STATIC_MAX_NODES = 65536
 
@@ -194,6 +201,34 @@ def budget_plan(n, entry_bytes, budget: int, fraction: float, priority=None):
     check(lib.pcs_budget_plan(na, ea, pa, c, budget, fraction, ko, ctypes.byref(sh),
                               ctypes.byref(dr)), "pcs_budget_plan")
     return list(ko)[:c], sh.value, dr.value
+
+
+def discover(k: int, probe, eps: int = 0):
+    """Sec. 4 discovery over k components; probe(keep: list[bool]) -> D.
+
+    Returns (PCS flags, probes run, consistent).  An exception inside the
+    probe stops the procedure and is raised again here.
+    """
+    lib = load_library()
+    failure = []
+
+    def cb(_user, keep, dist):
+        try:
+            dist[0] = int(probe([bool(keep[i]) for i in range(k)]))
+            return 0
+        except BaseException as ex:  # re-raised below
+            failure.append(ex)
+            return 1
+
+    fn = PROBE_FN(cb)
+    out = (ctypes.c_uint8 * max(k, 1))()
+    probes, ok = ctypes.c_int32(), ctypes.c_int32()
+    st = lib.pcs_discover(k, ctypes.cast(fn, ctypes.c_void_p), None, eps, out,
+                          ctypes.byref(probes), ctypes.byref(ok))
+    if failure:
+        raise failure[0]
+    check(st, "pcs_discover")
+    return [out[i] for i in range(k)], probes.value, bool(ok.value)
 
 
 class PcsError(RuntimeError):
@@ -461,6 +496,27 @@ class Context:
                                     _ptr(fp_after), _ptr(must), _stream_ptr(stream)),
               "pcs_classify")
         return must, fp_after
+
+    def mismatch(self, a, b, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        """Differing bytes of each pair (a[i], b[i]), plus their length difference."""
+        n = len(a)
+        assert len(b) == n
+        if out is None:
+            out = torch.empty(n, dtype=torch.int64, device="cuda:%d" % self.device)
+        check(self.lib.pcs_mismatch(self.h, self._bufs(a), self._bufs(b), n, _ptr(out),
+                                    _stream_ptr(stream)), "pcs_mismatch")
+        return out
+
+    def classify_reads(self, tensors, addr: torch.Tensor, nbytes: torch.Tensor,
+                       flags: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        """1 for each buffer some read [addr, addr + nbytes) overlaps (state), else 0."""
+        n = len(tensors)
+        if flags is None:
+            flags = torch.empty(n, dtype=torch.uint8, device="cuda:%d" % self.device)
+        check(self.lib.pcs_classify_reads(self.h, self._bufs(tensors), n, _ptr(addr),
+                                          _ptr(nbytes), addr.numel(), _ptr(flags),
+                                          _stream_ptr(stream)), "pcs_classify_reads")
+        return flags
 
     # -- prune ---------------------------------------------------------------
     @staticmethod
