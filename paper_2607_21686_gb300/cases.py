@@ -4,6 +4,9 @@
     python -m paper_2607_21686_gb300.cases classify --n 200 --hi-mib 32
     python -m paper_2607_21686_gb300.cases prune --sessions 256
     python -m paper_2607_21686_gb300.cases markov --sessions 4096
+    python -m paper_2607_21686_gb300.cases mismatch --n 200 --hi-mib 32
+    python -m paper_2607_21686_gb300.cases prune_global --sessions 256
+    python -m paper_2607_21686_gb300.cases cow --sessions 64
 
 Each case builds its seeded synthetic population on cuda:0, runs the step
 `--warmup` times, then once more, and prints the device time of that last
@@ -52,7 +55,10 @@ def case_kv(ctx, a, dev):
 def case_classify(ctx, a, dev):
     sw = synth.sweep(n=a.n, hi=a.hi_mib << 20, device=dev)
     fp0 = ctx.fingerprint(sw.before)
-    return _timed(lambda: ctx.classify(sw.after, fp0), a.warmup)
+    arr = ctx.buf_array(sw.after)
+    must = torch.empty(len(sw.after), dtype=torch.uint8, device=dev)
+    fp1 = torch.empty(len(sw.after), dtype=torch.int64, device=dev)
+    return _timed(lambda: ctx.classify(arr, fp0, fp1, must), a.warmup)
 
 
 def case_prune(ctx, a, dev):
@@ -78,7 +84,45 @@ def case_markov(ctx, a, dev):
     return _timed(step, a.warmup)
 
 
-CASES = {"kv": case_kv, "classify": case_classify, "prune": case_prune, "markov": case_markov}
+def case_mismatch(ctx, a, dev):
+    sw = synth.sweep(n=a.n, hi=a.hi_mib << 20, device=dev)
+    b0, b1 = ctx.buf_array(sw.before), ctx.buf_array(sw.after)
+    counts = torch.empty(len(sw.after), dtype=torch.int64, device=dev)
+    return _timed(lambda: ctx.mismatch(b0, b1, counts), a.warmup)
+
+
+def case_prune_global(ctx, a, dev):
+    b = synth.banks_config5(sessions=a.sessions, device=dev)
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(b.sessions)]
+    banks = ctx.banks_array(keys, [b.queries[s] for s in range(b.sessions)], 1024 + 2048)
+    kept = torch.empty(sum(b.n), dtype=torch.int32, device=dev)
+    koff = torch.empty(b.sessions + 1, dtype=torch.int32, device=dev)
+    budget = int(sum(b.n) * 3072 * 0.627)
+    return _timed(lambda: ctx.prune_global(banks, b.sessions, budget, kept, koff), a.warmup)
+
+
+def case_cow(ctx, a, dev):
+    # Every session's K and V pages shared by a fork, then the copy leg of one
+    # page per layer and K/V of each child.
+    S, layers, per = a.sessions, 24, 64
+    live = S * 2 * layers * per
+    pages = torch.empty(live + S * 2 * layers, 16, 16, 64, dtype=torch.bfloat16, device=dev)
+    pool = pcs.Pool(ctx, pages)
+    parent = pool.alloc(live)
+    child = torch.empty_like(parent)
+    ent = (torch.arange(S * 2 * layers) * per + 5).to(torch.int32).to(dev)
+
+    def step():
+        pool.share(parent, child)
+        pool.prepare_write(child, ent)
+        pool.release(child)
+    ms = _timed(step, a.warmup)
+    pool.destroy()
+    return ms
+
+
+CASES = {"kv": case_kv, "classify": case_classify, "prune": case_prune, "markov": case_markov,
+         "mismatch": case_mismatch, "prune_global": case_prune_global, "cow": case_cow}
 
 
 def main():

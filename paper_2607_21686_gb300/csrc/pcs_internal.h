@@ -218,7 +218,7 @@ cudaError_t launch_pool_release(const PoolDev& p, const int32_t* ids, int32_t n,
                                 cudaStream_t stream);
 
 // ---- Byte-mismatch distance (pcs_mismatch) --------------------------------
-constexpr uint32_t kMmTile = 16384;  // bytes of each pair per block iteration
+constexpr uint32_t kMmUnit = 2048;  // bytes of each pair per warp iteration
 
 struct MmPair {
   const uint8_t* a;
@@ -228,9 +228,9 @@ struct MmPair {
   uint32_t pad;
 };
 
-// Pair i owns tiles [tile_begin[i], tile_begin[i+1]); counts[i] += mismatches.
-cudaError_t launch_mismatch(const MmPair* pairs, const uint64_t* tile_begin, int32_t n,
-                            uint64_t tiles, uint64_t* counts, int sm_count, cudaStream_t stream);
+// Pair i owns units [unit_begin[i], unit_begin[i+1]); counts[i] += mismatches.
+cudaError_t launch_mismatch(const MmPair* pairs, const uint64_t* unit_begin, int32_t n,
+                            uint64_t units, uint64_t* counts, int sm_count, cudaStream_t stream);
 
 // ---- Reads against buffers (pcs_classify_reads) ---------------------------
 // Buffers sorted by start; maxend[i] = max(end[0..i]).

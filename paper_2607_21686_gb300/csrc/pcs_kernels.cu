@@ -1575,56 +1575,74 @@ __device__ __forceinline__ uint32_t bytes_ne(uint32_t x, uint32_t y) {
   return __popc(__vcmpne4(x, y)) >> 3;
 }
 
-__global__ void __launch_bounds__(kThreads)
-    k_mismatch(const MmPair* __restrict__ pairs, const uint64_t* __restrict__ tile_begin,
-               int32_t n, uint64_t tiles, uint64_t* counts) {
-  __shared__ uint32_t warp_sum[kWarps];
-  __shared__ int32_t s_pair;
-  for (uint64_t t = blockIdx.x; t < tiles; t += gridDim.x) {
-    if (threadIdx.x == 0) {
-      int lo = 0, hi = n - 1;  // the last pair whose first tile is <= t
-      while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (tile_begin[mid] <= t) lo = mid;
-        else hi = mid - 1;
-      }
-      s_pair = lo;
+// Every warp takes a contiguous range of 2 KiB units of the concatenated
+// pairs, finds the pair of its first unit once and walks forward; its count
+// is reduced across the warp and added to the pair when the pair changes.
+__global__ void __launch_bounds__(kThreads, 4)
+    k_mismatch(const MmPair* __restrict__ pairs, const uint64_t* __restrict__ unit_begin,
+               int32_t n, uint64_t units, uint64_t* counts) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t warps = static_cast<uint64_t>(gridDim.x) * kWarps;
+  const uint64_t w = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+  const uint64_t per = (units + warps - 1) / warps;
+  const uint64_t u0 = w * per;
+  const uint64_t u1 = u0 + per < units ? u0 + per : units;
+  if (u0 >= u1) return;
+  int lo = 0, hi = n - 1;  // the last pair whose first unit is <= u0
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (__ldg(unit_begin + mid) <= u0) lo = mid;
+    else hi = mid - 1;
+  }
+  int pi = lo;
+  MmPair P = pairs[pi];
+  uint64_t pbeg = __ldg(unit_begin + pi), pend = __ldg(unit_begin + pi + 1);
+  uint32_t c = 0;
+  for (uint64_t u = u0; u < u1; ++u) {
+    if (u >= pend) {
+      const uint32_t tot = __reduce_add_sync(kFull, c);
+      if (lane == 0 && tot)
+        atomicAdd(reinterpret_cast<unsigned long long*>(counts + pi),
+                  static_cast<unsigned long long>(tot));
+      c = 0;
+      do {
+        ++pi;
+        pend = __ldg(unit_begin + pi + 1);
+      } while (u >= pend);
+      P = pairs[pi];
+      pbeg = __ldg(unit_begin + pi);
     }
-    __syncthreads();
-    const MmPair P = pairs[s_pair];
-    const uint64_t off = (t - tile_begin[s_pair]) * kMmTile;
-    const uint64_t len = P.bytes - off < kMmTile ? P.bytes - off : kMmTile;
-    uint32_t c = 0;
+    const uint64_t off = (u - pbeg) * kMmUnit;
+    const uint32_t len = static_cast<uint32_t>(P.bytes - off < kMmUnit ? P.bytes - off : kMmUnit);
     if (P.vec) {
       const uint4* a = reinterpret_cast<const uint4*>(P.a + off);
       const uint4* b = reinterpret_cast<const uint4*>(P.b + off);
-      const uint32_t words = static_cast<uint32_t>(len / 16);
+      const uint32_t words = len >> 4;
       uint4 va[4], vb[4];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const uint32_t k = threadIdx.x + u * kThreads;
-        if (k < words) {
-          va[u] = __ldcs(a + k);
-          vb[u] = __ldcs(b + k);
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t x = lane + 32u * k;
+        if (x < words) {
+          va[k] = __ldcs(a + x);
+          vb[k] = __ldcs(b + x);
         }
       }
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const uint32_t k = threadIdx.x + u * kThreads;
-        if (k < words)
-          c += bytes_ne(va[u].x, vb[u].x) + bytes_ne(va[u].y, vb[u].y) +
-               bytes_ne(va[u].z, vb[u].z) + bytes_ne(va[u].w, vb[u].w);
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t x = lane + 32u * k;
+        if (x < words)
+          c += bytes_ne(va[k].x, vb[k].x) + bytes_ne(va[k].y, vb[k].y) +
+               bytes_ne(va[k].z, vb[k].z) + bytes_ne(va[k].w, vb[k].w);
       }
-      for (uint32_t k = words * 16 + threadIdx.x; k < len; k += kThreads)
-        c += P.a[off + k] != P.b[off + k];
+      for (uint32_t x = (words << 4) + lane; x < len; x += 32) c += P.a[off + x] != P.b[off + x];
     } else {
-      for (uint32_t k = threadIdx.x; k < len; k += kThreads) c += P.a[off + k] != P.b[off + k];
+      for (uint32_t x = lane; x < len; x += 32) c += P.a[off + x] != P.b[off + x];
     }
-    uint32_t total;
-    block_excl_scan(c, warp_sum, &total);
-    if (threadIdx.x == 0 && total) atomicAdd(reinterpret_cast<unsigned long long*>(counts + s_pair),
-                                             static_cast<unsigned long long>(total));
   }
+  const uint32_t tot = __reduce_add_sync(kFull, c);
+  if (lane == 0 && tot)
+    atomicAdd(reinterpret_cast<unsigned long long*>(counts + pi),
+              static_cast<unsigned long long>(tot));
 }
 
 // ---------------------------------------------------------------------------
@@ -1871,12 +1889,14 @@ cudaError_t launch_pool_cow(const PoolDev& p, int32_t* table, int64_t n_table,
   return cudaGetLastError();
 }
 
-cudaError_t launch_mismatch(const MmPair* pairs, const uint64_t* tile_begin, int32_t n,
-                            uint64_t tiles, uint64_t* counts, int sm_count, cudaStream_t stream) {
-  if (tiles == 0 || n <= 0) return cudaSuccess;
-  const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
-  k_mismatch<<<static_cast<unsigned>(tiles < cap ? tiles : cap), kThreads, 0, stream>>>(
-      pairs, tile_begin, n, tiles, counts);
+cudaError_t launch_mismatch(const MmPair* pairs, const uint64_t* unit_begin, int32_t n,
+                            uint64_t units, uint64_t* counts, int sm_count, cudaStream_t stream) {
+  if (units == 0 || n <= 0) return cudaSuccess;
+  // One resident wave (four blocks per SM), at least eight units per warp.
+  const uint64_t want = (units + 8 * kWarps - 1) / (8 * kWarps);
+  const uint64_t cap = static_cast<uint64_t>(sm_count) * 4;
+  k_mismatch<<<static_cast<unsigned>(want < cap ? want : cap), kThreads, 0, stream>>>(
+      pairs, unit_begin, n, units, counts);
   return cudaGetLastError();
 }
 

@@ -2116,7 +2116,7 @@ pcs_status pcs_mismatch(pcs_ctx* c, const pcs_buf* a, const pcs_buf* b, int32_t 
     pairs[i].vec = aligned16(a[i].ptr) && aligned16(b[i].ptr);
     extra[i] = std::max(a[i].bytes, b[i].bytes) - m;
     tb[i] = tiles;
-    tiles += (m + kMmTile - 1) / kMmTile;
+    tiles += (m + kMmUnit - 1) / kMmUnit;
   }
   tb[n] = tiles;
   std::lock_guard<std::mutex> lk(c->mu);

@@ -369,6 +369,33 @@ class Snapshot:
         self.ctx.delete(self)
 
 
+_BUF_DTYPE = np.dtype([("ptr", np.uint64), ("bytes", np.uint64), ("dtype", np.uint32),
+                       ("flags", np.uint32)])
+
+
+class BufArray:
+    """pcs_buf[n] describing contiguous tensors (keeps them alive)."""
+
+    def __init__(self, tensors):
+        tensors = list(tensors)
+        n = len(tensors)
+        a = np.zeros(max(n, 1), dtype=_BUF_DTYPE)
+        if n:
+            if not all(t.is_contiguous() for t in tensors):
+                raise ValueError("every buffer must be contiguous")
+            a["ptr"][:n] = [t.data_ptr() if t.numel() else 0 for t in tensors]
+            a["bytes"][:n] = [t.numel() * t.element_size() for t in tensors]
+            a["dtype"][:n] = [_DT_OF_TORCH.get(t.dtype, PCS_DT_RAW) for t in tensors]
+        self.keep = tensors
+        self.arr = a
+        self.n = n
+        self.ptr = a.ctypes.data_as(ctypes.POINTER(pcs_buf))
+        self.ptr._keep = a  # the pointer keeps the array alive
+
+    def __len__(self):
+        return self.n
+
+
 class Pool:
     """A copy-on-write page pool over the caller tensor `pages` ([n_pages, ...]).
 
@@ -469,12 +496,14 @@ class Context:
     # -- fingerprint / classify --------------------------------------------
     @staticmethod
     def _bufs(tensors):
-        arr = (pcs_buf * max(len(tensors), 1))()
-        for i, t in enumerate(tensors):
-            assert t.is_contiguous()
-            arr[i] = pcs_buf(ptr=_ptr(t), bytes=_nbytes(t),
-                             dtype=_DT_OF_TORCH.get(t.dtype, PCS_DT_RAW), flags=0)
-        return arr
+        if isinstance(tensors, BufArray):
+            return tensors.ptr
+        return BufArray(tensors).ptr
+
+    @staticmethod
+    def buf_array(tensors) -> "BufArray":
+        """A prebuilt pcs_buf array for repeated calls on the same tensors."""
+        return BufArray(tensors)
 
     def fingerprint(self, tensors, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
         n = len(tensors)
