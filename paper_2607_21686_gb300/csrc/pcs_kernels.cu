@@ -946,7 +946,7 @@ __device__ __forceinline__ float lane_tree_sum(float v) {
   return v;
 }
 
-constexpr int kScoreIlp = 4;  // entries a warp scores at once
+constexpr int kScoreIlp = 4;  // entries a warp scores at once (the tree below assumes 4)
 
 // Element i (0..7) of a 16-byte segment as fp32 (exact conversion).
 template <int DT>  // 1 = bf16, 0 = fp16
@@ -1007,7 +1007,8 @@ __global__ void __launch_bounds__(kThreads)
           if (t < segs) sq = __fadd_rn(sq, __fmul_rn(qf[j][i], qf[j][i]));
         }
       }
-      qnorm = __fsqrt_rn(lane_tree_sum(sq));
+      // The tree's full sum is lane 0's; every lane finalises an entry below.
+      qnorm = __shfl_sync(kFull, __fsqrt_rn(lane_tree_sum(sq)), 0);
       qbank = b;
     }
     const uint64_t bank_end = b + 1 < n_banks ? __ldg(&banks[b + 1].entry_begin) : n_entries;
@@ -1024,26 +1025,53 @@ __global__ void __launch_bounds__(kThreads)
         kv[q][j] = (q < cnt && t < segs) ? ld_stream(kbase + static_cast<uint64_t>(q) * B.D * 2 + 16 * t)
                                          : make_uint4(0, 0, 0, 0);
       }
+    // v[2q] = q.k and v[2q+1] = k.k of entry q, per lane: both chains step
+    // together in paired fp32 operations (each half rounded on its own, as
+    // the separate multiply and add).
+    static_assert(kScoreIlp == 4, "the transposed tree reduces 4 entries x 2 sums");
+    float v[2 * kScoreIlp];
 #pragma unroll
     for (int q = 0; q < kScoreIlp; ++q) {
-      float sd = 0.f, sk = 0.f;
+      float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
       for (int j = 0; j < SPL; ++j) {
         if (lane + 32 * j < segs) {
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const float ke = seg_elem<DT>(kv[q][j], i);
-            sd = __fadd_rn(sd, __fmul_rn(qf[j][i], ke));
-            sk = __fadd_rn(sk, __fmul_rn(ke, ke));
+            acc = __fadd2_rn(acc, __fmul2_rn(make_float2(qf[j][i], ke), make_float2(ke, ke)));
           }
         }
       }
-      const float d = lane_tree_sum(sd);
-      const float kk = lane_tree_sum(sk);
-      if (lane == 0 && q < cnt) {
-        const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
-        scores[e0 + q] = den == 0.f ? 0.f : __fdiv_rn(d, den);
-      }
+      v[2 * q] = acc.x;
+      v[2 * q + 1] = acc.y;
+    }
+    // The lane tree (s[l] += s[l + d], d = 1 .. 16) of all eight sums at
+    // once: at d = 1, 2, 4 each lane keeps half of its values and adds its
+    // partner's copy of them, so lane l ends with sum 4*(l&1) + 2*(l>>1&1) +
+    // (l>>2&1); d = 8, 16 finish it.  Addition is commutative, so every
+    // partial sum is the one the plain tree forms.
+    const bool b0 = lane & 1, b1 = lane & 2, b2 = lane & 4;
+    float w4[4], w2[2];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float give = b0 ? v[i] : v[4 + i];
+      w4[i] = __fadd_rn(b0 ? v[4 + i] : v[i], __shfl_xor_sync(kFull, give, 1));
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const float give = b1 ? w4[i] : w4[2 + i];
+      w2[i] = __fadd_rn(b1 ? w4[2 + i] : w4[i], __shfl_xor_sync(kFull, give, 2));
+    }
+    float w1 = __fadd_rn(b2 ? w2[1] : w2[0], __shfl_xor_sync(kFull, b2 ? w2[0] : w2[1], 4));
+    w1 = __fadd_rn(w1, __shfl_xor_sync(kFull, w1, 8));
+    w1 = __fadd_rn(w1, __shfl_xor_sync(kFull, w1, 16));
+    // Lanes 0..3 hold q.k of entry 2*(l&1) + (l>>1&1); lane l + 4 its k.k.
+    const float kk = __shfl_down_sync(kFull, w1, 4);
+    const int q = 2 * (lane & 1) + ((lane >> 1) & 1);
+    if (lane < 4 && q < cnt) {
+      const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
+      scores[e0 + q] = den == 0.f ? 0.f : __fdiv_rn(w1, den);
     }
     e0 = e0 + cnt - kScoreIlp;  // the loop adds kScoreIlp: next round starts at e0 + cnt
   }
