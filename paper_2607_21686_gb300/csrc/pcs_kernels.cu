@@ -1501,9 +1501,32 @@ __device__ __forceinline__ int32_t pool_pop(const PoolDev& P) {
   return q;
 }
 
+// Pops aggregated per warp: one atomic on the stack top for the warp's lanes.
 __global__ void __launch_bounds__(kThreads) k_pool_alloc(PoolDev P, int32_t* ids, int32_t n) {
   const int32_t j = blockIdx.x * kThreads + threadIdx.x;
-  if (j < n) ids[j] = pool_pop(P);
+  const int lane = threadIdx.x & 31;
+  const unsigned want = __ballot_sync(kFull, j < n);
+  if (j >= n) return;
+  const int cnt = __popc(want), r = __popc(want & ((1u << lane) - 1u));
+  const int leader = __ffs(want) - 1;
+  int32_t old = 0;
+  if (lane == leader) {
+    old = atomicSub(P.top, cnt);
+    const int32_t ok = old <= 0 ? 0 : (old < cnt ? old : cnt);
+    if (ok < cnt) {
+      atomicAdd(P.top, cnt - ok);
+      atomicOr(P.err, kDevErrNoPage);
+    }
+  }
+  old = __shfl_sync(want, old, leader);
+  const int32_t i = old - 1 - r;
+  if (i >= 0) {
+    const int32_t q = P.free_ids[i];
+    P.rc[q] = 1;
+    ids[j] = q;
+  } else {
+    ids[j] = -1;
+  }
 }
 
 __global__ void __launch_bounds__(kThreads)
@@ -1522,34 +1545,59 @@ __global__ void __launch_bounds__(kThreads)
 __global__ void __launch_bounds__(kThreads)
     k_pool_release(PoolDev P, const int32_t* ids, int32_t n) {
   const int32_t j = blockIdx.x * kThreads + threadIdx.x;
+  const unsigned live = __ballot_sync(kFull, j < n);  // lanes that reach the push
   if (j >= n) return;
   const int32_t p = ids[j];
-  if (!pool_id_ok(P, p)) return;
-  const uint32_t old = atomicSub(&P.rc[p], 1u);
-  if (old == 1u) {
-    const int32_t i = atomicAdd(P.top, 1);
+  bool freed = false;
+  if (pool_id_ok(P, p)) {
+    const uint32_t old = atomicSub(&P.rc[p], 1u);
+    if (old == 1u) {
+      freed = true;
+    } else if (old == 0u) {
+      atomicAdd(&P.rc[p], 1u);
+      atomicOr(P.err, kDevErrRefcount);
+    }
+  }
+  // Pushes aggregated per warp: one atomic on the stack top.
+  const unsigned push = __ballot_sync(live, freed);
+  if (!push) return;
+  const int lane = threadIdx.x & 31;
+  const int leader = __ffs(push) - 1;
+  int32_t i0 = 0;
+  if (lane == leader) i0 = atomicAdd(P.top, __popc(push));
+  i0 = __shfl_sync(live, i0, leader);
+  if (freed) {
+    const int32_t i = i0 + __popc(push & ((1u << lane) - 1u));
     if (i < P.n_pages) {
       P.free_ids[i] = p;
     } else {  // counts were inconsistent: never write past the stack
       atomicSub(P.top, 1);
       atomicOr(P.err, kDevErrRefcount);
     }
-  } else if (old == 0u) {
-    atomicAdd(&P.rc[p], 1u);
-    atomicOr(P.err, kDevErrRefcount);
   }
 }
 
-// One warp per table slot: lane 0 settles the hold, the warp copies the page.
+// One warp per table slot, eight slots per block round: lane 0 of each warp
+// settles its slot's hold; the slots that need a page take them off the free
+// stack with one atomic for the block (over-taking is given back, as in
+// pool_pop); then every warp copies its page, kCowDepth 16-byte loads in
+// flight per lane.
+constexpr int kCowDepth = 8;
+
 __global__ void __launch_bounds__(kThreads)
     k_pool_cow(PoolDev P, int32_t* table, int64_t n_table, const int32_t* entries, int32_t n) {
-  const int lane = threadIdx.x & 31;
-  const int64_t warps = static_cast<int64_t>(gridDim.x) * kWarps;
-  for (int64_t j = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5); j < n;
-       j += warps) {
-    int32_t p = -1, q = -1;
+  __shared__ uint32_t s_need;  // bit w: warp w needs a fresh page
+  __shared__ int32_t s_base;   // stack top before this round's pops
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  for (int64_t j0 = static_cast<int64_t>(blockIdx.x) * kWarps; j0 < n;
+       j0 += static_cast<int64_t>(gridDim.x) * kWarps) {
+    const int64_t j = j0 + wib;
+    int32_t p = -1;
     int64_t e = 0;
-    if (lane == 0) {
+    bool need = false;
+    if (threadIdx.x == 0) s_need = 0;
+    __syncthreads();
+    if (lane == 0 && j < n) {
       e = entries ? static_cast<int64_t>(entries[j]) : j;
       if (e < 0 || e >= n_table) {
         atomicOr(P.err, kDevErrIndex);
@@ -1563,32 +1611,57 @@ __global__ void __launch_bounds__(kThreads)
             atomicAdd(&P.rc[p], 1u);
             atomicOr(P.err, kDevErrRefcount);
           } else {
-            q = pool_pop(P);
-            if (q < 0) atomicAdd(&P.rc[p], 1u);  // no page: keep the shared hold
+            need = true;
+            atomicOr(&s_need, 1u << wib);
           }
         }
       }
     }
-    q = __shfl_sync(kFull, q, 0);
-    if (q < 0) continue;
-    p = __shfl_sync(kFull, p, 0);
-    const uint4* src = reinterpret_cast<const uint4*>(P.base + static_cast<uint64_t>(p) * P.page_bytes);
-    uint4* dst = reinterpret_cast<uint4*>(P.base + static_cast<uint64_t>(q) * P.page_bytes);
-    const uint64_t words = P.page_bytes / 16;
-    for (uint64_t k0 = lane; k0 < words; k0 += 32 * 8) {
-      uint4 v[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const uint64_t k = k0 + 32u * u;
-        if (k < words) v[u] = __ldcs(src + k);
+    __syncthreads();
+    const uint32_t mask = s_need;
+    if (threadIdx.x == 0 && mask) {
+      const int cnt = __popc(mask);
+      const int32_t old = atomicSub(P.top, cnt);
+      const int32_t ok = old <= 0 ? 0 : (old < cnt ? old : cnt);
+      if (ok < cnt) {
+        atomicAdd(P.top, cnt - ok);
+        atomicOr(P.err, kDevErrNoPage);
       }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const uint64_t k = k0 + 32u * u;
-        if (k < words) dst[k] = v[u];
+      s_base = old;
+    }
+    __syncthreads();
+    int32_t q = -1;
+    if (lane == 0 && need) {
+      const int32_t i = s_base - 1 - __popc(mask & ((1u << wib) - 1u));
+      if (i >= 0) {
+        q = P.free_ids[i];
+        P.rc[q] = 1;
+      } else {
+        atomicAdd(&P.rc[p], 1u);  // no page: keep the shared hold
       }
     }
-    if (lane == 0) table[e] = q;
+    q = __shfl_sync(kFull, q, 0);
+    if (q >= 0) {
+      p = __shfl_sync(kFull, p, 0);
+      const uint4* src =
+          reinterpret_cast<const uint4*>(P.base + static_cast<uint64_t>(p) * P.page_bytes);
+      uint4* dst = reinterpret_cast<uint4*>(P.base + static_cast<uint64_t>(q) * P.page_bytes);
+      const uint64_t words = P.page_bytes / 16;
+      for (uint64_t k0 = lane; k0 < words; k0 += 32 * kCowDepth) {
+        uint4 v[kCowDepth];
+#pragma unroll
+        for (int u = 0; u < kCowDepth; ++u) {
+          const uint64_t k = k0 + 32u * u;
+          if (k < words) v[u] = __ldcs(src + k);
+        }
+#pragma unroll
+        for (int u = 0; u < kCowDepth; ++u) {
+          const uint64_t k = k0 + 32u * u;
+          if (k < words) dst[k] = v[u];
+        }
+      }
+      if (lane == 0) table[e] = q;
+    }
   }
 }
 
