@@ -131,10 +131,16 @@ cudaError_t launch_small(int mode, const SecDesc* secs, WorkList wl, int group_l
                          const uint64_t* fp_before, uint8_t* flags, uint32_t* bad, int sm_count,
                          int blocks_per_sm, cudaStream_t stream);
 
+// One level of the node reduction of stream i: count nodes at src, reduced
+// by aligned groups of 32 to ceil(count / 32) nodes at dst.
+struct NodeLevel {
+  uint32_t src, count, dst, pad;
+};
+
 // Streams with many task nodes: reduce each aligned group of 32 nodes of
-// stream i (nodes[task_begin_i ...]) to one node at nodes[fin_begin_i + g].
-// Groups of all streams are numbered by fin_begin - base (monotone).
-cudaError_t launch_reduce_nodes(const SecDesc* secs, int n_secs, uint64_t* nodes, uint32_t base,
+// stream i (nodes[lv[i].src ...]) to one node at nodes[lv[i].dst + g].
+// Groups of all streams are numbered by dst - base (monotone).
+cudaError_t launch_reduce_nodes(const NodeLevel* lv, int n_secs, uint64_t* nodes, uint32_t base,
                                 uint32_t n_groups, int sm_count, cudaStream_t stream);
 
 // Section fps from the nodes [fin_begin, fin_begin + fin_count) (in place), then per mode:

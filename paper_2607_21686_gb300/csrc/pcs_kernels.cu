@@ -740,9 +740,9 @@ __device__ __forceinline__ uint64_t stream_fp(const SecDesc& s, uint64_t* nodes,
   return fmix(root ^ (s.bytes * kP));
 }
 
-// One warp per aligned group of 32 task nodes of one stream.
+// One warp per aligned group of 32 nodes of one stream (one reduction level).
 __global__ void __launch_bounds__(kThreads)
-    k_reduce_nodes(const SecDesc* __restrict__ secs, int n_secs, uint64_t* nodes, uint32_t base,
+    k_reduce_nodes(const NodeLevel* __restrict__ lv, int n_secs, uint64_t* nodes, uint32_t base,
                    uint32_t n_groups) {
   const int lane = threadIdx.x & 31;
   const uint32_t nw = gridDim.x * kWarps;
@@ -750,15 +750,15 @@ __global__ void __launch_bounds__(kThreads)
     int lo = 0, hi = n_secs - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (__ldg(&secs[mid].fin_begin) - base <= g) lo = mid;
+      if (__ldg(&lv[mid].dst) - base <= g) lo = mid;
       else hi = mid - 1;
     }
-    const SecDesc& s = secs[lo];
-    const uint32_t local = g - (s.fin_begin - base);
-    const uint32_t n = min(32u, s.n_tasks - 32u * local);
-    const uint64_t v = lane < static_cast<int>(n) ? nodes[s.task_begin + 32u * local + lane] : 0;
+    const NodeLevel L = lv[lo];
+    const uint32_t local = g - (L.dst - base);
+    const uint32_t n = min(32u, L.count - 32u * local);
+    const uint64_t v = lane < static_cast<int>(n) ? nodes[L.src + 32u * local + lane] : 0;
     const uint64_t r = warp_tree(v, static_cast<int>(n), lane);
-    if (lane == 0) nodes[s.fin_begin + local] = r;
+    if (lane == 0) nodes[L.dst + local] = r;
   }
 }
 
@@ -1907,13 +1907,13 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
   return cudaGetLastError();
 }
 
-cudaError_t launch_reduce_nodes(const SecDesc* secs, int n_secs, uint64_t* nodes, uint32_t base,
+cudaError_t launch_reduce_nodes(const NodeLevel* lv, int n_secs, uint64_t* nodes, uint32_t base,
                                 uint32_t n_groups, int sm_count, cudaStream_t stream) {
   if (n_groups == 0) return cudaSuccess;
   const uint64_t want = (static_cast<uint64_t>(n_groups) + kWarps - 1) / kWarps;
   const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
   const int blocks = static_cast<int>(want < cap ? want : cap);
-  k_reduce_nodes<<<blocks, kThreads, 0, stream>>>(secs, n_secs, nodes, base, n_groups);
+  k_reduce_nodes<<<blocks, kThreads, 0, stream>>>(lv, n_secs, nodes, base, n_groups);
   return cudaGetLastError();
 }
 

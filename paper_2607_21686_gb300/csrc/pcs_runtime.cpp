@@ -653,6 +653,10 @@ struct StreamPlan {
   uint64_t nodes = 0;          // task nodes
   uint32_t reduce_groups = 0;  // 32-to-1 groups reduced before finalising (0 = none)
   uint64_t nodes_total = 0;    // task nodes + reduced nodes
+  // Reduction levels: levels[k * n_streams + i] for stream i at level k,
+  // with level_groups[k] groups numbered from level_base[k].
+  std::vector<NodeLevel> levels;
+  std::vector<uint32_t> level_groups, level_base;
   int glog2 = 0;
 };
 
@@ -706,18 +710,36 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   P.reg_tasks = static_cast<uint32_t>(tr);
   P.nodes = node;
   // A stream with many task nodes would leave one finalising warp a long
-  // serial tree: reduce aligned groups of 32 nodes across the GPU first.
-  uint64_t max_tasks = 0;
-  for (const auto& x : d) max_tasks = std::max<uint64_t>(max_tasks, x.n_tasks);
-  uint64_t groups = 0;
+  // serial tree: reduce aligned groups of 32 nodes across the GPU, level by
+  // level, until no stream has more than 32 nodes left.  Aligned groups of
+  // 32^k nodes reduce to the nodes of the global pairwise tree.
   for (auto& x : d) {
-    if (allow_reduce && max_tasks > 64) {
-      x.fin_begin = static_cast<uint32_t>(node + groups);
-      x.fin_count = (x.n_tasks + 31) / 32;
-      groups += x.fin_count;
-    } else {
-      x.fin_begin = x.task_begin;
-      x.fin_count = x.n_tasks;
+    x.fin_begin = x.task_begin;
+    x.fin_count = x.n_tasks;
+  }
+  uint64_t max_count = 0;
+  for (const auto& x : d) max_count = std::max<uint64_t>(max_count, x.n_tasks);
+  uint64_t groups = 0;
+  if (allow_reduce && max_count > 64) {
+    while (max_count > 32) {
+      const uint64_t level_base = node + groups;
+      uint64_t level_groups = 0;
+      max_count = 0;
+      for (auto& x : d) {
+        NodeLevel L{};
+        L.src = x.fin_begin;
+        L.count = x.fin_count;
+        L.dst = static_cast<uint32_t>(level_base + level_groups);
+        const uint32_t out = (x.fin_count + 31) / 32;
+        level_groups += out;
+        x.fin_begin = L.dst;
+        x.fin_count = out;
+        max_count = std::max<uint64_t>(max_count, out);
+        P.levels.push_back(L);
+      }
+      P.level_base.push_back(static_cast<uint32_t>(level_base));
+      P.level_groups.push_back(static_cast<uint32_t>(level_groups));
+      groups += level_groups;
     }
   }
   P.reduce_groups = static_cast<uint32_t>(groups);
@@ -738,7 +760,7 @@ bool fused_ok(const std::vector<char>& bulk, bool small, int n_items) {
 
 // Workspace offsets of a stream plan's lists, after `base` bytes.
 struct ListLayout {
-  uint64_t bulk_ids, bulk_begin, reg_ids, reg_begin, end;
+  uint64_t bulk_ids, bulk_begin, reg_ids, reg_begin, levels, end;
 };
 
 ListLayout list_layout(const StreamPlan& P, uint64_t base) {
@@ -747,7 +769,8 @@ ListLayout list_layout(const StreamPlan& P, uint64_t base) {
   L.bulk_begin = L.bulk_ids + 4 * P.bulk_ids.size();
   L.reg_ids = L.bulk_begin + 4 * P.bulk_begin.size();
   L.reg_begin = L.reg_ids + 4 * P.reg_ids.size();
-  L.end = L.reg_begin + 4 * P.reg_begin.size();
+  L.levels = round_up(L.reg_begin + 4 * P.reg_begin.size(), 16);
+  L.end = L.levels + sizeof(NodeLevel) * P.levels.size();
   return L;
 }
 
@@ -761,6 +784,7 @@ void put_lists(std::vector<uint8_t>& plan, const StreamPlan& P, const ListLayout
   put(plan, L.bulk_begin, P.bulk_begin);
   put(plan, L.reg_ids, P.reg_ids);
   put(plan, L.reg_begin, P.reg_begin);
+  put(plan, L.levels, P.levels);
 }
 
 // Launch both streaming kernels of a plan (TMA-staged first).
@@ -848,9 +872,13 @@ cudaError_t launch_streams(pcs_ctx* c, int mode, const SecDesc* dsecs, const Str
     if (e != cudaSuccess) return e;
   }
   if (nodes && P.reduce_groups) {
-    LaunchScope ls(c, kKReduce, stream);
-    e = launch_reduce_nodes(dsecs, static_cast<int>(P.bulk_ids.size() + P.reg_ids.size()), nodes,
-                            static_cast<uint32_t>(P.nodes), P.reduce_groups, c->sm_count, stream);
+    const int n_streams = static_cast<int>(P.bulk_ids.size() + P.reg_ids.size());
+    const auto* lv = reinterpret_cast<const NodeLevel*>(ws + L.levels);
+    for (size_t k = 0; k < P.level_groups.size() && e == cudaSuccess; ++k) {
+      LaunchScope ls(c, kKReduce, stream);
+      e = launch_reduce_nodes(lv + k * n_streams, n_streams, nodes, P.level_base[k],
+                              P.level_groups[k], c->sm_count, stream);
+    }
   }
   return e;
 }
