@@ -1284,12 +1284,20 @@ __global__ void __launch_bounds__(kThreads) k_gselect(GPlan p, int pass) {
     const uint64_t end = start + kGTile < p.entries ? start + kGTile : p.entries;
     int b = p.tile_bank[t];
     const int hi = p.tile_bank[t + 1];
-#pragma unroll 4
-    for (int j = 0; j < kGTile / kThreads; ++j) {
+    // Every load of the tile in flight before any is used.
+    constexpr int kPer = kGTile / kThreads;
+    float sv[kPer];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
+      sv[j] = i < end ? __ldg(p.scores + i) : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
       const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
       uint32_t d = 256;  // not a candidate
       if (i < end) {
-        const uint64_t key = gkey(p.scores, i);
+        const uint64_t key = (static_cast<uint64_t>(ord32(sv[j])) << 32) | (0xFFFFFFFFull - i);
         if ((key & mask) == prefix) d = static_cast<uint32_t>(key >> shift) & 255u;
       }
       if (UNIFORM) {
@@ -1406,7 +1414,11 @@ __global__ void __launch_bounds__(kThreads) k_gcount(GPlan p) {
     const uint64_t start = static_cast<uint64_t>(t) * kGTile;
     const uint64_t end = start + kGTile < p.entries ? start + kGTile : p.entries;
     uint32_t c = 0;
-    for (uint64_t i = start + threadIdx.x; i < end; i += kThreads) c += gkey(p.scores, i) > T;
+#pragma unroll
+    for (int j = 0; j < kGTile / kThreads; ++j) {
+      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
+      if (i < end) c += gkey(p.scores, i) > T;
+    }
     uint32_t total;
     block_excl_scan(c, warp_sum, &total);
     if (threadIdx.x == 0) p.tile_cnt[t] = total;
@@ -1446,10 +1458,18 @@ __global__ void __launch_bounds__(kThreads) k_gwrite(GPlan p) {
     uint32_t base = p.tile_cnt[t];
     int b = p.tile_bank[t];
     const int hi = p.tile_bank[t + 1];
-    for (int j = 0; j < kGTile / kThreads; ++j) {
+    constexpr int kPer = kGTile / kThreads;
+    bool kp[kPer];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
+      kp[j] = i < end && gkey(p.scores, i) > T;
+    }
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
       const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
       const bool valid = i < end;
-      const bool keep = valid && gkey(p.scores, i) > T;
+      const bool keep = kp[j];
       uint32_t total;
       const uint32_t r = block_rank(keep, warp_cnt, &total);
       if (valid) {

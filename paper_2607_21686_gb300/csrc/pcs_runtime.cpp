@@ -459,7 +459,7 @@ pcs_status ws_acquire(pcs_ctx* c, uint64_t bytes, cudaStream_t stream, uint8_t**
   return PCS_OK;
 }
 
-constexpr uint64_t kPlanSlotBytes = 64 << 10;
+constexpr uint64_t kPlanSlotBytes = 256 << 10;  // per-call plans up to here copy asynchronously
 constexpr int kPlanSlots = 8;
 
 // Copy the call's descriptors (c->plan, `bytes`) into the workspace.  Small
