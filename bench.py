@@ -664,14 +664,22 @@ def run_e2e(a, ctx, kv, src, dst, stream, dev):
     copy_s = torch.cuda.Stream(device=dev)
     ready = [torch.cuda.Event(), torch.cuda.Event()]
     free = [torch.cuda.Event(), torch.cuda.Event()]
+    copy_marks = []  # (start, end) events of each step's copy, timed runs only
 
-    def h2d(i):
+    def h2d(i, mark=False):
         b = i % 2
         copy_s.wait_event(free[b])
+        if mark:
+            m0 = torch.cuda.Event(enable_timing=True)
+            m0.record(copy_s)
         with torch.cuda.stream(copy_s):
             pools[b][0].copy_(kh, non_blocking=True)
             pools[b][1].copy_(vh, non_blocking=True)
         ready[b].record(copy_s)
+        if mark:
+            m1 = torch.cuda.Event(enable_timing=True)
+            m1.record(copy_s)
+            copy_marks.append((m0, m1))
 
     def compute(i):
         b = i % 2
@@ -684,25 +692,26 @@ def run_e2e(a, ctx, kv, src, dst, stream, dev):
         ctx.delete_raw(hs, S)
         free[b].record(stream)
 
-    def run(n):
+    def run(n, mark=False):
         for e in free:
             e.record(stream)
-        h2d(0)
+        h2d(0, mark)
         for i in range(n):
             if i + 1 < n:
-                h2d(i + 1)
+                h2d(i + 1, mark)
             compute(i)
 
     run(2)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    run(steps)
+    run(steps, mark=True)
     e1.record(stream)
     torch.cuda.synchronize()
     ctx.sync()
     ms = e0.elapsed_time(e1) / steps
     h2d_b = kh.numel() * kh.element_size() * 2
+    copy_ms = sum(m0.elapsed_time(m1) for m0, m1 in copy_marks) / max(len(copy_marks), 1)
     d2h_b = fps_h.numel() * 8
     del kh, vh, kb, vb
     for h in host:
@@ -711,7 +720,8 @@ def run_e2e(a, ctx, kv, src, dst, stream, dev):
             "h2d_bytes_per_step": h2d_b, "d2h_bytes_per_step": d2h_b, "ms_per_step": round(ms, 3),
             "sessions_per_s": round(a.sessions / (ms / 1e3), 2), "steps": steps,
             "overlap": "double-buffered pools: copy of step i+1 under compute of step i",
-            "pinned": pinning}
+            "pinned": pinning,
+            "h2d_GBs_in_run": round(h2d_b / (copy_ms / 1e3) / 1e9, 1)}
 
 
 def main():
