@@ -712,7 +712,8 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   // A stream with many task nodes would leave one finalising warp a long
   // serial tree: reduce aligned groups of 32 nodes across the GPU, level by
   // level, until no stream has more than 32 nodes left.  Aligned groups of
-  // 32^k nodes reduce to the nodes of the global pairwise tree.
+  // 32^k nodes reduce to the nodes of the global pairwise tree.  Up to 256
+  // nodes (eight groups) the finalising warp is quicker than another launch.
   for (auto& x : d) {
     x.fin_begin = x.task_begin;
     x.fin_count = x.n_tasks;
@@ -720,7 +721,7 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   uint64_t max_count = 0;
   for (const auto& x : d) max_count = std::max<uint64_t>(max_count, x.n_tasks);
   uint64_t groups = 0;
-  if (allow_reduce && max_count > 64) {
+  if (allow_reduce && max_count > 256) {
     while (max_count > 32) {
       const uint64_t level_base = node + groups;
       uint64_t level_groups = 0;
