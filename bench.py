@@ -395,6 +395,22 @@ def run_pcs(a, rank, world, local_rank):
 # the headline `value` above is the KV checkpoint + restore step)
 # ---------------------------------------------------------------------------
 
+def _loop_ms(fn, stream, calls=10, warm=2):
+    """Device time per call of `calls` back-to-back calls between one pair of
+    events: the throughput of a repeated step (the host prepares call i+1
+    while the GPU runs call i), timed as the headline step is."""
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(calls):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / calls
+
+
 def _events_ms(fn, stream, reps=5, warm=2):
     """Best and median device time of fn() over reps, CUDA events on `stream`."""
     for _ in range(warm):
@@ -421,7 +437,7 @@ def measure_fork(ctx, src, stream):
 
     def fork_all():
         ctx.delete_raw(ctx.fork_raw(hs, n), n)
-    best, med = _events_ms(fork_all, stream, reps=3, warm=1)
+    med = _loop_ms(fork_all, stream, calls=5, warm=1)
     ctx.delete_raw(hs, n)
     peak = load_peaks()["hbm_gbs"]
     gbs = 2 * nbytes / (med / 1e3) / 1e9
@@ -459,7 +475,7 @@ def run_rows(ctx, dev, stream):
     after_arr, before_arr = ctx.buf_array(sw.after), ctx.buf_array(sw.before)
     must = torch.empty(len(sw.after), dtype=torch.uint8, device=dev)
     fp1 = torch.empty(len(sw.after), dtype=torch.int64, device=dev)
-    best, med = _events_ms(lambda: ctx.classify(after_arr, fp0, fp1, must), stream)
+    med = _loop_ms(lambda: ctx.classify(after_arr, fp0, fp1, must), stream)
     ctx.classify(after_arr, fp0, fp1, must)
     flips_ok = must.cpu().tolist() == [1 if f else 0 for f in sw.flipped]
     gbs = tot / (med / 1e3) / 1e9
@@ -468,7 +484,7 @@ def run_rows(ctx, dev, stream):
                        "frac_of_hbm": round(gbs / peak, 4), "flags_match_ground_truth": flips_ok}
     # The discovery distance on the same pairs: differing bytes of before / after.
     counts = torch.empty(len(sw.after), dtype=torch.int64, device=dev)
-    best, med = _events_ms(lambda: ctx.mismatch(before_arr, after_arr, counts), stream)
+    med = _loop_ms(lambda: ctx.mismatch(before_arr, after_arr, counts), stream)
     mm_ok = ctx.mismatch(before_arr, after_arr, counts).cpu().tolist() == \
         [1 if f else 0 for f in sw.flipped]
     gbs = 2 * tot / (med / 1e3) / 1e9
@@ -490,7 +506,7 @@ def run_rows(ctx, dev, stream):
     kept = torch.empty(sum(ks), dtype=torch.int32, device=dev)
     koff = torch.empty(S + 1, dtype=torch.int32, device=dev)
     kb = b.keys.numel() * b.keys.element_size()
-    best, med = _events_ms(lambda: ctx.prune(banks, S, params, kept, koff), stream)
+    med = _loop_ms(lambda: ctx.prune(banks, S, params, kept, koff), stream)
     gbs = kb / (med / 1e3) / 1e9
     out["prune"] = {"population": "2048 banks, n ~ U[256,4096], key bf16[512]",
                     "key_bytes_read": kb, "ms": round(med, 3), "GBs": round(gbs, 1),
@@ -498,7 +514,7 @@ def run_rows(ctx, dev, stream):
     # The same banks under one relevance threshold across all of them.
     gkept = torch.empty(sum(b.n), dtype=torch.int32, device=dev)
     gkoff = torch.empty(S + 1, dtype=torch.int32, device=dev)
-    bestg, medg = _events_ms(lambda: ctx.prune_global(banks, S, 8 << 30, gkept, gkoff), stream)
+    medg = _loop_ms(lambda: ctx.prune_global(banks, S, 8 << 30, gkept, gkoff), stream)
     gk = int(gkoff[-1].item())
     out["prune_global"] = {
         "population": "the same 2048 banks, one threshold across all under 8 GiB",
@@ -520,10 +536,9 @@ def run_rows(ctx, dev, stream):
 
     def ckpt_del():
         ctx.delete_raw(ctx.checkpoint_raw(sarr, S, pcs.PCS_PLACE_PINNED_HOST), S)
-    best, med = _events_ms(ckpt_del, stream, reps=3, warm=1)
+    med = _loop_ms(ckpt_del, stream, calls=3, warm=1)
     hs = ctx.checkpoint_raw(sarr, S, pcs.PCS_PLACE_PINNED_HOST)
-    bestr, medr = _events_ms(lambda: ctx.restore_raw(hs, S, tarr, verify=2), stream, reps=3,
-                             warm=1)
+    medr = _loop_ms(lambda: ctx.restore_raw(hs, S, tarr, verify=2), stream, calls=3, warm=1)
     ctx.sync()
     ctx.delete_raw(hs, S)
     out["suspend_to_host"] = {
@@ -566,7 +581,7 @@ def run_rows(ctx, dev, stream):
         hs = ctx.checkpoint_raw(barr, 4096)
         ctx.restore_raw(hs, 4096, barr)
         ctx.delete_raw(hs, 4096)
-    best, med = _events_ms(batch_step, stream, reps=3, warm=1)
+    med = _loop_ms(batch_step, stream, calls=5, warm=1)
     out["markov"] = {"one_session_checkpoint_us": round(ck_us, 2),
                      "one_session_restore_us": round(rs_us, 2),
                      "how": "wall clock per call (checkpoint incl. delete) through the ctypes "
