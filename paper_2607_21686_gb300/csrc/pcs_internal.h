@@ -89,8 +89,10 @@ struct alignas(16) BankDesc {
   int32_t D;
   int32_t k;
   uint32_t is_bf16;
+  uint64_t entry_bytes;    // bytes one kept entry costs (global threshold)
+  uint64_t pad;
 };
-static_assert(sizeof(BankDesc) == 48, "BankDesc layout");
+static_assert(sizeof(BankDesc) == 64, "BankDesc layout");
 
 // The streams one streaming kernel processes: item j is stream secs[ids[j]],
 // owning this kernel's tasks [begin[j], begin[j+1]) (the last up to n_tasks).
@@ -153,15 +155,16 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
                             const uint64_t* fp_before, uint8_t* flags, uint32_t* bad,
                             cudaStream_t stream);
 
-cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
-                         int key_types, float* scores, int sm_count, cudaStream_t stream);
+
 
 cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
                         int32_t* kept_idx, cudaStream_t stream);
 
 
 // ---- One relevance threshold across all banks (pcs_prune_global) ---------
-constexpr int kGTile = 4096;  // entries per tile of the global passes
+constexpr int kGTile = 4096;    // entries per tile of the global passes
+constexpr int kGPasses = 6;     // digits of the 64-bit key: 11, 11, 10, 11, 11, 10 bits
+constexpr int kGBins = 2048;    // bins of the widest digit
 
 // Select state: the kept set is every entry whose ranking key exceeds
 // `threshold`.  Set by the host, advanced by the last block of each pass.
@@ -170,8 +173,17 @@ struct alignas(16) GState {
   uint64_t remaining;     // budget left for keys inside the prefix
   uint64_t threshold;
   uint32_t done, ticket, total_kept, pad;
-  uint64_t whist[256];    // entry bytes per digit (mixed entry sizes)
-  uint32_t chist[256];    // entries per digit
+  uint64_t whist[kGBins]; // entry bytes per digit (mixed entry sizes)
+  uint32_t chist[kGBins]; // entries per digit
+};
+
+// The score kernel's optional epilogue: the first digit pass of the global
+// threshold (a histogram of the top key bits, then the digit choice).
+struct GHist {
+  GState* st;             // NULL: no histogram
+  uint64_t uniform_bytes; // entry bytes when every bank costs the same
+  int32_t mode;           // 1: uniform entry bytes, 2: per-bank entry bytes
+  int32_t pad;
 };
 
 // Passed by value as a kernel parameter.
@@ -192,8 +204,15 @@ struct GPlan {
   int32_t pad;
 };
 
-// Pass `pass` (0..7) of the byte-weighted radix select; a no-op once the
-// threshold is known.
+// Scores of every entry; with gh.st set (and a fixed-width kernel), also the
+// first digit pass of the global threshold.  Returns through *fused whether
+// that pass was done.
+cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
+                         int key_types, float* scores, int sm_count, cudaStream_t stream,
+                         GHist gh = GHist{}, bool* fused = nullptr);
+
+// Pass `pass` (0..kGPasses-1) of the byte-weighted radix select; a no-op
+// once the threshold is known.
 cudaError_t launch_gselect(const GPlan& p, int pass, int sm_count, cudaStream_t stream);
 // Count per tile and scan (first launch), then write kept indices and bank
 // offsets (second launch).

@@ -909,6 +909,104 @@ __global__ void __launch_bounds__(kThreads, 2)
 // Relevance score and top-k
 // ---------------------------------------------------------------------------
 
+// Order-preserving map float -> uint32 (-0 ranks as +0, NaN lowest).
+__device__ __forceinline__ uint32_t ord32(float s) {
+  if (isnan(s)) return 0u;
+  if (s == 0.f) s = 0.f;
+  const uint32_t u = __float_as_uint(s);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Digits of the 64-bit ranking key of the global threshold, most significant
+// first: 11, 11 and 10 bits of ord32(score), then the same of the position.
+__device__ __forceinline__ int gdigit_bits(int pass) { return pass % 3 == 2 ? 10 : 11; }
+__device__ __forceinline__ int gdigit_shift(int pass) {
+  return pass == 0 ? 53 : pass == 1 ? 42 : pass == 2 ? 32 : pass == 3 ? 21 : pass == 4 ? 10 : 0;
+}
+
+// The digit choice of one pass, by one warp, from the summed histograms
+// (staged in shared memory): scanning digits from the top, the first whose
+// bytes overrun the budget left is fixed into the prefix; if it holds a
+// single key, or it was the last digit, that key is the first that does not
+// fit and the threshold is set.
+template <bool UNIFORM>
+__device__ void gselect_pick(GState* st, int pass, uint64_t ubytes, const uint32_t* ch,
+                             const unsigned long long* wh) {
+  const int lane = threadIdx.x & 31;
+  const int bits = gdigit_bits(pass), shift = gdigit_shift(pass);
+  const int top = (1 << bits) - 1, per = (1 << bits) / 32;  // lane l: bins top-per*l ...
+  auto weight = [&](int bin) -> uint64_t {
+    return UNIFORM ? static_cast<uint64_t>(ch[bin]) * ubytes : static_cast<uint64_t>(wh[bin]);
+  };
+  uint64_t local = 0;
+  for (int j = 0; j < per; ++j) local += weight(top - per * lane - j);
+  uint64_t incl = local;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint64_t o = __shfl_up_sync(kFull, incl, d);
+    if (lane >= d) incl += o;
+  }
+  const uint64_t R = __ldcg(&st->remaining);
+  const unsigned hit = __ballot_sync(kFull, incl > R);
+  if (hit == 0) {  // every candidate fits (only when the whole population does)
+    if (lane == 0) {
+      st->threshold = 0;
+      st->done = 1;
+    }
+    return;
+  }
+  if (lane != __ffs(hit) - 1) return;
+  const uint64_t prefix = __ldcg(&st->prefix), mask = __ldcg(&st->mask);
+  uint64_t cum = incl - local;
+  for (int j = 0; j < per; ++j) {
+    const int bin = top - per * lane - j;
+    const uint64_t w = weight(bin);
+    if (cum + w > R) {
+      const uint64_t np = prefix | (static_cast<uint64_t>(bin) << shift);
+      const uint64_t nm = mask | (static_cast<uint64_t>(top) << shift);
+      st->prefix = np;
+      st->mask = nm;
+      st->remaining = R - cum;
+      if (ch[bin] == 1u || shift == 0) {
+        st->threshold = np | ~nm;
+        st->done = 1;
+      }
+      return;
+    }
+    cum += w;
+  }
+}
+
+// End of a histogram pass, by every block: add the block's bins (ch, wh in
+// shared memory) to the global ones; the last block to finish (atomic
+// ticket) stages the sums in the same shared arrays, picks the digit and
+// clears the global bins for the next pass.
+template <bool UNIFORM>
+__device__ void gpass_finish(GState* st, int pass, uint64_t ubytes, uint32_t* ch,
+                             unsigned long long* wh, bool* s_last) {
+  const int nb = 1 << gdigit_bits(pass);
+  __syncthreads();
+  for (int i = threadIdx.x; i < nb; i += blockDim.x) {
+    if (ch[i]) atomicAdd(&st->chist[i], ch[i]);
+    if (!UNIFORM && wh[i]) atomicAdd(reinterpret_cast<unsigned long long*>(&st->whist[i]), wh[i]);
+  }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) *s_last = atomicAdd(&st->ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!*s_last) return;
+  __threadfence();
+  for (int i = threadIdx.x; i < nb; i += blockDim.x) {
+    ch[i] = __ldcg(&st->chist[i]);
+    if (!UNIFORM) wh[i] = __ldcg(reinterpret_cast<const unsigned long long*>(&st->whist[i]));
+    st->chist[i] = 0;
+    st->whist[i] = 0;
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) gselect_pick<UNIFORM>(st, pass, ubytes, ch, wh);
+  if (threadIdx.x == 0) st->ticket = 0;
+}
+
 __device__ __forceinline__ float elem(uint32_t bits16, bool bf16) {
   return bf16 ? __uint_as_float(bits16 << 16)
               : __half2float(__ushort_as_half(static_cast<unsigned short>(bits16)));
@@ -962,10 +1060,10 @@ __device__ __forceinline__ float seg_elem(const uint4& v, int i) {
 // The bank's query is held in registers as fp32, with |q| computed once per
 // bank in the same fixed order; every key load of the kScoreIlp entries is
 // issued before any arithmetic.
-template <int SPL, int DT>
-__global__ void __launch_bounds__(kThreads)
-    k_score_fixed(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
-                  float* __restrict__ scores) {
+template <int SPL, int DT, int HM>
+__device__ __forceinline__ void score_range(const BankDesc* __restrict__ banks, int n_banks,
+                                            uint64_t n_entries, float* __restrict__ scores,
+                                            bool hist, uint32_t* s_cnt, unsigned long long* s_w) {
   const int lane = threadIdx.x & 31;
   const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
   const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kWarps;
@@ -1071,11 +1169,39 @@ __global__ void __launch_bounds__(kThreads)
     const int q = 2 * (lane & 1) + ((lane >> 1) & 1);
     if (lane < 4 && q < cnt) {
       const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
-      scores[e0 + q] = den == 0.f ? 0.f : __fdiv_rn(w1, den);
+      const float sc = den == 0.f ? 0.f : __fdiv_rn(w1, den);
+      scores[e0 + q] = sc;
+      if (HM && hist) {
+        const uint32_t d = ord32(sc) >> 21;  // key bits 63..53
+        atomicAdd(&s_cnt[d], 1u);
+        if (HM == 2) atomicAdd(&s_w[d], static_cast<unsigned long long>(B.entry_bytes));
+      }
     }
     e0 = e0 + cnt - kScoreIlp;  // the loop adds kScoreIlp: next round starts at e0 + cnt
   }
 }
+
+// HM (global threshold): 0 none; 1 / 2 also histogram the top 11 key bits of
+// every score (2: weighted by the bank's entry bytes) and pick the first digit.
+template <int SPL, int DT, int HM>
+__global__ void __launch_bounds__(kThreads)
+    k_score_fixed(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
+                  float* __restrict__ scores, GHist gh) {
+  __shared__ uint32_t s_cnt[HM ? kGBins : 1];
+  __shared__ unsigned long long s_w[HM == 2 ? kGBins : 1];
+  __shared__ bool s_last;
+  const bool hist = HM && !__ldcg(&gh.st->done);  // the same for every block
+  if (hist) {
+    for (int i = threadIdx.x; i < kGBins; i += kThreads) {
+      s_cnt[i] = 0;
+      if (HM == 2) s_w[i] = 0;
+    }
+    __syncthreads();
+  }
+  score_range<SPL, DT, HM>(banks, n_banks, n_entries, scores, hist, s_cnt, s_w);
+  if (hist) gpass_finish<HM == 1>(gh.st, 0, gh.uniform_bytes, s_cnt, s_w, &s_last);
+}
+
 
 // Any key width or a mix of key types: the query is re-read per entry.
 __global__ void __launch_bounds__(kThreads)
@@ -1123,12 +1249,6 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
-__device__ __forceinline__ uint32_t ord32(float s) {
-  if (isnan(s)) return 0u;
-  if (s == 0.f) s = 0.f;
-  const uint32_t u = __float_as_uint(s);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
 
 // Exclusive block scan of a 0/1 flag; returns the rank, *total = sum.
 __device__ __forceinline__ uint32_t block_rank(bool f, uint32_t* warp_cnt, uint32_t* total) {
@@ -1266,16 +1386,17 @@ __device__ __forceinline__ int gbank(const uint64_t* __restrict__ ebeg, int lo, 
 
 template <bool UNIFORM>
 __global__ void __launch_bounds__(kThreads) k_gselect(GPlan p, int pass) {
-  __shared__ uint64_t wh[256];
-  __shared__ uint32_t ch[256];
+  __shared__ uint32_t ch[kGBins];
+  __shared__ unsigned long long wh[UNIFORM ? 1 : kGBins];
   __shared__ bool s_last;
   GState* st = p.st;
   if (__ldcg(&st->done)) return;  // the same for every block of the launch
-  const int shift = 56 - 8 * pass;
+  const int shift = gdigit_shift(pass);
+  const uint32_t nb = 1u << gdigit_bits(pass);
   const uint64_t prefix = __ldcg(&st->prefix), mask = __ldcg(&st->mask);
-  for (int i = threadIdx.x; i < 256; i += kThreads) {
-    wh[i] = 0;
+  for (uint32_t i = threadIdx.x; i < nb; i += kThreads) {
     ch[i] = 0;
+    if (!UNIFORM) wh[i] = 0;
   }
   __syncthreads();
   const int lane = threadIdx.x & 31;
@@ -1295,89 +1416,23 @@ __global__ void __launch_bounds__(kThreads) k_gselect(GPlan p, int pass) {
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
       const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
-      uint32_t d = 256;  // not a candidate
+      uint32_t d = kGBins;  // not a candidate
       if (i < end) {
         const uint64_t key = (static_cast<uint64_t>(ord32(sv[j])) << 32) | (0xFFFFFFFFull - i);
-        if ((key & mask) == prefix) d = static_cast<uint32_t>(key >> shift) & 255u;
+        if ((key & mask) == prefix) d = static_cast<uint32_t>(key >> shift) & (nb - 1);
       }
       if (UNIFORM) {
         // Lanes with the same digit add once (the hot digits are few).
         const unsigned same = __match_any_sync(kFull, d);
-        if (d < 256 && lane == __ffs(same) - 1) atomicAdd(&ch[d], __popc(same));
-      } else if (d < 256) {
+        if (d < kGBins && lane == __ffs(same) - 1) atomicAdd(&ch[d], __popc(same));
+      } else if (d < kGBins) {
         b = gbank(p.ebeg, b, hi, i);
         atomicAdd(&ch[d], 1u);
-        atomicAdd(reinterpret_cast<unsigned long long*>(&wh[d]),
-                  static_cast<unsigned long long>(__ldg(p.ebytes + b)));
+        atomicAdd(&wh[d], static_cast<unsigned long long>(__ldg(p.ebytes + b)));
       }
     }
   }
-  __syncthreads();
-  for (int i = threadIdx.x; i < 256; i += kThreads) {
-    if (ch[i]) atomicAdd(&st->chist[i], ch[i]);
-    if (!UNIFORM && wh[i])
-      atomicAdd(reinterpret_cast<unsigned long long*>(&st->whist[i]),
-                static_cast<unsigned long long>(wh[i]));
-  }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(&st->ticket, 1u) == gridDim.x - 1;
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  if (threadIdx.x < 32) {
-    // Lane l covers digits 255-8l .. 248-8l (descending).
-    uint64_t w[8], local = 0;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int bin = 255 - 8 * lane - j;
-      w[j] = UNIFORM ? static_cast<uint64_t>(__ldcg(&st->chist[bin])) * p.uniform_bytes
-                     : __ldcg(&st->whist[bin]);
-      local += w[j];
-    }
-    uint64_t incl = local;
-#pragma unroll
-    for (int dd = 1; dd < 32; dd <<= 1) {
-      const uint64_t o = __shfl_up_sync(kFull, incl, dd);
-      if (lane >= dd) incl += o;
-    }
-    const uint64_t R = __ldcg(&st->remaining);
-    const unsigned hit = __ballot_sync(kFull, incl > R);
-    if (hit == 0) {
-      // Every candidate fits (only when the whole population does).
-      if (lane == 0) {
-        st->threshold = 0;
-        st->done = 1;
-      }
-    } else if (lane == __ffs(hit) - 1) {
-      uint64_t cum = incl - local;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        if (cum + w[j] > R) {
-          const int bin = 255 - 8 * lane - j;
-          const uint64_t np = prefix | (static_cast<uint64_t>(bin) << shift);
-          const uint64_t nm = mask | (0xFFull << shift);
-          st->prefix = np;
-          st->mask = nm;
-          st->remaining = R - cum;
-          // One key left in the digit, or the last digit: that key is the
-          // first that does not fit.
-          if (__ldcg(&st->chist[bin]) == 1u || shift == 0) {
-            st->threshold = np | ~nm;
-            st->done = 1;
-          }
-          break;
-        }
-        cum += w[j];
-      }
-    }
-  }
-  __syncthreads();
-  for (int i = threadIdx.x; i < 256; i += kThreads) {
-    st->chist[i] = 0;
-    st->whist[i] = 0;
-  }
-  if (threadIdx.x == 0) st->ticket = 0;
+  gpass_finish<UNIFORM>(st, pass, p.uniform_bytes, ch, wh, &s_last);
 }
 
 // Exclusive block scan of one uint32 per thread; *total = block sum.
@@ -1938,7 +1993,9 @@ cudaError_t launch_reduce_nodes(const NodeLevel* lv, int n_secs, uint64_t* nodes
 }
 
 cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
-                         int key_types, float* scores, int sm_count, cudaStream_t stream) {
+                         int key_types, float* scores, int sm_count, cudaStream_t stream,
+                         GHist gh, bool* fused) {
+  if (fused) *fused = false;
   if (n_entries == 0) return cudaSuccess;
   const uint64_t want = (n_entries + kWarps * kScoreIlp * 8 - 1) / (kWarps * kScoreIlp * 8);
   const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
@@ -1946,15 +2003,24 @@ cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
   // key_types: 0 = all fp16, 1 = all bf16, 2 = mixed.
   if (key_types == 2 || max_dim > 1024) {
     k_score_any<<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-  } else if (key_types == 1) {
-    if (max_dim <= 256) k_score_fixed<1, 1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-    else if (max_dim <= 512) k_score_fixed<2, 1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-    else k_score_fixed<4, 1><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-  } else {
-    if (max_dim <= 256) k_score_fixed<1, 0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-    else if (max_dim <= 512) k_score_fixed<2, 0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
-    else k_score_fixed<4, 0><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+    return cudaGetLastError();
   }
+  const int spl = max_dim <= 256 ? 1 : max_dim <= 512 ? 2 : 4;
+  const int hm = gh.st ? gh.mode : 0;
+#define PCS_SCORE(S, D, H) k_score_fixed<S, D, H><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores, gh)
+#define PCS_SCORE_H(S, D) (hm == 0 ? PCS_SCORE(S, D, 0) : hm == 1 ? PCS_SCORE(S, D, 1) : PCS_SCORE(S, D, 2))
+  if (key_types == 1) {
+    if (spl == 1) PCS_SCORE_H(1, 1);
+    else if (spl == 2) PCS_SCORE_H(2, 1);
+    else PCS_SCORE_H(4, 1);
+  } else {
+    if (spl == 1) PCS_SCORE_H(1, 0);
+    else if (spl == 2) PCS_SCORE_H(2, 0);
+    else PCS_SCORE_H(4, 0);
+  }
+#undef PCS_SCORE_H
+#undef PCS_SCORE
+  if (fused) *fused = hm != 0;
   return cudaGetLastError();
 }
 

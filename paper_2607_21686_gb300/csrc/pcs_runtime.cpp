@@ -1149,6 +1149,7 @@ pcs_status bank_descs(const pcs_bank* banks, int32_t n, const int32_t* k,
     x.D = b.key_dim;
     x.k = k ? k[s] : 0;
     x.is_bf16 = b.key_dtype == PCS_DT_BF16;
+    x.entry_bytes = b.entry_bytes;
     entries += b.n_entries;
     kept += x.k;
   }
@@ -1157,10 +1158,12 @@ pcs_status bank_descs(const pcs_bank* banks, int32_t n, const int32_t* k,
   return PCS_OK;
 }
 
-// The relevance score of every entry (descriptors already on the device).
+// The relevance score of every entry (descriptors already on the device);
+// with gh.st set, also the first digit pass of the global threshold where the
+// score kernel can take it (*fused says whether it did).
 cudaError_t launch_bank_scores(pcs_ctx* c, const pcs_bank* banks, int32_t n,
                                const BankDesc* dbanks, uint64_t entries, float* sc,
-                               cudaStream_t stream) {
+                               cudaStream_t stream, GHist gh = GHist{}, bool* fused = nullptr) {
   LaunchScope ls(c, kKScore, stream);
   int max_dim = 0, n_bf16 = 0;
   for (int s = 0; s < n; ++s) {
@@ -1168,7 +1171,7 @@ cudaError_t launch_bank_scores(pcs_ctx* c, const pcs_bank* banks, int32_t n,
     n_bf16 += banks[s].key_dtype == PCS_DT_BF16;
   }
   const int key_types = n_bf16 == 0 ? 0 : (n_bf16 == n ? 1 : 2);
-  return launch_score(dbanks, n, entries, max_dim, key_types, sc, c->sm_count, stream);
+  return launch_score(dbanks, n, entries, max_dim, key_types, sc, c->sm_count, stream, gh, fused);
 }
 
 pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_prune_params* p,
@@ -1329,8 +1332,15 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
   std::memcpy(c->plan.data() + o_st, &g0, sizeof g0);
   PCS_CUDA(plan_copy(c, ws, plan_bytes, stream));
   float* sc = scores ? scores : reinterpret_cast<float*>(ws + o_sc);
+  GHist gh{};
+  if (!g0.done) {
+    gh.st = reinterpret_cast<GState*>(ws + o_st);
+    gh.uniform_bytes = n > 0 ? banks[0].entry_bytes : 0;
+    gh.mode = uniform ? 1 : 2;
+  }
+  bool fused = false;
   PCS_CUDA(launch_bank_scores(c, banks, n, reinterpret_cast<const BankDesc*>(ws), entries, sc,
-                              stream));
+                              stream, gh, &fused));
   GPlan gp{};
   gp.scores = sc;
   gp.ebeg = reinterpret_cast<const uint64_t*>(ws + o_ebeg);
@@ -1346,8 +1356,9 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
   gp.tiles = static_cast<int32_t>(tiles);
   gp.uniform = uniform ? 1 : 0;
   if (!g0.done) {
-    // Eight digit passes at most; each is a no-op once the threshold is known.
-    for (int pass = 0; pass < 8; ++pass) {
+    // Six digit passes at most (the first inside the score kernel when it
+    // could take it); each is a no-op once the threshold is known.
+    for (int pass = fused ? 1 : 0; pass < kGPasses; ++pass) {
       LaunchScope ls(c, kKGSelect, stream);
       PCS_CUDA(launch_gselect(gp, pass, c->sm_count, stream));
     }
