@@ -107,7 +107,8 @@ typedef int32_t pcs_status;
 /* k-rules of pcs_prune. */
 #define PCS_K_FIXED 0     /* k = min(n, k_max)                               */
 #define PCS_K_BUDGET 1    /* T = sum n_s*entry_bytes_s; k_s = n_s if T <= B, */
-                          /* else floor(n_s * B / T)  (Sec. 7.5)             */
+                          /* else floor(n_s * B / T)  (Sec. 7.5); T may be  */
+                          /* given for a population split across processes  */
 #define PCS_K_FRACTION 2  /* k = round-half-even(fraction * n)              */
                           /* (Table tab:keepfrac)                           */
 
@@ -179,6 +180,10 @@ typedef struct pcs_prune_params {
     int32_t k_max;         /* PCS_K_FIXED                                   */
     uint64_t budget_bytes; /* PCS_K_BUDGET: host byte budget B              */
     double fraction;       /* PCS_K_FRACTION, in [0, 1]                     */
+    uint64_t total_bytes;  /* PCS_K_BUDGET: T of the whole population when */
+                           /* its banks are split over calls or processes   */
+                           /* (the sum of every part's T); 0 = the T of the */
+                           /* banks of this call                            */
 } pcs_prune_params;
 
 typedef struct pcs_snapshot_info {

@@ -1095,6 +1095,12 @@ pcs_status pcs_prune_counts(const pcs_bank* banks, int32_t n, const pcs_prune_pa
       for (int s = 0; s < n; ++s)
         T += static_cast<unsigned __int128>(static_cast<uint64_t>(banks[s].n_entries)) *
              banks[s].entry_bytes;
+      // A population split over processes: every part uses the whole T.
+      if (p->total_bytes != 0) {
+        if (p->total_bytes < T)
+          return fail(PCS_E_INVAL, "total_bytes is below the bytes of these banks");
+        T = p->total_bytes;
+      }
       for (int s = 0; s < n; ++s) {
         if (T <= p->budget_bytes) {
           k_out[s] = banks[s].n_entries;

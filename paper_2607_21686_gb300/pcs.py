@@ -76,7 +76,8 @@ class pcs_bank(ctypes.Structure):
 
 class pcs_prune_params(ctypes.Structure):
     _fields_ = [("rule", ctypes.c_int32), ("k_max", ctypes.c_int32),
-                ("budget_bytes", ctypes.c_uint64), ("fraction", ctypes.c_double)]
+                ("budget_bytes", ctypes.c_uint64), ("fraction", ctypes.c_double),
+                ("total_bytes", ctypes.c_uint64)]
 
 
 class pcs_snapshot_info(ctypes.Structure):
@@ -561,12 +562,17 @@ class Context:
         return arr
 
     @staticmethod
-    def params(rule: int, k_max: int = 0, budget: int = 0, fraction: float = 0.0):
-        return pcs_prune_params(rule=rule, k_max=k_max, budget_bytes=budget, fraction=fraction)
+    def params(rule: int, k_max: int = 0, budget: int = 0, fraction: float = 0.0,
+               total_bytes: int = 0):
+        return pcs_prune_params(rule=rule, k_max=k_max, budget_bytes=budget, fraction=fraction,
+                                total_bytes=total_bytes)
 
-    def prune_counts(self, banks, n: int, params) -> list:
+    @staticmethod
+    def prune_counts(banks, n: int, params) -> list:
+        """Host only: entries each bank keeps under `params`."""
         k = (ctypes.c_int32 * max(n, 1))()
-        check(self.lib.pcs_prune_counts(banks, n, ctypes.byref(params), k), "pcs_prune_counts")
+        check(load_library().pcs_prune_counts(banks, n, ctypes.byref(params), k),
+              "pcs_prune_counts")
         return list(k)[:n]
 
     def prune(self, banks, n: int, params, kept_idx: torch.Tensor, kept_off=None, scores=None,

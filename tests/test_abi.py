@@ -62,6 +62,7 @@ int main(void) {
   S(pcs_session) O(pcs_session, n_sections) O(pcs_session, sections)
   S(pcs_bank) O(pcs_bank, n_entries) O(pcs_bank, key_dtype) O(pcs_bank, entry_bytes)
   S(pcs_prune_params) O(pcs_prune_params, budget_bytes) O(pcs_prune_params, fraction)
+  O(pcs_prune_params, total_bytes)
   S(pcs_snapshot_info) O(pcs_snapshot_info, total_bytes) O(pcs_snapshot_info, data)
   S(pcs_section_info) O(pcs_section_info, offset) O(pcs_section_info, aux)
   S(pcs_stats) O(pcs_stats, live_snapshots)
@@ -139,6 +140,25 @@ def test_prune_counts_rejects_bad_params(lib):
     assert lib.pcs_prune_counts(_banks([3], 1), 1, ctypes.byref(p), k) == pcs.PCS_E_INVAL
     p = pcs.pcs_prune_params(rule=pcs.PCS_K_FRACTION, fraction=1.5)
     assert lib.pcs_prune_counts(_banks([3], 1), 1, ctypes.byref(p), k) == pcs.PCS_E_INVAL
+    # A whole-population T smaller than these banks' own bytes cannot be right.
+    p = pcs.pcs_prune_params(rule=pcs.PCS_K_BUDGET, budget_bytes=1, total_bytes=2)
+    assert lib.pcs_prune_counts(_banks([3], 1), 1, ctypes.byref(p), k) == pcs.PCS_E_INVAL
+
+
+def test_budget_counts_of_a_part_use_the_whole_population(lib):
+    # Counts of a part of the banks with the whole population's T equal the
+    # whole population's counts for those banks (the sharded budget rule).
+    rnd = np.random.default_rng(9)
+    n = rnd.integers(0, 5000, 400).astype(np.int32)
+    E = 3072
+    T = int(n.astype(np.int64).sum()) * E
+    for B in (T // 7, T // 2, T - 1, T):
+        want = oracle.k_budget(n, E, B).tolist()
+        for part in (slice(0, 150), slice(150, 400), slice(None, None, 3)):
+            p = pcs.pcs_prune_params(rule=pcs.PCS_K_BUDGET, budget_bytes=B, total_bytes=T)
+            assert _counts(lib, n[part].tolist(), p, E) == want[part]
+        p = pcs.pcs_prune_params(rule=pcs.PCS_K_BUDGET, budget_bytes=B, total_bytes=T)
+        assert _counts(lib, n.tolist(), p, E) == want
 
 
 def test_record_bytes_match_oracle(lib):

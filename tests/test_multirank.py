@@ -1,8 +1,11 @@
-"""The multi-rank path of bench.py on CPU with gloo (world size 2).
+"""The multi-rank paths on CPU with gloo (world size 2).
 
-Sessions are independent, so ranks share nothing on the data path; the only
-exchange is the max over ranks of the timed region.  These tests exercise that
-reduction and the launch contract of the reference arm under torchrun.
+Sessions are independent, so ranks share nothing on the data path of the
+step; bench.py's only exchange is the max over ranks of the timed region.
+The one real exchange of the method is the host budget of banks sharded
+across ranks (Sec. 7.5: every bank keeps the same fraction B / T of the whole
+population): one all-reduced scalar, T.  These tests exercise both
+reductions and the launch contract of the reference arm under torchrun.
 """
 import json
 import os
@@ -22,6 +25,28 @@ def _worker(rank, world, port, out):
     sys.path.insert(0, ROOT)
     import bench
     out[rank] = bench.max_over_ranks(10.0 + 5.0 * rank)
+    torch.distributed.destroy_process_group()
+
+
+def _budget_worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    torch.distributed.init_process_group("gloo", rank=rank, world_size=world)
+    sys.path.insert(0, ROOT)
+    from paper_2607_21686_gb300 import pcs
+    import numpy as np
+    rnd = np.random.default_rng(5)
+    n = rnd.integers(256, 4097, 2048)
+    E = rnd.choice([3072, 1024, 5000], 2048)
+    mine = range(rank, 2048, world)  # interleaved shards
+    banks = (pcs.pcs_bank * len(mine))()
+    for j, s in enumerate(mine):
+        banks[j] = pcs.pcs_bank(n_entries=int(n[s]), key_dim=8, key_dtype=pcs.PCS_DT_F16,
+                                entry_bytes=int(E[s]))
+    t_local = int(sum(int(n[s]) * int(E[s]) for s in mine))
+    t = torch.tensor([t_local], dtype=torch.int64)
+    torch.distributed.all_reduce(t)  # the one scalar the budget rule needs
+    p = pcs.Context.params(pcs.PCS_K_BUDGET, budget=8 << 30, total_bytes=int(t.item()))
+    out[rank] = dict(zip(mine, pcs.Context.prune_counts(banks, len(mine), p)))
     torch.distributed.destroy_process_group()
 
 
@@ -60,3 +85,24 @@ def test_reference_arm_under_torchrun():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_sharded_budget_matches_one_process():
+    ctx = mp.get_context("spawn")
+    with ctx.Manager() as m:
+        out = m.dict()
+        port = _free_port()
+        procs = [ctx.Process(target=_budget_worker, args=(r, 2, port, out)) for r in range(2)]
+        for p in procs:
+            p.start()
+        for p in procs:
+            p.join(120)
+            assert p.exitcode == 0
+        k = {**out[0], **out[1]}
+    import numpy as np
+    import oracle
+    rnd = np.random.default_rng(5)
+    n = rnd.integers(256, 4097, 2048)
+    E = rnd.choice([3072, 1024, 5000], 2048)
+    want = oracle.k_budget(n, E.astype(np.uint64), 8 << 30)
+    assert [k[s] for s in range(2048)] == want.tolist()
