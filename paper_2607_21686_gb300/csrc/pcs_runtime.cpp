@@ -889,6 +889,223 @@ pcs_snapshot* check_handle(pcs_ctx* c, const pcs_snapshot* h) {
   return c->live.count(p) ? p : nullptr;
 }
 
+// A checkpoint or a restore, planned: the descriptors (host bytes, uploaded
+// to [0, L.nodes) of a workspace) and how to launch its kernels.
+struct Prepared {
+  int mode = kModePack;  // kModePack, kModeRestore, kModeRestoreV
+  bool fused = false;    // one k_small launch (small calls)
+  int verify = 0;        // restore: 0, 1 or 2
+  int32_t n = 0;         // sessions
+  StreamPlan P;
+  ListLayout LL{};
+  WsLayout L;
+  std::vector<uint8_t> plan;
+};
+
+// Launch a prepared call whose descriptors are at `ws` (nodes after them).
+cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, cudaStream_t stream) {
+  const auto* dsecs = reinterpret_cast<const SecDesc*>(ws + pr.L.secs);
+  const auto* dsess = reinterpret_cast<const SessDesc*>(ws + pr.L.sess);
+  auto* nodes = reinterpret_cast<uint64_t*>(ws + pr.L.nodes);
+  WorkList wl{reinterpret_cast<const uint32_t*>(ws + pr.LL.reg_ids),
+              reinterpret_cast<const uint32_t*>(ws + pr.LL.reg_begin),
+              static_cast<int>(pr.P.reg_ids.size()), pr.P.reg_tasks};
+  if (pr.mode == kModePack) {
+    const auto* dent = reinterpret_cast<const Entry*>(ws + pr.L.entries);
+    if (pr.fused) {
+      LaunchScope ls(c, kKStreamPack, stream);
+      return launch_small(kModePack, dsecs, wl, pr.P.glog2, nodes, c->words, c->words + 3, pr.n,
+                          dsess, dent, nullptr, nullptr, nullptr, nullptr, c->sm_count,
+                          c->stream_bps, stream);
+    }
+    cudaError_t e = launch_streams(c, kModePack, dsecs, pr.P, pr.LL, ws, nodes, stream);
+    if (e != cudaSuccess) return e;
+    LaunchScope ls(c, kKFinalizePack, stream);
+    return launch_finalize(kModePack, dsecs, dsess, pr.n, dent, nodes, nullptr, nullptr, nullptr,
+                           nullptr, stream);
+  }
+  uint32_t* bad = c->words + (pr.verify == 1 ? 1 : 2);
+  if (pr.fused) {
+    LaunchScope ls(c, kKStreamRestoreV, stream);
+    return launch_small(kModeRestoreV, dsecs, wl, pr.P.glog2, nodes, c->words, c->words + 3, pr.n,
+                        dsess, nullptr, nullptr, nullptr, nullptr, bad, c->sm_count,
+                        c->stream_bps, stream);
+  }
+  cudaError_t e = launch_streams(c, pr.verify ? kModeRestoreV : kModeRestore, dsecs, pr.P, pr.LL,
+                                 ws, pr.verify ? nodes : nullptr, stream);
+  if (e != cudaSuccess || !pr.verify) return e;
+  LaunchScope ls(c, kKFinalizeRestoreV, stream);
+  return launch_finalize(kModeRestoreV, dsecs, dsess, pr.n, nullptr, nodes, nullptr, nullptr,
+                         nullptr, bad, stream);
+}
+
+// Plan a checkpoint of n sessions: validate, reserve one block for their
+// records (on `stream`), create the handles (not yet live), build the
+// descriptors.  On failure nothing is left reserved.
+pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, uint32_t placement,
+                            cudaStream_t stream, Prepared* pr, Block** blk_out,
+                            std::vector<std::unique_ptr<pcs_snapshot>>* handles) {
+  if (placement != PCS_PLACE_DEVICE && placement != PCS_PLACE_PINNED_HOST)
+    return fail(PCS_E_INVAL, "unknown placement %u", placement);
+  // Plan records: sizes, offsets, entries.
+  std::vector<uint64_t> rec_off(n + 1, 0), pstart(n);
+  uint64_t total_secs = 0;
+  for (int s = 0; s < n; ++s) {
+    const pcs_session& S = sessions[s];
+    if (S.n_sections < 1 || S.n_sections > 65535 || !S.sections)
+      return fail(PCS_E_INVAL, "session %d: needs 1..65535 sections", s);
+    for (int i = 0; i < S.n_sections; ++i) {
+      pcs_status st = check_section(S.sections[i], s, i, false);
+      if (st) return st;
+    }
+    uint64_t bytes = 0;
+    pcs_record_bytes(S.sections, S.n_sections, &bytes);
+    pstart[s] = round_up(kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * S.n_sections, kRecordAlign);
+    rec_off[s + 1] = rec_off[s] + bytes;
+    total_secs += S.n_sections;
+  }
+  if (total_secs > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many sections in one call");
+  Block* blk = nullptr;
+  pcs_status st = arena_of(c, placement)->alloc(rec_off[n], stream, &blk);
+  if (st) return st;
+  std::vector<SecDesc> d;
+  std::vector<SessDesc> sd(n);
+  std::vector<Entry> ent;
+  d.reserve(total_secs);
+  ent.reserve(total_secs);
+  handles->resize(n);
+  for (int s = 0; s < n; ++s) {
+    const pcs_session& S = sessions[s];
+    uint8_t* rec = blk->ptr + rec_off[s];
+    auto h = std::make_unique<pcs_snapshot>();
+    h->block = blk;
+    h->offset = rec_off[s];
+    h->total_bytes = rec_off[s + 1] - rec_off[s];
+    h->payload_start = pstart[s];
+    h->session_id = S.session_id;
+    h->kind = S.kind;
+    sd[s].record = rec;
+    sd[s].total_bytes = h->total_bytes;
+    sd[s].payload_start = pstart[s];
+    sd[s].sec_begin = static_cast<uint32_t>(d.size());
+    sd[s].n_sections = static_cast<uint32_t>(S.n_sections);
+    sd[s].session_id = S.session_id;
+    sd[s].kind = S.kind;
+    uint64_t off = pstart[s];
+    for (int i = 0; i < S.n_sections; ++i) {
+      const pcs_section& x = S.sections[i];
+      d.push_back(make_desc(x, rec + off, x.ring_start));
+      Entry e{};
+      e.type = x.type;
+      e.dtype = x.dtype;
+      e.layer = x.layer;
+      e.layout = x.layout;
+      e.offset = off;
+      e.bytes = x.bytes;
+      e.fp = 0;
+      e.dim0 = x.dim0;
+      e.dim1 = x.dim1;
+      e.aux = x.layout == PCS_LAYOUT_RING ? x.ring_start : 0;
+      ent.push_back(e);
+      h->table.push_back(e);
+      off = round_up(off + x.bytes, kRecordAlign);
+    }
+    (*handles)[s] = std::move(h);
+  }
+  PtrCache cache;
+  std::vector<char> bulk(d.size());
+  const bool small = total_bytes(d) <= kSmallCallBytes;
+  for (size_t i = 0; i < d.size(); ++i)
+    bulk[i] = bulk_eligible(c, d[i], placement == PCS_PLACE_DEVICE, small, cache);
+  uint32_t max_secs = 0;
+  for (int s = 0; s < n; ++s) max_secs = std::max<uint32_t>(max_secs, sd[s].n_sections);
+  pr->mode = kModePack;
+  pr->n = n;
+  pr->fused = fused_ok(bulk, small, n) && max_secs <= 2048;
+  if (!plan_streams(c, d, bulk, pr->P, !pr->fused)) {
+    arena_of(c, placement)->free(blk);
+    return fail(PCS_E_INVAL, "too much data in one call");
+  }
+  WsLayout& L = pr->L;
+  L.secs = 0;
+  L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
+  L.entries = round_up(L.sess + sizeof(SessDesc) * n, kRecordAlign);
+  pr->LL = list_layout(pr->P, L.entries + sizeof(Entry) * ent.size());
+  L.nodes = round_up(pr->LL.end, kRecordAlign);
+  L.total = L.nodes + 8 * pr->P.nodes_total;
+  pr->plan.resize(L.nodes);
+  put(pr->plan, L.secs, d);
+  put(pr->plan, L.sess, sd);
+  put(pr->plan, L.entries, ent);
+  put_lists(pr->plan, pr->P, pr->LL);
+  *blk_out = blk;
+  return PCS_OK;
+}
+
+// Plan a restore of n snapshots into n target sessions.
+pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
+                         const pcs_session* targets, int verify, Prepared* pr) {
+  std::vector<SecDesc> d;
+  std::vector<SessDesc> sd(n);
+  std::vector<char> payload_dev;
+  for (int s = 0; s < n; ++s) {
+    pcs_snapshot* h = check_handle(c, snaps[s]);
+    if (!h) return fail(PCS_E_HANDLE, "snapshot %d: unknown handle", s);
+    const pcs_session& T = targets[s];
+    if (T.n_sections != static_cast<int32_t>(h->table.size()) || !T.sections)
+      return fail(PCS_E_INVAL, "session %d: target has %d sections, snapshot %zu", s,
+                  T.n_sections, h->table.size());
+    sd[s].record = h->record();
+    sd[s].total_bytes = h->total_bytes;
+    sd[s].payload_start = h->payload_start;
+    sd[s].sec_begin = static_cast<uint32_t>(d.size());
+    sd[s].n_sections = static_cast<uint32_t>(T.n_sections);
+    sd[s].session_id = h->session_id;
+    sd[s].kind = h->kind;
+    for (int i = 0; i < T.n_sections; ++i) {
+      const pcs_section& x = T.sections[i];
+      pcs_status st = check_section(x, s, i, true);
+      if (st) return st;
+      const Entry& e = h->table[i];
+      if (x.bytes != e.bytes)
+        return fail(PCS_E_INVAL, "session %d section %d: target bytes %llu != snapshot %llu", s, i,
+                    static_cast<unsigned long long>(x.bytes), static_cast<unsigned long long>(e.bytes));
+      uint32_t rs = x.ring_start;
+      if (x.layout == PCS_LAYOUT_RING && rs == PCS_RING_START_FROM_SNAPSHOT) {
+        if (e.layout != PCS_LAYOUT_RING || e.aux >= x.window)
+          return fail(PCS_E_INVAL, "session %d section %d: no stored ring start fits", s, i);
+        rs = static_cast<uint32_t>(e.aux);
+      }
+      d.push_back(make_desc(x, h->record() + e.offset, rs));
+      payload_dev.push_back(h->block->placement == PCS_PLACE_DEVICE);
+    }
+  }
+  PtrCache cache;
+  std::vector<char> bulk(d.size());
+  const bool small = total_bytes(d) <= kSmallCallBytes;
+  for (size_t i = 0; i < d.size(); ++i) bulk[i] = bulk_eligible(c, d[i], payload_dev[i], small, cache);
+  uint32_t max_secs = 0;
+  for (int s = 0; s < n; ++s) max_secs = std::max<uint32_t>(max_secs, sd[s].n_sections);
+  pr->mode = verify ? kModeRestoreV : kModeRestore;
+  pr->verify = verify;
+  pr->n = n;
+  pr->fused = verify && fused_ok(bulk, small, n) && max_secs <= 2048;
+  if (!plan_streams(c, d, bulk, pr->P, !pr->fused))
+    return fail(PCS_E_INVAL, "too much data in one call");
+  WsLayout& L = pr->L;
+  L.secs = 0;
+  L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
+  pr->LL = list_layout(pr->P, L.sess + sizeof(SessDesc) * n);
+  L.nodes = round_up(pr->LL.end, kRecordAlign);
+  L.total = L.nodes + (verify ? 8 * pr->P.nodes_total : 0);
+  pr->plan.resize(L.nodes);
+  put(pr->plan, L.secs, d);
+  put(pr->plan, L.sess, sd);
+  put_lists(pr->plan, pr->P, pr->LL);
+  return PCS_OK;
+}
+
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -1438,131 +1655,26 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   if (n < 0 || (n > 0 && (!sessions || !out))) return fail(PCS_E_INVAL, "bad session list");
-  if (placement != PCS_PLACE_DEVICE && placement != PCS_PLACE_PINNED_HOST)
-    return fail(PCS_E_INVAL, "unknown placement %u", placement);
   if (n == 0) return PCS_OK;
-  // Plan records: sizes, offsets, entries.
-  std::vector<uint64_t> rec_off(n + 1, 0), pstart(n);
-  uint64_t total_secs = 0;
-  for (int s = 0; s < n; ++s) {
-    const pcs_session& S = sessions[s];
-    if (S.n_sections < 1 || S.n_sections > 65535 || !S.sections)
-      return fail(PCS_E_INVAL, "session %d: needs 1..65535 sections", s);
-    for (int i = 0; i < S.n_sections; ++i) {
-      pcs_status st = check_section(S.sections[i], s, i, false);
-      if (st) return st;
-    }
-    uint64_t bytes = 0;
-    pcs_record_bytes(S.sections, S.n_sections, &bytes);
-    pstart[s] = round_up(kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * S.n_sections, kRecordAlign);
-    rec_off[s + 1] = rec_off[s] + bytes;
-    total_secs += S.n_sections;
-  }
-  if (total_secs > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many sections in one call");
   std::lock_guard<std::mutex> lk(c->mu);
   pcs_status st = set_device(c);
   if (st) return st;
+  Prepared pr;
   Block* blk = nullptr;
-  st = arena_of(c, placement)->alloc(rec_off[n], stream, &blk);
+  std::vector<std::unique_ptr<pcs_snapshot>> handles;
+  st = build_checkpoint(c, sessions, n, placement, stream, &pr, &blk, &handles);
   if (st) return st;
-  std::vector<SecDesc> d;
-  std::vector<SessDesc> sd(n);
-  std::vector<Entry> ent;
-  d.reserve(total_secs);
-  ent.reserve(total_secs);
-  std::vector<std::unique_ptr<pcs_snapshot>> handles(n);
-  uint64_t chunks = 0;
-  for (int s = 0; s < n; ++s) {
-    const pcs_session& S = sessions[s];
-    uint8_t* rec = blk->ptr + rec_off[s];
-    auto h = std::make_unique<pcs_snapshot>();
-    h->block = blk;
-    h->offset = rec_off[s];
-    h->total_bytes = rec_off[s + 1] - rec_off[s];
-    h->payload_start = pstart[s];
-    h->session_id = S.session_id;
-    h->kind = S.kind;
-    sd[s].record = rec;
-    sd[s].total_bytes = h->total_bytes;
-    sd[s].payload_start = pstart[s];
-    sd[s].sec_begin = static_cast<uint32_t>(d.size());
-    sd[s].n_sections = static_cast<uint32_t>(S.n_sections);
-    sd[s].session_id = S.session_id;
-    sd[s].kind = S.kind;
-    uint64_t off = pstart[s];
-    for (int i = 0; i < S.n_sections; ++i) {
-      const pcs_section& x = S.sections[i];
-      SecDesc desc = make_desc(x, rec + off, x.ring_start);
-      chunks += desc.n_chunks;
-      d.push_back(desc);
-      Entry e{};
-      e.type = x.type;
-      e.dtype = x.dtype;
-      e.layer = x.layer;
-      e.layout = x.layout;
-      e.offset = off;
-      e.bytes = x.bytes;
-      e.fp = 0;
-      e.dim0 = x.dim0;
-      e.dim1 = x.dim1;
-      e.aux = x.layout == PCS_LAYOUT_RING ? x.ring_start : 0;
-      ent.push_back(e);
-      h->table.push_back(e);
-      off = round_up(off + x.bytes, kRecordAlign);
-    }
-    handles[s] = std::move(h);
-  }
-  (void)chunks;
-  PtrCache cache;
-  std::vector<char> bulk(d.size());
-  const bool small = total_bytes(d) <= kSmallCallBytes;
-  for (size_t i = 0; i < d.size(); ++i)
-    bulk[i] = bulk_eligible(c, d[i], placement == PCS_PLACE_DEVICE, small, cache);
-  uint32_t max_secs = 0;
-  for (int s = 0; s < n; ++s) max_secs = std::max<uint32_t>(max_secs, sd[s].n_sections);
-  const bool fused = fused_ok(bulk, small, n) && max_secs <= 2048;
-  StreamPlan P;
-  const bool fits = plan_streams(c, d, bulk, P, !fused);
-  WsLayout L;
-  L.secs = 0;
-  L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
-  L.entries = round_up(L.sess + sizeof(SessDesc) * n, kRecordAlign);
-  const ListLayout LL = list_layout(P, L.entries + sizeof(Entry) * ent.size());
-  L.nodes = round_up(LL.end, kRecordAlign);
-  L.total = L.nodes + 8 * P.nodes_total;
   auto undo = [&](pcs_status s) {
     arena_of(c, placement)->free(blk);
     return s;
   };
-  if (!fits) return undo(fail(PCS_E_INVAL, "too much data in one call"));
   uint8_t* ws = nullptr;
-  st = ws_acquire(c, L.total, stream, &ws);
+  st = ws_acquire(c, pr.L.total, stream, &ws);
   if (st) return undo(st);
-  c->plan.resize(L.nodes);
-  put(c->plan, L.secs, d);
-  put(c->plan, L.sess, sd);
-  put(c->plan, L.entries, ent);
-  put_lists(c->plan, P, LL);
-  cudaError_t e = plan_copy(c, ws, L.nodes, stream);
-  auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
-  auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
-  auto* dent = reinterpret_cast<const Entry*>(ws + L.entries);
-  auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
-  if (fused && e == cudaSuccess) {
-    WorkList wl{reinterpret_cast<const uint32_t*>(ws + LL.reg_ids),
-                reinterpret_cast<const uint32_t*>(ws + LL.reg_begin),
-                static_cast<int>(P.reg_ids.size()), P.reg_tasks};
-    LaunchScope ls(c, kKStreamPack, stream);
-    e = launch_small(kModePack, dsecs, wl, P.glog2, nodes, c->words, c->words + 3, n, dsess, dent,
-                     nullptr, nullptr, nullptr, nullptr, c->sm_count, c->stream_bps, stream);
-  } else {
-    if (e == cudaSuccess) e = launch_streams(c, kModePack, dsecs, P, LL, ws, nodes, stream);
-    if (e == cudaSuccess) {
-      LaunchScope ls(c, kKFinalizePack, stream);
-      e = launch_finalize(kModePack, dsecs, dsess, n, dent, nodes, nullptr, nullptr, nullptr,
-                          nullptr, stream);
-    }
-  }
+  c->plan.swap(pr.plan);
+  cudaError_t e = plan_copy(c, ws, pr.L.nodes, stream);
+  c->plan.swap(pr.plan);
+  if (e == cudaSuccess) e = launch_prepared(c, pr, ws, stream);
   if (e != cudaSuccess) return undo(cuda_fail(e, "checkpoint launch"));
   blk->written = record_event(c->events, stream);
   st = ws_release(c, stream, blk->written);
@@ -1677,95 +1789,24 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   std::lock_guard<std::mutex> lk(c->mu);
   pcs_status st = set_device(c);
   if (st) return st;
-  std::vector<SecDesc> d;
-  std::vector<SessDesc> sd(n);
-  std::vector<char> payload_dev;
-  uint64_t chunks = 0;
-  for (int s = 0; s < n; ++s) {
-    pcs_snapshot* h = check_handle(c, snaps[s]);
-    if (!h) return fail(PCS_E_HANDLE, "snapshot %d: unknown handle", s);
-    const pcs_session& T = targets[s];
-    if (T.n_sections != static_cast<int32_t>(h->table.size()) || !T.sections)
-      return fail(PCS_E_INVAL, "session %d: target has %d sections, snapshot %zu", s,
-                  T.n_sections, h->table.size());
-    sd[s].record = h->record();
-    sd[s].total_bytes = h->total_bytes;
-    sd[s].payload_start = h->payload_start;
-    sd[s].sec_begin = static_cast<uint32_t>(d.size());
-    sd[s].n_sections = static_cast<uint32_t>(T.n_sections);
-    sd[s].session_id = h->session_id;
-    sd[s].kind = h->kind;
-    for (int i = 0; i < T.n_sections; ++i) {
-      const pcs_section& x = T.sections[i];
-      st = check_section(x, s, i, true);
-      if (st) return st;
-      const Entry& e = h->table[i];
-      if (x.bytes != e.bytes)
-        return fail(PCS_E_INVAL, "session %d section %d: target bytes %llu != snapshot %llu", s, i,
-                    static_cast<unsigned long long>(x.bytes), static_cast<unsigned long long>(e.bytes));
-      uint32_t rs = x.ring_start;
-      if (x.layout == PCS_LAYOUT_RING && rs == PCS_RING_START_FROM_SNAPSHOT) {
-        if (e.layout != PCS_LAYOUT_RING || e.aux >= x.window)
-          return fail(PCS_E_INVAL, "session %d section %d: no stored ring start fits", s, i);
-        rs = static_cast<uint32_t>(e.aux);
-      }
-      SecDesc desc = make_desc(x, h->record() + e.offset, rs);
-      chunks += desc.n_chunks;
-      d.push_back(desc);
-      payload_dev.push_back(h->block->placement == PCS_PLACE_DEVICE);
-    }
-  }
+  Prepared pr;
+  st = build_restore(c, snaps, n, targets, verify, &pr);
+  if (st) return st;
   for (int s = 0; s < n; ++s) {
     st = wait_written(snaps[s]->block, stream);
     if (st) return st;
   }
-  (void)chunks;
-  PtrCache cache;
-  std::vector<char> bulk(d.size());
-  const bool small = total_bytes(d) <= kSmallCallBytes;
-  for (size_t i = 0; i < d.size(); ++i) bulk[i] = bulk_eligible(c, d[i], payload_dev[i], small, cache);
-  uint32_t max_secs = 0;
-  for (int s = 0; s < n; ++s) max_secs = std::max<uint32_t>(max_secs, sd[s].n_sections);
-  const bool fused = verify && fused_ok(bulk, small, n) && max_secs <= 2048;
-  StreamPlan P;
-  if (!plan_streams(c, d, bulk, P, !fused)) return fail(PCS_E_INVAL, "too much data in one call");
-  WsLayout L;
-  L.secs = 0;
-  L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
-  const ListLayout LL = list_layout(P, L.sess + sizeof(SessDesc) * n);
-  L.nodes = round_up(LL.end, kRecordAlign);
-  L.total = L.nodes + (verify ? 8 * P.nodes_total : 0);
   uint8_t* ws = nullptr;
-  st = ws_acquire(c, L.total, stream, &ws);
+  st = ws_acquire(c, pr.L.total, stream, &ws);
   if (st) return st;
-  c->plan.resize(L.nodes);
-  put(c->plan, L.secs, d);
-  put(c->plan, L.sess, sd);
-  put_lists(c->plan, P, LL);
-  PCS_CUDA(plan_copy(c, ws, L.nodes, stream));
-  auto* dsecs = reinterpret_cast<const SecDesc*>(ws + L.secs);
-  auto* dsess = reinterpret_cast<const SessDesc*>(ws + L.sess);
-  auto* nodes = reinterpret_cast<uint64_t*>(ws + L.nodes);
+  c->plan.swap(pr.plan);
+  cudaError_t e = plan_copy(c, ws, pr.L.nodes, stream);
+  c->plan.swap(pr.plan);
+  PCS_CUDA(e);
   // verify == 1: count failures of this call in words[1] and wait for them;
   // verify == 2: accumulate them in words[2] for the next pcs_sync.
   if (verify == 1) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
-  if (fused) {
-    WorkList wl{reinterpret_cast<const uint32_t*>(ws + LL.reg_ids),
-                reinterpret_cast<const uint32_t*>(ws + LL.reg_begin),
-                static_cast<int>(P.reg_ids.size()), P.reg_tasks};
-    LaunchScope ls(c, kKStreamRestoreV, stream);
-    PCS_CUDA(launch_small(kModeRestoreV, dsecs, wl, P.glog2, nodes, c->words, c->words + 3, n,
-                          dsess, nullptr, nullptr, nullptr, nullptr,
-                          c->words + (verify == 1 ? 1 : 2), c->sm_count, c->stream_bps, stream));
-  } else {
-    PCS_CUDA(launch_streams(c, verify ? kModeRestoreV : kModeRestore, dsecs, P, LL, ws,
-                            verify ? nodes : nullptr, stream));
-    if (verify) {
-      LaunchScope ls(c, kKFinalizeRestoreV, stream);
-      PCS_CUDA(launch_finalize(kModeRestoreV, dsecs, dsess, n, nullptr, nodes, nullptr, nullptr,
-                               nullptr, c->words + (verify == 1 ? 1 : 2), stream));
-    }
-  }
+  PCS_CUDA(launch_prepared(c, pr, ws, stream));
   for (int s = 0; s < n; ++s) {
     st = note_use(c, snaps[s]->block, stream);
     if (st) return st;
