@@ -571,6 +571,26 @@ def run_rows(ctx, dev, stream):
     torch.cuda.synchronize()
     rs_us = (time.perf_counter() - t0) / n * 1e6
     ctx.delete_raw(h0, 1)
+    # One session as prepared calls: launches only.
+    p1, ph = ctx.plan_checkpoint(oarr, 1)
+    pr1 = ctx.plan_restore(ph, 1, oarr, verify=0)
+    for _ in range(20):
+        ctx.plan_run(p1)
+        ctx.plan_run(pr1)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(n):
+        ctx.plan_run(p1)
+    torch.cuda.synchronize()
+    pck_us = (time.perf_counter() - t0) / n * 1e6
+    t0 = time.perf_counter()
+    for _ in range(n):
+        ctx.plan_run(pr1)
+    torch.cuda.synchronize()
+    prs_us = (time.perf_counter() - t0) / n * 1e6
+    ctx.plan_destroy(pr1)
+    ctx.plan_destroy(p1)
+    ctx.delete_raw(ph, 1)
     g = torch.Generator(device=dev).manual_seed(synth.seed_for(1))
     obs = torch.randint(0, 256, (4096, 3, 256, 256), generator=g, device=dev, dtype=torch.uint8)
     rng = torch.randint(-2**62, 2**62, (4096, 2), generator=g, device=dev, dtype=torch.int64)
@@ -582,13 +602,31 @@ def run_rows(ctx, dev, stream):
         ctx.restore_raw(hs, 4096, barr)
         ctx.delete_raw(hs, 4096)
     med = _loop_ms(batch_step, stream, calls=5, warm=1)
+    # The same step as prepared calls: planned once, then launches only.
+    cplan, phs = ctx.plan_checkpoint(barr, 4096)
+    rplan = ctx.plan_restore(phs, 4096, barr, verify=2)
+
+    def prepared_step():
+        ctx.plan_run(cplan)
+        ctx.plan_run(rplan)
+    medp = _loop_ms(prepared_step, stream, calls=20, warm=2)
+    ctx.sync()
+    ctx.plan_destroy(rplan)
+    ctx.plan_destroy(cplan)
+    ctx.delete_raw(phs, 4096)
     out["markov"] = {"one_session_checkpoint_us": round(ck_us, 2),
                      "one_session_restore_us": round(rs_us, 2),
+                     "one_session_prepared_checkpoint_us": round(pck_us, 2),
+                     "one_session_prepared_restore_us": round(prs_us, 2),
                      "how": "wall clock per call (checkpoint incl. delete) through the ctypes "
                             "binding with a prebuilt session array, 1000 calls",
                      "paper_context_us": 12.0,
                      "batch_4096_sessions_per_s": round(4096 / (med / 1e3), 1),
-                     "batch_GBs": round(4 * 4096 * (196608 + 16) / (med / 1e3) / 1e9, 1)}
+                     "batch_GBs": round(4 * 4096 * (196608 + 16) / (med / 1e3) / 1e9, 1),
+                     "prepared_4096_sessions_per_s": round(4096 / (medp / 1e3), 1),
+                     "prepared_GBs": round(4 * 4096 * (196608 + 16) / (medp / 1e3) / 1e9, 1),
+                     "prepared_frac_of_hbm": round(4 * 4096 * (196608 + 16) / (medp / 1e3) / 1e9
+                                                   / peak, 4)}
     del obs, rng, batch, barr
     out["cow_fork"] = measure_cow_fork(ctx, dev, stream, peak)
     return out

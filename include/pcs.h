@@ -115,6 +115,7 @@ typedef int32_t pcs_status;
 typedef struct pcs_ctx pcs_ctx;
 typedef struct pcs_snapshot pcs_snapshot;
 typedef struct pcs_pool pcs_pool;
+typedef struct pcs_plan pcs_plan;
 
 /* A runtime buffer to fingerprint: `bytes` bytes at device pointer `ptr`. */
 typedef struct pcs_buf {
@@ -485,6 +486,32 @@ pcs_status pcs_fork_many(pcs_ctx *ctx, pcs_snapshot *const *parents, int32_t n,
  */
 pcs_status pcs_restore(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n,
                        const pcs_session *targets, int32_t verify, void *stream);
+
+/*
+ * Prepared calls, for the same checkpoint or restore repeated (a periodic
+ * checkpoint of a fixed set of sessions, a restore that recurs): the call is
+ * planned once -- validation, descriptors, launch shape, uploaded into a
+ * device buffer of the plan -- and each pcs_plan_run only launches kernels.
+ * Everything a section describes (pointers, sizes, layouts, ring starts) is
+ * fixed at plan time; the bytes it points at are read at run time.  Runs of
+ * one plan must be ordered (they share its scratch).
+ *
+ * pcs_plan_checkpoint: plans checkpoint(s) of n sessions, creates their n
+ * snapshots (out, host array) and runs the first checkpoint on `stream`.
+ * Every later run overwrites the same records in place (the snapshots are
+ * the plan's latest checkpoint); the records stay valid until both the
+ * snapshots are deleted and the plan destroyed.
+ * pcs_plan_restore: plans restore(c) of n snapshots into n targets; verify
+ * 0 or 2 (mismatches reported by pcs_sync).  The plan keeps the snapshots'
+ * records alive until it is destroyed.
+ */
+pcs_status pcs_plan_checkpoint(pcs_ctx *ctx, const pcs_session *sessions, int32_t n,
+                               uint32_t placement, pcs_snapshot **out, pcs_plan **plan,
+                               void *stream);
+pcs_status pcs_plan_restore(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n,
+                            const pcs_session *targets, int32_t verify, pcs_plan **plan);
+pcs_status pcs_plan_run(pcs_ctx *ctx, pcs_plan *plan, void *stream);
+pcs_status pcs_plan_destroy(pcs_ctx *ctx, pcs_plan *plan);
 
 /* delete(c): release a snapshot (its memory is reused once pending work
  * that reads it has finished). */

@@ -318,6 +318,8 @@ struct pcs_pool {
   void* meta = nullptr;  // counts, free stack and top in one allocation
 };
 
+struct pcs_plan;
+
 struct pcs_ctx {
   int device = 0;
   int sm_count = 0;
@@ -353,6 +355,7 @@ struct pcs_ctx {
   double kernel_ms[32] = {};
   uint64_t kernel_n[32] = {};
   std::unordered_set<pcs_pool*> pools;  // live page pools
+  std::unordered_set<pcs_plan*> plans;  // live prepared calls
 };
 
 namespace {
@@ -902,6 +905,37 @@ struct Prepared {
   std::vector<uint8_t> plan;
 };
 
+}  // namespace
+
+// A prepared call: its descriptors in a device buffer of its own, and one
+// reference on every record block it writes or reads.
+struct pcs_plan {
+  Prepared pr;
+  uint8_t* dev = nullptr;
+  std::vector<Block*> blocks;
+};
+
+namespace {
+
+void destroy_plan(pcs_ctx* c, pcs_plan* p) {
+  if (p->dev) cudaFree(p->dev);  // waits for the device
+  for (Block* b : p->blocks) release_block(c, b);
+  delete p;
+}
+
+void destroy_plans(pcs_ctx* c) {
+  for (auto* p : c->plans) destroy_plan(c, p);
+  c->plans.clear();
+}
+
+// The plan's own device copy of its descriptors, with room for its nodes.
+pcs_status plan_upload(pcs_plan* p) {
+  PCS_CUDA(cudaMalloc(&p->dev, std::max<uint64_t>(p->pr.L.total, 16)));
+  if (!p->pr.plan.empty())
+    PCS_CUDA(cudaMemcpy(p->dev, p->pr.plan.data(), p->pr.plan.size(), cudaMemcpyHostToDevice));
+  return PCS_OK;
+}
+
 // Launch a prepared call whose descriptors are at `ws` (nodes after them).
 cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, cudaStream_t stream) {
   const auto* dsecs = reinterpret_cast<const SecDesc*>(ws + pr.L.secs);
@@ -1174,6 +1208,7 @@ pcs_status pcs_destroy(pcs_ctx* c) {
       delete pl;
     }
     c->pools.clear();
+    destroy_plans(c);
     c->ws_busy.reset();
     if (c->ws) cudaFree(c->ws);
     if (c->words) cudaFree(c->words);
@@ -1819,6 +1854,116 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
     PCS_CUDA(cudaStreamSynchronize(stream));
     if (bad) return fail(PCS_E_CORRUPT, "%u of %d restored sessions failed verification", bad, n);
   }
+  return PCS_OK;
+}
+
+// ---- Prepared calls ---------------------------------------------------------
+
+pcs_status pcs_plan_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n,
+                               uint32_t placement, pcs_snapshot** out, pcs_plan** plan,
+                               void* stream_) {
+  if (!c || !plan) return fail(PCS_E_INVAL, "bad arguments");
+  *plan = nullptr;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  if (n <= 0 || !sessions || !out) return fail(PCS_E_INVAL, "bad session list");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  auto p = std::make_unique<pcs_plan>();
+  Block* blk = nullptr;
+  std::vector<std::unique_ptr<pcs_snapshot>> handles;
+  st = build_checkpoint(c, sessions, n, placement, stream, &p->pr, &blk, &handles);
+  if (st) return st;
+  st = plan_upload(p.get());
+  cudaError_t e = st ? cudaSuccess : launch_prepared(c, p->pr, p->dev, stream);
+  if (st || e != cudaSuccess) {
+    if (p->dev) cudaFree(p->dev);
+    arena_of(c, placement)->free(blk);
+    return st ? st : cuda_fail(e, "checkpoint launch");
+  }
+  blk->written = record_event(c->events, stream);
+  blk->refs = n + 1;  // the snapshots and the plan
+  p->blocks.push_back(blk);
+  for (int s = 0; s < n; ++s) {
+    out[s] = handles[s].release();
+    c->live.insert(out[s]);
+  }
+  *plan = p.release();
+  c->plans.insert(*plan);
+  return PCS_OK;
+}
+
+pcs_status pcs_plan_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
+                            const pcs_session* targets, int32_t verify, pcs_plan** plan) {
+  if (!c || !plan) return fail(PCS_E_INVAL, "bad arguments");
+  *plan = nullptr;
+  if (n <= 0 || !snaps || !targets) return fail(PCS_E_INVAL, "bad arguments");
+  if (verify != 0 && verify != 2)
+    return fail(PCS_E_INVAL, "a prepared restore verifies with 0 or 2 (reported at pcs_sync)");
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  auto p = std::make_unique<pcs_plan>();
+  st = build_restore(c, snaps, n, targets, verify, &p->pr);
+  if (st) return st;
+  st = plan_upload(p.get());
+  if (st) {
+    if (p->dev) cudaFree(p->dev);
+    return st;
+  }
+  for (int s = 0; s < n; ++s) {
+    Block* b = snaps[s]->block;
+    if (std::find(p->blocks.begin(), p->blocks.end(), b) == p->blocks.end()) {
+      ++b->refs;
+      p->blocks.push_back(b);
+    }
+  }
+  *plan = p.release();
+  c->plans.insert(*plan);
+  return PCS_OK;
+}
+
+pcs_status pcs_plan_run(pcs_ctx* c, pcs_plan* p, void* stream_) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+  std::lock_guard<std::mutex> lk(c->mu);
+  if (!p || !c->plans.count(p)) return fail(PCS_E_HANDLE, "not a live plan of this context");
+  pcs_status st = set_device(c);
+  if (st) return st;
+  const bool ckpt = p->pr.mode == kModePack;
+  for (Block* b : p->blocks) {
+    if (!ckpt) {
+      st = wait_written(b, stream);  // the records' latest checkpoint
+      if (st) return st;
+      continue;
+    }
+    // Rewriting records: after every queued reader of them, on any stream.
+    for (auto& u : b->uses)
+      if (u.first != stream && u.second && !u.second->done())
+        PCS_CUDA(cudaStreamWaitEvent(stream, u.second->ev, 0));
+  }
+  PCS_CUDA(launch_prepared(c, p->pr, p->dev, stream));
+  for (Block* b : p->blocks) {
+    if (ckpt) {
+      b->written = record_event(c->events, stream);
+      if (!b->written) return fail(PCS_E_CUDA, "cudaEventRecord failed");
+    } else {
+      st = note_use(c, b, stream);
+      if (st) return st;
+    }
+  }
+  return PCS_OK;
+}
+
+pcs_status pcs_plan_destroy(pcs_ctx* c, pcs_plan* p) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  if (!p) return PCS_OK;
+  std::lock_guard<std::mutex> lk(c->mu);
+  if (!c->plans.count(p)) return fail(PCS_E_HANDLE, "not a live plan of this context");
+  pcs_status st = set_device(c);
+  if (st) return st;
+  c->plans.erase(p);
+  destroy_plan(c, p);
   return PCS_OK;
 }
 

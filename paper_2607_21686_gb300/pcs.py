@@ -159,6 +159,12 @@ SIGNATURES = {
                                  _vp]),
     "pcs_discover": (_st, [_i32, _vp, _vp, _u64, ctypes.POINTER(ctypes.c_uint8),
                            ctypes.POINTER(_i32), ctypes.POINTER(_i32)]),
+    "pcs_plan_checkpoint": (_st, [_vp, ctypes.POINTER(pcs_session), _i32, _u32,
+                                  ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp]),
+    "pcs_plan_restore": (_st, [_vp, ctypes.POINTER(_vp), _i32, ctypes.POINTER(pcs_session), _i32,
+                               ctypes.POINTER(_vp)]),
+    "pcs_plan_run": (_st, [_vp, _vp, _vp]),
+    "pcs_plan_destroy": (_st, [_vp, _vp]),
     "pcs_fingerprint_static": (_st, [ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
 }
 # int32 probe(void* user, const uint8_t* keep, uint64_t* distance)
@@ -637,6 +643,28 @@ class Context:
 
     def delete_raw(self, handles, n: int) -> None:
         check(self.lib.pcs_delete_many(self.h, handles, n), "pcs_delete_many")
+
+    # -- prepared calls ---------------------------------------------------------
+    def plan_checkpoint(self, arr, n: int, placement: int = PCS_PLACE_DEVICE, stream=None):
+        """Plan checkpoint(s) of a prebuilt session array and run it once:
+        (plan handle, ctypes array of the n snapshot handles)."""
+        out = (ctypes.c_void_p * max(n, 1))()
+        plan = ctypes.c_void_p()
+        check(self.lib.pcs_plan_checkpoint(self.h, arr, n, placement, out, ctypes.byref(plan),
+                                           _stream_ptr(stream)), "pcs_plan_checkpoint")
+        return plan, out
+
+    def plan_restore(self, handles, n: int, arr, verify: int = 0):
+        plan = ctypes.c_void_p()
+        check(self.lib.pcs_plan_restore(self.h, handles, n, arr, verify, ctypes.byref(plan)),
+              "pcs_plan_restore")
+        return plan
+
+    def plan_run(self, plan, stream=None) -> None:
+        check(self.lib.pcs_plan_run(self.h, plan, _stream_ptr(stream)), "pcs_plan_run")
+
+    def plan_destroy(self, plan) -> None:
+        check(self.lib.pcs_plan_destroy(self.h, plan), "pcs_plan_destroy")
 
     def fork(self, snap: Snapshot, stream=None) -> Snapshot:
         out = ctypes.c_void_p()
