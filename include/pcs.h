@@ -228,6 +228,14 @@ const char *pcs_last_error(void);
 const char *pcs_status_string(pcs_status s);
 
 /*
+ * Cap the memory the context reserves for snapshots of one placement
+ * (bytes; 0 = no cap, the default).  Reservations already made stay; empty
+ * ones over the cap are returned.  A call that would need more fails with
+ * PCS_E_NOMEM before any launch and leaves no snapshot behind.
+ */
+pcs_status pcs_set_arena_limit(pcs_ctx *ctx, uint32_t placement, uint64_t bytes);
+
+/*
  * Create a context on CUDA device `device`: it owns the snapshot arenas,
  * the workspace of the kernels and the snapshot table.  PCS_E_CUDA if the
  * device cannot be used.

@@ -251,10 +251,21 @@ class Arena {
     return t;
   }
 
+  // Cap on the bytes this arena reserves (0: none).
+  void set_limit(uint64_t bytes) {
+    limit_ = bytes;
+    if (limit_ && reserved() > limit_) trim();
+  }
+
  private:
   pcs_status new_slab(uint64_t bytes) {
     const uint64_t min_slab = placement_ == PCS_PLACE_DEVICE ? (256ull << 20) : (64ull << 20);
-    const uint64_t size = round_up(std::max(bytes, min_slab), 2ull << 20);
+    uint64_t size = round_up(std::max(bytes, min_slab), 2ull << 20);
+    if (limit_) {
+      const uint64_t have = reserved();
+      if (have + size > limit_) size = round_up(bytes, 2ull << 20);  // no headroom slab
+      if (have + size > limit_) return PCS_E_NOMEM;
+    }
     void* p = nullptr;
     if (placement_ == PCS_PLACE_DEVICE) {
       if (cudaMalloc(&p, size) != cudaSuccess) return PCS_E_NOMEM;
@@ -291,6 +302,7 @@ class Arena {
   }
 
   uint32_t placement_;
+  uint64_t limit_ = 0;
   std::shared_ptr<EventPool> pool_;
   std::vector<std::unique_ptr<Slab>> slabs_;
   std::map<void*, void*> host_of_;
@@ -1224,6 +1236,17 @@ pcs_status pcs_destroy(pcs_ctx* c) {
     c->host_arena.reset();
   }
   delete c;
+  return PCS_OK;
+}
+
+pcs_status pcs_set_arena_limit(pcs_ctx* c, uint32_t placement, uint64_t bytes) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  if (placement != PCS_PLACE_DEVICE && placement != PCS_PLACE_PINNED_HOST)
+    return fail(PCS_E_INVAL, "unknown placement %u", placement);
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  arena_of(c, placement)->set_limit(bytes);
   return PCS_OK;
 }
 

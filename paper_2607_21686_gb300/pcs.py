@@ -165,6 +165,7 @@ SIGNATURES = {
                                ctypes.POINTER(_vp)]),
     "pcs_plan_run": (_st, [_vp, _vp, _vp]),
     "pcs_plan_destroy": (_st, [_vp, _vp]),
+    "pcs_set_arena_limit": (_st, [_vp, _u32, _u64]),
     "pcs_fingerprint_static": (_st, [ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
 }
 # int32 probe(void* user, const uint8_t* keep, uint64_t* distance)
@@ -480,6 +481,9 @@ class Context:
 
     def __exit__(self, *exc):
         self.close()
+
+    def set_arena_limit(self, placement: int, nbytes: int) -> None:
+        check(self.lib.pcs_set_arena_limit(self.h, placement, nbytes), "pcs_set_arena_limit")
 
     def stats(self) -> pcs_stats:
         s = pcs_stats()
