@@ -229,7 +229,7 @@ const char *pcs_status_string(pcs_status s);
 
 /*
  * Cap the memory the context reserves for snapshots of one placement
- * (bytes; 0 = no cap, the default).  Reservations already made stay; empty
+ * (no paper counterpart: a runtime control; bytes; 0 = no cap, the default).  Reservations already made stay; empty
  * ones over the cap are returned.  A call that would need more fails with
  * PCS_E_NOMEM before any launch and leaves no snapshot behind.
  */
@@ -496,8 +496,10 @@ pcs_status pcs_restore(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n,
                        const pcs_session *targets, int32_t verify, void *stream);
 
 /*
- * Prepared calls, for the same checkpoint or restore repeated (a periodic
- * checkpoint of a fixed set of sessions, a restore that recurs): the call is
+ * Prepared calls (no paper counterpart: a runtime form of checkpoint(s) and
+ * restore(c) of Sec. 3 "The contract", same records, same verification),
+ * for the same checkpoint or restore repeated (a periodic checkpoint of a
+ * fixed set of sessions, a restore that recurs): the call is
  * planned once -- validation, descriptors, launch shape, uploaded into a
  * device buffer of the plan -- and each pcs_plan_run only launches kernels.
  * Everything a section describes (pointers, sizes, layouts, ring starts) is
