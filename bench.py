@@ -491,7 +491,27 @@ def run_rows(ctx, dev, stream):
     out["mismatch"] = {"population": "the same 200 buffer pairs (before, after)",
                        "bytes_read": 2 * tot, "ms": round(med, 3), "GBs": round(gbs, 1),
                        "frac_of_hbm": round(gbs / peak, 4), "counts_match_ground_truth": mm_ok}
-    del sw, fp0, must, fp1, counts, after_arr, before_arr
+    # State versus witness: a read log of 16M byte ranges (what a resume
+    # touched) against the same 200 buffers.
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(4) + 9)
+    bases = torch.tensor([t.data_ptr() for t in sw.after], dtype=torch.int64, device=dev)
+    lens = torch.tensor([t.numel() * t.element_size() for t in sw.after], dtype=torch.int64,
+                        device=dev)
+    m = 1 << 24
+    which = torch.randint(0, 140, (m,), generator=g, device=dev)  # 60 buffers never read
+    off = (torch.rand(m, generator=g, device=dev) * lens[which]).long()
+    addr = bases[which] + off
+    nbytes = torch.minimum(torch.randint(1, 4097, (m,), generator=g, device=dev,
+                                         dtype=torch.int64), lens[which] - off)  # within the buffer
+    flags = torch.empty(len(sw.after), dtype=torch.uint8, device=dev)
+    med = _loop_ms(lambda: ctx.classify_reads(after_arr, addr, nbytes, flags), stream)
+    read_ok = flags.cpu().tolist()[140:] == [0] * 60 and all(flags.cpu().tolist()[:140])
+    out["classify_reads"] = {"population": "16M reads (1 B-4 KiB) over 140 of the 200 buffers",
+                             "reads": m, "ms": round(med, 3),
+                             "Mreads_per_s": round(m / (med / 1e3) / 1e6, 1),
+                             "GBs_of_log": round(16 * m / (med / 1e3) / 1e9, 1),
+                             "flags_match_ground_truth": read_ok}
+    del sw, fp0, must, fp1, counts, after_arr, before_arr, addr, nbytes, which, bases, lens, off
 
     # a4-a5, a7, a10: 2048 banks, relevance top-k under an 8 GiB host budget,
     # pack to pinned host, verified restore to HBM.
@@ -523,6 +543,17 @@ def run_rows(ctx, dev, stream):
         "kept_fraction": round(gk / sum(b.n), 4),
         "kept_bytes": gk * (1024 + 2048)}
     del gkept, gkoff
+    # Recency-keyed retention (lru): the same banks kept by last-use step.
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(5) + 3)
+    last_use = torch.randint(0, 1 << 20, (sum(b.n),), generator=g, device=dev).float()
+    rk = [int(x * 0.627) for x in b.n]
+    rkept = torch.empty(sum(rk), dtype=torch.int32, device=dev)
+    n_arr, k_arr = ctx.int32_array(b.n), ctx.int32_array(rk)
+    med = _loop_ms(lambda: ctx.topk(last_use, n_arr, k_arr, rkept), stream)
+    out["topk_recency"] = {"population": "the same 2048 banks, lru keys, 62.7% kept per bank",
+                           "entries": sum(b.n), "ms": round(med, 3),
+                           "Mentries_per_s": round(sum(b.n) / (med / 1e3) / 1e6, 1)}
+    del last_use, rkept
     koff_h = koff.cpu().tolist()
     sess = [pcs.bank_session(s, keys[s], vals[s], kept[koff_h[s]:koff_h[s + 1]]) for s in range(S)]
     kept_bytes = sum(ks) * (1024 + 2048)

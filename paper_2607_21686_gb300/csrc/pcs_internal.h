@@ -268,7 +268,7 @@ struct ReadPlan {
   int32_t pad;
 };
 cudaError_t launch_classify_reads(const ReadPlan& p, const uint64_t* addr, const uint64_t* bytes,
-                                  int64_t m, uint8_t* flags, cudaStream_t stream);
+                                  int64_t m, uint8_t* flags, int sm_count, cudaStream_t stream);
 
 // Occupancy of the streaming kernel (blocks per SM) for the launch shape.
 int stream_blocks_per_sm();

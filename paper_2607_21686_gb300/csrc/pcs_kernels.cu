@@ -1829,30 +1829,67 @@ __global__ void __launch_bounds__(kThreads, 4)
 // passes the read's start.
 // ---------------------------------------------------------------------------
 
+// Threads stride over the reads; a block marks the buffers it saw in a
+// shared bitmap and writes each flag once at the end (many reads hit few
+// buffers, so stores to the flags would otherwise pile up on a few lines).
+// With few buffers the sorted arrays are staged in shared memory too.
+constexpr int kReadStage = 512;  // buffers staged in shared memory
+
 __global__ void __launch_bounds__(kThreads)
     k_classify_reads(ReadPlan P, const uint64_t* __restrict__ addr,
                      const uint64_t* __restrict__ bytes, int64_t m, uint8_t* flags) {
-  const int64_t j = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x;
-  if (j >= m) return;
-  const uint64_t a = addr[j], len = bytes[j];
-  if (len == 0) return;
-  const uint64_t e = a + len < a ? ~0ull : a + len;
-  int lo = 0, hi = P.n;  // hi: first buffer starting at or after e
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (P.start[mid] < e) lo = mid + 1;
-    else hi = mid;
+  extern __shared__ __align__(16) uint8_t rd_smem[];
+  uint32_t* const seen = reinterpret_cast<uint32_t*>(rd_smem);  // [words] bitmap
+  const int words = (P.n + 31) / 32;
+  const bool staged = P.n <= kReadStage;
+  uint64_t* s_start = reinterpret_cast<uint64_t*>(seen + ((words + 1) & ~1));
+  uint64_t* s_end = s_start + (staged ? P.n : 0);
+  uint64_t* s_max = s_end + (staged ? P.n : 0);
+  for (int w = threadIdx.x; w < words; w += kThreads) seen[w] = 0;
+  if (staged)
+    for (int i = threadIdx.x; i < P.n; i += kThreads) {
+      s_start[i] = P.start[i];
+      s_end[i] = P.end[i];
+      s_max[i] = P.maxend[i];
+    }
+  __syncthreads();
+  const uint64_t* st = staged ? s_start : P.start;
+  const uint64_t* en = staged ? s_end : P.end;
+  const uint64_t* mx = staged ? s_max : P.maxend;
+  for (int64_t j = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; j < m;
+       j += static_cast<int64_t>(gridDim.x) * kThreads) {
+    const uint64_t a = addr[j], len = bytes[j];
+    if (len == 0) continue;
+    const uint64_t e = a + len < a ? ~0ull : a + len;
+    int lo = 0, hi = P.n;  // hi: first buffer starting at or after e
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (st[mid] < e) lo = mid + 1;
+      else hi = mid;
+    }
+    const int end_i = lo;
+    lo = 0;
+    hi = end_i;  // first buffer whose running maximum end exceeds a
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (mx[mid] > a) hi = mid;
+      else lo = mid + 1;
+    }
+    for (int i = lo; i < end_i; ++i) {
+      const uint32_t bit = 1u << (i & 31);
+      // Most reads hit a buffer already marked: look before the atomic.
+      if (en[i] > a && en[i] > st[i] && !(seen[i >> 5] & bit)) atomicOr(&seen[i >> 5], bit);
+    }
   }
-  const int end_i = lo;
-  lo = 0;
-  hi = end_i;  // first buffer whose running maximum end exceeds a
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (P.maxend[mid] > a) hi = mid;
-    else lo = mid + 1;
+  __syncthreads();
+  for (int w = threadIdx.x; w < words; w += kThreads) {
+    uint32_t bits = seen[w];
+    while (bits) {
+      const int b = __ffs(bits) - 1;
+      bits &= bits - 1;
+      flags[P.orig[32 * w + b]] = 1;
+    }
   }
-  for (int i = lo; i < end_i; ++i)
-    if (P.end[i] > a && P.end[i] > P.start[i]) flags[P.orig[i]] = 1;
 }
 
 template <int MODE>
@@ -2088,9 +2125,21 @@ cudaError_t launch_mismatch(const MmPair* pairs, const uint64_t* unit_begin, int
 }
 
 cudaError_t launch_classify_reads(const ReadPlan& p, const uint64_t* addr, const uint64_t* bytes,
-                                  int64_t m, uint8_t* flags, cudaStream_t stream) {
+                                  int64_t m, uint8_t* flags, int sm_count, cudaStream_t stream) {
   if (m <= 0 || p.n <= 0) return cudaSuccess;
-  k_classify_reads<<<grid_for(m), kThreads, 0, stream>>>(p, addr, bytes, m, flags);
+  const size_t words = (static_cast<size_t>(p.n) + 31) / 32;
+  size_t smem = ((words + 1) & ~static_cast<size_t>(1)) * 4;
+  if (p.n <= kReadStage) smem += 24ull * p.n;
+  if (smem > 48 * 1024) {  // more buffers than a block's bitmap can hold
+    cudaError_t e = cudaFuncSetAttribute(k_classify_reads,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  const uint64_t want = (static_cast<uint64_t>(m) + kThreads - 1) / kThreads;
+  const uint64_t cap = static_cast<uint64_t>(sm_count) * 4;
+  k_classify_reads<<<static_cast<unsigned>(want < cap ? want : cap), kThreads, smem, stream>>>(
+      p, addr, bytes, m, flags);
   return cudaGetLastError();
 }
 

@@ -2444,7 +2444,7 @@ pcs_status pcs_classify_reads(pcs_ctx* c, const pcs_buf* bufs, int32_t n, const 
   rp.n = n;
   if (m > 0) {
     LaunchScope ls(c, kKClassifyReads, stream);
-    PCS_CUDA(launch_classify_reads(rp, addr, bytes, m, flags, stream));
+    PCS_CUDA(launch_classify_reads(rp, addr, bytes, m, flags, c->sm_count, stream));
   }
   return ws_release(c, stream);
 }

@@ -591,11 +591,17 @@ class Context:
                                  _ptr(kept_idx), _ptr(kept_off), _stream_ptr(stream)),
               "pcs_prune")
 
+    @staticmethod
+    def int32_array(values):
+        """A ctypes int32 array (prebuilt once for repeated calls)."""
+        return (ctypes.c_int32 * max(len(values), 1))(*values)
+
     def topk(self, keys: torch.Tensor, n, k, kept_idx: torch.Tensor, kept_off=None, stream=None):
-        """Keep-k per bank by caller rank keys (CSR float32 `keys`)."""
+        """Keep-k per bank by caller rank keys (CSR float32 `keys`); n and k
+        are sequences of ints or prebuilt int32_array()s."""
         nb = len(n)
-        na = (ctypes.c_int32 * max(nb, 1))(*n)
-        ka = (ctypes.c_int32 * max(nb, 1))(*k)
+        na = n if isinstance(n, ctypes.Array) else self.int32_array(n)
+        ka = k if isinstance(k, ctypes.Array) else self.int32_array(k)
         check(self.lib.pcs_topk(self.h, _ptr(keys), na, ka, nb, _ptr(kept_idx), _ptr(kept_off),
                                 _stream_ptr(stream)), "pcs_topk")
 
