@@ -1044,7 +1044,7 @@ __device__ __forceinline__ float lane_tree_sum(float v) {
   return v;
 }
 
-constexpr int kScoreIlp = 4;  // entries a warp scores at once (the tree below assumes 4)
+constexpr int kScoreIlp = 4;  // entries a warp scores at once (a multiple of 4)
 
 // Element i (0..7) of a 16-byte segment as fp32 (exact conversion).
 template <int DT>  // 1 = bf16, 0 = fp16
@@ -1126,7 +1126,7 @@ __device__ __forceinline__ void score_range(const BankDesc* __restrict__ banks, 
     // v[2q] = q.k and v[2q+1] = k.k of entry q, per lane: both chains step
     // together in paired fp32 operations (each half rounded on its own, as
     // the separate multiply and add).
-    static_assert(kScoreIlp == 4, "the transposed tree reduces 4 entries x 2 sums");
+    static_assert(kScoreIlp % 4 == 0, "the transposed tree reduces groups of 4 entries x 2 sums");
     float v[2 * kScoreIlp];
 #pragma unroll
     for (int q = 0; q < kScoreIlp; ++q) {
@@ -1144,37 +1144,41 @@ __device__ __forceinline__ void score_range(const BankDesc* __restrict__ banks, 
       v[2 * q] = acc.x;
       v[2 * q + 1] = acc.y;
     }
-    // The lane tree (s[l] += s[l + d], d = 1 .. 16) of all eight sums at
-    // once: at d = 1, 2, 4 each lane keeps half of its values and adds its
-    // partner's copy of them, so lane l ends with sum 4*(l&1) + 2*(l>>1&1) +
-    // (l>>2&1); d = 8, 16 finish it.  Addition is commutative, so every
-    // partial sum is the one the plain tree forms.
+    // The lane tree (s[l] += s[l + d], d = 1 .. 16) of the eight sums of
+    // each group of four entries at once: at d = 1, 2, 4 each lane keeps half
+    // of its values and adds its partner's copy of them, so lane l ends with
+    // sum 4*(l&1) + 2*(l>>1&1) + (l>>2&1); d = 8, 16 finish it.  Addition is
+    // commutative, so every partial sum is the one the plain tree forms.
     const bool b0 = lane & 1, b1 = lane & 2, b2 = lane & 4;
-    float w4[4], w2[2];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float give = b0 ? v[i] : v[4 + i];
-      w4[i] = __fadd_rn(b0 ? v[4 + i] : v[i], __shfl_xor_sync(kFull, give, 1));
-    }
+    for (int g = 0; g < kScoreIlp / 4; ++g) {
+      const float* vg = v + 8 * g;
+      float w4[4], w2[2];
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const float give = b1 ? w4[i] : w4[2 + i];
-      w2[i] = __fadd_rn(b1 ? w4[2 + i] : w4[i], __shfl_xor_sync(kFull, give, 2));
-    }
-    float w1 = __fadd_rn(b2 ? w2[1] : w2[0], __shfl_xor_sync(kFull, b2 ? w2[0] : w2[1], 4));
-    w1 = __fadd_rn(w1, __shfl_xor_sync(kFull, w1, 8));
-    w1 = __fadd_rn(w1, __shfl_xor_sync(kFull, w1, 16));
-    // Lanes 0..3 hold q.k of entry 2*(l&1) + (l>>1&1); lane l + 4 its k.k.
-    const float kk = __shfl_down_sync(kFull, w1, 4);
-    const int q = 2 * (lane & 1) + ((lane >> 1) & 1);
-    if (lane < 4 && q < cnt) {
-      const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
-      const float sc = den == 0.f ? 0.f : __fdiv_rn(w1, den);
-      scores[e0 + q] = sc;
-      if (HM && hist) {
-        const uint32_t d = ord32(sc) >> 21;  // key bits 63..53
-        atomicAdd(&s_cnt[d], 1u);
-        if (HM == 2) atomicAdd(&s_w[d], static_cast<unsigned long long>(B.entry_bytes));
+      for (int i = 0; i < 4; ++i) {
+        const float give = b0 ? vg[i] : vg[4 + i];
+        w4[i] = __fadd_rn(b0 ? vg[4 + i] : vg[i], __shfl_xor_sync(kFull, give, 1));
+      }
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const float give = b1 ? w4[i] : w4[2 + i];
+        w2[i] = __fadd_rn(b1 ? w4[2 + i] : w4[i], __shfl_xor_sync(kFull, give, 2));
+      }
+      float w1 = __fadd_rn(b2 ? w2[1] : w2[0], __shfl_xor_sync(kFull, b2 ? w2[0] : w2[1], 4));
+      w1 = __fadd_rn(w1, __shfl_xor_sync(kFull, w1, 8));
+      w1 = __fadd_rn(w1, __shfl_xor_sync(kFull, w1, 16));
+      // Lanes 0..3 hold q.k of entry 4g + 2*(l&1) + (l>>1&1); lane l + 4 its k.k.
+      const float kk = __shfl_down_sync(kFull, w1, 4);
+      const int q = 4 * g + 2 * (lane & 1) + ((lane >> 1) & 1);
+      if (lane < 4 && q < cnt) {
+        const float den = __fmul_rn(qnorm, __fsqrt_rn(kk));
+        const float sc = den == 0.f ? 0.f : __fdiv_rn(w1, den);
+        scores[e0 + q] = sc;
+        if (HM && hist) {
+          const uint32_t d = ord32(sc) >> 21;  // key bits 63..53
+          atomicAdd(&s_cnt[d], 1u);
+          if (HM == 2) atomicAdd(&s_w[d], static_cast<unsigned long long>(B.entry_bytes));
+        }
       }
     }
     e0 = e0 + cnt - kScoreIlp;  // the loop adds kScoreIlp: next round starts at e0 + cnt
