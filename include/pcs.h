@@ -344,6 +344,32 @@ pcs_status pcs_prune_global(pcs_ctx *ctx, const pcs_bank *banks, int32_t n, uint
                             float *scores, int32_t *kept_idx, int32_t *kept_off, void *stream);
 
 /*
+ * The histogram exchange of a global threshold over banks split across
+ * processes: called once per digit pass (the same number of times in every
+ * part) with this part's histograms -- counts[i] entries and bytes[i] entry
+ * bytes per digit i < bins -- which it must replace, in place, by their sums
+ * over all parts (an all-reduce).  Returns 0, or non-zero to stop.
+ */
+typedef int32_t (*pcs_hist_exchange_fn)(void *user, uint64_t *counts, uint64_t *bytes,
+                                        int32_t bins);
+
+/*
+ * pcs_prune_global for one part of a population whose banks are split
+ * across processes (Sec. 7.5's budget over the whole population; the one
+ * exchange is a histogram per digit pass, done by the caller's `exchange`).
+ * Entries are ranked over the whole population by (score desc, position
+ * asc), this part's entry 0 being at position `pos_base` (the entries of the
+ * parts before it); the kept set is the longest prefix of that order within
+ * `budget`, and this call writes this part's share of it (kept_idx /
+ * kept_off as for pcs_prune_global).  Synchronises `stream` once per pass.
+ * PCS_E_INVAL if the exchange fails or positions pass 2^32 - 1.
+ */
+pcs_status pcs_prune_global_part(pcs_ctx *ctx, const pcs_bank *banks, int32_t n, uint64_t budget,
+                                 uint64_t pos_base, pcs_hist_exchange_fn exchange, void *user,
+                                 float *scores, int32_t *kept_idx, int32_t *kept_off,
+                                 void *stream);
+
+/*
  * Host only: the reactive shrink-then-drop plan of a host budget (Sec. 7.10:
  * the runtime escalates shrink -> nothing left to shrink -> drop, and acts
  * only when the budget binds).  Sessions are visited in ascending priority

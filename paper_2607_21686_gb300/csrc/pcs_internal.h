@@ -201,7 +201,8 @@ struct GPlan {
   int32_t n_banks;
   int32_t tiles;
   int32_t uniform;
-  int32_t pad;
+  int32_t local;              // 1: histogram only, the host sums the parts and picks
+  uint64_t pos_base;          // position of entry 0 in the whole (split) population
 };
 
 // Scores of every entry; with gh.st set (and a fixed-width kernel), also the

@@ -983,13 +983,14 @@ __device__ void gselect_pick(GState* st, int pass, uint64_t ubytes, const uint32
 // clears the global bins for the next pass.
 template <bool UNIFORM>
 __device__ void gpass_finish(GState* st, int pass, uint64_t ubytes, uint32_t* ch,
-                             unsigned long long* wh, bool* s_last) {
+                             unsigned long long* wh, bool* s_last, bool pick = true) {
   const int nb = 1 << gdigit_bits(pass);
   __syncthreads();
   for (int i = threadIdx.x; i < nb; i += blockDim.x) {
     if (ch[i]) atomicAdd(&st->chist[i], ch[i]);
     if (!UNIFORM && wh[i]) atomicAdd(reinterpret_cast<unsigned long long*>(&st->whist[i]), wh[i]);
   }
+  if (!pick) return;  // a part of a split population: the host sums and picks
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) *s_last = atomicAdd(&st->ticket, 1u) == gridDim.x - 1;
@@ -1372,8 +1373,8 @@ __global__ void __launch_bounds__(kThreads)
 // budget runs out.
 // ---------------------------------------------------------------------------
 
-__device__ __forceinline__ uint64_t gkey(const float* sc, uint64_t i) {
-  return (static_cast<uint64_t>(ord32(__ldg(sc + i))) << 32) | (0xFFFFFFFFull - i);
+__device__ __forceinline__ uint64_t gkey(const float* sc, uint64_t i, uint64_t base) {
+  return (static_cast<uint64_t>(ord32(__ldg(sc + i))) << 32) | (0xFFFFFFFFull - (base + i));
 }
 
 // The bank holding entry i: the last bank in [lo, hi] whose first entry is
@@ -1422,7 +1423,8 @@ __global__ void __launch_bounds__(kThreads) k_gselect(GPlan p, int pass) {
       const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
       uint32_t d = kGBins;  // not a candidate
       if (i < end) {
-        const uint64_t key = (static_cast<uint64_t>(ord32(sv[j])) << 32) | (0xFFFFFFFFull - i);
+        const uint64_t key =
+            (static_cast<uint64_t>(ord32(sv[j])) << 32) | (0xFFFFFFFFull - (p.pos_base + i));
         if ((key & mask) == prefix) d = static_cast<uint32_t>(key >> shift) & (nb - 1);
       }
       if (UNIFORM) {
@@ -1436,7 +1438,7 @@ __global__ void __launch_bounds__(kThreads) k_gselect(GPlan p, int pass) {
       }
     }
   }
-  gpass_finish<UNIFORM>(st, pass, p.uniform_bytes, ch, wh, &s_last);
+  gpass_finish<UNIFORM>(st, pass, p.uniform_bytes, ch, wh, &s_last, !p.local);
 }
 
 // Exclusive block scan of one uint32 per thread; *total = block sum.
@@ -1476,7 +1478,7 @@ __global__ void __launch_bounds__(kThreads) k_gcount(GPlan p) {
 #pragma unroll
     for (int j = 0; j < kGTile / kThreads; ++j) {
       const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
-      if (i < end) c += gkey(p.scores, i) > T;
+      if (i < end) c += gkey(p.scores, i, p.pos_base) > T;
     }
     uint32_t total;
     block_excl_scan(c, warp_sum, &total);
@@ -1522,7 +1524,7 @@ __global__ void __launch_bounds__(kThreads) k_gwrite(GPlan p) {
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
       const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
-      kp[j] = i < end && gkey(p.scores, i) > T;
+      kp[j] = i < end && gkey(p.scores, i, p.pos_base) > T;
     }
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {

@@ -1544,8 +1544,83 @@ pcs_status pcs_topk(pcs_ctx* c, const float* keys, const int32_t* n, const int32
   return ws_release(c, stream);
 }
 
-pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64_t budget,
-                            float* scores, int32_t* kept_idx, int32_t* kept_off, void* stream_) {
+// Digit schedule of the 64-bit ranking key (the same as the kernels'):
+// 11, 11, 10 bits of ord32(score), then 11, 11, 10 bits of the position.
+static const int kGDigitBits[kGPasses] = {11, 11, 10, 11, 11, 10};
+static const int kGDigitShift[kGPasses] = {53, 42, 32, 21, 10, 0};
+
+// The digit choice of one pass from histograms summed over all parts (the
+// device's gselect_pick, on the host).  Returns true once the threshold is
+// known.
+static bool host_pick(int pass, const uint64_t* counts, const uint64_t* bytes, GState* g) {
+  const int bits = kGDigitBits[pass], shift = kGDigitShift[pass];
+  const uint64_t top = (1ull << bits) - 1;
+  uint64_t cum = 0;
+  for (int64_t bin = static_cast<int64_t>(top); bin >= 0; --bin) {
+    if (cum + bytes[bin] > g->remaining) {
+      g->prefix |= static_cast<uint64_t>(bin) << shift;
+      g->mask |= top << shift;
+      g->remaining -= cum;
+      if (counts[bin] == 1 || shift == 0) {
+        g->threshold = g->prefix | ~g->mask;
+        return true;
+      }
+      return false;
+    }
+    cum += bytes[bin];
+  }
+  g->threshold = 0;  // every candidate fits
+  return true;
+}
+
+// The digit passes of one part of a split population: histogram here, sum
+// over the parts through `ex`, pick on the host, send the state back.
+static pcs_status exchange_passes(pcs_ctx* c, const GPlan& gp, uint64_t budget,
+                                  pcs_hist_exchange_fn ex, void* user, cudaStream_t stream) {
+  std::vector<uint32_t> c32(kGBins);
+  std::vector<uint64_t> counts(kGBins), bytes(kGBins);
+  GState g{};
+  g.remaining = budget;
+  for (int pass = 0; pass < kGPasses; ++pass) {
+    const int nb = 1 << kGDigitBits[pass];
+    std::fill(counts.begin(), counts.end(), 0);
+    std::fill(bytes.begin(), bytes.end(), 0);
+    if (gp.tiles > 0) {
+      {
+        LaunchScope ls(c, kKGSelect, stream);
+        PCS_CUDA(launch_gselect(gp, pass, c->sm_count, stream));
+      }
+      PCS_CUDA(cudaMemcpyAsync(c32.data(), gp.st->chist, 4ull * nb, cudaMemcpyDeviceToHost, stream));
+      if (!gp.uniform)
+        PCS_CUDA(cudaMemcpyAsync(bytes.data(), gp.st->whist, 8ull * nb, cudaMemcpyDeviceToHost,
+                                 stream));
+      PCS_CUDA(cudaMemsetAsync(gp.st->chist, 0, 4ull * kGBins, stream));
+      PCS_CUDA(cudaMemsetAsync(gp.st->whist, 0, 8ull * kGBins, stream));
+      PCS_CUDA(cudaStreamSynchronize(stream));
+      for (int i = 0; i < nb; ++i) {
+        counts[i] = c32[i];
+        if (gp.uniform) bytes[i] = counts[i] * gp.uniform_bytes;
+      }
+    }
+    const int32_t rc = ex(user, counts.data(), bytes.data(), nb);
+    if (rc != 0) return fail(PCS_E_INVAL, "histogram exchange of pass %d returned %d", pass, rc);
+    const bool done = host_pick(pass, counts.data(), bytes.data(), &g);
+    g.done = done ? 1 : 0;
+    // The header fields (prefix .. done) for the next pass and the compaction.
+    PCS_CUDA(cudaMemcpyAsync(gp.st, &g, offsetof(GState, ticket), cudaMemcpyHostToDevice, stream));
+    PCS_CUDA(cudaStreamSynchronize(stream));
+    if (done) break;
+  }
+  return PCS_OK;
+}
+
+// The global threshold over these banks; with `ex`, these banks are one part
+// of a population split over processes: each digit pass's histogram is
+// summed over the parts by `ex` and the digit is picked on the host.
+static pcs_status prune_global_impl(pcs_ctx* c, const pcs_bank* banks, int32_t n,
+                                    uint64_t budget, float* scores, int32_t* kept_idx,
+                                    int32_t* kept_off, void* stream_, pcs_hist_exchange_fn ex,
+                                    void* user, uint64_t pos_base) {
   if (!c || n < 0 || (n > 0 && !banks)) return fail(PCS_E_INVAL, "bad arguments");
   if (!kept_off) return fail(PCS_E_INVAL, "kept_off is null");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
@@ -1569,7 +1644,9 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
   std::lock_guard<std::mutex> lk(c->mu);
   st = set_device(c);
   if (st) return st;
-  if (entries == 0) {
+  if (pos_base + entries > 0xFFFFFFFFull)
+    return fail(PCS_E_INVAL, "positions past 2^32 - 1 in the whole population");
+  if (entries == 0 && !ex) {
     // Nothing to rank: every bank keeps nothing.
     PCS_CUDA(cudaMemsetAsync(kept_off, 0, 4ull * (n + 1), stream));
     return PCS_OK;
@@ -1579,7 +1656,7 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
   std::vector<uint32_t> tile_bank(tiles + 1);
   {
     int b = 0;
-    for (uint64_t t = 0; t <= tiles; ++t) {
+    for (uint64_t t = 0; t <= tiles && entries > 0; ++t) {
       const uint64_t i = std::min<uint64_t>(t * kGTile, entries - 1);
       while (b + 1 < n && ebeg[b + 1] <= i) ++b;
       tile_bank[t] = static_cast<uint32_t>(b);
@@ -1587,7 +1664,9 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
   }
   GState g0{};
   g0.remaining = budget;
-  g0.done = total <= budget;  // the budget does not bind: threshold 0 keeps all
+  // The budget does not bind: threshold 0 keeps all.  (A part cannot tell:
+  // the first summed histogram shows it.)
+  g0.done = !ex && total <= budget;
   uint64_t at = round_up(sizeof(BankDesc) * n, kRecordAlign);
   const uint64_t o_ebeg = at;
   at = round_up(at + 8ull * (n + 1), 16);
@@ -1614,7 +1693,7 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
   PCS_CUDA(plan_copy(c, ws, plan_bytes, stream));
   float* sc = scores ? scores : reinterpret_cast<float*>(ws + o_sc);
   GHist gh{};
-  if (!g0.done) {
+  if (!g0.done && !ex) {
     gh.st = reinterpret_cast<GState*>(ws + o_st);
     gh.uniform_bytes = n > 0 ? banks[0].entry_bytes : 0;
     gh.mode = uniform ? 1 : 2;
@@ -1636,7 +1715,12 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
   gp.n_banks = n;
   gp.tiles = static_cast<int32_t>(tiles);
   gp.uniform = uniform ? 1 : 0;
-  if (!g0.done) {
+  gp.pos_base = pos_base;
+  if (ex) {
+    gp.local = 1;
+    st = exchange_passes(c, gp, budget, ex, user, stream);
+    if (st) return st;
+  } else if (!g0.done) {
     // Six digit passes at most (the first inside the score kernel when it
     // could take it); each is a no-op once the threshold is known.
     for (int pass = fused ? 1 : 0; pass < kGPasses; ++pass) {
@@ -1644,12 +1728,29 @@ pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64
       PCS_CUDA(launch_gselect(gp, pass, c->sm_count, stream));
     }
   }
-  {
+  if (entries == 0) {
+    PCS_CUDA(cudaMemsetAsync(kept_off, 0, 4ull * (n + 1), stream));
+  } else {
     LaunchScope ls(c, kKGCompact, stream);
     c->launches += 1;  // count and write
     PCS_CUDA(launch_gcompact(gp, c->sm_count, stream));
   }
   return ws_release(c, stream);
+}
+
+pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64_t budget,
+                            float* scores, int32_t* kept_idx, int32_t* kept_off, void* stream) {
+  return prune_global_impl(c, banks, n, budget, scores, kept_idx, kept_off, stream, nullptr,
+                           nullptr, 0);
+}
+
+pcs_status pcs_prune_global_part(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64_t budget,
+                                 uint64_t pos_base, pcs_hist_exchange_fn exchange, void* user,
+                                 float* scores, int32_t* kept_idx, int32_t* kept_off,
+                                 void* stream) {
+  if (!exchange) return fail(PCS_E_INVAL, "exchange is null");
+  return prune_global_impl(c, banks, n, budget, scores, kept_idx, kept_off, stream, exchange,
+                           user, pos_base);
 }
 
 pcs_status pcs_budget_plan(const int32_t* n, const uint64_t* entry_bytes, const double* priority,

@@ -166,8 +166,12 @@ SIGNATURES = {
     "pcs_plan_run": (_st, [_vp, _vp, _vp]),
     "pcs_plan_destroy": (_st, [_vp, _vp]),
     "pcs_set_arena_limit": (_st, [_vp, _u32, _u64]),
+    "pcs_prune_global_part": (_st, [_vp, ctypes.POINTER(pcs_bank), _i32, _u64, _u64, _vp, _vp,
+                                    _vp, _vp, _vp, _vp]),
     "pcs_fingerprint_static": (_st, [ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
 }
+# int32 exchange(void* user, uint64_t* counts, uint64_t* bytes, int32 bins)
+EXCHANGE_FN = ctypes.CFUNCTYPE(_i32, _vp, ctypes.POINTER(_u64), ctypes.POINTER(_u64), _i32)
 # int32 probe(void* user, const uint8_t* keep, uint64_t* distance)
 PROBE_FN = ctypes.CFUNCTYPE(_i32, _vp, ctypes.POINTER(ctypes.c_uint8), ctypes.POINTER(_u64))
 PCS_STATIC_MAX_BUFFERS = 64
@@ -610,6 +614,32 @@ class Context:
         """One relevance threshold across all banks under a byte budget."""
         check(self.lib.pcs_prune_global(self.h, banks, n, budget, _ptr(scores), _ptr(kept_idx),
                                         _ptr(kept_off), _stream_ptr(stream)), "pcs_prune_global")
+
+    def prune_global_part(self, banks, n: int, budget: int, pos_base: int, exchange,
+                          kept_idx: torch.Tensor, kept_off: torch.Tensor, scores=None,
+                          stream=None):
+        """One part of a split population: exchange(counts, bytes) receives
+        this part's per-digit histograms (numpy uint64 views) and must sum
+        them over all parts in place."""
+        failure = []
+
+        def cb(_user, counts, nbytes, bins):
+            try:
+                c = np.ctypeslib.as_array(counts, shape=(bins,))
+                b = np.ctypeslib.as_array(nbytes, shape=(bins,))
+                exchange(c, b)
+                return 0
+            except BaseException as ex:  # re-raised below
+                failure.append(ex)
+                return 1
+
+        fn = EXCHANGE_FN(cb)
+        st = self.lib.pcs_prune_global_part(self.h, banks, n, budget, pos_base,
+                                            ctypes.cast(fn, ctypes.c_void_p), None, _ptr(scores),
+                                            _ptr(kept_idx), _ptr(kept_off), _stream_ptr(stream))
+        if failure:
+            raise failure[0]
+        check(st, "pcs_prune_global_part")
 
     # -- snapshots -------------------------------------------------------------
     def record_bytes(self, session: Session) -> int:

@@ -5,7 +5,10 @@ banks: scores bit-equal to the oracle's fixed-order fp32 score, kept sets and
 bank offsets identical, across several 4096-entry tiles with a ragged tail,
 with uniform and mixed entry sizes (the two select paths), empty banks at
 either end and in the middle, exact ties across banks, and budgets that keep
-nothing, one entry, a fraction, all but one, and all.
+nothing, one entry, a fraction, all but one, and all.  The same population
+split into two parts (two threads, two contexts, the histograms summed on the
+host each pass, as ranks would all-reduce them) gives each part its share of
+the one-population answer.
 """
 import numpy as np
 import pytest
@@ -123,3 +126,79 @@ def test_global_threshold_keeps_relevant_sessions(ctx, dev):
     qs = [q.half().to(dev)] * 2
     kept, koff, _ = _run(ctx, dev, keys, qs, 10, 2000)
     assert koff.tolist() == [0, 200, 200]
+
+
+def _split_run(dev, keys, qs, E, budget, cut):
+    """Two parts (banks [:cut] and [cut:]) run as two threads with their own
+    contexts and streams; the exchange sums the histograms through a barrier."""
+    import threading
+    parts = [(keys[:cut], qs[:cut], E[:cut]), (keys[cut:], qs[cut:], E[cut:])]
+    base = [0, sum(k.shape[0] for k in keys[:cut])]
+    barrier = threading.Barrier(2)
+    slot_c, slot_b, out, errs = [None, None], [None, None], [None, None], []
+
+    def worker(r):
+        try:
+            pk, pq, pe = parts[r]
+            with pcs.Context(0) as c:
+                s = torch.cuda.Stream(device=dev)
+                banks = c.banks_array(pk, pq, pe) if pk else (pcs.pcs_bank * 1)()
+                total = sum(k.shape[0] for k in pk)
+                kept = torch.full((max(total, 1),), -7, dtype=torch.int32, device=dev)
+                koff = torch.full((len(pk) + 1,), -7, dtype=torch.int32, device=dev)
+
+                def ex(cnt, byt):
+                    slot_c[r], slot_b[r] = cnt.copy(), byt.copy()
+                    barrier.wait(60)
+                    tc, tb = slot_c[0] + slot_c[1], slot_b[0] + slot_b[1]
+                    barrier.wait(60)
+                    cnt[:] = tc
+                    byt[:] = tb
+                c.prune_global_part(banks, len(pk), budget, base[r], ex, kept, koff, stream=s)
+                s.synchronize()
+                ko = koff.cpu().numpy()
+                out[r] = (kept.cpu().numpy()[:ko[-1]], ko)
+        except BaseException as e:  # surfaced below
+            errs.append(e)
+            barrier.abort()
+
+    ts = [threading.Thread(target=worker, args=(r,)) for r in range(2)]
+    for t in ts:
+        t.start()
+    for t in ts:
+        t.join(300)
+    assert not errs, errs
+    return out
+
+
+@pytest.mark.parametrize("budget_frac", [0.0, 0.3, 0.62, 1.0])
+def test_global_threshold_split_across_parts(dev, budget_frac):
+    b = synth.banks(310, 30, 0, 600, 128, torch.bfloat16, (8,), torch.uint8)
+    keys, qs = _views(b, dev)
+    rnd = np.random.default_rng(11)
+    E = [int(x) for x in rnd.integers(1, 4000, len(keys))]
+    T = sum(k.shape[0] * e for k, e in zip(keys, E))
+    B = int(T * budget_frac)
+    s32 = _oracle_scores(keys, qs)
+    want, woff = oracle.prune_global(s32, [k.shape[0] for k in keys], E, B)
+    for cut in (12, 0):  # the second split gives part 0 no banks at all
+        got = _split_run(dev, keys, qs, E, B, cut)
+        for r, (lo, hi) in enumerate(((0, cut), (cut, len(keys)))):
+            kept, ko = got[r]
+            assert ko.tolist() == (woff[lo:hi + 1] - woff[lo]).tolist(), (cut, r)
+            assert kept.tolist() == want[woff[lo]:woff[hi]].tolist(), (cut, r)
+
+
+def test_global_threshold_one_part_equals_whole(ctx, dev):
+    b = synth.banks(311, 25, 1, 400, 64, torch.float16, (8,), torch.uint8)
+    keys, qs = _views(b, dev)
+    banks = ctx.banks_array(keys, qs, 300)
+    total = sum(b.n)
+    B = total * 300 // 3
+    kept = torch.empty(total, dtype=torch.int32, device=dev)
+    koff = torch.empty(len(keys) + 1, dtype=torch.int32, device=dev)
+    ctx.prune_global_part(banks, len(keys), B, 0, lambda c, x: None, kept, koff)
+    ctx.sync()
+    want, woff = oracle.prune_global(_oracle_scores(keys, qs), b.n, 300, B)
+    assert koff.cpu().tolist() == woff.tolist()
+    assert kept.cpu().tolist()[:woff[-1]] == want.tolist()
