@@ -1569,19 +1569,6 @@ __device__ __forceinline__ bool pool_id_ok(const PoolDev& P, int32_t p) {
   return true;
 }
 
-// Take one free page (count 1), or -1 with the error recorded.
-__device__ __forceinline__ int32_t pool_pop(const PoolDev& P) {
-  const int32_t i = atomicSub(P.top, 1);
-  if (i <= 0) {
-    atomicAdd(P.top, 1);
-    atomicOr(P.err, kDevErrNoPage);
-    return -1;
-  }
-  const int32_t q = P.free_ids[i - 1];
-  P.rc[q] = 1;
-  return q;
-}
-
 // Pops aggregated per warp: one atomic on the stack top for the warp's lanes.
 __global__ void __launch_bounds__(kThreads) k_pool_alloc(PoolDev P, int32_t* ids, int32_t n) {
   const int32_t j = blockIdx.x * kThreads + threadIdx.x;
@@ -1660,9 +1647,9 @@ __global__ void __launch_bounds__(kThreads)
 
 // One warp per table slot, eight slots per block round: lane 0 of each warp
 // settles its slot's hold; the slots that need a page take them off the free
-// stack with one atomic for the block (over-taking is given back, as in
-// pool_pop); then every warp copies its page, kCowDepth 16-byte loads in
-// flight per lane.
+// stack with one atomic for the block (pages taken past an empty stack are
+// given back and reported); then every warp copies its page, kCowDepth
+// 16-byte loads in flight per lane.
 constexpr int kCowDepth = 8;
 
 __global__ void __launch_bounds__(kThreads)
