@@ -7,6 +7,8 @@
     python -m paper_2607_21686_gb300.cases mismatch --n 200 --hi-mib 32
     python -m paper_2607_21686_gb300.cases prune_global --sessions 256
     python -m paper_2607_21686_gb300.cases cow --sessions 64
+    python -m paper_2607_21686_gb300.cases reads --n 200 --hi-mib 32
+    python -m paper_2607_21686_gb300.cases topk --sessions 2048
 
 Each case builds its seeded synthetic population on cuda:0, runs the step
 `--warmup` times, then once more, and prints the device time of that last
@@ -121,8 +123,38 @@ def case_cow(ctx, a, dev):
     return ms
 
 
+def case_reads(ctx, a, dev):
+    # A read log over the sweep's buffers: 140 of them read, 60 never.
+    sw = synth.sweep(n=a.n, hi=a.hi_mib << 20, device=dev)
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(4) + 9)
+    bases = torch.tensor([t.data_ptr() for t in sw.after], dtype=torch.int64, device=dev)
+    lens = torch.tensor([t.numel() * t.element_size() for t in sw.after], dtype=torch.int64,
+                        device=dev)
+    m = 1 << 24
+    which = torch.randint(0, int(0.7 * len(sw.after)), (m,), generator=g, device=dev)
+    off = (torch.rand(m, generator=g, device=dev) * lens[which]).long()
+    nbytes = torch.minimum(torch.randint(1, 4097, (m,), generator=g, device=dev,
+                                         dtype=torch.int64), lens[which] - off)
+    arr = ctx.buf_array(sw.after)
+    flags = torch.empty(len(sw.after), dtype=torch.uint8, device=dev)
+    addr = bases[which] + off
+    return _timed(lambda: ctx.classify_reads(arr, addr, nbytes, flags), a.warmup)
+
+
+def case_topk(ctx, a, dev):
+    # Recency-keyed retention: last-use steps as rank keys, 62.7% kept per bank.
+    b = synth.banks_config5(sessions=a.sessions, device=dev)
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(5) + 3)
+    keys = torch.randint(0, 1 << 20, (sum(b.n),), generator=g, device=dev).float()
+    k = [int(x * 0.627) for x in b.n]
+    kept = torch.empty(sum(k), dtype=torch.int32, device=dev)
+    na, ka = ctx.int32_array(b.n), ctx.int32_array(k)
+    return _timed(lambda: ctx.topk(keys, na, ka, kept), a.warmup)
+
+
 CASES = {"kv": case_kv, "classify": case_classify, "prune": case_prune, "markov": case_markov,
-         "mismatch": case_mismatch, "prune_global": case_prune_global, "cow": case_cow}
+         "mismatch": case_mismatch, "prune_global": case_prune_global, "cow": case_cow,
+         "reads": case_reads, "topk": case_topk}
 
 
 def main():
