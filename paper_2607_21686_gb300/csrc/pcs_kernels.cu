@@ -2130,7 +2130,7 @@ cudaError_t launch_classify_reads(const ReadPlan& p, const uint64_t* addr, const
     if (e != cudaSuccess) return e;
   }
   const uint64_t want = (static_cast<uint64_t>(m) + kThreads - 1) / kThreads;
-  const uint64_t cap = static_cast<uint64_t>(sm_count) * 4;
+  const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;  // 32 registers: 8 blocks per SM
   k_classify_reads<<<static_cast<unsigned>(want < cap ? want : cap), kThreads, smem, stream>>>(
       p, addr, bytes, m, flags);
   return cudaGetLastError();
