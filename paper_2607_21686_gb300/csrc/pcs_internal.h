@@ -172,9 +172,16 @@ struct alignas(16) GState {
   uint64_t prefix, mask;  // key bits fixed so far
   uint64_t remaining;     // budget left for keys inside the prefix
   uint64_t threshold;
-  uint32_t done, ticket, total_kept, pad;
+  uint32_t done, ticket, total_kept, n_cand;
+  uint32_t bar_count, bar_gen, pad[2];  // k_gfinish: arrivals, last barrier released
   uint64_t whist[kGBins]; // entry bytes per digit (mixed entry sizes)
   uint32_t chist[kGBins]; // entries per digit
+};
+
+// Summed bins of one later digit pass inside k_gfinish.
+struct GBinSet {
+  uint64_t w[kGBins];
+  uint32_t c[kGBins];
 };
 
 // The score kernel's optional epilogue: the first digit pass of the global
@@ -192,7 +199,7 @@ struct GPlan {
   const uint64_t* ebeg;       // [n_banks + 1]: first entry of each bank; ebeg[n_banks] = entries
   const uint64_t* ebytes;     // [n_banks]: bytes one entry of the bank costs
   const uint32_t* tile_bank;  // [tiles + 1]: bank of entry min(t * kGTile, entries - 1)
-  uint32_t* tile_cnt;         // [tiles]: kept per tile, then its exclusive scan
+  uint32_t* tile_cnt;         // [tiles]: kept per tile
   GState* st;
   int32_t* kept_idx;          // [<= entries], CSR by bank
   int32_t* kept_off;          // [n_banks + 1]
@@ -203,6 +210,14 @@ struct GPlan {
   int32_t uniform;
   int32_t local;              // 1: histogram only, the host sums the parts and picks
   uint64_t pos_base;          // position of entry 0 in the whole (split) population
+  int32_t vec;                // 1: scores 16-byte aligned (whole runs read as float4)
+  int32_t pad;
+  // k_gfinish scratch
+  uint32_t* ucand;            // [tiles * 8]: candidates of each 512-entry unit
+  uint64_t* ckey;             // [tiles * kGTile]: their keys, unit u's from 512 u
+  uint32_t* cbank;            // the same slots: their banks (mixed entry sizes only)
+  GBinSet* hb;                // [kGPasses]: summed bins of the passes after the first
+  uint32_t* err;              // the context's error word (a barrier that timed out)
 };
 
 // Scores of every entry; with gh.st set (and a fixed-width kernel), also the
@@ -212,12 +227,13 @@ cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
                          int key_types, float* scores, int sm_count, cudaStream_t stream,
                          GHist gh = GHist{}, bool* fused = nullptr);
 
-// Pass `pass` (0..kGPasses-1) of the byte-weighted radix select; a no-op
-// once the threshold is known.
+// The bins of pass `pass` (0..kGPasses-1) of the byte-weighted radix select
+// over a part of a split population (local plan: the host sums and picks);
+// a no-op once the threshold is known.
 cudaError_t launch_gselect(const GPlan& p, int pass, int sm_count, cudaStream_t stream);
-// Count per tile and scan (first launch), then write kept indices and bank
-// offsets (second launch).
-cudaError_t launch_gcompact(const GPlan& p, int sm_count, cudaStream_t stream);
+// The digit passes from `first_pass` on (none once the state is done) and
+// the compaction: kept indices and bank offsets.  One cooperative launch.
+cudaError_t launch_gfinish(const GPlan& p, int first_pass, int sm_count, cudaStream_t stream);
 
 // ---- Copy-on-write page pool (pcs_pool_*) ---------------------------------
 // Reference counts and a free stack over caller memory.  A kernel either only

@@ -15,9 +15,14 @@
 // k_topk          per-bank radix select of the k largest (score, -index),
 //                 kept indices written in ascending order (Sec. 7.5).
 //
-// No kernel waits on another block: every pass is a plain data-parallel
-// sweep, so nothing here can spin.  Index values read from device memory are
-// bounds-checked; a bad one is reported through the error word and skipped.
+// k_gfinish       the global threshold's later digit passes and its
+//                 compaction, in one cooperative launch (Sec. 7.5 variant).
+//
+// Only k_gfinish has blocks that wait on one another, at grid barriers of a
+// cooperative launch (all blocks resident); every wait here, there and on an
+// mbarrier, gives up after about two seconds and sets the timeout bit.
+// Index values read from device memory are bounds-checked; a bad one is
+// reported through the error word and skipped.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
@@ -1367,15 +1372,13 @@ __global__ void __launch_bounds__(kThreads)
 // (score descending, then bank, then index ascending; unique keys).  The kept
 // set is the longest prefix of the descending key order whose entry bytes
 // fit the budget: every key above the key of the first entry that does not
-// fit.  That key is found most significant byte first, each pass summing the
-// bytes (not the count) of the candidate keys per digit; the last block of a
-// pass (atomic ticket, no block waits for another) picks the digit where the
-// budget runs out.
+// fit.  That key is found most significant digit first, each pass summing
+// the bytes (not the count) of the candidate keys per digit and picking the
+// digit where the budget runs out.  The first pass rides on the score kernel
+// (its last block, by atomic ticket, picks); k_gfinish runs the rest.
+// k_gselect bins one pass of a part of a population split over processes;
+// the host sums the parts' bins and picks.
 // ---------------------------------------------------------------------------
-
-__device__ __forceinline__ uint64_t gkey(const float* sc, uint64_t i, uint64_t base) {
-  return (static_cast<uint64_t>(ord32(__ldg(sc + i))) << 32) | (0xFFFFFFFFull - (base + i));
-}
 
 // The bank holding entry i: the last bank in [lo, hi] whose first entry is
 // <= i (empty banks share their successor's first entry and come before it).
@@ -1465,86 +1468,550 @@ __device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_s
   return before + incl - v;
 }
 
-// Kept entries per tile; the last block scans the tile counts into offsets
-// and closes the bank offsets of trailing empty banks.
-__global__ void __launch_bounds__(kThreads) k_gcount(GPlan p) {
-  __shared__ uint32_t warp_sum[kWarps];
-  __shared__ bool s_last;
-  const uint64_t T = __ldcg(&p.st->threshold);
-  for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
-    const uint64_t start = static_cast<uint64_t>(t) * kGTile;
-    const uint64_t end = start + kGTile < p.entries ? start + kGTile : p.entries;
-    uint32_t c = 0;
-#pragma unroll
-    for (int j = 0; j < kGTile / kThreads; ++j) {
-      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
-      if (i < end) c += gkey(p.scores, i, p.pos_base) > T;
-    }
-    uint32_t total;
-    block_excl_scan(c, warp_sum, &total);
-    if (threadIdx.x == 0) p.tile_cnt[t] = total;
-  }
-  __threadfence();
+// ---------------------------------------------------------------------------
+// The rest of the global threshold in one cooperative launch (k_gfinish):
+// the digit passes after the first and the compaction.  Its blocks are all
+// resident at once and meet at grid barriers; the last block to arrive makes
+// the digit choice from the summed bins before it releases the others.
+//
+//   pass 0 (only when the score kernel could not take it): bins of the top
+//     digit of every key;
+//   the first full scan: keys above the digits fixed so far are kept for
+//     sure and counted per tile; keys inside them (the candidates) are
+//     binned by the next digit and stored in their 512-entry unit's slots;
+//   later passes bin the candidates only;
+//   once the threshold is known, the kept candidates join their tiles'
+//   counts; each block sums the counts before its contiguous tile range and
+//   writes the kept indices and bank offsets of its tiles in order.
+// ---------------------------------------------------------------------------
+
+// One block's copy of the select state.
+struct GLocal {
+  uint64_t prefix, mask, remaining, threshold;
+  uint32_t done;
+};
+
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.add.acq_rel.gpu.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Bounded grid barrier number k (1, 2, ...) of a cooperative launch.  The
+// arrival count only grows (barrier k is full at k x blocks); the last block
+// to arrive runs `last` (every thread of it), then publishes k.  A block that
+// waits past kWaitCycles sets the timeout bit and returns false; the others
+// then give up at their next barrier.
+template <typename F>
+__device__ bool grid_barrier(GState* st, uint32_t* err, uint32_t k, bool* s_flag, F&& last) {
   __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(&p.st->ticket, 1u) == gridDim.x - 1;
+  if (threadIdx.x == 0) *s_flag = atom_add_acq_rel(&st->bar_count, 1u) == k * gridDim.x - 1;
   __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  uint32_t run = 0;
-  for (int base = 0; base < p.tiles; base += kThreads) {
-    const int t = base + threadIdx.x;
-    const uint32_t v = t < p.tiles ? __ldcg(&p.tile_cnt[t]) : 0u;
-    uint32_t total;
-    const uint32_t ex = block_excl_scan(v, warp_sum, &total);
-    if (t < p.tiles) p.tile_cnt[t] = run + ex;
-    run += total;
+  if (*s_flag) {  // the last block: everybody else's writes are visible
+    last();
+    __syncthreads();
+    if (threadIdx.x == 0) st_release(&st->bar_gen, k);
+    return true;  // *s_flag stays set until the next barrier rewrites it
   }
+  __syncthreads();  // every thread has read *s_flag
   if (threadIdx.x == 0) {
-    p.st->total_kept = run;
-    p.kept_off[p.n_banks] = static_cast<int32_t>(run);
-    for (int b = p.n_banks - 1; b >= 0 && p.ebeg[b] == p.entries; --b)
-      p.kept_off[b] = static_cast<int32_t>(run);
-    p.st->ticket = 0;
+    bool ok = true;
+    const long long t0 = clock64();
+    while (ld_acquire(&st->bar_gen) < k) {
+      if (clock64() - t0 > kWaitCycles) {
+        atomicOr(err, kDevErrTimeout);
+        ok = false;
+        break;
+      }
+      __nanosleep(20);
+    }
+    *s_flag = ok;
+  }
+  __syncthreads();
+  return *s_flag;
+}
+
+// Inclusive block scan of one uint64 per thread.
+__device__ __forceinline__ uint64_t block_incl_scan64(uint64_t v, uint64_t* warp_sum) {
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  uint64_t incl = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint64_t o = __shfl_up_sync(kFull, incl, d);
+    if (lane >= d) incl += o;
+  }
+  if (lane == 31) warp_sum[wib] = incl;
+  __syncthreads();
+  uint64_t before = 0;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w)
+    if (w < wib) before += warp_sum[w];
+  __syncthreads();
+  return before + incl;
+}
+
+// The digit choice of a pass from the summed bins, by the whole block:
+// thread t holds the bins top - per*t - j (j < per), highest digits first;
+// the first thread whose running bytes overrun the budget left finds the
+// digit, as in gselect_pick.
+template <bool UNIFORM>
+__device__ void gpick_block(GLocal* s, int pass, uint64_t ubytes, const uint32_t* gc,
+                            const unsigned long long* gw, uint64_t* scan64) {
+  const int bits = gdigit_bits(pass), shift = gdigit_shift(pass);
+  const int nb = 1 << bits, top = nb - 1, per = nb / kThreads;
+  uint32_t cn[kGBins / kThreads];
+  uint64_t wt[kGBins / kThreads];
+  uint64_t local = 0;
+#pragma unroll
+  for (int j = 0; j < kGBins / kThreads; ++j) {
+    cn[j] = 0;
+    wt[j] = 0;
+    if (j < per) {
+      const int bin = top - per * static_cast<int>(threadIdx.x) - j;
+      cn[j] = __ldcg(gc + bin);
+      wt[j] = UNIFORM ? static_cast<uint64_t>(cn[j]) * ubytes
+                      : static_cast<uint64_t>(__ldcg(gw + bin));
+      local += wt[j];
+    }
+  }
+  const uint64_t incl = block_incl_scan64(local, scan64);
+  const uint64_t R = s->remaining;
+  const int fit = __syncthreads_count(incl <= R);
+  if (fit == kThreads) {  // every candidate fits (only when the whole population does)
+    if (threadIdx.x == 0) {
+      s->threshold = 0;
+      s->done = 1;
+    }
+  } else if (static_cast<int>(threadIdx.x) == fit) {
+    uint64_t cum = incl - local;
+#pragma unroll
+    for (int j = 0; j < kGBins / kThreads; ++j) {
+      if (j < per && cum + wt[j] > R) {
+        const int bin = top - per * static_cast<int>(threadIdx.x) - j;
+        const uint64_t np = s->prefix | (static_cast<uint64_t>(bin) << shift);
+        const uint64_t nm = s->mask | (static_cast<uint64_t>(top) << shift);
+        s->prefix = np;
+        s->mask = nm;
+        s->remaining = R - cum;
+        if (cn[j] == 1u || shift == 0) {
+          s->threshold = np | ~nm;
+          s->done = 1;
+        }
+        break;
+      }
+      cum += wt[j];
+    }
+  }
+  __syncthreads();
+}
+
+// The bins of pass `pass`: the state's own for the first pass this launch
+// bins (zero at launch), a scratch set (zeroed here) for the later ones.
+__device__ __forceinline__ uint32_t* gbins_c(const GPlan& p, int pass, int first) {
+  return pass == first ? p.st->chist : p.hb[pass].c;
+}
+__device__ __forceinline__ unsigned long long* gbins_w(const GPlan& p, int pass, int first) {
+  return reinterpret_cast<unsigned long long*>(pass == first ? p.st->whist : p.hb[pass].w);
+}
+
+// Add a block's bins to the summed ones.
+template <bool UNIFORM>
+__device__ __forceinline__ void gbins_add(const uint32_t* ch, const unsigned long long* wh, int nb,
+                                          uint32_t* gc, unsigned long long* gw) {
+  __syncthreads();
+  for (int i = threadIdx.x; i < nb; i += kThreads) {
+    if (ch[i]) atomicAdd(gc + i, ch[i]);
+    if (!UNIFORM && wh[i]) atomicAdd(gw + i, wh[i]);
   }
 }
 
-// Kept indices (bank-local, ascending) at their global rank, and the offset
-// of every bank at the rank of its first entry.
-__global__ void __launch_bounds__(kThreads) k_gwrite(GPlan p) {
-  __shared__ uint32_t warp_cnt[kWarps];
-  const uint64_t T = __ldcg(&p.st->threshold);
-  for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
-    const uint64_t start = static_cast<uint64_t>(t) * kGTile;
-    const uint64_t end = start + kGTile < p.entries ? start + kGTile : p.entries;
-    uint32_t base = p.tile_cnt[t];
-    int b = p.tile_bank[t];
-    const int hi = p.tile_bank[t + 1];
-    constexpr int kPer = kGTile / kThreads;
-    bool kp[kPer];
+// Bin digit d (kGBins: not a candidate) with the given weight.  Uniform
+// weights: every lane of the warp calls it and lanes with the same digit add
+// once (the hot digits are few).
+template <bool UNIFORM>
+__device__ __forceinline__ void gbin(uint32_t* ch, unsigned long long* wh, uint32_t d,
+                                     uint64_t bytes) {
+  if (UNIFORM) {
+    const unsigned same = __match_any_sync(kFull, d);
+    if (d < kGBins && (threadIdx.x & 31) == __ffs(same) - 1) atomicAdd(&ch[d], __popc(same));
+  } else if (d < kGBins) {
+    atomicAdd(&ch[d], 1u);
+    atomicAdd(&wh[d], static_cast<unsigned long long>(bytes));
+  }
+}
+
+// Entries of tile t handled by this thread: warp w takes the 512 entries
+// from t * kGTile + 512 w (its unit), lane l the 16 entries from 16 l of them.
+constexpr int kGPer = kGTile / kThreads;
+constexpr int kGUnit = 32 * kGPer;
+static_assert(kGPer == 16, "tile layout: 16 entries per thread");
+
+__device__ __forceinline__ uint64_t glane0(int t) {
+  return static_cast<uint64_t>(t) * kGTile + (threadIdx.x >> 5) * kGUnit + (threadIdx.x & 31) * kGPer;
+}
+
+// The 16 scores from entry i0 (zero past `end`): four 16-byte loads when the
+// run is whole and the scores are 16-byte aligned.
+__device__ __forceinline__ void gload(const GPlan& p, uint64_t i0, uint64_t end, float (&sc)[kGPer]) {
+  if (p.vec && i0 + kGPer <= end) {
+    const float4* v = reinterpret_cast<const float4*>(p.scores + i0);
 #pragma unroll
-    for (int j = 0; j < kPer; ++j) {
-      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
-      kp[j] = i < end && gkey(p.scores, i, p.pos_base) > T;
+    for (int q = 0; q < kGPer / 4; ++q) {
+      const float4 x = __ldg(v + q);
+      sc[4 * q] = x.x;
+      sc[4 * q + 1] = x.y;
+      sc[4 * q + 2] = x.z;
+      sc[4 * q + 3] = x.w;
     }
+  } else {
 #pragma unroll
-    for (int j = 0; j < kPer; ++j) {
-      const uint64_t i = start + static_cast<uint64_t>(j) * kThreads + threadIdx.x;
-      const bool valid = i < end;
-      const bool keep = kp[j];
-      uint32_t total;
-      const uint32_t r = block_rank(keep, warp_cnt, &total);
-      if (valid) {
-        b = gbank(p.ebeg, b, hi, i);
-        const uint64_t first = __ldg(p.ebeg + b);
-        if (keep) p.kept_idx[base + r] = static_cast<int32_t>(i - first);
-        if (i == first) {
-          p.kept_off[b] = static_cast<int32_t>(base + r);
-          for (int e = b - 1; e >= 0 && __ldg(p.ebeg + e) == i; --e)
-            p.kept_off[e] = static_cast<int32_t>(base + r);
+    for (int j = 0; j < kGPer; ++j) sc[j] = i0 + j < end ? __ldg(p.scores + i0 + j) : 0.f;
+  }
+}
+
+__device__ __forceinline__ uint64_t gkey_of(float sc, uint64_t pos) {
+  return (static_cast<uint64_t>(ord32(sc)) << 32) | (0xFFFFFFFFull - pos);
+}
+
+// Exclusive warp scan of one uint32 per lane; *total = warp sum.
+__device__ __forceinline__ uint32_t warp_excl_scan(uint32_t v, uint32_t* total) {
+  const int lane = threadIdx.x & 31;
+  uint32_t incl = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint32_t o = __shfl_up_sync(kFull, incl, d);
+    if (lane >= d) incl += o;
+  }
+  *total = __shfl_sync(kFull, incl, 31);
+  return incl - v;
+}
+
+// The bank of entry i of a tile whose entries lie in banks lo .. hi, with
+// its first entry and the next bank's.  Every lane of the warp calls it.
+// When the tile touches at most 31 banks, lane k holds the first entry of
+// bank lo + k and the search runs over the warp's registers.
+__device__ __forceinline__ int gbank_tile(const GPlan& p, int lo, int hi, uint64_t i,
+                                          uint64_t* first, uint64_t* next) {
+  const int lane = threadIdx.x & 31;
+  if (hi - lo <= 30) {  // the same for the whole warp
+    const uint64_t eb = __ldg(p.ebeg + lo + min(lane, hi - lo + 1));
+    int k = 0;  // the last k <= hi - lo with first entry <= i
+#pragma unroll
+    for (int step = 16; step > 0; step >>= 1) {
+      const int c = k + step;
+      const uint64_t v = __shfl_sync(kFull, eb, c < 31 ? c : 31);
+      if (c <= hi - lo && v <= i) k = c;
+    }
+    *first = __shfl_sync(kFull, eb, k);
+    *next = __shfl_sync(kFull, eb, k + 1);
+    return lo + k;
+  }
+  const int b = gbank(p.ebeg, lo, hi, i);
+  *first = __ldg(p.ebeg + b);
+  *next = __ldg(p.ebeg + b + 1);
+  return b;
+}
+
+template <bool UNIFORM>
+__global__ void __launch_bounds__(kThreads, 4) k_gfinish(GPlan p, int first_pass) {
+  __shared__ uint32_t ch[kGBins];
+  __shared__ unsigned long long wh[UNIFORM ? 1 : kGBins];
+  __shared__ GLocal s;
+  __shared__ uint64_t scan64[kWarps];
+  __shared__ uint32_t scan32[kWarps];
+  __shared__ bool s_ok;
+  GState* st = p.st;
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const uint64_t nthreads = static_cast<uint64_t>(gridDim.x) * kThreads;
+  const uint64_t gtid = static_cast<uint64_t>(blockIdx.x) * kThreads + threadIdx.x;
+  const uint32_t units = static_cast<uint32_t>(p.tiles) * kWarps;
+  const uint32_t gwarp = blockIdx.x * kWarps + wib, nwarps = gridDim.x * kWarps;
+  if (threadIdx.x == 0) {
+    s.prefix = __ldcg(&st->prefix);
+    s.mask = __ldcg(&st->mask);
+    s.remaining = __ldcg(&st->remaining);
+    s.threshold = __ldcg(&st->threshold);
+    s.done = __ldcg(&st->done);
+  }
+  // Scratch bins of the passes after the first binned here; nothing adds to
+  // them before the first barrier.
+  for (uint64_t i = gtid; i < static_cast<uint64_t>(kGPasses) * kGBins; i += nthreads) {
+    const int ps = static_cast<int>(i / kGBins);
+    if (ps > first_pass) {
+      p.hb[ps].c[i % kGBins] = 0;
+      p.hb[ps].w[i % kGBins] = 0;
+    }
+  }
+  auto zero_bins = [&]() {
+    for (int i = threadIdx.x; i < kGBins; i += kThreads) {
+      ch[i] = 0;
+      if (!UNIFORM) wh[i] = 0;
+    }
+    __syncthreads();
+  };
+  // The digit choice of a pass, by the last block to reach the barrier after
+  // it; every block then reads the new state.
+  auto pick = [&](int ps) {
+    gpick_block<UNIFORM>(&s, ps, p.uniform_bytes, gbins_c(p, ps, first_pass),
+                         gbins_w(p, ps, first_pass), scan64);
+    if (threadIdx.x == 0) {
+      st->prefix = s.prefix;
+      st->mask = s.mask;
+      st->remaining = s.remaining;
+      st->threshold = s.threshold;
+      st->done = s.done;
+    }
+  };
+  auto load_state = [&]() {
+    if (threadIdx.x == 0) {
+      s.prefix = __ldcg(&st->prefix);
+      s.mask = __ldcg(&st->mask);
+      s.remaining = __ldcg(&st->remaining);
+      s.threshold = __ldcg(&st->threshold);
+      s.done = __ldcg(&st->done);
+    }
+    __syncthreads();
+  };
+  // Each warp's units in turn (unit u: the candidates of entries
+  // [512 u, 512 u + 512)), the next unit's count fetched ahead.
+  auto for_units = [&](auto&& body) {
+    uint32_t u = gwarp;
+    uint32_t nc = u < units ? __ldcg(p.ucand + u) : 0u;
+    while (u < units) {
+      const uint32_t un = u + nwarps;
+      const uint32_t nn = un < units ? __ldcg(p.ucand + un) : 0u;
+      if (nc) body(u, nc);
+      u = un;
+      nc = nn;
+    }
+  };
+  uint32_t nbar = 0;  // barriers passed
+  __syncthreads();
+  int pass = first_pass;
+
+  // Pass 0: the top digit of every key.
+  if (pass == 0 && !s.done) {
+    zero_bins();
+    for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
+      const uint64_t end = min(static_cast<uint64_t>(t + 1) * kGTile, p.entries);
+      const uint64_t i0 = glane0(t);
+      float sc[kGPer];
+      gload(p, i0, end, sc);
+      int b = 0, hi = 0;
+      if (!UNIFORM && i0 < end) {
+        hi = p.tile_bank[t + 1];
+        b = gbank(p.ebeg, p.tile_bank[t], hi, i0);
+      }
+#pragma unroll
+      for (int j = 0; j < kGPer; ++j) {
+        const uint64_t i = i0 + j;
+        uint64_t bytes = 0;
+        if (!UNIFORM && i < end) {
+          while (b < hi && __ldg(p.ebeg + b + 1) <= i) ++b;
+          bytes = __ldg(p.ebytes + b);
+        }
+        gbin<UNIFORM>(ch, wh, i < end ? ord32(sc[j]) >> 21 : kGBins, bytes);
+      }
+    }
+    gbins_add<UNIFORM>(ch, wh, kGBins, gbins_c(p, 0, first_pass), gbins_w(p, 0, first_pass));
+    if (!grid_barrier(st, p.err, ++nbar, &s_ok, [&] { pick(0); })) return;
+    load_state();
+    pass = 1;
+  }
+
+  // The first full scan: kept-for-sure counts per tile; candidates (keys
+  // inside the digits fixed so far) binned by the next digit and stored in
+  // their unit's slots.
+  const bool cand_scan = !s.done;
+  if (cand_scan) zero_bins();
+  {
+    const int shift = gdigit_shift(pass);
+    const uint32_t dmask = (1u << gdigit_bits(pass)) - 1u;
+    const uint64_t prefix = s.prefix, mask = s.mask;
+    const uint64_t above = s.done ? s.threshold : (prefix | ~mask);
+    for (int t = blockIdx.x; t < p.tiles; t += gridDim.x) {
+      const uint64_t end = min(static_cast<uint64_t>(t + 1) * kGTile, p.entries);
+      const uint64_t i0 = glane0(t);
+      float sc[kGPer];
+      gload(p, i0, end, sc);
+      uint32_t sure = 0, cm = 0;
+#pragma unroll
+      for (int j = 0; j < kGPer; ++j) {
+        if (i0 + j < end) {
+          const uint64_t key = gkey_of(sc[j], p.pos_base + i0 + j);
+          if (key > above) ++sure;
+          else if (cand_scan && (key & mask) == prefix) cm |= 1u << j;
         }
       }
-      base += total;
+      uint32_t nc, sure_w;
+      const uint32_t at0 = warp_excl_scan(__popc(cm), &nc);
+      warp_excl_scan(sure, &sure_w);
+      if (cm) {  // few lanes: bin the candidates and store them in the unit's slots
+        const uint64_t slot = (static_cast<uint64_t>(t) * kWarps + wib) * kGUnit + at0;
+        int b = 0, hi = 0;
+        if (!UNIFORM) {
+          hi = p.tile_bank[t + 1];
+          b = gbank(p.ebeg, p.tile_bank[t], hi, i0);
+        }
+        uint32_t k = 0;
+#pragma unroll
+        for (int j = 0; j < kGPer; ++j) {
+          if (cm & (1u << j)) {
+            const uint64_t i = i0 + j;
+            const uint64_t key = gkey_of(sc[j], p.pos_base + i);
+            const uint32_t d = static_cast<uint32_t>(key >> shift) & dmask;
+            p.ckey[slot + k] = key;
+            atomicAdd(&ch[d], 1u);
+            if (!UNIFORM) {
+              while (b < hi && __ldg(p.ebeg + b + 1) <= i) ++b;
+              p.cbank[slot + k] = static_cast<uint32_t>(b);
+              atomicAdd(&wh[d], static_cast<unsigned long long>(__ldg(p.ebytes + b)));
+            }
+            ++k;
+          }
+        }
+      }
+      if (lane == 0) {
+        p.ucand[static_cast<uint64_t>(t) * kWarps + wib] = nc;
+        scan32[wib] = sure_w;
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        uint32_t sum = 0;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) sum += scan32[w];
+        p.tile_cnt[t] = sum;
+      }
+      __syncthreads();
     }
+  }
+  if (cand_scan) {
+    gbins_add<UNIFORM>(ch, wh, 1 << gdigit_bits(pass), gbins_c(p, pass, first_pass),
+                       gbins_w(p, pass, first_pass));
+    if (!grid_barrier(st, p.err, ++nbar, &s_ok, [&] { pick(pass); })) return;
+    load_state();
+    ++pass;
+  }
+
+  // Later passes over the candidates only.
+  while (!s.done && pass < kGPasses) {
+    zero_bins();
+    const int shift = gdigit_shift(pass);
+    const uint32_t dmask = (1u << gdigit_bits(pass)) - 1u;
+    const uint64_t prefix = s.prefix, mask = s.mask;
+    for_units([&](uint32_t u, uint32_t nc) {
+      const uint64_t slot = static_cast<uint64_t>(u) * kGUnit;
+      for (uint32_t k = lane; k < nc; k += 32) {
+        const uint64_t key = __ldcg(p.ckey + slot + k);
+        if ((key & mask) == prefix) {
+          const uint32_t d = static_cast<uint32_t>(key >> shift) & dmask;
+          atomicAdd(&ch[d], 1u);
+          if (!UNIFORM)
+            atomicAdd(&wh[d], static_cast<unsigned long long>(
+                                  __ldg(p.ebytes + __ldcg(p.cbank + slot + k))));
+        }
+      }
+    });
+    gbins_add<UNIFORM>(ch, wh, 1 << gdigit_bits(pass), gbins_c(p, pass, first_pass),
+                       gbins_w(p, pass, first_pass));
+    if (!grid_barrier(st, p.err, ++nbar, &s_ok, [&] { pick(pass); })) return;
+    load_state();
+    ++pass;
+  }
+  const uint64_t T = s.threshold;
+
+  // Kept candidates join their tiles' counts.
+  if (cand_scan) {
+    for_units([&](uint32_t u, uint32_t nc) {
+      const uint64_t slot = static_cast<uint64_t>(u) * kGUnit;
+      uint32_t kept = 0;
+      for (uint32_t k = lane; k < nc; k += 32) kept += __ldcg(p.ckey + slot + k) > T;
+#pragma unroll
+      for (int d = 16; d > 0; d >>= 1) kept += __shfl_xor_sync(kFull, kept, d);
+      if (lane == 0 && kept) atomicAdd(p.tile_cnt + u / kWarps, kept);
+    });
+  }
+  if (!grid_barrier(st, p.err, ++nbar, &s_ok, [] {})) return;
+
+  // Write: block b takes tiles [t0, t1) and starts at the kept count before t0.
+  const int t0 = static_cast<int>(static_cast<int64_t>(p.tiles) * blockIdx.x / gridDim.x);
+  const int t1 = static_cast<int>(static_cast<int64_t>(p.tiles) * (blockIdx.x + 1) / gridDim.x);
+  uint32_t before = 0;
+  {
+    uint32_t part = 0;
+    for (int t = threadIdx.x; t < t0; t += kThreads) part += __ldcg(p.tile_cnt + t);
+    uint32_t total;
+    block_excl_scan(part, scan32, &total);
+    before = total;
+  }
+  if (blockIdx.x == 0) {  // the total and the offsets of trailing empty banks
+    uint32_t part = 0;
+    for (int t = threadIdx.x; t < p.tiles; t += kThreads) part += __ldcg(p.tile_cnt + t);
+    uint32_t total;
+    block_excl_scan(part, scan32, &total);
+    if (threadIdx.x == 0) {
+      st->total_kept = total;
+      st->threshold = T;
+      p.kept_off[p.n_banks] = static_cast<int32_t>(total);
+      for (int b = p.n_banks - 1; b >= 0 && p.ebeg[b] == p.entries; --b)
+        p.kept_off[b] = static_cast<int32_t>(total);
+    }
+  }
+  for (int t = t0; t < t1; ++t) {
+    const uint64_t end = min(static_cast<uint64_t>(t + 1) * kGTile, p.entries);
+    const uint64_t i0 = glane0(t);
+    uint32_t keep = 0;  // bit j: entry i0 + j is kept
+    {
+      float sc[kGPer];
+      gload(p, i0, end, sc);
+#pragma unroll
+      for (int j = 0; j < kGPer; ++j)
+        if (i0 + j < end && gkey_of(sc[j], p.pos_base + i0 + j) > T) keep |= 1u << j;
+    }
+    uint32_t wtot;
+    const uint32_t lane_before = warp_excl_scan(__popc(keep), &wtot);
+    if (lane == 0) scan32[wib] = wtot;
+    __syncthreads();
+    uint32_t rank = before + lane_before, all = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const uint32_t v = scan32[w];
+      if (w < wib) rank += v;
+      all += v;
+    }
+    __syncthreads();
+    // The lane's bank cursor: bank b holds entries [first, next).
+    const int hi = p.tile_bank[t + 1];
+    uint64_t first, next;
+    int b = gbank_tile(p, p.tile_bank[t], hi, i0, &first, &next);
+    if (i0 < end) {
+#pragma unroll
+      for (int j = 0; j < kGPer; ++j) {
+        const uint64_t i = i0 + j;
+        if (i < end) {
+          while (b < hi && next <= i) {
+            ++b;
+            first = next;
+            next = __ldg(p.ebeg + b + 1);
+          }
+          if (i == first) {
+            p.kept_off[b] = static_cast<int32_t>(rank);
+            for (int e = b - 1; e >= 0 && __ldg(p.ebeg + e) == i; --e)
+              p.kept_off[e] = static_cast<int32_t>(rank);
+          }
+          if (keep & (1u << j)) p.kept_idx[rank++] = static_cast<int32_t>(i - first);
+        }
+      }
+    }
+    before += all;
   }
 }
 
@@ -1892,6 +2359,28 @@ int occupancy() {
   return b > 0 ? b : 1;
 }
 
+// Blocks of kThreads threads (no dynamic shared memory) of `kernel` that one
+// SM holds at once, asked once per kernel.  A grid of SMs x this many blocks
+// is one resident wave: a larger grid of equal blocks leaves its last wave
+// part-full, with fewer loads in flight while it runs.
+int resident_blocks(const void* kernel) {
+  static std::mutex mu;
+  static const void* keys[64];
+  static int vals[64];
+  static int n = 0;
+  std::lock_guard<std::mutex> lk(mu);
+  for (int i = 0; i < n; ++i)
+    if (keys[i] == kernel) return vals[i];
+  int b = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, kernel, kThreads, 0) != cudaSuccess || b < 1)
+    b = 1;
+  if (n < 64) {
+    keys[n] = kernel;
+    vals[n++] = b;
+  }
+  return b;
+}
+
 template <int MODE>
 cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, uint32_t* err,
                              int sm_count, cudaStream_t stream) {
@@ -2027,17 +2516,23 @@ cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
                          GHist gh, bool* fused) {
   if (fused) *fused = false;
   if (n_entries == 0) return cudaSuccess;
+  // At least eight rounds per warp; at most one resident wave.
   const uint64_t want = (n_entries + kWarps * kScoreIlp * 8 - 1) / (kWarps * kScoreIlp * 8);
-  const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
-  const int blocks = static_cast<int>(want < cap ? want : cap);
+  auto grid = [&](const void* k) {
+    const uint64_t cap = static_cast<uint64_t>(sm_count) * resident_blocks(k);
+    return static_cast<int>(want < cap ? want : cap);
+  };
   // key_types: 0 = all fp16, 1 = all bf16, 2 = mixed.
   if (key_types == 2 || max_dim > 1024) {
-    k_score_any<<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores);
+    k_score_any<<<grid(reinterpret_cast<const void*>(k_score_any)), kThreads, 0, stream>>>(
+        banks, n_banks, n_entries, scores);
     return cudaGetLastError();
   }
   const int spl = max_dim <= 256 ? 1 : max_dim <= 512 ? 2 : 4;
   const int hm = gh.st ? gh.mode : 0;
-#define PCS_SCORE(S, D, H) k_score_fixed<S, D, H><<<blocks, kThreads, 0, stream>>>(banks, n_banks, n_entries, scores, gh)
+#define PCS_SCORE(S, D, H)                                                                    \
+  k_score_fixed<S, D, H><<<grid(reinterpret_cast<const void*>(k_score_fixed<S, D, H>)), kThreads, \
+                           0, stream>>>(banks, n_banks, n_entries, scores, gh)
 #define PCS_SCORE_H(S, D) (hm == 0 ? PCS_SCORE(S, D, 0) : hm == 1 ? PCS_SCORE(S, D, 1) : PCS_SCORE(S, D, 2))
   if (key_types == 1) {
     if (spl == 1) PCS_SCORE_H(1, 1);
@@ -2062,15 +2557,20 @@ cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
   return cudaGetLastError();
 }
 
-static int gblocks(const GPlan& p, int sm_count) {
-  const int cap = 4 * sm_count;
+static int gblocks(const GPlan& p, int sm_count, const void* kernel) {
+  const int cap = sm_count * resident_blocks(kernel);
   return p.tiles < cap ? p.tiles : cap;
 }
 
 cudaError_t launch_gselect(const GPlan& p, int pass, int sm_count, cudaStream_t stream) {
   if (p.tiles <= 0) return cudaSuccess;
-  if (p.uniform) k_gselect<true><<<gblocks(p, sm_count), kThreads, 0, stream>>>(p, pass);
-  else k_gselect<false><<<gblocks(p, sm_count), kThreads, 0, stream>>>(p, pass);
+  if (p.uniform) {
+    const int g = gblocks(p, sm_count, reinterpret_cast<const void*>(k_gselect<true>));
+    k_gselect<true><<<g, kThreads, 0, stream>>>(p, pass);
+  } else {
+    const int g = gblocks(p, sm_count, reinterpret_cast<const void*>(k_gselect<false>));
+    k_gselect<false><<<g, kThreads, 0, stream>>>(p, pass);
+  }
   return cudaGetLastError();
 }
 
@@ -2100,7 +2600,8 @@ cudaError_t launch_pool_cow(const PoolDev& p, int32_t* table, int64_t n_table,
                             const int32_t* entries, int32_t n, int sm_count, cudaStream_t stream) {
   if (n <= 0) return cudaSuccess;
   const int64_t want = (static_cast<int64_t>(n) + kWarps - 1) / kWarps;
-  const int64_t cap = static_cast<int64_t>(sm_count) * 8;
+  const int64_t cap = static_cast<int64_t>(sm_count) *
+                      resident_blocks(reinterpret_cast<const void*>(k_pool_cow));
   k_pool_cow<<<static_cast<unsigned>(want < cap ? want : cap), kThreads, 0, stream>>>(
       p, table, n_table, entries, n);
   return cudaGetLastError();
@@ -2136,13 +2637,17 @@ cudaError_t launch_classify_reads(const ReadPlan& p, const uint64_t* addr, const
   return cudaGetLastError();
 }
 
-cudaError_t launch_gcompact(const GPlan& p, int sm_count, cudaStream_t stream) {
+cudaError_t launch_gfinish(const GPlan& p, int first_pass, int sm_count, cudaStream_t stream) {
   if (p.tiles <= 0) return cudaSuccess;
-  k_gcount<<<gblocks(p, sm_count), kThreads, 0, stream>>>(p);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  k_gwrite<<<gblocks(p, sm_count), kThreads, 0, stream>>>(p);
-  return cudaGetLastError();
+  const void* k = p.uniform ? reinterpret_cast<const void*>(k_gfinish<true>)
+                            : reinterpret_cast<const void*>(k_gfinish<false>);
+  // Every block must be resident at once: at most one wave.
+  const int cap = sm_count * resident_blocks(k);
+  const int grid = p.tiles < cap ? p.tiles : cap;
+  GPlan a = p;
+  int fp = first_pass;
+  void* args[] = {&a, &fp};
+  return cudaLaunchCooperativeKernel(k, dim3(grid), dim3(kThreads), args, 0, stream);
 }
 
 

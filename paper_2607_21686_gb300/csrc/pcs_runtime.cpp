@@ -383,7 +383,7 @@ pcs_status set_device(pcs_ctx* c) {
 enum KernelKind {
   kKStreamHash, kKStreamPack, kKStreamRestore, kKStreamRestoreV, kKFinalizeHash,
   kKFinalizePack, kKFinalizeRestoreV, kKScore, kKTopk, kKBulkHash, kKBulkPack,
-  kKBulkRestore, kKBulkRestoreV, kKReduce, kKGSelect, kKGCompact, kKPoolAlloc, kKPoolShare,
+  kKBulkRestore, kKBulkRestoreV, kKReduce, kKGSelect, kKGFinish, kKPoolAlloc, kKPoolShare,
   kKPoolCow, kKPoolRelease, kKMismatch, kKClassifyReads, kKernelKinds
 };
 static_assert(kKernelKinds <= 32, "kernel timing table");
@@ -391,7 +391,7 @@ const char* kKernelNames[kKernelKinds] = {
     "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
     "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
-    "k_reduce_nodes", "k_gselect", "k_gcompact", "k_pool_alloc", "k_pool_share", "k_pool_cow",
+    "k_reduce_nodes", "k_gselect", "k_gfinish", "k_pool_alloc", "k_pool_share", "k_pool_cow",
     "k_pool_release", "k_mismatch", "k_classify_reads"};
 
 cudaEvent_t timing_event(pcs_ctx* c) {
@@ -1679,6 +1679,14 @@ static pcs_status prune_global_impl(pcs_ctx* c, const pcs_bank* banks, int32_t n
   const uint64_t plan_bytes = at;
   const uint64_t o_tc = at;
   at = round_up(at + 4ull * tiles, kRecordAlign);
+  const uint64_t o_ucand = at;
+  at = round_up(at + 4ull * 8 * tiles, kRecordAlign);
+  const uint64_t o_hb = at;
+  at = round_up(at + sizeof(GBinSet) * kGPasses, kRecordAlign);
+  const uint64_t o_ckey = at;
+  at = round_up(at + 8ull * kGTile * tiles, kRecordAlign);
+  const uint64_t o_cbank = at;
+  if (!uniform) at = round_up(at + 4ull * kGTile * tiles, kRecordAlign);
   const uint64_t o_sc = at;
   const uint64_t ws_bytes = at + (scores ? 0 : 4ull * entries);
   uint8_t* ws = nullptr;
@@ -1716,24 +1724,26 @@ static pcs_status prune_global_impl(pcs_ctx* c, const pcs_bank* banks, int32_t n
   gp.tiles = static_cast<int32_t>(tiles);
   gp.uniform = uniform ? 1 : 0;
   gp.pos_base = pos_base;
+  gp.vec = aligned16(sc) ? 1 : 0;
+  gp.ucand = reinterpret_cast<uint32_t*>(ws + o_ucand);
+  gp.ckey = reinterpret_cast<uint64_t*>(ws + o_ckey);
+  gp.cbank = uniform ? nullptr : reinterpret_cast<uint32_t*>(ws + o_cbank);
+  gp.hb = reinterpret_cast<GBinSet*>(ws + o_hb);
+  gp.err = c->words;
   if (ex) {
+    // Every pass summed over the parts and picked on the host; the state
+    // reaches k_gfinish done.
     gp.local = 1;
     st = exchange_passes(c, gp, budget, ex, user, stream);
     if (st) return st;
-  } else if (!g0.done) {
-    // Six digit passes at most (the first inside the score kernel when it
-    // could take it); each is a no-op once the threshold is known.
-    for (int pass = fused ? 1 : 0; pass < kGPasses; ++pass) {
-      LaunchScope ls(c, kKGSelect, stream);
-      PCS_CUDA(launch_gselect(gp, pass, c->sm_count, stream));
-    }
   }
   if (entries == 0) {
     PCS_CUDA(cudaMemsetAsync(kept_off, 0, 4ull * (n + 1), stream));
   } else {
-    LaunchScope ls(c, kKGCompact, stream);
-    c->launches += 1;  // count and write
-    PCS_CUDA(launch_gcompact(gp, c->sm_count, stream));
+    // The passes the score kernel did not take (at most six, none once the
+    // threshold is known) and the compaction, in one launch.
+    LaunchScope ls(c, kKGFinish, stream);
+    PCS_CUDA(launch_gfinish(gp, fused ? 1 : 0, c->sm_count, stream));
   }
   return ws_release(c, stream);
 }

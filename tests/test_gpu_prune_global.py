@@ -4,8 +4,9 @@ pcs_prune_global through the C ABI against the oracle on the same seeded
 banks: scores bit-equal to the oracle's fixed-order fp32 score, kept sets and
 bank offsets identical, across several 4096-entry tiles with a ragged tail,
 with uniform and mixed entry sizes (the two select paths), empty banks at
-either end and in the middle, exact ties across banks, and budgets that keep
-nothing, one entry, a fraction, all but one, and all.  The same population
+either end and in the middle, exact ties across banks, mixed key types and
+keys wider than 1024 (the first digit binned after the score kernel), and
+budgets that keep nothing, one entry, a fraction, all but one, and all.  The same population
 split into two parts (two threads, two contexts, the histograms summed on the
 host each pass, as ranks would all-reduce them) gives each part its share of
 the one-population answer.
@@ -126,6 +127,33 @@ def test_global_threshold_keeps_relevant_sessions(ctx, dev):
     qs = [q.half().to(dev)] * 2
     kept, koff, _ = _run(ctx, dev, keys, qs, 10, 2000)
     assert koff.tolist() == [0, 200, 200]
+
+
+@pytest.mark.parametrize("mixed_bytes", [False, True])
+def test_global_threshold_mixed_key_types(ctx, dev, mixed_bytes):
+    # fp16 and bf16 banks together (and, below, keys wider than 1024): the
+    # score kernel takes no digit pass, so the first is binned after it.
+    g = torch.Generator().manual_seed(21)
+    D = 96
+    keys, qs = [], []
+    for s in range(14):
+        dt = torch.float16 if s % 2 else torch.bfloat16
+        n = int(torch.randint(0, 900, (1,), generator=g))
+        keys.append(torch.randn(n, D, generator=g).to(dt).to(dev))
+        qs.append(torch.randn(D, generator=g).to(dt).to(dev))
+    E = [int(x) for x in np.random.default_rng(4).integers(1, 3000, 14)] if mixed_bytes else 700
+    Eb = E if mixed_bytes else [E] * 14
+    T = sum(k.shape[0] * e for k, e in zip(keys, Eb))
+    _check(ctx, dev, keys, qs, E, [0, 1, T // 9, T // 2, T - 1, T])
+
+
+def test_global_threshold_wide_keys(ctx, dev):
+    g = torch.Generator().manual_seed(22)
+    D = 1536
+    keys = [torch.randn(int(n), D, generator=g).half().to(dev) for n in (300, 0, 1200, 77)]
+    qs = [torch.randn(D, generator=g).half().to(dev) for _ in range(4)]
+    T = sum(k.shape[0] for k in keys) * 50
+    _check(ctx, dev, keys, qs, 50, [0, 50, T // 3, T - 50, T])
 
 
 def _split_run(dev, keys, qs, E, budget, cut):
