@@ -1279,13 +1279,124 @@ __device__ __forceinline__ uint32_t block_rank(bool f, uint32_t* warp_cnt, uint3
   return before + in_warp;
 }
 
+// Exclusive block scan of one uint32 per thread; *total = block sum.
+__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_sum,
+                                                    uint32_t* total) {
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  uint32_t incl = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint32_t o = __shfl_up_sync(kFull, incl, d);
+    if (lane >= d) incl += o;
+  }
+  if (lane == 31) warp_sum[wib] = incl;
+  __syncthreads();
+  uint32_t before = 0, sum = 0;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) {
+    const uint32_t c = warp_sum[w];
+    if (w < wib) before += c;
+    sum += c;
+  }
+  __syncthreads();
+  *total = sum;
+  return before + incl - v;
+}
+
+// The digit of one radix-select pass (warp 0, histogram in shared memory):
+// scanning bins from the top, the first whose running count reaches the
+// rank still wanted is fixed into the prefix.
+__device__ __forceinline__ void topk_pick(const uint32_t* hist, int shift, uint32_t* s_prefix,
+                                          uint32_t* s_mask, uint32_t* s_remaining) {
+  const int lane = threadIdx.x & 31;
+  // Lane l covers bins 255-8l .. 248-8l (descending).
+  uint32_t local = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) local += hist[255 - 8 * lane - j];
+  uint32_t incl = local;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint32_t o = __shfl_up_sync(kFull, incl, d);
+    if (lane >= d) incl += o;
+  }
+  const uint32_t remaining = *s_remaining;
+  const unsigned hit = __ballot_sync(kFull, incl >= remaining);
+  const int first = __ffs(hit) - 1;  // remaining <= count, so hit != 0
+  if (lane == first) {
+    uint32_t cum = incl - local;
+    for (int j = 0; j < 8; ++j) {
+      const int bin = 255 - 8 * lane - j;
+      if (cum + hist[bin] >= remaining) {
+        *s_prefix |= static_cast<uint32_t>(bin) << shift;
+        *s_mask |= 0xFFu << shift;
+        *s_remaining = remaining - cum;
+        break;
+      }
+      cum += hist[bin];
+    }
+  }
+}
+
+constexpr int kTopkPer = 16;                    // entries a thread holds
+constexpr int kTopkReg = kThreads * kTopkPer;   // banks up to this size stay in registers
+
+// One bank of at most kTopkReg entries, 0 < k < n: thread t holds the keys of
+// entries [16 t, 16 t + 16) for all four passes; the kept entries (every key
+// above the threshold, then the first ones equal to it) are ranked with two
+// block scans and written in ascending index order.
+__device__ void topk_bank_reg(const float* __restrict__ sc, int n, int k, int32_t* __restrict__ out,
+                              uint32_t* hist, uint32_t* warp_sum, uint32_t* s_prefix,
+                              uint32_t* s_mask, uint32_t* s_remaining) {
+  const int base = threadIdx.x * kTopkPer;
+  uint32_t u[kTopkPer];
+#pragma unroll
+  for (int j = 0; j < kTopkPer; ++j) u[j] = base + j < n ? ord32(__ldg(sc + base + j)) : 0u;
+  if (threadIdx.x == 0) {
+    *s_prefix = 0;
+    *s_mask = 0;
+    *s_remaining = static_cast<uint32_t>(k);
+  }
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    for (int i = threadIdx.x; i < 256; i += kThreads) hist[i] = 0;
+    __syncthreads();
+    const uint32_t prefix = *s_prefix, mask = *s_mask;
+#pragma unroll
+    for (int j = 0; j < kTopkPer; ++j)
+      if (base + j < n && (u[j] & mask) == prefix) atomicAdd(&hist[(u[j] >> shift) & 255u], 1u);
+    __syncthreads();
+    if (threadIdx.x < 32) topk_pick(hist, shift, s_prefix, s_mask, s_remaining);
+    __syncthreads();
+  }
+  const uint32_t t = *s_prefix, take_eq = *s_remaining;
+  uint32_t gt = 0, eq = 0;
+#pragma unroll
+  for (int j = 0; j < kTopkPer; ++j) {
+    if (base + j < n) {
+      gt |= static_cast<uint32_t>(u[j] > t) << j;
+      eq |= static_cast<uint32_t>(u[j] == t) << j;
+    }
+  }
+  uint32_t total;
+  uint32_t r = block_excl_scan(__popc(eq), warp_sum, &total);  // equal keys before this thread's
+  uint32_t keep = gt;
+  for (uint32_t m = eq; m; m &= m - 1) {
+    if (r >= take_eq) break;
+    keep |= m & (~m + 1u);
+    ++r;
+  }
+  uint32_t pos = block_excl_scan(__popc(keep), warp_sum, &total);
+  for (uint32_t m = keep; m; m &= m - 1) out[pos++] = base + __ffs(m) - 1;
+  __syncthreads();
+}
+
 __global__ void __launch_bounds__(kThreads)
     k_topk(const BankDesc* __restrict__ banks, int n_banks, const float* __restrict__ scores,
            int32_t* __restrict__ kept_idx) {
   __shared__ uint32_t hist[256];
   __shared__ uint32_t warp_cnt[kWarps];
   __shared__ uint32_t s_prefix, s_mask, s_remaining;
-  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const int wib = threadIdx.x >> 5;
   for (int b = blockIdx.x; b < n_banks; b += gridDim.x) {
     const BankDesc B = banks[b];
     const int n = B.n, k = B.k;
@@ -1296,6 +1407,10 @@ __global__ void __launch_bounds__(kThreads)
       continue;
     }
     if (k <= 0) continue;
+    if (n <= kTopkReg) {
+      topk_bank_reg(sc, n, k, out, hist, warp_cnt, &s_prefix, &s_mask, &s_remaining);
+      continue;
+    }
     if (threadIdx.x == 0) {
       s_prefix = 0;
       s_mask = 0;
@@ -1313,34 +1428,7 @@ __global__ void __launch_bounds__(kThreads)
         if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & 255u], 1u);
       }
       __syncthreads();
-      if (wib == 0) {
-        // Lane l covers bins 255-8l .. 248-8l (descending).
-        uint32_t local = 0;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) local += hist[255 - 8 * lane - j];
-        uint32_t incl = local;
-#pragma unroll
-        for (int d = 1; d < 32; d <<= 1) {
-          const uint32_t o = __shfl_up_sync(kFull, incl, d);
-          if (lane >= d) incl += o;
-        }
-        const uint32_t remaining = s_remaining;
-        const unsigned hit = __ballot_sync(kFull, incl >= remaining);
-        const int first = __ffs(hit) - 1;  // remaining <= count, so hit != 0
-        if (lane == first) {
-          uint32_t cum = incl - local;
-          for (int j = 0; j < 8; ++j) {
-            const int bin = 255 - 8 * lane - j;
-            if (cum + hist[bin] >= remaining) {
-              s_prefix = prefix | (static_cast<uint32_t>(bin) << shift);
-              s_mask = mask | (0xFFu << shift);
-              s_remaining = remaining - cum;
-              break;
-            }
-            cum += hist[bin];
-          }
-        }
-      }
+      if (wib == 0) topk_pick(hist, shift, &s_prefix, &s_mask, &s_remaining);
       __syncthreads();
     }
     // Keep every entry above the threshold and the first `remaining` equal
@@ -1444,29 +1532,6 @@ __global__ void __launch_bounds__(kThreads) k_gselect(GPlan p, int pass) {
   gpass_finish<UNIFORM>(st, pass, p.uniform_bytes, ch, wh, &s_last, !p.local);
 }
 
-// Exclusive block scan of one uint32 per thread; *total = block sum.
-__device__ __forceinline__ uint32_t block_excl_scan(uint32_t v, uint32_t* warp_sum,
-                                                    uint32_t* total) {
-  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-  uint32_t incl = v;
-#pragma unroll
-  for (int d = 1; d < 32; d <<= 1) {
-    const uint32_t o = __shfl_up_sync(kFull, incl, d);
-    if (lane >= d) incl += o;
-  }
-  if (lane == 31) warp_sum[wib] = incl;
-  __syncthreads();
-  uint32_t before = 0, sum = 0;
-#pragma unroll
-  for (int w = 0; w < kWarps; ++w) {
-    const uint32_t c = warp_sum[w];
-    if (w < wib) before += c;
-    sum += c;
-  }
-  __syncthreads();
-  *total = sum;
-  return before + incl - v;
-}
 
 // ---------------------------------------------------------------------------
 // The rest of the global threshold in one cooperative launch (k_gfinish):

@@ -465,6 +465,28 @@ def test_topk_by_recency_keys(ctx, dev, policy):
         assert kh[oh[0]:oh[1]].tolist() == list(range(n[0] - k[0], n[0]))
 
 
+@pytest.mark.parametrize("ties", [False, True])
+def test_topk_bank_sizes(ctx, dev, ties):
+    # Banks up to 4096 entries are selected from registers, larger ones by
+    # re-reading their keys: sizes on both sides of the switch, several k.
+    rnd = np.random.default_rng(17 + ties)
+    n = [1, 17, 255, 256, 257, 4095, 4096, 4097, 10000, 3000]
+    k = [1, 5, 1, 128, 256, 4094, 1000, 4096, 3333, 2999]
+    if ties:
+        keys = [rnd.integers(0, 40, x).astype(np.float32) for x in n]
+    else:
+        keys = [rnd.normal(size=x).astype(np.float32) for x in n]
+    keys[3][:] = 0.0  # one bank of equal keys
+    flat = torch.from_numpy(np.concatenate(keys)).to(dev)
+    kept = torch.empty(sum(k), dtype=torch.int32, device=dev)
+    koff = torch.empty(len(n) + 1, dtype=torch.int32, device=dev)
+    ctx.topk(flat, n, k, kept, koff)
+    ctx.sync()
+    kh, oh = kept.cpu().numpy(), koff.cpu().numpy()
+    for b, (kk, x) in enumerate(zip(keys, k)):
+        assert kh[oh[b]:oh[b + 1]].tolist() == oracle.topk(kk, x).tolist(), b
+
+
 def test_fork_many_mixed_placements(ctx, dev):
     # Device records over 1 MiB take the TMA copy; pinned-host ones the register copy.
     kv = synth.kv(seed=90, sessions=3, layers=2, heads=16, head_dim=64, window=256, page_rows=16)
