@@ -153,7 +153,7 @@ cudaError_t launch_reduce_nodes(const NodeLevel* lv, int n_secs, uint64_t* nodes
 cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess, int n_sess,
                             const Entry* entries, uint64_t* nodes, uint64_t* fp_out,
                             const uint64_t* fp_before, uint8_t* flags, uint32_t* bad,
-                            cudaStream_t stream);
+                            int max_secs, cudaStream_t stream);
 
 
 

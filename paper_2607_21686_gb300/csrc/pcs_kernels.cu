@@ -881,6 +881,66 @@ __global__ void __launch_bounds__(kThreads)
                                 gridDim.x, smem, &s_bad);
 }
 
+// Sessions of at most 32 sections: one warp per session (lane j keeps
+// section j's fp), the same outputs as finalize_sessions_block.
+template <int MODE>
+__global__ void __launch_bounds__(kThreads)
+    k_finalize_sessions_warp(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
+                             int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
+                             uint8_t* corrupt, uint32_t* bad) {
+  const int lane = threadIdx.x & 31;
+  const int nw = gridDim.x * kWarps;
+  for (int b = blockIdx.x * kWarps + (threadIdx.x >> 5); b < n_sess; b += nw) {
+    const SessDesc S = sess[b];
+    Entry* table = reinterpret_cast<Entry*>(S.record + kHeaderBytes);
+    const int ns = static_cast<int>(S.n_sections);
+    uint64_t mine = 0;
+    bool bad_sec = false;
+    for (int j = 0; j < ns; ++j) {
+      const SecDesc s = secs[S.sec_begin + j];
+      const uint64_t fp = stream_fp(s, nodes, lane);
+      if (MODE == kModePack) {
+        if (lane < 4) {
+          Entry e = entries[S.sec_begin + j];
+          e.fp = fp;
+          reinterpret_cast<uint4*>(&table[j])[lane] = reinterpret_cast<const uint4*>(&e)[lane];
+        }
+        if (lane == j) mine = fp;
+      } else {
+        if (lane == j) {
+          mine = table[j].fp;
+          bad_sec = mine != fp;
+        }
+      }
+    }
+    // Session fp = fmix(tree(fps) ^ n), the fps being the table's.
+    const uint64_t sfp = fmix(warp_tree(mine, ns, lane) ^ static_cast<uint64_t>(ns));
+    const bool any_bad = __any_sync(kFull, bad_sec);
+    if (lane == 0) {
+      if (MODE == kModePack) {
+        uint4* h = reinterpret_cast<uint4*>(S.record);
+        h[0] = make_uint4(kMagic, kVersion | (S.n_sections << 16), S.session_id, S.kind);
+        h[1] = make_uint4(static_cast<uint32_t>(S.total_bytes),
+                          static_cast<uint32_t>(S.total_bytes >> 32), static_cast<uint32_t>(sfp),
+                          static_cast<uint32_t>(sfp >> 32));
+        h[2] = make_uint4(0, 0, 0, 0);
+        h[3] = make_uint4(0, 0, 0, 0);
+      } else {
+        const uint64_t stored = *reinterpret_cast<const uint64_t*>(S.record + 24);
+        const bool broken = any_bad || stored != sfp;
+        if (corrupt) corrupt[b] = broken ? 1 : 0;
+        if (broken) atomicAdd(bad, 1u);
+      }
+    }
+    if (MODE == kModePack) {
+      // Zero the gap between the end of the table and the first payload.
+      const uint64_t from = kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * S.n_sections;
+      for (uint64_t o = from + 16u * lane; o < S.payload_start; o += 16u * 32)
+        *reinterpret_cast<uint4*>(S.record + o) = make_uint4(0, 0, 0, 0);
+    }
+  }
+}
+
 // Small calls in one launch: the streaming pass, then the finalisation by
 // the last block to finish (an atomic ticket; no block waits for another).
 // `ticket` is zero on entry and reset by the last block.
@@ -2548,8 +2608,22 @@ cudaError_t launch_small(int mode, const SecDesc* secs, WorkList wl, int group_l
 cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess, int n_sess,
                             const Entry* entries, uint64_t* nodes, uint64_t* fp_out,
                             const uint64_t* fp_before, uint8_t* flags, uint32_t* bad,
-                            cudaStream_t stream) {
+                            int max_secs, cudaStream_t stream) {
   if (n_sess <= 0) return cudaSuccess;
+  if (mode != kModeHash && max_secs <= 32) {
+    // Few sections per session: a warp each, not a block each.
+    const int want = (n_sess + kWarps - 1) / kWarps;
+    const int blocks = want < 65535 ? want : 65535;
+    if (mode == kModePack)
+      k_finalize_sessions_warp<kModePack><<<blocks, kThreads, 0, stream>>>(secs, sess, n_sess,
+                                                                          entries, nodes, flags, bad);
+    else if (mode == kModeRestoreV)
+      k_finalize_sessions_warp<kModeRestoreV><<<blocks, kThreads, 0, stream>>>(
+          secs, sess, n_sess, entries, nodes, flags, bad);
+    else
+      return cudaErrorInvalidValue;
+    return cudaGetLastError();
+  }
   if (mode == kModeHash) {
     const int blocks = (n_sess + kWarps - 1) / kWarps;
     k_finalize_hash<<<blocks < 4096 ? blocks : 4096, kThreads, 0, stream>>>(secs, n_sess, nodes, fp_out,

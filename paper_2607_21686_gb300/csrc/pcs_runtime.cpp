@@ -861,7 +861,7 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   {
     LaunchScope ls(c, kKFinalizeHash, stream);
     PCS_CUDA(launch_finalize(kModeHash, dsecs, nullptr, n, nullptr, nodes, fp_out, fp_before,
-                             flags, nullptr, stream));
+                             flags, nullptr, 0, stream));
   }
   return ws_release(c, stream);
 }
@@ -911,6 +911,7 @@ struct Prepared {
   bool fused = false;    // one k_small launch (small calls)
   int verify = 0;        // restore: 0, 1 or 2
   int32_t n = 0;         // sessions
+  int32_t max_secs = 0;  // most sections in one session
   StreamPlan P;
   ListLayout LL{};
   WsLayout L;
@@ -968,7 +969,7 @@ cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, cudaStr
     if (e != cudaSuccess) return e;
     LaunchScope ls(c, kKFinalizePack, stream);
     return launch_finalize(kModePack, dsecs, dsess, pr.n, dent, nodes, nullptr, nullptr, nullptr,
-                           nullptr, stream);
+                           nullptr, pr.max_secs, stream);
   }
   uint32_t* bad = c->words + (pr.verify == 1 ? 1 : 2);
   if (pr.fused) {
@@ -982,7 +983,7 @@ cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, cudaStr
   if (e != cudaSuccess || !pr.verify) return e;
   LaunchScope ls(c, kKFinalizeRestoreV, stream);
   return launch_finalize(kModeRestoreV, dsecs, dsess, pr.n, nullptr, nodes, nullptr, nullptr,
-                         nullptr, bad, stream);
+                         nullptr, bad, pr.max_secs, stream);
 }
 
 // Plan a checkpoint of n sessions: validate, reserve one block for their
@@ -1067,6 +1068,7 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
   for (int s = 0; s < n; ++s) max_secs = std::max<uint32_t>(max_secs, sd[s].n_sections);
   pr->mode = kModePack;
   pr->n = n;
+  pr->max_secs = static_cast<int32_t>(max_secs);
   pr->fused = fused_ok(bulk, small, n) && max_secs <= 2048;
   if (!plan_streams(c, d, bulk, pr->P, !pr->fused)) {
     arena_of(c, placement)->free(blk);
@@ -1135,6 +1137,7 @@ pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
   pr->mode = verify ? kModeRestoreV : kModeRestore;
   pr->verify = verify;
   pr->n = n;
+  pr->max_secs = static_cast<int32_t>(max_secs);
   pr->fused = verify && fused_ok(bulk, small, n) && max_secs <= 2048;
   if (!plan_streams(c, d, bulk, pr->P, !pr->fused))
     return fail(PCS_E_INVAL, "too much data in one call");
