@@ -101,6 +101,32 @@ __device__ uint64_t warp_tree_inplace(uint64_t* a, uint32_t n, int lane) {
   return a[0];
 }
 
+// The same tree for n <= 1024: up to eight groups of 32 are read at once,
+// group g's root is kept in lane g, then the roots' tree.  Nothing is
+// written.  Called by one whole warp; every lane returns the root.
+__device__ uint64_t warp_tree_regs(const uint64_t* a, uint32_t n, int lane) {
+  const uint32_t groups = (n + 31) / 32;
+  uint64_t mine = 0;
+  for (uint32_t g0 = 0; g0 < groups; g0 += 8) {
+    uint64_t v[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const uint32_t i = 32 * (g0 + q) + lane;
+      v[q] = i < n ? a[i] : 0;
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const uint32_t g = g0 + q;
+      if (g < groups) {  // the same for the whole warp
+        const uint64_t r = __shfl_sync(kFull, warp_tree(v[q], static_cast<int>(min(32u, n - 32 * g)), lane), 0);
+        if (lane == static_cast<int>(g)) mine = r;
+      }
+    }
+  }
+  const uint64_t root = groups > 1 ? warp_tree(mine, static_cast<int>(groups), lane) : mine;
+  return __shfl_sync(kFull, root, 0);
+}
+
 // Tree of a 2-chunk tile, both chunks at once.  Lane l holds a0 = lane value
 // l of chunk 0 and a1 = lane value l of chunk 1.  Level 1 puts chunk q's pair
 // (2i, 2i+1) in lane 16q + i; from then on the pair of every level is in lanes
@@ -741,7 +767,8 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
 // ---------------------------------------------------------------------------
 
 __device__ __forceinline__ uint64_t stream_fp(const SecDesc& s, uint64_t* nodes, int lane) {
-  const uint64_t root = warp_tree_inplace(nodes + s.fin_begin, s.fin_count, lane);
+  const uint64_t root = s.fin_count <= 1024 ? warp_tree_regs(nodes + s.fin_begin, s.fin_count, lane)
+                                             : warp_tree_inplace(nodes + s.fin_begin, s.fin_count, lane);
   return fmix(root ^ (s.bytes * kP));
 }
 
