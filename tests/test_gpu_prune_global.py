@@ -115,6 +115,27 @@ def test_global_threshold_scores_optional_and_no_entries(ctx, dev):
     assert koff.tolist() == [0, 0, 0, 0]
 
 
+def test_global_threshold_unaligned_scores(ctx, dev):
+    # A scores buffer that starts 4 bytes past a 16-byte boundary: the scans
+    # read it one float at a time.
+    b = synth.banks(304, 9, 100, 900, 64, torch.float16, (8,), torch.uint8)
+    keys, qs = _views(b, dev)
+    total = sum(b.n)
+    banks = ctx.banks_array(keys, qs, 200)
+    buf = torch.zeros(total + 4, dtype=torch.float32, device=dev)
+    scores = buf[1:1 + total]
+    kept = torch.empty(total, dtype=torch.int32, device=dev)
+    koff = torch.empty(len(keys) + 1, dtype=torch.int32, device=dev)
+    B = total * 200 * 2 // 5
+    ctx.prune_global(banks, len(keys), B, kept, koff, scores)
+    ctx.sync()
+    s32 = _oracle_scores(keys, qs)
+    assert np.array_equal(scores.cpu().numpy().view(np.uint32), s32.view(np.uint32))
+    want, woff = oracle.prune_global(s32, b.n, 200, B)
+    assert koff.cpu().tolist() == woff.tolist()
+    assert kept.cpu().tolist()[:woff[-1]] == want.tolist()
+
+
 def test_global_threshold_keeps_relevant_sessions(ctx, dev):
     # Against the same-fraction rule: a bank aligned with its query keeps
     # more under the global threshold.
