@@ -847,21 +847,26 @@ __device__ void finalize_sessions_block(const SecDesc* __restrict__ secs,
                                         uint64_t* smem, uint32_t* s_bad) {
   const int lane = threadIdx.x & 31;
   const int wib = threadIdx.x >> 5;
+  const uint32_t nwarps = blockDim.x >> 5;
   for (int b = b0; b < n_sess; b += stride) {
     const SessDesc S = sess[b];
     Entry* table = reinterpret_cast<Entry*>(S.record + kHeaderBytes);
     if (threadIdx.x == 0) *s_bad = 0;
     __syncthreads();
-    for (uint32_t j = wib; j < S.n_sections; j += kWarps) {
+    for (uint32_t j = wib; j < S.n_sections; j += nwarps) {
       const SecDesc s = secs[S.sec_begin + j];
+      uint4 ew = make_uint4(0, 0, 0, 0);  // lanes 0..3: the entry, read before the tree
+      if (MODE == kModePack && lane < 4)
+        ew = reinterpret_cast<const uint4*>(&entries[S.sec_begin + j])[lane];
       const uint64_t fp = stream_fp(s, nodes, lane);
       if (MODE == kModePack) {
-        // Lanes 0..3 write the 64-byte entry as four 16-byte words.
-        if (lane < 4) {
-          Entry e = entries[S.sec_begin + j];
-          e.fp = fp;
-          reinterpret_cast<uint4*>(&table[j])[lane] = reinterpret_cast<const uint4*>(&e)[lane];
+        // Lanes 0..3 write the 64-byte entry as four 16-byte words; the fp
+        // (bytes 32..39) is the first half of lane 2's word.
+        if (lane == 2) {
+          ew.x = static_cast<uint32_t>(fp);
+          ew.y = static_cast<uint32_t>(fp >> 32);
         }
+        if (lane < 4) reinterpret_cast<uint4*>(&table[j])[lane] = ew;
       } else {
         if (lane == 0 && table[j].fp != fp) atomicOr(s_bad, 1u);
       }
@@ -890,15 +895,16 @@ __device__ void finalize_sessions_block(const SecDesc* __restrict__ secs,
     if (MODE == kModePack) {
       // Zero the gap between the end of the table and the first payload.
       const uint64_t from = kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * S.n_sections;
-      for (uint64_t o = from + 16u * threadIdx.x; o < S.payload_start; o += 16u * kThreads)
+      for (uint64_t o = from + 16u * threadIdx.x; o < S.payload_start; o += 16u * blockDim.x)
         *reinterpret_cast<uint4*>(S.record + o) = make_uint4(0, 0, 0, 0);
     }
     __syncthreads();
   }
 }
 
+// Any block size up to 512 threads (a warp per section in turn).
 template <int MODE>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(512)
     k_finalize_sessions(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
                         int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
                         uint8_t* corrupt, uint32_t* bad) {
@@ -2655,12 +2661,17 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
     const int blocks = (n_sess + kWarps - 1) / kWarps;
     k_finalize_hash<<<blocks < 4096 ? blocks : 4096, kThreads, 0, stream>>>(secs, n_sess, nodes, fp_out,
                                                                             fp_before, flags);
-  } else if (mode == kModePack) {
-    k_finalize_sessions<kModePack><<<n_sess < 65535 ? n_sess : 65535, kThreads, 0, stream>>>(
-        secs, sess, n_sess, entries, nodes, flags, bad);
-  } else if (mode == kModeRestoreV) {
-    k_finalize_sessions<kModeRestoreV><<<n_sess < 65535 ? n_sess : 65535, kThreads, 0, stream>>>(
-        secs, sess, n_sess, entries, nodes, flags, bad);
+  } else if (mode == kModePack || mode == kModeRestoreV) {
+    // A block per session, a warp per section (up to 16 at once: two
+    // blocks of 64-register threads fit an SM).
+    const int warps = max_secs < 8 ? 8 : max_secs > 16 ? 16 : max_secs;
+    const int blocks = n_sess < 65535 ? n_sess : 65535;
+    if (mode == kModePack)
+      k_finalize_sessions<kModePack><<<blocks, 32 * warps, 0, stream>>>(secs, sess, n_sess, entries,
+                                                                       nodes, flags, bad);
+    else
+      k_finalize_sessions<kModeRestoreV><<<blocks, 32 * warps, 0, stream>>>(
+          secs, sess, n_sess, entries, nodes, flags, bad);
   } else {
     return cudaErrorInvalidValue;
   }
