@@ -487,6 +487,34 @@ def test_topk_bank_sizes(ctx, dev, ties):
         assert kh[oh[b]:oh[b + 1]].tolist() == oracle.topk(kk, x).tolist(), b
 
 
+def test_topk_digit_boundaries(ctx, dev):
+    # Keys that share their leading bits and differ only in the last digit,
+    # keys straddling digit boundaries, special values (NaN lowest, -0 == +0,
+    # infinities, subnormals) and runs of equal keys at the threshold.
+    rnd = np.random.default_rng(29)
+    banks = []
+    one = np.float32(1.0).view(np.uint32)
+    banks.append((one + rnd.integers(0, 1024, 3000)).astype(np.uint32).view(np.float32))
+    banks.append((one + rnd.integers(0, 1 << 21, 2048)).astype(np.uint32).view(np.float32))
+    spec = np.array([np.nan, 0.0, -0.0, np.inf, -np.inf, 1e-45, -1e-45, 1e-38, -2.5, 2.5],
+                    dtype=np.float32)
+    banks.append(rnd.choice(spec, 1500))
+    eq = rnd.normal(size=4096).astype(np.float32)
+    eq[rnd.integers(0, 4096, 1500)] = np.float32(0.125)
+    banks.append(eq)
+    banks.append(-np.abs(rnd.normal(size=700)).astype(np.float32))
+    k = [1500, 1024, 700, 2000, 350]
+    flat = torch.from_numpy(np.concatenate(banks)).to(dev)
+    n = [len(x) for x in banks]
+    kept = torch.empty(sum(k), dtype=torch.int32, device=dev)
+    koff = torch.empty(len(n) + 1, dtype=torch.int32, device=dev)
+    ctx.topk(flat, n, k, kept, koff)
+    ctx.sync()
+    kh, oh = kept.cpu().numpy(), koff.cpu().numpy()
+    for b, (kk, x) in enumerate(zip(banks, k)):
+        assert kh[oh[b]:oh[b + 1]].tolist() == oracle.topk(kk, x).tolist(), b
+
+
 def test_fork_many_mixed_placements(ctx, dev):
     # Device records over 1 MiB take the TMA copy; pinned-host ones the register copy.
     kv = synth.kv(seed=90, sessions=3, layers=2, heads=16, head_dim=64, window=256, page_rows=16)
