@@ -267,6 +267,20 @@ pcs_status pcs_timing_read(pcs_ctx *ctx, pcs_kernel_time *out, int32_t max, int3
 pcs_status pcs_sync(pcs_ctx *ctx, void *stream);
 
 /*
+ * Self-test of the bounded device waits (no paper counterpart: a check of
+ * the failure path).  Enqueues on `stream` one kernel thread that waits,
+ * with the same helpers and the same bound (about two seconds of SM clock)
+ * as the library's kernels, for something that never happens: which = 0,
+ * the second arrival at a shared-memory mbarrier that expects two (the wait
+ * of the TMA pipeline); which = 1, a device flag that nothing writes (the
+ * poll of the grid barrier).  The wait gives up, sets the timeout bit and
+ * the kernel returns, so the next pcs_sync on the stream reports
+ * PCS_E_TIMEOUT and the context stays usable.  PCS_E_INVAL for another
+ * `which`.
+ */
+pcs_status pcs_selftest_wait(pcs_ctx *ctx, int32_t which, void *stream);
+
+/*
  * Content fingerprint PCSFP64-v1 of n buffers (the measurement that decides
  * must-snapshot, Sec. 4 step 1 at epsilon = 0).  fp_out: device uint64[n].
  * Definition: 4096-byte chunks (bytes past the end read as 0); in chunk c,

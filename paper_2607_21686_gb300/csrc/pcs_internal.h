@@ -159,6 +159,11 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
 
 cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
                         int32_t* kept_idx, cudaStream_t stream);
+// One thread waits for what never happens (which = 0: an mbarrier's second
+// arrival; 1: *never_set >= 1), gives up after the kernels' wait bound and
+// sets the timeout bit in *err.
+cudaError_t launch_selftest_wait(int which, const uint32_t* never_set, uint32_t* err,
+                                 cudaStream_t stream);
 
 
 // ---- One relevance threshold across all banks (pcs_prune_global) ---------

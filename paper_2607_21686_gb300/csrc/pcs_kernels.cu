@@ -1663,6 +1663,17 @@ __device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
   asm volatile("st.release.gpu.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
+// Bounded wait (one thread) until *p >= k, read with acquire semantics;
+// false if about kWaitCycles of SM clock passed first.
+__device__ __forceinline__ bool wait_flag_geq(const uint32_t* p, uint32_t k) {
+  const long long t0 = clock64();
+  while (ld_acquire(p) < k) {
+    if (clock64() - t0 > kWaitCycles) return false;
+    __nanosleep(20);
+  }
+  return true;
+}
+
 // Bounded grid barrier number k (1, 2, ...) of a cooperative launch.  The
 // arrival count only grows (barrier k is full at k x blocks); the last block
 // to arrive runs `last` (every thread of it), then publishes k.  A block that
@@ -1681,16 +1692,8 @@ __device__ bool grid_barrier(GState* st, uint32_t* err, uint32_t k, bool* s_flag
   }
   __syncthreads();  // every thread has read *s_flag
   if (threadIdx.x == 0) {
-    bool ok = true;
-    const long long t0 = clock64();
-    while (ld_acquire(&st->bar_gen) < k) {
-      if (clock64() - t0 > kWaitCycles) {
-        atomicOr(err, kDevErrTimeout);
-        ok = false;
-        break;
-      }
-      __nanosleep(20);
-    }
+    const bool ok = wait_flag_geq(&st->bar_gen, k);
+    if (!ok) atomicOr(err, kDevErrTimeout);
     *s_flag = ok;
   }
   __syncthreads();
@@ -2510,6 +2513,33 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// ---------------------------------------------------------------------------
+// Self-test of the bounded waits: one thread waits, through the helpers the
+// production kernels use and with their bound, for something that never
+// happens -- the second arrival at an mbarrier that expects two (the TMA
+// pipeline's wait) or a flag nothing writes (the grid barrier's poll) --
+// then records the timeout in the context's error word and returns.
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__global__ void k_selftest_wait(int which, const uint32_t* never_set, uint32_t* err) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x != 0) return;
+  bool ok;
+  if (which == 0) {
+    mbar_init(&bar, 2);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    mbar_arrive(&bar);
+    ok = mbar_wait(&bar, 0);
+  } else {
+    ok = wait_flag_geq(never_set, 1);
+  }
+  if (!ok) atomicOr(err, kDevErrTimeout);
+}
+
 template <int MODE>
 int occupancy() {
   int b = 0;
@@ -2827,6 +2857,12 @@ cudaError_t launch_gfinish(const GPlan& p, int first_pass, int sm_count, cudaStr
   return cudaLaunchCooperativeKernel(k, dim3(grid), dim3(kThreads), args, 0, stream);
 }
 
+
+cudaError_t launch_selftest_wait(int which, const uint32_t* never_set, uint32_t* err,
+                                 cudaStream_t stream) {
+  k_selftest_wait<<<1, 32, 0, stream>>>(which, never_set, err);
+  return cudaGetLastError();
+}
 
 // ---------------------------------------------------------------------------
 // Fingerprints with no allocation

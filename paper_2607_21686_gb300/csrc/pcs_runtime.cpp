@@ -1337,6 +1337,18 @@ pcs_status pcs_sync(pcs_ctx* c, void* stream) {
   return PCS_OK;
 }
 
+pcs_status pcs_selftest_wait(pcs_ctx* c, int32_t which, void* stream) {
+  if (!c) return fail(PCS_E_INVAL, "ctx is null");
+  if (which != 0 && which != 1) return fail(PCS_E_INVAL, "which must be 0 or 1, got %d", which);
+  std::lock_guard<std::mutex> lk(c->mu);
+  pcs_status st = set_device(c);
+  if (st) return st;
+  // words[4] is zeroed at creation and never written: nothing will set it.
+  PCS_CUDA(launch_selftest_wait(which, c->words + 4, c->words, static_cast<cudaStream_t>(stream)));
+  ++c->launches;
+  return PCS_OK;
+}
+
 pcs_status pcs_fingerprint(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t* fp_out,
                            void* stream) {
   if (!c) return fail(PCS_E_INVAL, "ctx is null");

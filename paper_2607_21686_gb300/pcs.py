@@ -120,6 +120,7 @@ SIGNATURES = {
     "pcs_destroy": (_st, [_vp]),
     "pcs_get_stats": (_st, [_vp, ctypes.POINTER(pcs_stats)]),
     "pcs_sync": (_st, [_vp, _vp]),
+    "pcs_selftest_wait": (_st, [_vp, _i32, _vp]),
     "pcs_timing_enable": (_st, [_vp, _i32]),
     "pcs_timing_read": (_st, [_vp, ctypes.POINTER(pcs_kernel_time), _i32, ctypes.POINTER(_i32)]),
     "pcs_fingerprint": (_st, [_vp, ctypes.POINTER(pcs_buf), _i32, _vp, _vp]),
@@ -507,6 +508,10 @@ class Context:
 
     def sync(self, stream=None) -> None:
         check(self.lib.pcs_sync(self.h, _stream_ptr(stream)), "pcs_sync")
+
+    def selftest_wait(self, which: int, stream=None) -> None:
+        """Enqueue the bounded-wait self-test; the next sync raises PCS_E_TIMEOUT."""
+        check(self.lib.pcs_selftest_wait(self.h, which, _stream_ptr(stream)), "pcs_selftest_wait")
 
     # -- fingerprint / classify --------------------------------------------
     @staticmethod

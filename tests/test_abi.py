@@ -102,6 +102,10 @@ def test_create_without_gpu_fails_loudly(lib):
     assert b"CUDA" in lib.pcs_last_error() or lib.pcs_last_error()
 
 
+def test_selftest_wait_rejects_a_null_context(lib):
+    assert lib.pcs_selftest_wait(None, 0, None) == pcs.PCS_E_INVAL
+
+
 def _banks(n_list, entry_bytes):
     arr = (pcs.pcs_bank * len(n_list))()
     for i, n in enumerate(n_list):
