@@ -636,7 +636,8 @@ int32_t pcso_restore(const uint8_t *rec, pcso_section *t, int32_t n, int32_t ver
     uint64_t total, sfp, offset, bytes, fp, aux;
     uint64_t *fps;
     int32_t i, bad = 0;
-    if (!pcso_record_header(rec, &ns, &sid, &kind, &total, &sfp) || (int32_t)ns != n) return -1;
+    if (n < 1 || !pcso_record_header(rec, &ns, &sid, &kind, &total, &sfp) || (int32_t)ns != n)
+        return -1; /* a record holds at least one section */
     fps = (uint64_t *)malloc((size_t)n * sizeof(uint64_t));
     if (!fps) return -1;
     for (i = 0; i < n; i++) {
