@@ -106,6 +106,7 @@ struct WorkList {
 
 // Chunks per task of the TMA-staged kernel (an 8 KiB tile).
 constexpr int kBulkTileChunks = 2;
+constexpr uint32_t kFinRegNodes = 1024;  // nodes a finalising warp trees from registers
 // Smallest row size the TMA-staged kernel takes for ROWS / RING streams.
 constexpr uint64_t kBulkMinRowBytes = 512;
 

@@ -767,7 +767,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
 // ---------------------------------------------------------------------------
 
 __device__ __forceinline__ uint64_t stream_fp(const SecDesc& s, uint64_t* nodes, int lane) {
-  const uint64_t root = s.fin_count <= 1024 ? warp_tree_regs(nodes + s.fin_begin, s.fin_count, lane)
+  const uint64_t root = s.fin_count <= kFinRegNodes ? warp_tree_regs(nodes + s.fin_begin, s.fin_count, lane)
                                              : warp_tree_inplace(nodes + s.fin_begin, s.fin_count, lane);
   return fmix(root ^ (s.bytes * kP));
 }
