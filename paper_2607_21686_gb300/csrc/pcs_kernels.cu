@@ -589,20 +589,8 @@ __device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, con
     // One contiguous piece: the record payload, or a contiguous buffer.
     if (lane == 0) {
       const uint32_t bytes = pe > p0 ? static_cast<uint32_t>(pe - p0) : 0u;
-      const uint8_t* src = T::kLoadLayout ? s.lbase + p0 : s.payload + p0;
-      if (MODE == kModePack) {
-        // Pacing, measured: a pack from a contiguous buffer issues its bulk
-        // copy after one L2 round trip -- the tile's offset recomputed from
-        // its work-list entry read through L2 (the same value as p0).  4,096
-        // contiguous 192 KiB sources pack 8 % faster that way (0.296 ->
-        // 0.273 ms); a sleep of the same length does not do it, and the
-        // read-only hash pass gets slower, so only packs pace.
-        uint32_t b;
-        asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(b) : "l"(wl.begin + item) : "memory");
-        src = s.lbase + static_cast<uint64_t>(t - b) * kTileBytes;
-      }
       mbar_arrive_expect_tx(bar, bytes);
-      if (bytes) bulk_g2s(tile, src, bytes, bar);
+      if (bytes) bulk_g2s(tile, T::kLoadLayout ? s.lbase + p0 : s.payload + p0, bytes, bar);
     }
     return;
   }
