@@ -4,6 +4,7 @@
     python -m paper_2607_21686_gb300.cases classify --n 200 --hi-mib 32
     python -m paper_2607_21686_gb300.cases prune --sessions 256
     python -m paper_2607_21686_gb300.cases markov --sessions 4096
+    python -m paper_2607_21686_gb300.cases markov_layouts --sessions 4096
     python -m paper_2607_21686_gb300.cases mismatch --n 200 --hi-mib 32
     python -m paper_2607_21686_gb300.cases prune_global --sessions 256
     python -m paper_2607_21686_gb300.cases cow --sessions 64
@@ -86,6 +87,29 @@ def case_markov(ctx, a, dev):
     return _timed(step, a.warmup)
 
 
+def case_markov_layouts(ctx, a, dev):
+    # The same observation bytes packed twice: as one contiguous section per
+    # session, then as the same tensor addressed through 32 KiB rows
+    # (identity row index).  Records, sizes and addresses are identical; only
+    # the kernel's staging path differs.
+    rows_per = 196608 // 32768
+    pool = torch.randint(0, 256, (a.sessions * rows_per, 32768), device=dev, dtype=torch.uint8)
+    flat = pool.view(a.sessions, 196608)
+    idx = torch.arange(a.sessions * rows_per, dtype=torch.int32, device=dev)
+    contig = ctx.session_array([pcs.Session(s, pcs.PCS_KIND_MARKOV,
+                                            [pcs.contig_section(pcs.PCS_SEC_OBS, flat[s])],
+                                            keep=[pool]) for s in range(a.sessions)])
+    rows = ctx.session_array([pcs.Session(s, pcs.PCS_KIND_MARKOV,
+                                          [pcs.rows_section(pcs.PCS_SEC_OBS, pool,
+                                                            idx[rows_per * s:rows_per * (s + 1)])],
+                                          keep=[pool, idx]) for s in range(a.sessions)])
+
+    def step():
+        for arr in (contig, rows):
+            ctx.delete_raw(ctx.checkpoint_raw(arr, a.sessions), a.sessions)
+    return _timed(step, a.warmup)
+
+
 def case_mismatch(ctx, a, dev):
     sw = synth.sweep(n=a.n, hi=a.hi_mib << 20, device=dev)
     b0, b1 = ctx.buf_array(sw.before), ctx.buf_array(sw.after)
@@ -153,6 +177,7 @@ def case_topk(ctx, a, dev):
 
 
 CASES = {"kv": case_kv, "classify": case_classify, "prune": case_prune, "markov": case_markov,
+         "markov_layouts": case_markov_layouts,
          "mismatch": case_mismatch, "prune_global": case_prune_global, "cow": case_cow,
          "reads": case_reads, "topk": case_topk}
 
