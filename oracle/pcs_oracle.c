@@ -15,11 +15,11 @@
  *     acceptance test D <= epsilon is byte identity, so "must snapshot" is
  *     decided by comparing a buffer's content before and after a recompute
  *     (Sec. 3 "The partition"; Sec. 4 procedure FINGERPRINT, step 1).
- *   - It gives no hash, no pack format and no relevance formula.  The
- *     frozen readings used here (content fingerprint PCSFP64-v1, the PCS1
- *     record layout, fixed-order fp32 cosine, (score, -index) ranking and
- *     the three k-rules) are the ones listed in the design notes; each
- *     function names the reading it implements.
+ *   - It gives no hash, no pack format and no relevance formula.  Where
+ *     it is silent this file fixes one reading (content fingerprint
+ *     PCSFP64-v1, the PCS1 record layout, fixed-order fp32 cosine,
+ *     (score, -index) ranking and the three k-rules), and each function
+ *     states the reading it implements.
  *
  * Parity status of each function against the paper
  *   pcso_fmix              pinned: published SplitMix64 output vectors
