@@ -182,7 +182,7 @@ void pcso_classify(const uint64_t *fp_before, const uint64_t *fp_after, int32_t 
 }
 
 /* ------------------------------------------------------------------------ */
-/* Relevance score (Sec. 5 "relevance-keyed" eviction; Sec. 7.5).  The paper */
+/* Relevance score (Sec. 5, eviction by relevance; Sec. 7.5).  The paper     */
 /* ranks bank frames by relevance to the return viewpoint but gives no      */
 /* formula; the reading is cosine(query, key) in fp32 with a fixed order.    */
 /* ------------------------------------------------------------------------ */
