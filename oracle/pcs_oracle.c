@@ -23,12 +23,22 @@
  *
  * Parity status of each function against the paper
  *   pcso_fmix              pinned: published SplitMix64 output vectors
- *   pcso_fingerprint       parity unpinned against the paper (it prints no
- *                          hash); pinned to the definition's invariants
- *                          (per-word bijection, order and length sensitivity,
- *                          aligned-group decomposition) and to brute force
+ *   pcso_lane_value,       the paper prints no hash, so these are pinned to
+ *   pcso_chunk_hash,       the frozen definition: a second statement of the
+ *   pcso_fingerprint       lane chain vectorised over the 32 lanes (a chunk
+ *                          viewed as u64[8][32][2]) with a top-down buffer
+ *                          tree, equal bit for bit, and planted slips (rotation,
+ *                          word order, seed, segment map) that it catches; and
+ *                          to the definition's invariants (per-word bijection,
+ *                          order and length sensitivity, aligned-group
+ *                          decomposition) and brute force
  *   pcso_classify          pinned: seeded ground truth of which buffers changed
- *   pcso_score_f32/_f64    pinned: numpy cosine, closed forms (parallel,
+ *   pcso_score_f32         pinned: a second statement of the summation order
+ *                          (lanes as a float32[blocks][32][8] view, numpy
+ *                          binary32 steps), equal bit for bit, that catches a
+ *                          lane map of e mod 32, a sequential sum and a folded
+ *                          lane tree; within 1e-3 of the fp64 cosine
+ *   pcso_score_f64         pinned: numpy cosine, closed forms (parallel,
  *                          antiparallel, orthogonal, scaled copies)
  *   pcso_topk              pinned: brute-force ranking on tiny inputs, ties
  *   pcso_k_*               pinned: Table tab:keepfrac frame counts (fraction
