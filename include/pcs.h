@@ -222,9 +222,10 @@ typedef struct pcs_kernel_time {
     double total_ms;           /* sum of CUDA-event durations               */
 } pcs_kernel_time;
 
-/* Message of the calling thread's last error ("" if none). */
+/* Message of the calling thread's last error ("" if none).  No paper
+ * counterpart: error reporting of this C interface. */
 const char *pcs_last_error(void);
-/* Name of a status code. */
+/* Name of a status code (no paper counterpart). */
 const char *pcs_status_string(pcs_status s);
 
 /*
@@ -237,24 +238,30 @@ pcs_status pcs_set_arena_limit(pcs_ctx *ctx, uint32_t placement, uint64_t bytes)
 
 /*
  * Create a context on CUDA device `device`: it owns the snapshot arenas,
- * the workspace of the kernels and the snapshot table.  PCS_E_CUDA if the
- * device cannot be used.
+ * the workspace of the kernels and the snapshot table.  A context is this
+ * library's form of the session runtime's session table and PCS store
+ * (Sec. 5, Figure fig:arch; Sec. 8), with the paged allocation that Sec. 3
+ * "Boundary" leaves to the lower runtime.  PCS_E_CUDA if the device cannot
+ * be used.
  */
 pcs_status pcs_create(int32_t device, pcs_ctx **out);
-/* Destroy a context: waits for its work, frees every snapshot it owns. */
+/* Destroy a context (the end of the store of Sec. 5 / Sec. 8): waits for
+ * its work, frees every snapshot it owns. */
 pcs_status pcs_destroy(pcs_ctx *ctx);
-/* Fill `out` with the context's counters (host only, no synchronisation). */
+/* Fill `out` with the context's counters (host only, no synchronisation).
+ * No paper counterpart: monitoring of this library. */
 pcs_status pcs_get_stats(pcs_ctx *ctx, pcs_stats *out);
 
 /*
- * Per-kernel timing: with on != 0 every kernel launch of the context is
- * bracketed by CUDA events on its own stream; on == 0 stops.  Either call
- * clears the accumulated times.
+ * Per-kernel timing (no paper counterpart: a measurement aid): with on != 0
+ * every kernel launch of the context is bracketed by CUDA events on its own
+ * stream; on == 0 stops.  Either call clears the accumulated times.
  */
 pcs_status pcs_timing_enable(pcs_ctx *ctx, int32_t on);
 /*
  * Wait for the timed launches and write up to `max` per-kernel totals to
- * `out` (host); *n = number of kernels with at least one timed launch.
+ * `out` (host); *n = number of kernels with at least one timed launch.  No
+ * paper counterpart.
  */
 pcs_status pcs_timing_read(pcs_ctx *ctx, pcs_kernel_time *out, int32_t max, int32_t *n);
 
@@ -262,7 +269,9 @@ pcs_status pcs_timing_read(pcs_ctx *ctx, pcs_kernel_time *out, int32_t max, int3
  * Wait for `stream`, then report what kernels recorded since the last
  * pcs_sync -- failed asynchronous verifications (PCS_E_CORRUPT), a bounded
  * wait that gave up (PCS_E_TIMEOUT), an out-of-range index (PCS_E_RANGE) --
- * or a CUDA error (PCS_E_CUDA).  Clears them.
+ * or a CUDA error (PCS_E_CUDA).  Clears them.  No paper counterpart: the
+ * paper's runtime is synchronous Python; this is where the asynchronous
+ * outcome of a verified restore (the I1 check of Sec. 3) reaches the host.
  */
 pcs_status pcs_sync(pcs_ctx *ctx, void *stream);
 
@@ -305,8 +314,10 @@ pcs_status pcs_classify(pcs_ctx *ctx, const pcs_buf *bufs, int32_t n, const uint
                         uint64_t *fp_after, uint8_t *must_snapshot, void *stream);
 
 /*
- * Host only: how many entries each bank keeps under `params`.  k_out: host
- * int32[n].  PCS_E_INVAL on a bad rule or fraction.
+ * Host only: how many entries each bank keeps under `params` (the k-rules:
+ * a fixed cap, the same fraction of every bank under a host budget, Sec. 7.5,
+ * or a retention fraction, Table tab:keepfrac).  k_out: host int32[n].
+ * PCS_E_INVAL on a bad rule or fraction.
  */
 pcs_status pcs_prune_counts(const pcs_bank *banks, int32_t n, const pcs_prune_params *params,
                             int32_t *k_out);
@@ -416,21 +427,26 @@ pcs_status pcs_budget_plan(const int32_t *n, const uint64_t *entry_bytes, const 
  */
 pcs_status pcs_pool_create(pcs_ctx *ctx, void *base, uint64_t page_bytes, int32_t n_pages,
                            pcs_pool **out);
+/* Destroy a pool (of the copy-on-write pool above; the pages' bytes stay the
+ * caller's). */
 pcs_status pcs_pool_destroy(pcs_ctx *ctx, pcs_pool *pool);
 
-/* n free pages, each held once: ids: device int32[n]. */
+/* n free pages, each held once: ids: device int32[n].  Paged allocation of
+ * the lower runtime (Sec. 3 "Boundary"). */
 pcs_status pcs_pool_alloc(pcs_ctx *ctx, pcs_pool *pool, int32_t *ids, int32_t n, void *stream);
 
 /*
- * Fork of the tables holding src: every page of src gains one holder and,
- * if dst is not NULL, src is copied to dst (the child's table).  No page
- * bytes move.  src, dst: device int32[n].
+ * Fork of the tables holding src (fork(c) by copy-on-write, Sec. 3 I3;
+ * Sec. 7.3): every page of src gains one holder and, if dst is not NULL,
+ * src is copied to dst (the child's table).  No page bytes move.  src, dst:
+ * device int32[n].
  */
 pcs_status pcs_pool_share(pcs_ctx *ctx, pcs_pool *pool, const int32_t *src, int32_t *dst,
                           int32_t n, void *stream);
 
 /*
- * The copy leg, before the caller writes the pages at table[entries[j]]
+ * The copy leg of copy-on-write (Sec. 7.3: it fires on the first write),
+ * before the caller writes the pages at table[entries[j]]
  * (j < n; entries NULL: table[0 .. n)): a slot whose page is also held
  * elsewhere gets a fresh page holding a copy of it and gives up its hold on
  * the old one; a page held by that slot alone stays.  Of several holders of
@@ -440,11 +456,13 @@ pcs_status pcs_pool_share(pcs_ctx *ctx, pcs_pool *pool, const int32_t *src, int3
 pcs_status pcs_pool_prepare_write(pcs_ctx *ctx, pcs_pool *pool, int32_t *table, int64_t n_table,
                                   const int32_t *entries, int32_t n, void *stream);
 
-/* Every page of ids loses one holder; pages held by nobody become free. */
+/* Every page of ids loses one holder; pages held by nobody become free
+ * (delete(c) of a shared table, Sec. 3 "The contract"). */
 pcs_status pcs_pool_release(pcs_ctx *ctx, pcs_pool *pool, const int32_t *ids, int32_t n,
                             void *stream);
 
 /*
+ * No paper counterpart (inspection of the pool above).
  * Synchronises `stream`, then reads the pool's state: free page count; the
  * holder count of every page (host uint32[n_pages] or NULL); the free pages
  * (host int32[n_pages] or NULL; the first *free_pages entries are valid).
@@ -499,7 +517,8 @@ pcs_status pcs_discover(int32_t k, pcs_probe_fn probe, void *user, uint64_t eps,
 /*
  * Host only: bytes of the PCS1 record a session of these sections packs to:
  * 256-byte aligned header + 64-byte entries, then each payload at a
- * 256-byte aligned offset.
+ * 256-byte aligned offset.  The record layout is this library's (Sec. 3
+ * "Boundary": storage owns serialisation; the paper fixes no format).
  */
 pcs_status pcs_record_bytes(const pcs_section *sections, int32_t n_sections, uint64_t *out);
 
@@ -515,16 +534,21 @@ pcs_status pcs_checkpoint(pcs_ctx *ctx, const pcs_session *sessions, int32_t n,
                           uint32_t placement, pcs_snapshot **out, void *stream);
 
 /*
- * fork(c): an independent byte copy of a snapshot, same placement (I3).
+ * fork(c) (Sec. 3 "The contract"): an independent byte copy of a snapshot,
+ * same placement, so the child's continuation cannot affect the parent's
+ * (I3).  A full copy because a bank consumed in place cannot share pages
+ * (Sec. 7.3); pcs_pool_share is the copy-on-write form.
  */
 pcs_status pcs_fork(pcs_ctx *ctx, const pcs_snapshot *parent, pcs_snapshot **child,
                     void *stream);
-/* fork(c) for n snapshots in one call; children: host array of n handles. */
+/* fork(c) (Sec. 3 "The contract") for n snapshots in one call; children:
+ * host array of n handles. */
 pcs_status pcs_fork_many(pcs_ctx *ctx, pcs_snapshot *const *parents, int32_t n,
                          pcs_snapshot **children, void *stream);
 
 /*
- * restore(c) for n snapshots (I1): scatter each section payload to the
+ * restore(c) (Sec. 3 "The contract") for n snapshots, byte-identical to the
+ * checkpointed state (I1): scatter each section payload to the
  * target section of targets[i] (same section count and byte counts; any
  * layout).  verify = 1 also recomputes every section fingerprint and the
  * session fp, waits for `stream`, and returns PCS_E_CORRUPT if any differs
@@ -563,21 +587,25 @@ pcs_status pcs_plan_restore(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n,
 pcs_status pcs_plan_run(pcs_ctx *ctx, pcs_plan *plan, void *stream);
 pcs_status pcs_plan_destroy(pcs_ctx *ctx, pcs_plan *plan);
 
-/* delete(c): release a snapshot (its memory is reused once pending work
- * that reads it has finished). */
+/* delete(c) (Sec. 3 "The contract"): release a snapshot (its memory is
+ * reused once pending work that reads it has finished). */
 pcs_status pcs_delete(pcs_ctx *ctx, pcs_snapshot *snap);
 
-/* delete(c) for n snapshots at once; PCS_E_HANDLE (and nothing deleted)
- * if any handle is unknown. */
+/* delete(c) (Sec. 3 "The contract") for n snapshots at once; PCS_E_HANDLE
+ * (and nothing deleted) if any handle is unknown. */
 pcs_status pcs_delete_many(pcs_ctx *ctx, pcs_snapshot *const *snaps, int32_t n);
 
-/* Header fields of a snapshot; waits for the work that wrote it. */
+/* Header fields of a snapshot; waits for the work that wrote it.  No paper
+ * counterpart: inspection of this library's record (Sec. 3 "Boundary":
+ * storage owns serialisation). */
 pcs_status pcs_snapshot_get_info(pcs_ctx *ctx, const pcs_snapshot *snap, pcs_snapshot_info *out);
-/* Section entry i of a snapshot; waits for the work that wrote it. */
+/* Section entry i of a snapshot; waits for the work that wrote it.  No
+ * paper counterpart (inspection, as above). */
 pcs_status pcs_snapshot_get_section(pcs_ctx *ctx, const pcs_snapshot *snap, int32_t i,
                                 pcs_section_info *out);
 /* Copy record bytes [offset, offset + bytes) to dst (device or host),
- * enqueued on stream. */
+ * enqueued on stream.  No paper counterpart: raw access to the serialised
+ * record that storage owns (Sec. 3 "Boundary"). */
 pcs_status pcs_snapshot_copy_out(pcs_ctx *ctx, const pcs_snapshot *snap, uint64_t offset,
                                  uint64_t bytes, void *dst, void *stream);
 
