@@ -73,6 +73,12 @@ def workload_name(a) -> str:
             % (a.sessions, a.layers, a.heads, a.head_dim, a.window, a.page_rows))
 
 
+def bench_config(a, world: int) -> dict:
+    """The `config` of both arms' JSON lines (the same workload and settings)."""
+    return {"workload": workload_name(a), "sessions": a.sessions * world, "layers": a.layers,
+            "verify": not a.no_verify, "l2": "inputs larger than L2 (24 GiB pools)"}
+
+
 def step_bytes(a) -> int:
     """Algorithmic bytes per step: pack R+W and restore R+W of every section."""
     sec = a.window * a.heads * a.head_dim * 2
@@ -274,8 +280,7 @@ def run_reference(a, rank, world):
             "warmup": a.warmup, "ms_per_step": round(a.sessions / sps * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
             "data": "synthetic", "impl": "reference",
-            "config": {"workload": workload_name(a), "sessions": a.sessions,
-                       "l2": "inputs larger than L2"},
+            "config": bench_config(a, world),
             "sessions_per_s": sps,
             "cpu_baseline": dict(rates[-1], value=v),
             "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -947,10 +952,7 @@ def main():
                 "steps": a.steps, "warmup": a.warmup, "ms_per_step": round(ms_step, 4),
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
                 "data": "synthetic",
-                "config": {"workload": workload_name(a), "sessions": a.sessions * world,
-                           "layers": a.layers, "verify": not a.no_verify,
-                           "l2": "inputs larger than L2 (24 GiB pools)",
-                           "host_cpus": r["host_cpus"]},
+                "config": bench_config(a, world), "host_cpus": r["host_cpus"],
                 "sessions_per_s": round(sps, 2),
                 "frac_of_nominal_8tbs": round(gbs / 8000.0, 4),
                 "roofline": roof, "cpu_baseline": cpu, "e2e": r["e2e"],

@@ -1,15 +1,15 @@
 """Run one workload of the PCS hot path once (for profiling a single kernel).
 
-    python -m paper_2607_21686_gb300.cases kv --sessions 8
-    python -m paper_2607_21686_gb300.cases classify --n 200 --hi-mib 32
-    python -m paper_2607_21686_gb300.cases prune --sessions 256
-    python -m paper_2607_21686_gb300.cases markov --sessions 4096
-    python -m paper_2607_21686_gb300.cases markov_layouts --sessions 4096
-    python -m paper_2607_21686_gb300.cases mismatch --n 200 --hi-mib 32
-    python -m paper_2607_21686_gb300.cases prune_global --sessions 256
-    python -m paper_2607_21686_gb300.cases cow --sessions 64
-    python -m paper_2607_21686_gb300.cases reads --n 200 --hi-mib 32
-    python -m paper_2607_21686_gb300.cases topk --sessions 2048
+    python profile_cases.py kv --sessions 8
+    python profile_cases.py classify --n 200 --hi-mib 32
+    python profile_cases.py prune --sessions 256
+    python profile_cases.py markov --sessions 4096
+    python profile_cases.py markov_layouts --sessions 4096
+    python profile_cases.py mismatch --n 200 --hi-mib 32
+    python profile_cases.py prune_global --sessions 256
+    python profile_cases.py cow --sessions 64
+    python profile_cases.py reads --n 200 --hi-mib 32
+    python profile_cases.py topk --sessions 2048
 
 Each case builds its seeded synthetic population on cuda:0, runs the step
 `--warmup` times, then once more, and prints the device time of that last
@@ -23,7 +23,7 @@ import json
 
 import torch
 
-from . import build, pcs, synth
+from paper_2607_21686_gb300 import build, pcs, synth
 
 
 def _timed(fn, warmup):
