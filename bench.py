@@ -380,11 +380,13 @@ def run_pcs(a, rank, world, local_rank):
     # End to end through the public API with the state coming from host memory.
     e2e = None
     if not a.no_e2e:
-        e2e = run_e2e(a, ctx, kv, src, dst, stream, dev)
+        e2e = run_e2e(a, ctx, kv, dst, stream, dev)
 
     rows = None
     if not a.no_rows and rank == 0:
-        rows = {"fork": measure_fork(ctx, src, stream)}
+        rows = {"fork": measure_fork(ctx, src, stream),
+                "kv_suspend_resume": measure_suspend_resume(a, ctx, src, dst, stream, dev,
+                                                            steps=5)}
         del src, dst, kv, k2, v2, meta2
         torch.cuda.empty_cache()
         rows.update(run_rows(ctx, dev, stream))
@@ -433,6 +435,30 @@ def _events_ms(fn, stream, reps=5, warm=2):
     return ts[0], ts[len(ts) // 2]
 
 
+def measure_link(dev, stream) -> dict:
+    """The host link with pinned cudaMemcpyAsync of 1 GiB (best of 5): each
+    direction alone, and both at once on two streams (per direction)."""
+    x = torch.empty(1 << 30, dtype=torch.uint8, pin_memory=True)
+    x2 = torch.empty(1 << 30, dtype=torch.uint8, pin_memory=True)
+    y = torch.empty(1 << 30, dtype=torch.uint8, device=dev)
+    y2 = torch.empty(1 << 30, dtype=torch.uint8, device=dev)
+    h2d = (1 << 30) / (_events_ms(lambda: y.copy_(x, non_blocking=True), stream)[0] / 1e3) / 1e9
+    d2h = (1 << 30) / (_events_ms(lambda: x.copy_(y, non_blocking=True), stream)[0] / 1e3) / 1e9
+    other = torch.cuda.Stream(device=dev)
+
+    def both():
+        other.wait_stream(stream)
+        y.copy_(x, non_blocking=True)
+        with torch.cuda.stream(other):
+            x2.copy_(y2, non_blocking=True)
+        stream.wait_stream(other)
+    duplex = (1 << 30) / (_events_ms(both, stream)[0] / 1e3) / 1e9
+    del x, x2, y, y2
+    return {"h2d_GBs": round(h2d, 1), "d2h_GBs": round(d2h, 1),
+            "duplex_GBs_each_way": round(duplex, 1),
+            "how": "pinned cudaMemcpyAsync 1 GiB, best of 5; duplex: one copy each way at once"}
+
+
 def measure_fork(ctx, src, stream):
     """a9: fork every snapshot of the KV step in one call (independent copies)."""
     arr = ctx.session_array(src)
@@ -461,15 +487,8 @@ def run_rows(ctx, dev, stream):
 
     peak = load_peaks()["hbm_gbs"]
     out = {}
-    # Host link (pinned cudaMemcpyAsync, 1 GiB, best of 5): the roofline of
-    # host placement.
-    x = torch.empty(1 << 30, dtype=torch.uint8, pin_memory=True)
-    y = torch.empty(1 << 30, dtype=torch.uint8, device=dev)
-    h2d = (1 << 30) / (_events_ms(lambda: y.copy_(x, non_blocking=True), stream)[0] / 1e3) / 1e9
-    d2h = (1 << 30) / (_events_ms(lambda: x.copy_(y, non_blocking=True), stream)[0] / 1e3) / 1e9
-    del x, y
-    out["host_link"] = {"h2d_GBs": round(h2d, 1), "d2h_GBs": round(d2h, 1),
-                        "how": "pinned cudaMemcpyAsync 1 GiB, best of 5"}
+    out["host_link"] = measure_link(dev, stream)
+    h2d, d2h = out["host_link"]["h2d_GBs"], out["host_link"]["d2h_GBs"]
 
     # a1-a3: classification sweep, 200 buffers of 64 B .. 256 MiB.
     sw = synth.sweep(device=dev)
@@ -517,6 +536,8 @@ def run_rows(ctx, dev, stream):
                              "GBs_of_log": round(16 * m / (med / 1e3) / 1e9, 1),
                              "flags_match_ground_truth": read_ok}
     del sw, fp0, must, fp1, counts, after_arr, before_arr, addr, nbytes, which, bases, lens, off
+
+    out["banks_config2"] = measure_banks_config2(ctx, dev, stream, peak)
 
     # a4-a5, a7, a10: 2048 banks, relevance top-k under an 8 GiB host budget,
     # pack to pinned host, verified restore to HBM.
@@ -668,6 +689,78 @@ def run_rows(ctx, dev, stream):
     return out
 
 
+def measure_banks_config2(ctx, dev, stream, peak):
+    """a4-a5, a7-a10 on 64 memory banks: prune to k = min(n, 128) by relevance,
+    checkpoint the kept entries to HBM, verified restore into compacted banks,
+    delete -- one step, enqueued without a host wait (the kept counts are
+    known on the host, so the sessions are described before the prune has
+    written the indices they gather by)."""
+    from paper_2607_21686_gb300 import pcs, synth
+
+    b = synth.banks_config2(device=dev)
+    S = b.sessions
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    vals = [b.values[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    banks = ctx.banks_array(keys, [b.queries[s] for s in range(S)], 512 + b.value_bytes)
+    params = ctx.params(pcs.PCS_K_FIXED, k_max=128)
+    ks = ctx.prune_counts(banks, S, params)
+    koff = [0]
+    for k in ks:
+        koff.append(koff[-1] + k)
+    kept = torch.empty(koff[-1], dtype=torch.int32, device=dev)
+    sess = [pcs.bank_session(s, keys[s], vals[s], kept[koff[s]:koff[s + 1]]) for s in range(S)]
+    outs = [(torch.empty(ks[s], dtype=torch.int32, device=dev),
+             torch.empty(ks[s], 256, dtype=torch.float16, device=dev),
+             torch.empty((ks[s],) + tuple(b.values.shape[1:]), dtype=b.values.dtype, device=dev))
+            for s in range(S)]
+    sarr = ctx.session_array(sess)
+    tarr = ctx.session_array([pcs.bank_targets(s, *outs[s]) for s in range(S)])
+
+    def step():
+        ctx.prune(banks, S, params, kept)
+        hs = ctx.checkpoint_raw(sarr, S)
+        ctx.restore_raw(hs, S, tarr, verify=2)
+        ctx.delete_raw(hs, S)
+    med = _loop_ms(step, stream, calls=20, warm=3)
+    ctx.sync()
+    # The restored banks hold exactly the kept rows, in ascending index.
+    kept_h = kept.cpu()
+    ok = True
+    for s in (0, S // 2, S - 1):
+        ki = kept_h[koff[s]:koff[s + 1]]
+        ok &= bool(torch.equal(outs[s][0].cpu(), ki)) and bool(torch.all(ki[1:] > ki[:-1]))
+        ok &= bool(torch.equal(outs[s][2], vals[s][ki.long().to(dev)]))
+    # Planned once, then launches only (prune, checkpoint, restore).
+    cplan, phs = ctx.plan_checkpoint(sarr, S)
+    rplan = ctx.plan_restore(phs, S, tarr, verify=2)
+
+    def prepared_step():
+        ctx.prune(banks, S, params, kept)
+        ctx.plan_run(cplan)
+        ctx.plan_run(rplan)
+    medp = _loop_ms(prepared_step, stream, calls=20, warm=3)
+    ctx.sync()
+    ctx.plan_destroy(rplan)
+    ctx.plan_destroy(cplan)
+    ctx.delete_raw(phs, S)
+    kb = sum(b.n) * 512
+    payload = koff[-1] * (4 + 512 + b.value_bytes)
+    moved = kb + 4 * payload
+    return {"population": "64 banks, n ~ U[1,512], key fp16[256], latent bf16[16,32,32], "
+                          "k = min(n,128)",
+            "entries": sum(b.n), "kept": koff[-1], "key_bytes_read": kb,
+            "bytes_per_step": moved, "how": "prune + checkpoint to HBM + verified restore + "
+            "delete, 20 back-to-back steps between one pair of events",
+            "ms": round(med, 4), "GBs": round(moved / (med / 1e3) / 1e9, 1),
+            "sessions_per_s": round(S / (med / 1e3), 1),
+            "frac_of_hbm": round(moved / (med / 1e3) / 1e9 / peak, 4),
+            "prepared_ms": round(medp, 4),
+            "prepared_GBs": round(moved / (medp / 1e3) / 1e9, 1),
+            "prepared_sessions_per_s": round(S / (medp / 1e3), 1),
+            "prepared_frac_of_hbm": round(moved / (medp / 1e3) / 1e9 / peak, 4),
+            "restored_rows_match": ok}
+
+
 def measure_cow_fork(ctx, dev, stream, peak):
     """Copy-on-write fork of the 256 KV sessions: share every K and V page
     (no bytes move), then the copy leg of each child's first token append
@@ -768,31 +861,55 @@ class HostBuffer:
             self.mm = None
 
 
-def run_e2e(a, ctx, kv, src, dst, stream, dev):
-    """Each step: H2D of the KV pools from pinned memory, checkpoint, verified
-    restore, D2H of the session fingerprints.  The pools are double-buffered:
-    step i+1's copy (on a copy stream) runs while step i computes, so a step
-    costs max(copy, compute) -- the host link, here."""
+def run_e2e(a, ctx, kv, dst, stream, dev):
+    """End to end through the library with the state in host memory: each
+    step checkpoints every session from K and V page pools that live in
+    pinned host memory (the caller hands the library host pointers; its
+    kernels read the pages over the host link, pack the records into HBM and
+    fingerprint them), restores the records verified into the freshly
+    permuted pool in HBM, reads the session fingerprints back to the host and
+    deletes the snapshots.  Host -> device: every payload byte, once per
+    step; device -> host: one 8-byte session fingerprint per session."""
     from paper_2607_21686_gb300 import pcs
 
+    S = a.sessions
     nb = kv.k_pool.numel() * kv.k_pool.element_size()
     probes = {}
 
-    def probe(name, a, b):
-        # One full copy of both pools: huge pages or not shows at this size.
-        a.copy_(kv.k_pool)
-        b.copy_(kv.v_pool)
+    def sessions_on(kh, vh):
+        return ctx.session_array([pcs.kv_session(s, kv.meta[s], kh, vh, kv.page_table[s],
+                                                 kv.ring_start[s], a.window) for s in range(S)])
+
+    dst_arr = ctx.session_array(dst)
+    verify = 0 if a.no_verify else 2
+
+    def step(arr):
+        hs = ctx.checkpoint_raw(arr, S)
+        ctx.restore_raw(hs, S, dst_arr, verify=verify)
+        for k in range(S):
+            ctx.copy_out(pcs.Snapshot(ctx, hs[k]), 24, 8, fps_d[k:k + 1])
+        fps_h.copy_(fps_d, non_blocking=True)
+        ctx.delete_raw(hs, S)
+
+    def probe(name, kh, vh):
+        # One whole step from these host pools: how the pages were pinned
+        # shows at this size.
+        kh.copy_(kv.k_pool)
+        vh.copy_(kv.v_pool)
+        arr = sessions_on(kh, vh)
+        step(arr)
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        kv.k_pool.copy_(a, non_blocking=True)
-        kv.v_pool.copy_(b, non_blocking=True)
+        step(arr)
         e1.record(stream)
         torch.cuda.synchronize()
         probes[name] = round(2 * nb / (e0.elapsed_time(e1) / 1e3) / 1e9, 1)
-        return probes[name]
+        return probes[name], arr
 
-    host, kh, vh, pinning = [], None, None, None
+    fps_h = torch.empty(S, dtype=torch.int64, pin_memory=True)
+    fps_d = torch.empty(S, dtype=torch.int64, device=dev)
+    host, kh, vh, arr, pinning, rate = [], None, None, None, None, 0.0
     huge0 = _anon_huge_bytes()
     try:
         host = [HostBuffer(nb), HostBuffer(nb)]
@@ -800,99 +917,127 @@ def run_e2e(a, ctx, kv, src, dst, stream, dev):
         vh = host[1].view(kv.v_pool.shape, kv.v_pool.dtype)
         pinning = "huge-page mapping, cudaHostRegister"
         probes["huge_pages_GiB"] = round((_anon_huge_bytes() - huge0) / 2**30, 1)
-        rate = probe("mapping_GBs", kh, vh)
+        rate, arr = probe("mapping_GBs_of_pools", kh, vh)
     except Exception:
         for h in host:
             h.close()
-        host, rate = [], 0.0
+        host, kh, vh, rate = [], None, None, 0.0
     if rate < 150.0:
-        # Without huge pages the mapping's DMA can crawl; the driver's own
-        # pinned allocation may do better on this host.  Keep the faster.
+        # Without huge pages the host's address translation can slow the link
+        # down; the driver's own pinned allocation may do better.  Keep the faster.
         try:
             kt = torch.empty(kv.k_pool.shape, dtype=kv.k_pool.dtype, pin_memory=True)
             vt = torch.empty(kv.v_pool.shape, dtype=kv.v_pool.dtype, pin_memory=True)
-            if probe("cudaHostAlloc_GBs", kt, vt) > rate:
+            r2, arr2 = probe("cudaHostAlloc_GBs_of_pools", kt, vt)
+            if r2 > rate:
                 for h in host:
                     h.close()
-                host, kh, vh, pinning = [], kt, vt, "cudaHostAlloc"
+                host, kh, vh, arr, pinning, rate = [], kt, vt, arr2, "cudaHostAlloc", r2
             else:
-                del kt, vt
+                del kt, vt, arr2
         except Exception as ex:  # pinned memory could not be had
             if kh is None:
                 return {"value": None, "unit": "GB/s", "note": "pinned allocation failed: %s" % ex}
-    kh.copy_(kv.k_pool)
-    vh.copy_(kv.v_pool)
-    fps_h = torch.empty(a.sessions, dtype=torch.int64, pin_memory=True)
-    fps_d = torch.empty(a.sessions, dtype=torch.int64, device=dev)
-    steps = max(2, min(a.steps, 5))
-    S = a.sessions
-    kb, vb = torch.empty_like(kv.k_pool), torch.empty_like(kv.v_pool)
-    src_b = [pcs.kv_session(s, kv.meta[s], kb, vb, kv.page_table[s], kv.ring_start[s], a.window)
-             for s in range(S)]
-    arrs = [ctx.session_array(src), ctx.session_array(src_b)]
-    pools = [(kv.k_pool, kv.v_pool), (kb, vb)]
-    dst_arr = ctx.session_array(dst)
-    copy_s = torch.cuda.Stream(device=dev)
-    ready = [torch.cuda.Event(), torch.cuda.Event()]
-    free = [torch.cuda.Event(), torch.cuda.Event()]
-    copy_marks = []  # (start, end) events of each step's copy, timed runs only
-
-    def h2d(i, mark=False):
-        b = i % 2
-        copy_s.wait_event(free[b])
-        if mark:
-            m0 = torch.cuda.Event(enable_timing=True)
-            m0.record(copy_s)
-        with torch.cuda.stream(copy_s):
-            pools[b][0].copy_(kh, non_blocking=True)
-            pools[b][1].copy_(vh, non_blocking=True)
-        ready[b].record(copy_s)
-        if mark:
-            m1 = torch.cuda.Event(enable_timing=True)
-            m1.record(copy_s)
-            copy_marks.append((m0, m1))
-
-    def compute(i):
-        b = i % 2
-        stream.wait_event(ready[b])
-        hs = ctx.checkpoint_raw(arrs[b], S)
-        ctx.restore_raw(hs, S, dst_arr, verify=0 if a.no_verify else 2)
-        for k in range(S):
-            ctx.copy_out(pcs.Snapshot(ctx, hs[k]), 24, 8, fps_d[k:k + 1])
-        fps_h.copy_(fps_d, non_blocking=True)
-        ctx.delete_raw(hs, S)
-        free[b].record(stream)
-
-    def run(n, mark=False):
-        for e in free:
-            e.record(stream)
-        h2d(0, mark)
-        for i in range(n):
-            if i + 1 < n:
-                h2d(i + 1, mark)
-            compute(i)
-
-    run(2)
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    run(steps, mark=True)
-    e1.record(stream)
+    for _ in range(max(1, a.warmup)):
+        step(arr)
     torch.cuda.synchronize()
     ctx.sync()
-    ms = e0.elapsed_time(e1) / steps
-    h2d_b = kh.numel() * kh.element_size() * 2
-    copy_ms = sum(m0.elapsed_time(m1) for m0, m1 in copy_marks) / max(len(copy_marks), 1)
-    d2h_b = fps_h.numel() * 8
-    del kh, vh, kb, vb
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(a.steps):
+        step(arr)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ctx.sync()  # raises if a verified restore found a mismatch
+    ms = e0.elapsed_time(e1) / a.steps
+    del arr, kh, vh
     for h in host:
         h.close()
     return {"value": round(step_bytes(a) / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
-            "h2d_bytes_per_step": h2d_b, "d2h_bytes_per_step": d2h_b, "ms_per_step": round(ms, 3),
-            "sessions_per_s": round(a.sessions / (ms / 1e3), 2), "steps": steps,
-            "overlap": "double-buffered pools: copy of step i+1 under compute of step i",
-            "pinned": pinning, "pinned_probes": probes,
-            "h2d_GBs_in_run": round(h2d_b / (copy_ms / 1e3) / 1e9, 1)}
+            "h2d_bytes_per_step": 2 * nb, "d2h_bytes_per_step": fps_h.numel() * 8,
+            "ms_per_step": round(ms, 3), "sessions_per_s": round(S / (ms / 1e3), 2),
+            "steps": a.steps,
+            "how": "pcs_checkpoint of the sessions from K/V page pools in pinned host memory "
+                   "(the library reads them over the host link), verified pcs_restore into "
+                   "HBM, session fingerprints copied to the host, delete",
+            "h2d_GBs_in_run": round(2 * nb / (ms / 1e3) / 1e9, 1),
+            "pinned": pinning, "pinned_probes": probes}
+
+
+def measure_suspend_resume(a, ctx, src, dst, stream, dev, groups: int = 8,
+                           steps: int | None = None):
+    """The KV population crossing the host link both ways every step: suspend
+    every session to pinned host memory (checkpoint with
+    PCS_PLACE_PINNED_HOST: the library's kernels pack HBM into host records,
+    fingerprints fused) and resume it from there (verified restore from the
+    host records into the freshly permuted pool in HBM).  The sessions go in
+    `groups` groups, each a prepared checkpoint on one stream and a prepared
+    restore on another: group g resumes while group g + 1 is suspended, so
+    the link carries both directions at once (a call that only crosses the
+    link takes half the SMs, so the two kernels can run side by side).
+    The library orders every record's rewrite after its last read.  Bytes
+    over the link per step: every record written to the host, and read back."""
+    from paper_2607_21686_gb300 import pcs
+
+    S = a.sessions
+    G = max(1, min(groups, S))
+    steps = a.steps if steps is None else steps
+    bounds = [S * g // G for g in range(G + 1)]
+    verify = 0 if a.no_verify else 2
+    cplans, rplans, handles, rec_bytes = [], [], [], 0
+    for g in range(G):
+        lo, hi = bounds[g], bounds[g + 1]
+        cp, hs = ctx.plan_checkpoint(ctx.session_array(src[lo:hi]), hi - lo,
+                                     pcs.PCS_PLACE_PINNED_HOST, stream=stream)
+        rplans.append(ctx.plan_restore(hs, hi - lo, ctx.session_array(dst[lo:hi]), verify=verify))
+        cplans.append(cp)
+        handles.append((hs, hi - lo))
+        rec_bytes += sum(ctx.info(pcs.Snapshot(ctx, hs[i])).total_bytes for i in range(hi - lo))
+    s_out = torch.cuda.Stream(device=dev)
+    s_in = torch.cuda.Stream(device=dev)
+    suspended = [torch.cuda.Event() for _ in range(G)]
+
+    def run(n):
+        s_out.wait_stream(stream)
+        s_in.wait_stream(stream)
+        for _ in range(n):
+            for g in range(G):
+                ctx.plan_run(cplans[g], stream=s_out)
+                suspended[g].record(s_out)
+                s_in.wait_event(suspended[g])
+                ctx.plan_run(rplans[g], stream=s_in)
+        stream.wait_stream(s_out)
+        stream.wait_stream(s_in)
+
+    probe = measure_link(dev, stream)
+    run(max(1, a.warmup))
+    torch.cuda.synchronize()
+    ctx.sync()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    run(steps)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ctx.sync()  # raises if a verified resume found a mismatch
+    ms = e0.elapsed_time(e1) / steps
+    # The step's result as the host sees it: every session fingerprint, read
+    # from the records in host memory.
+    fps = [ctx.info(pcs.Snapshot(ctx, hs[i])).session_fp for hs, n in handles for i in range(n)]
+    for p in rplans + cplans:
+        ctx.plan_destroy(p)
+    for hs, n in handles:
+        ctx.delete_raw(hs, n)
+    link = rec_bytes / (ms / 1e3) / 1e9
+    return {"value": round(step_bytes(a) / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": rec_bytes, "d2h_bytes_per_step": rec_bytes,
+            "ms_per_step": round(ms, 3), "sessions_per_s": round(S / (ms / 1e3), 2),
+            "steps": steps, "groups": G,
+            "how": "suspend to pinned host (pcs_checkpoint, PCS_PLACE_PINNED_HOST) + verified "
+                   "resume into HBM (pcs_restore from the host records), prepared calls, "
+                   "%d groups on two streams" % G,
+            "link_GBs_each_way": round(link, 1), "host_link": probe,
+            "frac_of_duplex_link": round(link / probe["duplex_GBs_each_way"], 4),
+            "session_fps_read": len(fps)}
 
 
 def main():

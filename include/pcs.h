@@ -639,7 +639,10 @@ pcs_status pcs_snapshot_read_file(pcs_ctx *ctx, const char *path, uint32_t place
  * A call beyond a limit returns PCS_E_INVAL before anything is enqueued.
  * The first call on a device looks up the array's device address with that
  * device current (this may load the library's GPU code on that device); make
- * that first call before any stream capture.  All calls share the array: two
+ * that first call before any stream capture.  The address is kept for the
+ * rest of the process: after cudaDeviceReset on a device, the module is
+ * loaded anew and the kept address is stale, so a process that resets a
+ * device must not call this entry point on it again.  All calls share the array: two
  * calls whose work overlaps on the GPU (unordered streams) corrupt each
  * other's results, so order them.  No part of the array needs to start at
  * zero; each call writes every node it later reads.  On success the call

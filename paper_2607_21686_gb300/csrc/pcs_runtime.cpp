@@ -348,8 +348,11 @@ struct pcs_ctx {
   // Small device words: [0] kernel error bits, [1] verification failures.
   uint32_t* words = nullptr;
   std::vector<uint8_t> plan;   // host staging of the descriptors
-  // Pinned ring for small plans: a true async copy, no driver-side staging.
-  uint8_t* plan_ring = nullptr;
+  // Pinned slots for the plans of calls: a true async copy, no driver-side
+  // staging of pageable memory (which can hold the host until the stream
+  // has caught up).  Each slot grows to the largest plan it has carried.
+  uint8_t* plan_slot_buf[8] = {};
+  uint64_t plan_slot_cap[8] = {};
   Ev plan_slot_busy[8];
   int plan_slot = 0;
   int plan_slot_used = -1;     // slot of the call in progress, or -1
@@ -474,24 +477,36 @@ pcs_status ws_acquire(pcs_ctx* c, uint64_t bytes, cudaStream_t stream, uint8_t**
   return PCS_OK;
 }
 
-constexpr uint64_t kPlanSlotBytes = 256 << 10;  // per-call plans up to here copy asynchronously
+constexpr uint64_t kPlanSlotBytes = 256 << 10;  // smallest pinned plan slot
+constexpr uint64_t kPlanSlotMax = 64ull << 20;  // larger plans are copied from pageable memory
 constexpr int kPlanSlots = 8;
 
-// Copy the call's descriptors (c->plan, `bytes`) into the workspace.  Small
-// plans go through a slot of a pinned ring, reusable once the call that last
-// used it has passed its end event; larger ones are copied from pageable memory.
+// Copy the call's descriptors (c->plan, `bytes`) into the workspace.  Plans
+// go through a pinned slot (round robin over kPlanSlots), reusable once the
+// call that last used it has passed its end event; a slot too small for the
+// plan is replaced by a larger one.  When the slot is still busy, or the plan
+// is huge, it is copied from pageable memory.
 cudaError_t plan_copy(pcs_ctx* c, uint8_t* ws, uint64_t bytes, cudaStream_t stream) {
-  if (bytes <= kPlanSlotBytes) {
-    if (!c->plan_ring &&
-        cudaHostAlloc(&c->plan_ring, kPlanSlotBytes * kPlanSlots, cudaHostAllocDefault) != cudaSuccess) {
-      cudaGetLastError();
-      c->plan_ring = nullptr;
-    }
-    if (c->plan_ring) {
-      const int i = c->plan_slot;
-      Ev& busy = c->plan_slot_busy[i];
-      if (!busy || busy->done()) {
-        uint8_t* slot = c->plan_ring + kPlanSlotBytes * i;
+  if (bytes <= kPlanSlotMax) {
+    const int i = c->plan_slot;
+    Ev& busy = c->plan_slot_busy[i];
+    if (!busy || busy->done()) {
+      if (c->plan_slot_cap[i] < bytes) {
+        if (c->plan_slot_buf[i]) cudaFreeHost(c->plan_slot_buf[i]);
+        c->plan_slot_buf[i] = nullptr;
+        c->plan_slot_cap[i] = 0;
+        uint64_t cap = kPlanSlotBytes;
+        while (cap < bytes) cap *= 2;
+        void* p = nullptr;
+        if (cudaHostAlloc(&p, cap, cudaHostAllocDefault) == cudaSuccess) {
+          c->plan_slot_buf[i] = static_cast<uint8_t*>(p);
+          c->plan_slot_cap[i] = cap;
+        } else {
+          cudaGetLastError();
+        }
+      }
+      if (c->plan_slot_buf[i]) {
+        uint8_t* slot = c->plan_slot_buf[i];
         std::memcpy(slot, c->plan.data(), bytes);
         c->plan_slot = (i + 1) % kPlanSlots;
         // Held until ws_release records the call's end; a call that fails
@@ -673,6 +688,7 @@ struct StreamPlan {
   std::vector<NodeLevel> levels;
   std::vector<uint32_t> level_groups, level_base;
   int glog2 = 0;
+  bool link_bound = false;     // every stream crosses the host link (see link_bound_call)
 };
 
 // The TMA-staged kernel takes a stream whose bytes on both sides live in
@@ -684,6 +700,35 @@ bool bulk_eligible(const pcs_ctx* c, const SecDesc& d, bool payload_device, bool
   if (!is_device_ptr(d.lbase, cache)) return false;
   if (d.layout == kContig) return d.align == 16 || d.bytes == 0;
   return d.row_bytes >= kBulkMinRowBytes && d.row_bytes % 16 == 0;
+}
+
+// A call whose every non-empty stream has one side in host memory (a record
+// in pinned host memory, or a section that lives there) moves its bytes over
+// the host link, a few hundred GB/s that half the SMs keep busy (measured:
+// 256 KV sessions suspend at 193 GB/s and resume at 210 GB/s on half the SMs,
+// as on all of them; on a quarter the resume lost 6 %, on an eighth 43 %): its
+// register kernel gets a grid of 1 / kLinkSmDiv of the GPU, so a suspend and
+// a resume on two streams, or a suspend beside other work, can run side by
+// side instead of one after the other.
+#ifndef PCS_LINK_SM_DIV
+#define PCS_LINK_SM_DIV 2
+#endif
+constexpr int kLinkSmDiv = PCS_LINK_SM_DIV;
+
+bool link_bound_call(const std::vector<SecDesc>& d, const std::vector<char>& bulk,
+                     const std::vector<char>& payload_device, PtrCache& cache) {
+  bool any = false;
+  for (size_t i = 0; i < d.size(); ++i) {
+    if (d[i].bytes == 0) continue;
+    if (bulk[i]) return false;
+    if (payload_device[i] && is_device_ptr(d[i].lbase, cache)) return false;
+    any = true;
+  }
+  return any;
+}
+
+int grid_sms(const pcs_ctx* c, const StreamPlan& P) {
+  return P.link_bound ? std::max(1, c->sm_count / kLinkSmDiv) : c->sm_count;
 }
 
 // Calls moving at most this many bytes take the register kernel: their time
@@ -836,6 +881,7 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   const bool fused = fused_ok(bulk, small, n);
   StreamPlan P;
   if (!plan_streams(c, d, bulk, P, !fused)) return fail(PCS_E_INVAL, "too much data in one call");
+  P.link_bound = link_bound_call(d, bulk, std::vector<char>(n, 1), cache);
   WsLayout L;
   L.secs = 0;
   const ListLayout LL = list_layout(P, sizeof(SecDesc) * n);
@@ -886,7 +932,7 @@ cudaError_t launch_streams(pcs_ctx* c, int mode, const SecDesc* dsecs, const Str
                 reinterpret_cast<const uint32_t*>(ws + L.reg_begin),
                 static_cast<int>(P.reg_ids.size()), P.reg_tasks};
     LaunchScope ls(c, stream_kind(mode), stream);
-    e = launch_stream(mode, dsecs, wl, P.glog2, nodes, c->words, c->sm_count, c->stream_bps,
+    e = launch_stream(mode, dsecs, wl, P.glog2, nodes, c->words, grid_sms(c, P), c->stream_bps,
                       stream);
     if (e != cudaSuccess) return e;
   }
@@ -1077,6 +1123,8 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
     arena_of(c, placement)->free(blk);
     return fail(PCS_E_INVAL, "too much data in one call");
   }
+  pr->P.link_bound =
+      link_bound_call(d, bulk, std::vector<char>(d.size(), placement == PCS_PLACE_DEVICE), cache);
   WsLayout& L = pr->L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
@@ -1144,6 +1192,7 @@ pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
   pr->fused = verify && fused_ok(bulk, small, n) && max_secs <= 2048;
   if (!plan_streams(c, d, bulk, pr->P, !pr->fused))
     return fail(PCS_E_INVAL, "too much data in one call");
+  pr->P.link_bound = link_bound_call(d, bulk, payload_dev, cache);
   WsLayout& L = pr->L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
@@ -1232,7 +1281,8 @@ pcs_status pcs_destroy(pcs_ctx* c) {
     if (c->words) cudaFree(c->words);
     if (c->stage) cudaFreeHost(c->stage);
     for (auto& e : c->plan_slot_busy) e.reset();
-    if (c->plan_ring) cudaFreeHost(c->plan_ring);
+    for (uint8_t* b : c->plan_slot_buf)
+      if (b) cudaFreeHost(b);
     for (auto& t : c->timed) {
       cudaEventDestroy(t.start);
       cudaEventDestroy(t.stop);
@@ -1903,7 +1953,10 @@ pcs_status pcs_fork_many(pcs_ctx* c, pcs_snapshot* const* parents, int32_t n,
     st = arena_of(c, pl)->alloc(need[pl], stream, &blk[pl]);
     if (st) return undo(st);
   }
+  // Snapshots of one call share a block: one wait (one event query) per run
+  // of equal blocks, not per snapshot.
   for (int i = 0; i < n; ++i) {
+    if (i > 0 && parents[i]->block == parents[i - 1]->block) continue;
     st = wait_written(parents[i]->block, stream);
     if (st) return undo(st);
   }
@@ -1942,7 +1995,8 @@ pcs_status pcs_fork_many(pcs_ctx* c, pcs_snapshot* const* parents, int32_t n,
   Ev done = record_event(c->events, stream);
   st = ws_release(c, stream, done);
   if (st) return undo(st);
-  for (int i = 0; i < n; ++i) note_use(c, parents[i]->block, stream);
+  for (int i = 0; i < n; ++i)
+    if (i == 0 || parents[i]->block != parents[i - 1]->block) note_use(c, parents[i]->block, stream);
   for (int pl = 0; pl < 2; ++pl) {
     if (!blk[pl]) continue;
     blk[pl]->written = done;
@@ -1980,6 +2034,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   st = build_restore(c, snaps, n, targets, verify, &pr);
   if (st) return st;
   for (int s = 0; s < n; ++s) {
+    if (s > 0 && snaps[s]->block == snaps[s - 1]->block) continue;  // one wait per run of a block
     st = wait_written(snaps[s]->block, stream);
     if (st) return st;
   }
@@ -1995,6 +2050,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   if (verify == 1) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
   PCS_CUDA(launch_prepared(c, pr, ws, stream));
   for (int s = 0; s < n; ++s) {
+    if (s > 0 && snaps[s]->block == snaps[s - 1]->block) continue;
     st = note_use(c, snaps[s]->block, stream);
     if (st) return st;
   }

@@ -1,11 +1,15 @@
 """GPU parity at the full workload sizes, in the launch shape bench.py times.
 
-The oracle is too slow for every byte, so each test checks sampled outputs
-against the oracle one by one (whole records of sampled sessions, scores and
-kept sets of sampled banks) and checks properties that hold at any size on
-every output (every restored row equals its source row; every section's
-stored fingerprint is re-verified by the restore).
+Every fingerprint the GPU stores or returns at full size is compared with
+the oracle's: the oracle's C calls release the GIL, so host threads (one per
+core) fingerprint the records' payloads side by side.  Whole records are
+compared byte for byte with the oracle's on sampled sessions (its pack would
+re-gather every page on the host), and every payload byte of every record is
+compared on the device with a gather of the source rows in logical order.
 """
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 import pytest
 import torch
@@ -22,6 +26,41 @@ def _session_pages(pool, pt):
     flat = pt.reshape(-1).long()
     pages = pool[flat].cpu()
     return pages, torch.arange(flat.numel(), dtype=torch.int32).view(pt.shape)
+
+
+def _host_threads() -> int:
+    return max(1, len(os.sched_getaffinity(0)))
+
+
+def _check_record_fps(ctx, snaps, batch=32):
+    """Every section fp and the session fp of every record against the
+    oracle: fp of each payload as the record holds it, and the session fp
+    composed from the oracle's section fps by the oracle's tree and mixer."""
+    sizes = [ctx.info(x).total_bytes for x in snaps]
+    stage = torch.empty(max(sizes) * min(batch, len(snaps)), dtype=torch.uint8, pin_memory=True)
+    host = stage.numpy()
+    checked = 0
+    with ThreadPoolExecutor(_host_threads()) as pool:
+        for b0 in range(0, len(snaps), batch):
+            group = snaps[b0:b0 + batch]
+            offs = np.cumsum([0] + sizes[b0:b0 + len(group)]).tolist()
+            for i, x in enumerate(group):
+                ctx.copy_out(x, 0, sizes[b0 + i], stage[offs[i]:offs[i + 1]])
+            torch.cuda.current_stream().synchronize()
+            jobs = []
+            for i, x in enumerate(group):
+                info = ctx.info(x)
+                secs = [ctx.section(x, j) for j in range(info.n_sections)]
+                futs = [pool.submit(oracle.fingerprint,
+                                    host[offs[i] + e.offset: offs[i] + e.offset + e.bytes])
+                        for e in secs]
+                jobs.append((b0 + i, info, secs, futs))
+            for s, info, secs, futs in jobs:
+                fps = [f.result() for f in futs]
+                assert [e.fp for e in secs] == fps, s
+                assert info.session_fp == oracle.fmix(oracle.tree(fps) ^ info.n_sections), s
+                checked += 1
+    assert checked == len(snaps)
 
 
 def test_kv_full_size(ctx, dev):
@@ -48,6 +87,24 @@ def test_kv_full_size(ctx, dev):
         assert torch.equal(kv.k_pool[a, r], k2[b, r]), s
         assert torch.equal(kv.v_pool[a, r], v2[b, r]), s
     assert torch.equal(meta2, kv.meta)
+    # Every payload byte of every record: META, then K_l and V_l of every
+    # layer in logical order (token j = ring slot (start + j) mod window).
+    layer_bytes = W * kv.k_pool[0, 0].numel() * 2
+    rec = torch.empty(ctx.info(snaps[0]).total_bytes, dtype=torch.uint8, device=dev)
+    for s in range(S):
+        ctx.copy_out(snaps[s], 0, rec.numel(), rec)
+        slot = (kv.ring_start[s] + j) % W
+        e0 = ctx.section(snaps[s], 0)
+        assert torch.equal(rec[e0.offset:e0.offset + e0.bytes], kv.meta[s].view(torch.uint8)), s
+        for l in range(Lyr):
+            rows = slot // P
+            for i, pool in ((1 + 2 * l, kv.k_pool), (2 + 2 * l, kv.v_pool)):
+                e = ctx.section(snaps[s], i)
+                assert e.bytes == layer_bytes
+                want = pool[kv.page_table[s, l].long()[rows], slot % P].contiguous()
+                assert torch.equal(rec[e.offset:e.offset + e.bytes], want.view(-1).view(torch.uint8)), (s, l, i)
+    # Every section fp and session fp of every record against the oracle.
+    _check_record_fps(ctx, snaps)
     # Sampled whole records against the oracle.
     for s in (0, 127, S - 1):
         kp, ptc = _session_pages(kv.k_pool, kv.page_table[s])

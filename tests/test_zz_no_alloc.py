@@ -64,6 +64,51 @@ def test_static_matches_context_twice(ctx, dev):
     assert u64(out) == [oracle.fingerprint(np_bytes(t)) for t in second]
 
 
+def _task_log2(sizes):
+    """2^g chunks per warp task, as the entry point picks it: the smallest g
+    whose tasks fit the fixed node array and leave fewer than 2 x 8192 tasks'
+    worth of chunks per doubling (a larger call takes larger tasks)."""
+    chunks = [max(1, -(-n // 4096)) for n in sizes]
+    g = 0
+    while g < 5 and (sum(-(-c // (1 << g)) for c in chunks) > pcs.PCS_STATIC_MAX_NODES
+                     or (sum(chunks) >> (g + 1)) >= 8192):
+        g += 1
+    return g
+
+
+# Totals from about 100 MiB to 1.3 GiB: one case per task size 2^1 .. 2^5
+# chunks, chunk counts not multiples of 2^g, with empty and unaligned views.
+_LARGE = {
+    1: [(60 << 20) + 4097, (40 << 20) + 3, 0],
+    2: [(150 << 20) + 12345, 7, (50 << 20) + 4096 * 3 + 1],
+    3: [(300 << 20) + 4096 * 5 + 9, 0, (100 << 20) + 1],
+    4: [(500 << 20) + 4096 * 13 + 5, (200 << 20) + 4096 * 7],
+    5: [(900 << 20) + 4096 * 29 + 11, 4095, (400 << 20) + 4096 * 31 + 3],
+}
+
+
+@pytest.mark.parametrize("g", sorted(_LARGE))
+def test_static_large_task_groups(ctx, dev, g):
+    # Every call past 64 MiB groups 2^g chunks per warp task: the per-warp
+    # loop over the group, the lane that keeps each chunk's hash and the
+    # warp tree over a partial last group.
+    sizes = _LARGE[g]
+    assert _task_log2(sizes) == g
+    lib = pcs.load_library()
+    gen = torch.Generator(device=dev).manual_seed(100 + g)
+    tensors = []
+    for i, n in enumerate(sizes):
+        t = torch.randint(0, 256, (n + 3,), generator=gen, dtype=torch.uint8, device=dev)
+        tensors.append(t[3:] if i % 2 else t[:n])  # odd buffers: views off a 16-byte boundary
+    for _ in range(2):
+        out = torch.full((len(tensors),), -1, dtype=torch.int64, device=dev)
+        assert _static(lib, tensors, out) == pcs.PCS_OK, lib.pcs_last_error()
+        want = ctx.fingerprint(tensors)
+        torch.cuda.synchronize()
+        assert u64(out) == u64(want)
+    assert u64(out) == [oracle.fingerprint(np_bytes(t)) for t in tensors]
+
+
 def test_static_limits_are_rejected_before_any_work(dev):
     lib = pcs.load_library()
     t = torch.zeros(16, dtype=torch.uint8, device=dev)
