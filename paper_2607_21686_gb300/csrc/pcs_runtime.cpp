@@ -341,11 +341,21 @@ struct pcs_ctx {
   std::shared_ptr<EventPool> events = std::make_shared<EventPool>();
   std::unique_ptr<Arena> dev_arena, host_arena;
   std::unordered_set<pcs_snapshot*> live;
-  // Workspace: descriptors and tree nodes of one call.
-  uint8_t* ws = nullptr;
-  uint64_t ws_bytes = 0;
-  Ev ws_busy;
-  // Small device words: [0] kernel error bits, [1] verification failures.
+  // Workspaces, one per stream: the descriptors and tree nodes of a call,
+  // after a header of per-call device words ([0] the fused kernel's ticket,
+  // [1] failures of a verify = 1 restore).  Calls on one stream are ordered
+  // by the stream; calls on different streams do not share one, so they can
+  // run side by side.
+  struct Workspace {
+    uint8_t* buf = nullptr;
+    uint64_t bytes = 0;
+    Ev busy;  // the last call's end
+  };
+  std::unordered_map<cudaStream_t, Workspace> ws;
+  Workspace* ws_cur = nullptr;    // of the call in progress (calls hold mu)
+  uint32_t* call_words = nullptr;  // its header words
+  // Context-wide device words: [0] kernel error bits, [2] verify = 2
+  // failures until the next pcs_sync, [4] a flag nothing writes (self-test).
   uint32_t* words = nullptr;
   std::vector<uint8_t> plan;   // host staging of the descriptors
   // Pinned slots for the plans of calls: a true async copy, no driver-side
@@ -453,27 +463,37 @@ Arena* arena_of(pcs_ctx* c, uint32_t placement) {
   return placement == PCS_PLACE_DEVICE ? c->dev_arena.get() : c->host_arena.get();
 }
 
-// Make `stream` wait for the previous call's use of the workspace, grow it
-// if needed.  Returns the workspace base.
+constexpr uint64_t kWsHeader = 256;  // per-call device words before the descriptors
+
+// The workspace of `stream` for the call in progress: grown if needed (after
+// its last call has finished), else `stream` waits for its last call (a no-op
+// on the same stream; a stream handle may be reused after its stream was
+// destroyed).  Returns the base of the call's descriptors; the call's header
+// words are c->call_words, zero on entry.
 pcs_status ws_acquire(pcs_ctx* c, uint64_t bytes, cudaStream_t stream, uint8_t** out) {
-  bytes = round_up(std::max<uint64_t>(bytes, 1), kRecordAlign);
-  if (bytes > c->ws_bytes) {
-    if (c->ws_busy) PCS_CUDA(cudaEventSynchronize(c->ws_busy->ev));
-    c->ws_busy.reset();
-    if (c->ws) cudaFree(c->ws);
-    c->ws = nullptr;
-    c->ws_bytes = 0;
+  bytes = round_up(std::max<uint64_t>(bytes, 1), kRecordAlign) + kWsHeader;
+  pcs_ctx::Workspace& W = c->ws[stream];
+  if (bytes > W.bytes) {
+    if (W.busy) PCS_CUDA(cudaEventSynchronize(W.busy->ev));
+    W.busy.reset();
+    if (W.buf) cudaFree(W.buf);
+    W.buf = nullptr;
+    W.bytes = 0;
     const uint64_t want = round_up(std::max<uint64_t>(bytes, 1ull << 20) * 5 / 4, 2ull << 20);
-    if (cudaMalloc(&c->ws, want) != cudaSuccess) {
+    if (cudaMalloc(&W.buf, want) != cudaSuccess) {
       cudaGetLastError();
+      W.buf = nullptr;
       return fail(PCS_E_NOMEM, "cannot allocate %llu bytes of workspace",
                   static_cast<unsigned long long>(want));
     }
-    c->ws_bytes = want;
-  } else if (c->ws_busy && !c->ws_busy->done()) {
-    PCS_CUDA(cudaStreamWaitEvent(stream, c->ws_busy->ev, 0));
+    PCS_CUDA(cudaMemset(W.buf, 0, kWsHeader));
+    W.bytes = want;
+  } else if (W.busy && !W.busy->done()) {
+    PCS_CUDA(cudaStreamWaitEvent(stream, W.busy->ev, 0));
   }
-  *out = c->ws;
+  c->ws_cur = &W;
+  c->call_words = reinterpret_cast<uint32_t*>(W.buf);
+  *out = W.buf + kWsHeader;
   return PCS_OK;
 }
 
@@ -524,9 +544,10 @@ cudaError_t plan_copy(pcs_ctx* c, uint8_t* ws, uint64_t bytes, cudaStream_t stre
 // End of a call's use of the workspace (and of its plan slot): `done`, if
 // given, is an event already recorded at this point of the stream.
 pcs_status ws_release(pcs_ctx* c, cudaStream_t stream, Ev done = nullptr) {
-  c->ws_busy = done ? done : record_event(c->events, stream);
-  if (!c->ws_busy) return fail(PCS_E_CUDA, "cudaEventRecord failed");
-  if (c->plan_slot_used >= 0) c->plan_slot_busy[c->plan_slot_used] = c->ws_busy;
+  Ev& busy = c->ws_cur->busy;
+  busy = done ? done : record_event(c->events, stream);
+  if (!busy) return fail(PCS_E_CUDA, "cudaEventRecord failed");
+  if (c->plan_slot_used >= 0) c->plan_slot_busy[c->plan_slot_used] = busy;
   c->plan_slot_used = -1;
   return PCS_OK;
 }
@@ -901,7 +922,7 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
                 reinterpret_cast<const uint32_t*>(ws + LL.reg_begin),
                 static_cast<int>(P.reg_ids.size()), P.reg_tasks};
     LaunchScope ls(c, kKStreamHash, stream);
-    PCS_CUDA(launch_small(kModeHash, dsecs, wl, P.glog2, nodes, c->words, c->words + 3, n, nullptr,
+    PCS_CUDA(launch_small(kModeHash, dsecs, wl, P.glog2, nodes, c->words, c->call_words, n, nullptr,
                           nullptr, fp_out, fp_before, flags, nullptr, c->sm_count, c->stream_bps,
                           stream));
     return ws_release(c, stream);
@@ -990,16 +1011,24 @@ void destroy_plans(pcs_ctx* c) {
   c->plans.clear();
 }
 
-// The plan's own device copy of its descriptors, with room for its nodes.
+// The plan's own device copy of its descriptors, with room for its nodes,
+// after a header of its own device words (zero), as in a workspace.
 pcs_status plan_upload(pcs_plan* p) {
-  PCS_CUDA(cudaMalloc(&p->dev, std::max<uint64_t>(p->pr.L.total, 16)));
+  PCS_CUDA(cudaMalloc(&p->dev, kWsHeader + std::max<uint64_t>(p->pr.L.total, 16)));
+  PCS_CUDA(cudaMemset(p->dev, 0, kWsHeader));
   if (!p->pr.plan.empty())
-    PCS_CUDA(cudaMemcpy(p->dev, p->pr.plan.data(), p->pr.plan.size(), cudaMemcpyHostToDevice));
+    PCS_CUDA(cudaMemcpy(p->dev + kWsHeader, p->pr.plan.data(), p->pr.plan.size(),
+                        cudaMemcpyHostToDevice));
   return PCS_OK;
 }
 
-// Launch a prepared call whose descriptors are at `ws` (nodes after them).
-cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, cudaStream_t stream) {
+uint8_t* plan_ws(const pcs_plan* p) { return p->dev + kWsHeader; }
+uint32_t* plan_words(const pcs_plan* p) { return reinterpret_cast<uint32_t*>(p->dev); }
+
+// Launch a prepared call whose descriptors are at `ws` (nodes after them);
+// `words` are the call's header words (ticket of the fused kernel).
+cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, uint32_t* words,
+                            cudaStream_t stream) {
   const auto* dsecs = reinterpret_cast<const SecDesc*>(ws + pr.L.secs);
   const auto* dsess = reinterpret_cast<const SessDesc*>(ws + pr.L.sess);
   auto* nodes = reinterpret_cast<uint64_t*>(ws + pr.L.nodes);
@@ -1010,7 +1039,7 @@ cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, cudaStr
     const auto* dent = reinterpret_cast<const Entry*>(ws + pr.L.entries);
     if (pr.fused) {
       LaunchScope ls(c, kKStreamPack, stream);
-      return launch_small(kModePack, dsecs, wl, pr.P.glog2, nodes, c->words, c->words + 3, pr.n,
+      return launch_small(kModePack, dsecs, wl, pr.P.glog2, nodes, c->words, words, pr.n,
                           dsess, dent, nullptr, nullptr, nullptr, nullptr, c->sm_count,
                           c->stream_bps, stream);
     }
@@ -1020,10 +1049,10 @@ cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, cudaStr
     return launch_finalize(kModePack, dsecs, dsess, pr.n, dent, nodes, nullptr, nullptr, nullptr,
                            nullptr, pr.max_secs, stream);
   }
-  uint32_t* bad = c->words + (pr.verify == 1 ? 1 : 2);
+  uint32_t* bad = pr.verify == 1 ? words + 1 : c->words + 2;
   if (pr.fused) {
     LaunchScope ls(c, kKStreamRestoreV, stream);
-    return launch_small(kModeRestoreV, dsecs, wl, pr.P.glog2, nodes, c->words, c->words + 3, pr.n,
+    return launch_small(kModeRestoreV, dsecs, wl, pr.P.glog2, nodes, c->words, words, pr.n,
                         dsess, nullptr, nullptr, nullptr, nullptr, bad, c->sm_count,
                         c->stream_bps, stream);
   }
@@ -1276,8 +1305,11 @@ pcs_status pcs_destroy(pcs_ctx* c) {
     }
     c->pools.clear();
     destroy_plans(c);
-    c->ws_busy.reset();
-    if (c->ws) cudaFree(c->ws);
+    for (auto& kv : c->ws) {
+      kv.second.busy.reset();
+      if (kv.second.buf) cudaFree(kv.second.buf);
+    }
+    c->ws.clear();
     if (c->words) cudaFree(c->words);
     if (c->stage) cudaFreeHost(c->stage);
     for (auto& e : c->plan_slot_busy) e.reset();
@@ -1911,7 +1943,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   c->plan.swap(pr.plan);
   cudaError_t e = plan_copy(c, ws, pr.L.nodes, stream);
   c->plan.swap(pr.plan);
-  if (e == cudaSuccess) e = launch_prepared(c, pr, ws, stream);
+  if (e == cudaSuccess) e = launch_prepared(c, pr, ws, c->call_words, stream);
   if (e != cudaSuccess) return undo(cuda_fail(e, "checkpoint launch"));
   blk->written = record_event(c->events, stream);
   st = ws_release(c, stream, blk->written);
@@ -2047,8 +2079,9 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   PCS_CUDA(e);
   // verify == 1: count failures of this call in words[1] and wait for them;
   // verify == 2: accumulate them in words[2] for the next pcs_sync.
-  if (verify == 1) PCS_CUDA(cudaMemsetAsync(c->words + 1, 0, 4, stream));
-  PCS_CUDA(launch_prepared(c, pr, ws, stream));
+  uint32_t* words = c->call_words;
+  if (verify == 1) PCS_CUDA(cudaMemsetAsync(words + 1, 0, 4, stream));
+  PCS_CUDA(launch_prepared(c, pr, ws, words, stream));
   for (int s = 0; s < n; ++s) {
     if (s > 0 && snaps[s]->block == snaps[s - 1]->block) continue;
     st = note_use(c, snaps[s]->block, stream);
@@ -2058,7 +2091,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   if (st) return st;
   if (verify == 1) {
     uint32_t bad = 0;
-    PCS_CUDA(cudaMemcpyAsync(&bad, c->words + 1, 4, cudaMemcpyDeviceToHost, stream));
+    PCS_CUDA(cudaMemcpyAsync(&bad, words + 1, 4, cudaMemcpyDeviceToHost, stream));
     PCS_CUDA(cudaStreamSynchronize(stream));
     if (bad) return fail(PCS_E_CORRUPT, "%u of %d restored sessions failed verification", bad, n);
   }
@@ -2083,7 +2116,7 @@ pcs_status pcs_plan_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t 
   st = build_checkpoint(c, sessions, n, placement, stream, &p->pr, &blk, &handles);
   if (st) return st;
   st = plan_upload(p.get());
-  cudaError_t e = st ? cudaSuccess : launch_prepared(c, p->pr, p->dev, stream);
+  cudaError_t e = st ? cudaSuccess : launch_prepared(c, p->pr, plan_ws(p.get()), plan_words(p.get()), stream);
   if (st || e != cudaSuccess) {
     if (p->dev) cudaFree(p->dev);
     arena_of(c, placement)->free(blk);
@@ -2150,7 +2183,7 @@ pcs_status pcs_plan_run(pcs_ctx* c, pcs_plan* p, void* stream_) {
       if (u.first != stream && u.second && !u.second->done())
         PCS_CUDA(cudaStreamWaitEvent(stream, u.second->ev, 0));
   }
-  PCS_CUDA(launch_prepared(c, p->pr, p->dev, stream));
+  PCS_CUDA(launch_prepared(c, p->pr, plan_ws(p), plan_words(p), stream));
   for (Block* b : p->blocks) {
     if (ckpt) {
       b->written = record_event(c->events, stream);

@@ -4,6 +4,8 @@
     python profile_cases.py classify --n 200 --hi-mib 32
     python profile_cases.py prune --sessions 256
     python profile_cases.py markov --sessions 4096
+    python profile_cases.py markov_prepared --sessions 4096
+    python profile_cases.py banks2 --sessions 64
     python profile_cases.py markov_layouts --sessions 4096
     python profile_cases.py mismatch --n 200 --hi-mib 32
     python profile_cases.py prune_global --sessions 256
@@ -84,6 +86,57 @@ def case_markov(ctx, a, dev):
         hs = ctx.checkpoint_raw(arr, a.sessions)
         ctx.restore_raw(hs, a.sessions, arr)
         ctx.delete_raw(hs, a.sessions)
+    return _timed(step, a.warmup)
+
+
+def case_markov_prepared(ctx, a, dev):
+    # The Markov batch as prepared calls: checkpoint, then verified restore
+    # (mismatches counted on the device), launches only.
+    g = torch.Generator(device=dev).manual_seed(synth.seed_for(1))
+    obs = torch.randint(0, 256, (a.sessions, 3, 256, 256), generator=g, device=dev, dtype=torch.uint8)
+    rng = torch.randint(-2**62, 2**62, (a.sessions, 2), generator=g, device=dev, dtype=torch.int64)
+    arr = ctx.session_array([pcs.markov_session(s, obs[s], rng[s]) for s in range(a.sessions)])
+    cplan, hs = ctx.plan_checkpoint(arr, a.sessions)
+    rplan = ctx.plan_restore(hs, a.sessions, arr, verify=2)
+
+    def step():
+        ctx.plan_run(cplan)
+        ctx.plan_run(rplan)
+    ms = _timed(step, a.warmup)
+    ctx.sync()
+    ctx.plan_destroy(rplan)
+    ctx.plan_destroy(cplan)
+    ctx.delete_raw(hs, a.sessions)
+    return ms
+
+
+def case_banks2(ctx, a, dev):
+    # Memory banks (64 by default): prune to k = min(n, 128), checkpoint the
+    # kept entries to HBM, verified restore into compacted banks, delete.
+    b = synth.banks_config2(device=dev, sessions=a.sessions)
+    S = b.sessions
+    keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    vals = [b.values[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
+    banks = ctx.banks_array(keys, [b.queries[s] for s in range(S)], 512 + b.value_bytes)
+    params = ctx.params(pcs.PCS_K_FIXED, k_max=128)
+    ks = ctx.prune_counts(banks, S, params)
+    koff = [0]
+    for k in ks:
+        koff.append(koff[-1] + k)
+    kept = torch.empty(koff[-1], dtype=torch.int32, device=dev)
+    sarr = ctx.session_array([pcs.bank_session(s, keys[s], vals[s], kept[koff[s]:koff[s + 1]])
+                              for s in range(S)])
+    outs = [(torch.empty(ks[s], dtype=torch.int32, device=dev),
+             torch.empty(ks[s], 256, dtype=torch.float16, device=dev),
+             torch.empty((ks[s],) + tuple(b.values.shape[1:]), dtype=b.values.dtype, device=dev))
+            for s in range(S)]
+    tarr = ctx.session_array([pcs.bank_targets(s, *outs[s]) for s in range(S)])
+
+    def step():
+        ctx.prune(banks, S, params, kept)
+        hs = ctx.checkpoint_raw(sarr, S)
+        ctx.restore_raw(hs, S, tarr, verify=2)
+        ctx.delete_raw(hs, S)
     return _timed(step, a.warmup)
 
 
@@ -177,6 +230,7 @@ def case_topk(ctx, a, dev):
 
 
 CASES = {"kv": case_kv, "classify": case_classify, "prune": case_prune, "markov": case_markov,
+         "markov_prepared": case_markov_prepared, "banks2": case_banks2,
          "markov_layouts": case_markov_layouts,
          "mismatch": case_mismatch, "prune_global": case_prune_global, "cow": case_cow,
          "reads": case_reads, "topk": case_topk}
