@@ -40,10 +40,10 @@ METRIC = "snapshot+restore GB/s and sessions/s on 1 GB300; % of HBM (PCIe) roofl
 # capture summarised in profiles/k_bulk_kv8x24_full.md (8 sessions, scaled by
 # sessions / 8), valid only for the streaming-kernel source it was taken on.
 NCU_TRAFFIC = {
-    "source_sha256_prefix": "3edbcd422d109bd3",
+    "source_sha256_prefix": "64f3b87a0c0b9b6e",
     "sessions": 8,
-    "k_bulk<pack>": 805711616 + 754301440,
-    "k_bulk<restore_verify>": 805729280 + 754210816,
+    "k_bulk<pack>": 805710848 + 754139648,
+    "k_bulk<restore_verify>": 805741056 + 754459648,
 }
 
 

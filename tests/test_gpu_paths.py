@@ -127,3 +127,54 @@ def test_timing_reports_both_kernels(ctx, dev):
     ctx.timing(False)
     assert t["k_bulk<hash>"][0] == 1 and t["k_stream<hash>"][0] == 1
     assert t["k_finalize<hash>"][0] == 1
+
+
+def test_small_unaligned_sources_in_large_calls(ctx, ctx_reg, dev):
+    # A call past the small-call size mixes both kernels: the aligned
+    # buffer goes through the TMA kernel, sections off a 16-byte boundary
+    # (sources and restore targets) through the register kernel, in one call.
+    g = torch.Generator().manual_seed(31)
+    big = torch.randint(0, 256, (3 << 20,), generator=g, dtype=torch.uint8).to(dev)
+    pool = torch.randint(0, 256, (1 << 18,), generator=g, dtype=torch.uint8).to(dev)
+    views, off = [big], 0
+    for n in [1, 3, 4, 15, 16, 17, 100, 511, 4095, 4096, 4097, 8191, 8192, 8193]:
+        for shift in (1, 2, 4, 8, 12):
+            off += shift
+            views.append(pool[off:off + n])
+            off += n
+    assert off <= pool.numel()
+    want = [oracle.fingerprint(np_bytes(x)) for x in views]
+    assert u64(ctx.fingerprint(views)) == want
+    assert u64(ctx_reg.fingerprint(views)) == want
+    # Checkpoint: one big aligned section and small unaligned ones per session.
+    sess = []
+    for s in range(6):
+        secs = [pcs.contig_section(pcs.PCS_SEC_OBS, big[s << 18:(s + 1) << 18])]
+        secs += [pcs.contig_section(pcs.PCS_SEC_KEPT_IDX, v) for v in views[1 + s::6]]
+        sess.append(pcs.Session(s, pcs.PCS_KIND_MARKOV, secs, keep=[big, pool]))
+    snaps = ctx.checkpoint(sess)
+    for s, sn in enumerate(snaps):
+        sp = oracle.SessionSpec(s, oracle.KIND_MARKOV)
+        sp.contig(pcs.PCS_SEC_OBS, oracle.DT_U8, np_bytes(big[s << 18:(s + 1) << 18]))
+        for v in views[1 + s::6]:
+            sp.contig(pcs.PCS_SEC_KEPT_IDX, oracle.DT_U8, np_bytes(v))
+        assert np.array_equal(ctx.record(sn).numpy(), oracle.pack(sp)), s
+    # Restore into targets that are themselves off a 16-byte boundary.
+    tpool = torch.zeros(1 << 18, dtype=torch.uint8, device=dev)
+    tb = torch.zeros(6 << 18, dtype=torch.uint8, device=dev)
+    tg, toff, tv = [], 3, []
+    for s in range(6):
+        secs = [pcs.contig_section(pcs.PCS_SEC_OBS, tb[s << 18:(s + 1) << 18])]
+        for v in views[1 + s::6]:
+            t = tpool[toff:toff + v.numel()]
+            toff += v.numel() + 5
+            tv.append((t, v))
+            secs.append(pcs.contig_section(pcs.PCS_SEC_KEPT_IDX, t))
+        tg.append(pcs.Session(s, pcs.PCS_KIND_MARKOV, secs, keep=[tb, tpool]))
+    ctx.restore(snaps, tg, verify=True)
+    torch.cuda.synchronize()
+    assert torch.equal(tb, big[:6 << 18])
+    for t, v in tv:
+        assert torch.equal(t, v)
+    for sn in snaps:
+        ctx.delete(sn)

@@ -136,3 +136,50 @@ def test_plan_argument_errors(ctx, dev):
     assert e.value.status == pcs.PCS_E_INVAL
     ctx.plan_destroy(plan)
     ctx.delete_raw(hs, 2)
+
+
+@pytest.mark.parametrize("n", [3, 70])  # the fused small-call kernel and the general path
+def test_calls_on_two_streams_run_side_by_side(ctx, dev, n):
+    # Plain calls on two streams have a workspace each, and prepared calls a
+    # buffer each, so nothing orders them against each other: many rounds on
+    # both streams at once, nothing synchronised in between, every record
+    # and every restored byte as the oracle says.
+    streams = [torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)]
+    sets = [_markov(n, dev, seed=800 + 100 * k) for k in range(2)]
+    arrs = [ctx.session_array([pcs.markov_session(i, o[i], r[i]) for i in range(n)])
+            for o, r in sets]
+    outs = [[(torch.zeros_like(o), torch.zeros_like(r)) for o, r in zip(*sets[k])]
+            for k in range(2)]
+    tarrs = [ctx.session_array([pcs.markov_session(i, a, b) for i, (a, b) in enumerate(outs[k])])
+             for k in range(2)]
+    plans = []
+    for k in range(2):
+        cp, phs = ctx.plan_checkpoint(arrs[k], n, stream=streams[k])
+        plans.append((cp, phs, ctx.plan_restore(phs, n, tarrs[k], verify=2)))
+    torch.cuda.synchronize()
+    kept = []
+    for round_ in range(6):
+        for k in range(2):
+            hs = ctx.checkpoint_raw(arrs[k], n, stream=streams[k])
+            ctx.restore_raw(hs, n, tarrs[k], verify=2, stream=streams[k])
+            kept.append((k, hs))
+            ctx.plan_run(plans[k][0], stream=streams[k])
+            ctx.plan_run(plans[k][2], stream=streams[k])
+    torch.cuda.synchronize()
+    ctx.sync()  # no verified restore failed, no kernel error
+    for k in range(2):
+        obs, rng = sets[k]
+        for i in range(n):
+            assert torch.equal(outs[k][i][0], obs[i]) and torch.equal(outs[k][i][1], rng[i])
+            want = _oracle_rec(i, obs[i], rng[i])
+            assert np.array_equal(ctx.record(pcs.Snapshot(ctx, plans[k][1][i])).numpy(), want)
+    for k, hs in kept[-2:]:
+        for i in (0, n - 1):
+            assert np.array_equal(ctx.record(pcs.Snapshot(ctx, hs[i])).numpy(),
+                                  _oracle_rec(i, sets[k][0][i], sets[k][1][i]))
+    for k, hs in kept:
+        ctx.delete_raw(hs, n)
+    for cp, phs, rp in plans:
+        ctx.plan_destroy(rp)
+        ctx.plan_destroy(cp)
+        ctx.delete_raw(phs, n)
