@@ -40,10 +40,10 @@ METRIC = "snapshot+restore GB/s and sessions/s on 1 GB300; % of HBM (PCIe) roofl
 # capture summarised in profiles/k_bulk_kv8x24_full.md (8 sessions, scaled by
 # sessions / 8), valid only for the streaming-kernel source it was taken on.
 NCU_TRAFFIC = {
-    "source_sha256_prefix": "64f3b87a0c0b9b6e",
+    "source_sha256_prefix": "65775241df3a934b",
     "sessions": 8,
-    "k_bulk<pack>": 805710848 + 754139648,
-    "k_bulk<restore_verify>": 805741056 + 754459648,
+    "k_bulk<pack>": 805709568 + 754288128,
+    "k_bulk<restore_verify>": 805732608 + 754471168,
 }
 
 
@@ -88,14 +88,20 @@ def step_bytes(a) -> int:
 
 
 def kernel_source_sha() -> str:
-    """sha256 prefix of the streaming kernels' source: pcs_kernels.cu up to the
-    finalisation kernels (helpers, the register kernel, the TMA kernel)."""
+    """sha256 prefix of the streaming kernels' code: pcs_kernels.cu up to the
+    finalisation kernels (helpers, the register kernel, the TMA kernel, the
+    hash kernel), with // comments and blank lines left out, so that a change
+    of wording does not disown a capture of the same code."""
     import hashlib
+    import re
     p = os.path.join(ROOT, "paper_2607_21686_gb300", "csrc", "pcs_kernels.cu")
     with open(p, "rb") as f:
         text = f.read()
     cut = text.find(b"// Finalisation: stream fps")
-    return hashlib.sha256(text[:cut if cut > 0 else len(text)]).hexdigest()[:16]
+    code = text[:cut if cut > 0 else len(text)].decode()
+    lines = [re.sub(r"//.*$", "", ln).rstrip() for ln in code.splitlines()]
+    code = "\n".join(ln for ln in lines if ln.strip())
+    return hashlib.sha256(code.encode()).hexdigest()[:16]
 
 
 def ncu_traffic(kernel: str, sessions: int):

@@ -7,6 +7,11 @@
 //                 paged-ring layout, and folds them into the PCSFP64-v1 lane
 //                 chain; a shuffle tree makes the chunk hash and then the
 //                 task's aligned-group node (Sec. 4 FINGERPRINT, step 1).
+// k_bulk<MODE>    the moving passes (pack, restore) of aligned streams: per-warp
+//                 TMA pipelines of 8 KiB tiles through shared memory, the
+//                 fingerprint of each tile fused into the copy.
+// k_hash          the read-only fingerprint pass of aligned buffers: a warp per
+//                 8 KiB tile, plain loads into registers, 20 warps per SM.
 // k_finalize<MODE> trees the task nodes of each stream into its fingerprint and
 //                 writes outputs: fps / classification flags, record headers
 //                 and section tables (checkpoint, Sec. 3 "The contract", I4),
@@ -393,13 +398,14 @@ __global__ void __launch_bounds__(kThreads, 2)
 constexpr int kTileChunks = kBulkTileChunks;
 constexpr uint32_t kTileBytes = kTileChunks * kChunkBytes;
 
-// Shape of the TMA kernel per mode: warps per block and stages per warp.
-// Moving modes keep 3 tiles per warp in flight; the read-only hash mode,
-// bound by the hash chains' latency, trades a stage for more warps.
+// Shape of the TMA kernel (the moving modes: pack, restore, verified
+// restore): warps per block and stages per warp, 3 tiles per warp in flight.
+// The read-only hash pass has a kernel of its own (k_hash, below).
 template <int MODE>
 struct BulkShape {
-  static constexpr int kWarps = MODE == kModeHash ? 12 : 8;
-  static constexpr int kStages = MODE == kModeHash ? 2 : 3;
+  static_assert(MODE != kModeHash, "the hash-only pass runs in k_hash");
+  static constexpr int kWarps = 8;
+  static constexpr int kStages = 3;
   static constexpr int kThreads = 32 * kWarps;
 };
 constexpr int kTileRows = 32;  // rows >= 512 bytes touching an 8 KiB tile: at most 17
@@ -686,36 +692,6 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     }
     fence_async_smem();
     __syncwarp();
-    if (MODE == kModeHash) {
-      // Read-only pass: the tile goes into registers and its stage is handed
-      // to tile i + kWarpStages before the hashing starts, so both stages
-      // load while the chains run (measured: the 200-buffer sweep 6.22 ->
-      // 6.27 TB/s).  The two chunks share each level of one tree.
-      const uint64_t c0 = p0 / kChunkBytes;
-      const int nc = static_cast<int>((p1 - p0) / kChunkBytes);
-      const uint32_t node = m.node;
-      uint4 va[kSegs], vb[kSegs];
-#pragma unroll
-      for (int k = 0; k < kSegs; ++k) {
-        va[k] = *reinterpret_cast<const uint4*>(tile + 512 * k + 16 * lane);
-        vb[k] = nc > 1 ? *reinterpret_cast<const uint4*>(tile + kChunkBytes + 512 * k + 16 * lane) : zero;
-      }
-      fence_async_smem();  // the reads above before the next bulk copy into the stage
-      __syncwarp();
-      const uint32_t tn = t0 + i + kWarpStages;
-      if (tn < t1) stage_tile<MODE>(secs, wl, item_of(tn), tn, m, tile, bar, err, lane);
-      uint64_t ha = fmix(kSeed ^ (c0 * 32u + lane));
-      uint64_t hb = fmix(kSeed ^ ((c0 + 1) * 32u + lane));
-#pragma unroll
-      for (int k = 0; k < kSegs; ++k) {
-        ha = absorb(ha, va[k]);
-        hb = absorb(hb, vb[k]);
-      }
-      static_assert(kTileChunks == 2, "tile_tree2 reduces two chunks");
-      const uint64_t root = tile_tree2(fmix(ha), fmix(hb), nc, lane);
-      if (lane == 0) nodes[node] = root;
-      continue;
-    }
     bool issued = false;
     if (MODE == kModePack) {
       // Contiguous payload, through the record's 256-byte padding.
@@ -761,8 +737,8 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
         }
       }
       // Moving passes are bound by DRAM; one tree per chunk paces the warps
-      // so that loads and stores interleave best (measured: the hash pass's
-      // shared tree makes pack and restore slower).
+      // so that loads and stores interleave best (measured: the shared tree
+      // of tile_tree2 makes pack and restore slower).
       uint64_t mine = 0;
 #pragma unroll
       for (int q = 0; q < kTileChunks; ++q) {
@@ -782,6 +758,73 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     if (tn < t1) stage_tile<MODE>(secs, wl, item_of(tn), tn, m, tile, bar, err, lane);
   }
   if (any_issued) bulk_wait_all();
+}
+
+// ---------------------------------------------------------------------------
+// Read-only fingerprint pass (hash mode of the streams the TMA kernel would
+// take: 16-byte aligned contiguous device buffers)
+//
+// Every warp walks a contiguous range of 8 KiB tiles; per tile each lane
+// issues its sixteen 16-byte loads (segments lane + 32k of both chunks) into
+// registers, then runs the two lane chains interleaved and one shared tree
+// (tile_tree2).  No shared memory: 20 warps per SM fit in the register file
+// (88 registers), and their loads hide each other's hashing.  Measured on
+// the 200-buffer classify sweep: 6.68 TB/s, against 6.27 TB/s for the TMA
+// pipeline with two 8 KiB stages per warp (which shared memory capped at 12
+// warps) and 6.99 TB/s for a plain-load byte compare of the same pairs;
+// 16 warps 6.49, 24 warps (spilling) 6.08, two tiles in flight per warp
+// (166 registers, 12 warps) 5.42.
+// ---------------------------------------------------------------------------
+
+constexpr int kHashWarps = 20;
+constexpr int kHashThreads = 32 * kHashWarps;
+
+__global__ void __launch_bounds__(kHashThreads, 1)
+    k_hash(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes) {
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  // This warp's tiles: a contiguous, balanced range [t0, t1).
+  const uint64_t T_all = wl.n_tasks;
+  const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kHashWarps + warp;
+  const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kHashWarps;
+  const uint32_t t0 = static_cast<uint32_t>(T_all * gw / nw);
+  const uint32_t t1 = static_cast<uint32_t>(T_all * (gw + 1) / nw);
+  if (t0 >= t1) return;
+  int item = find_item(wl.begin, wl.n_items, t0);
+  for (uint32_t t = t0; t < t1; ++t) {
+    while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= t) ++item;
+    const SecDesc* s = secs + __ldg(wl.ids + item);
+    const uint8_t* base = reinterpret_cast<const uint8_t*>(
+        __ldg(reinterpret_cast<const unsigned long long*>(&s->lbase)));
+    const uint64_t L = __ldg(reinterpret_cast<const unsigned long long*>(&s->bytes));
+    const uint64_t nch = __ldg(reinterpret_cast<const unsigned long long*>(&s->n_chunks));
+    const uint32_t loc = t - __ldg(wl.begin + item);
+    const uint64_t p0 = static_cast<uint64_t>(loc) * kTileBytes;
+    const uint64_t c0 = p0 / kChunkBytes;
+    // Bytes at or past L read as zero (the chunk's padding).
+    uint4 v[2 * kSegs];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+#pragma unroll
+      for (int k = 0; k < kSegs; ++k) {
+        const uint64_t off = p0 + q * kChunkBytes + 512u * k + 16u * lane;
+        uint4 x = make_uint4(0, 0, 0, 0);
+        if (off + 16 <= L) x = ld_stream(base + off);
+        else if (off < L) x = ld_small(base + off, static_cast<int>(L - off), true);
+        v[q * kSegs + k] = x;
+      }
+    }
+    uint64_t ha = fmix(kSeed ^ (c0 * 32u + lane));
+    uint64_t hb = fmix(kSeed ^ ((c0 + 1) * 32u + lane));
+#pragma unroll
+    for (int k = 0; k < kSegs; ++k) {
+      ha = absorb(ha, v[k]);
+      hb = absorb(hb, v[kSegs + k]);
+    }
+    static_assert(kTileChunks == 2, "tile_tree2 reduces two chunks");
+    const uint64_t root = tile_tree2(fmix(ha), fmix(hb), nch - c0 >= 2 ? 2 : 1, lane);
+    if (lane == 0) nodes[__ldg(&s->task_begin) + loc] = root;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -2649,7 +2692,12 @@ cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* no
                         uint32_t* dev_err, int sm_count, cudaStream_t stream) {
   if (wl.n_tasks == 0) return cudaSuccess;
   switch (mode) {
-    case kModeHash: return launch_bulk_mode<kModeHash>(secs, wl, nodes, dev_err, sm_count, stream);
+    case kModeHash: {
+      const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + kHashWarps - 1) / kHashWarps;
+      const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
+      k_hash<<<blocks, kHashThreads, 0, stream>>>(secs, wl, nodes);
+      return cudaGetLastError();
+    }
     case kModePack: return launch_bulk_mode<kModePack>(secs, wl, nodes, dev_err, sm_count, stream);
     case kModeRestore:
       return launch_bulk_mode<kModeRestore>(secs, wl, nodes, dev_err, sm_count, stream);

@@ -403,7 +403,7 @@ static_assert(kKernelKinds <= 32, "kernel timing table");
 const char* kKernelNames[kKernelKinds] = {
     "k_stream<hash>", "k_stream<pack>", "k_stream<restore>", "k_stream<restore_verify>",
     "k_finalize<hash>", "k_finalize<pack>", "k_finalize<restore_verify>", "k_score", "k_topk",
-    "k_bulk<hash>", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
+    "k_hash", "k_bulk<pack>", "k_bulk<restore>", "k_bulk<restore_verify>",
     "k_reduce_nodes", "k_gselect", "k_gfinish", "k_pool_alloc", "k_pool_share", "k_pool_cow",
     "k_pool_release", "k_mismatch", "k_classify_reads"};
 
