@@ -294,14 +294,22 @@ __device__ __forceinline__ void store_seg(const SecDesc& s, uint64_t off, uint4 
   }
 }
 
-// Section of warp task `task` in a work list: last j with begin[j] <= task.
+// Section of warp task `task` in a work list: the last j with begin[j] <=
+// task (begin[0] = 0 and begin rises).  Called by a whole warp with a
+// warp-uniform task: each round the lanes probe 32 evenly spaced entries of
+// the range still open and keep the part after the last probe <= task, so
+// that 12,544 items take three dependent loads instead of fourteen.
 __device__ __forceinline__ int find_item(const uint32_t* __restrict__ begin, int n_items,
-                                        uint32_t task) {
-  int lo = 0, hi = n_items - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (__ldg(begin + mid) <= task) lo = mid;
-    else hi = mid - 1;
+                                        uint32_t task, int lane) {
+  int lo = 0, span = n_items;  // the answer lies in [lo, lo + span)
+  while (span > 1) {
+    const int step = (span + 31) >> 5;
+    const int i = lo + lane * step;
+    const bool le = i < lo + span && __ldg(begin + i) <= task;
+    const unsigned m = __ballot_sync(kFull, le);  // lane 0 probes lo: never empty
+    const int last = 31 - __clz(m);
+    lo += last * step;
+    span = min(step, span - last * step);
   }
   return lo;
 }
@@ -317,7 +325,7 @@ __device__ __forceinline__ void run_stream_tasks(const SecDesc* __restrict__ sec
   const uint32_t nw = gridDim.x * kWarps;
   int cur = -1;
   for (uint32_t task = blockIdx.x * kWarps + wib; task < wl.n_tasks; task += nw) {
-    const int j = find_item(wl.begin, wl.n_items, task);
+    const int j = find_item(wl.begin, wl.n_items, task, lane);
     if (j != cur) {
       __syncwarp();
       const SecDesc* src = &secs[__ldg(wl.ids + j)];
@@ -408,6 +416,15 @@ struct BulkShape {
   static constexpr int kStages = 3;
   static constexpr int kThreads = 32 * kWarps;
 };
+// Copies one contiguous 8 KiB load of a hashing pass is split into (1 KiB
+// each).  Measured, 4,096 and 16,384 Markov sessions of 192 KiB: pack 0.308
+// -> 0.276 ms and 1.105 -> 1.001 ms, verified restore 0.304 -> 0.268 ms and
+// 1.108 -> 0.993 ms (2, 4 and 16 pieces gained less).  Plain
+// restores keep one copy (a fork of 256 KV records lost 1.3 % with pieces),
+// and so do loads of a restore into rows (split, the KV step's verified
+// restore took twice as long).
+constexpr int kContigPieces = 8;
+static_assert(kTileBytes / kContigPieces % 16 == 0 && kContigPieces <= 32, "pieces");
 constexpr int kTileRows = 32;  // rows >= 512 bytes touching an 8 KiB tile: at most 17
 constexpr long long kWaitCycles = 4000000000ll;  // give up a wait after ~2 s of SM clock
 static_assert(kTileBytes / kBulkMinRowBytes + 1 <= kTileRows, "tile rows");
@@ -592,11 +609,19 @@ __device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, con
   }
   __syncwarp();
   if (!T::kLoadLayout || s.layout == kContig) {
-    // One contiguous piece: the record payload, or a contiguous buffer.
-    if (lane == 0) {
-      const uint32_t bytes = pe > p0 ? static_cast<uint32_t>(pe - p0) : 0u;
-      mbar_arrive_expect_tx(bar, bytes);
-      if (bytes) bulk_g2s(tile, T::kLoadLayout ? s.lbase + p0 : s.payload + p0, bytes, bar);
+    // One contiguous piece: the record payload, or a contiguous buffer.  A
+    // hashing pass whose layout side is contiguous (a pack from a
+    // contiguous buffer, a verified restore into one) loads it as
+    // kContigPieces copies issued by as many lanes.
+    const uint32_t bytes = pe > p0 ? static_cast<uint32_t>(pe - p0) : 0u;
+    const int pieces = (T::kHash && s.layout == kContig) ? kContigPieces : 1;
+    if (lane == 0) mbar_arrive_expect_tx(bar, bytes);
+    __syncwarp();
+    if (lane < pieces && bytes) {
+      const uint32_t piece = ((bytes + pieces - 1) / pieces + 15u) & ~15u;
+      const uint32_t lo = static_cast<uint32_t>(lane) * piece;
+      const uint32_t hi = lo + piece < bytes ? lo + piece : bytes;
+      if (hi > lo) bulk_g2s(tile + lo, (T::kLoadLayout ? s.lbase : s.payload) + p0 + lo, hi - lo, bar);
     }
     return;
   }
@@ -647,7 +672,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
   const uint32_t t0 = static_cast<uint32_t>(T_all * gw / nw);
   const uint32_t t1 = static_cast<uint32_t>(T_all * (gw + 1) / nw);
   if (t0 >= t1) return;
-  int item = find_item(wl.begin, wl.n_items, t0);  // item of the next tile to stage
+  int item = find_item(wl.begin, wl.n_items, t0, lane);  // item of the next tile to stage
   auto item_of = [&](uint32_t t) {
     while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= t) ++item;
     return item;
@@ -790,7 +815,7 @@ __global__ void __launch_bounds__(kHashThreads, 1)
   const uint32_t t0 = static_cast<uint32_t>(T_all * gw / nw);
   const uint32_t t1 = static_cast<uint32_t>(T_all * (gw + 1) / nw);
   if (t0 >= t1) return;
-  int item = find_item(wl.begin, wl.n_items, t0);
+  int item = find_item(wl.begin, wl.n_items, t0, lane);
   for (uint32_t t = t0; t < t1; ++t) {
     while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= t) ++item;
     const SecDesc* s = secs + __ldg(wl.ids + item);
