@@ -119,9 +119,12 @@ cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_
                           cudaStream_t stream);
 
 // TMA-staged kernel: tasks of kBulkTileChunks chunks staged through shared
-// memory with cp.async.bulk; one persistent block per SM.
+// memory with cp.async.bulk; one persistent block per SM.  `sched`: two
+// device words of the call (zero on entry, left zero) that share out the
+// launch's last tiles at run time; launches using the same words must be
+// ordered.  (Hash mode runs k_hash and does not use them.)
 cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* nodes,
-                        uint32_t* dev_err, int sm_count, cudaStream_t stream);
+                        uint32_t* dev_err, uint32_t* sched, int sm_count, cudaStream_t stream);
 size_t bulk_shared_bytes();
 
 // One launch for a small call: the register streaming pass over wl (no

@@ -9,7 +9,9 @@
 //                 task's aligned-group node (Sec. 4 FINGERPRINT, step 1).
 // k_bulk<MODE>    the moving passes (pack, restore) of aligned streams: per-warp
 //                 TMA pipelines of 8 KiB tiles through shared memory, the
-//                 fingerprint of each tile fused into the copy.
+//                 fingerprint of each tile fused into the copy
+//                 (k_bulk_shared: the same for small launches, the last
+//                 tiles handed out at run time).
 // k_hash          the read-only fingerprint pass of aligned buffers: a warp per
 //                 8 KiB tile, plain loads into registers, 20 warps per SM.
 // k_finalize<MODE> trees the task nodes of each stream into its fingerprint and
@@ -295,13 +297,14 @@ __device__ __forceinline__ void store_seg(const SecDesc& s, uint64_t off, uint4 
 }
 
 // Section of warp task `task` in a work list: the last j with begin[j] <=
-// task (begin[0] = 0 and begin rises).  Called by a whole warp with a
+// task (begin rises), searched from item `lo` on (begin[lo] <= task; lo = 0
+// searches the whole list, begin[0] = 0).  Called by a whole warp with a
 // warp-uniform task: each round the lanes probe 32 evenly spaced entries of
 // the range still open and keep the part after the last probe <= task, so
 // that 12,544 items take three dependent loads instead of fourteen.
-__device__ __forceinline__ int find_item(const uint32_t* __restrict__ begin, int n_items,
+__device__ __forceinline__ int find_item(const uint32_t* __restrict__ begin, int lo, int n_items,
                                         uint32_t task, int lane) {
-  int lo = 0, span = n_items;  // the answer lies in [lo, lo + span)
+  int span = n_items - lo;  // the answer lies in [lo, lo + span)
   while (span > 1) {
     const int step = (span + 31) >> 5;
     const int i = lo + lane * step;
@@ -325,7 +328,7 @@ __device__ __forceinline__ void run_stream_tasks(const SecDesc* __restrict__ sec
   const uint32_t nw = gridDim.x * kWarps;
   int cur = -1;
   for (uint32_t task = blockIdx.x * kWarps + wib; task < wl.n_tasks; task += nw) {
-    const int j = find_item(wl.begin, wl.n_items, task, lane);
+    const int j = find_item(wl.begin, 0, wl.n_items, task, lane);
     if (j != cur) {
       __syncwarp();
       const SecDesc* src = &secs[__ldg(wl.ids + j)];
@@ -425,6 +428,20 @@ struct BulkShape {
 // restore took twice as long).
 constexpr int kContigPieces = 8;
 static_assert(kTileBytes / kContigPieces % 16 == 0 && kContigPieces <= 32, "pieces");
+// Work sharing of the TMA kernel.  With static ranges alone, warps given
+// equal tile counts finish up to 10-25 % apart (a per-warp %globaltimer
+// probe: 4,096 Markov sessions 226-263 us, median 236; 64 banks 69-92 us,
+// median 79).  A launch of fewer than kDynMaxTilesPerWarp tiles per warp
+// runs k_bulk_shared: 1 / kDynShare of its tiles (the last ones) are handed
+// out at run time, in chunks of up to kDynChunkMax tiles, about
+// kDynGrabsPerWarp per warp.  Measured (alternating builds, one box): the
+// 64-bank step 0.273 -> 0.261 ms; at 84 tiles per warp (4,096 Markov
+// sessions) no change; at 2,587 (the 256-session KV step) sharing 1/4 or 1/8
+// made the step 0.7-1.5 % slower, so large launches keep static ranges.
+constexpr uint32_t kDynMaxTilesPerWarp = 64;
+constexpr uint32_t kDynShare = 8;
+constexpr uint32_t kDynGrabsPerWarp = 8;
+constexpr uint32_t kDynChunkMax = 32;
 constexpr int kTileRows = 32;  // rows >= 512 bytes touching an 8 KiB tile: at most 17
 constexpr long long kWaitCycles = 4000000000ll;  // give up a wait after ~2 s of SM clock
 static_assert(kTileBytes / kBulkMinRowBytes + 1 <= kTileRows, "tile rows");
@@ -647,11 +664,100 @@ __device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, con
   issue_runs<true>(st, rp, pe, tile, bar, lane);
 }
 
+// One staged tile whose loads have landed: complete it, issue its stores
+// (one bulk group), fold its chunks into the fingerprint and write its node.
+// Returns whether stores were issued.  Called by a whole warp.
+template <int MODE>
+__device__ __forceinline__ bool bulk_tile(const WarpStage& m, uint8_t* tile,
+                                          uint64_t* __restrict__ nodes, int lane) {
+  using T = ModeTraits<MODE>;
+  const uint4 zero = make_uint4(0, 0, 0, 0);
+  const SecDesc& s = m.d;
+  const uint64_t L = s.bytes, p0 = m.p0, p1 = m.p1;
+  const uint64_t pe = staged_end<MODE>(s, p1);
+  // Complete the tile: [pe, p1) holds the stream's unaligned tail (layout
+  // side) and zeros past its end.
+  for (uint64_t o = pe + 16u * lane; o < p1; o += 512u) {
+    uint4 v = zero;
+    if (T::kLoadLayout && o < L) {
+      const uint64_t left = L - o;
+      v = ld_small(s.lbase + o, left < 16 ? static_cast<int>(left) : 16, true);
+    }
+    *reinterpret_cast<uint4*>(tile + (o - p0)) = v;
+  }
+  if (!T::kLoadLayout && (L & 15u) && L >= p0 && L < p1 && lane == 0) {
+    // Restore: payload bytes past the logical end read as zero.
+    const uint64_t o = L & ~15ull;
+    uint4* q = reinterpret_cast<uint4*>(tile + (o - p0));
+    *q = mask_tail(*q, static_cast<int>(L - o));
+  }
+  fence_async_smem();
+  __syncwarp();
+  bool issued = false;
+  if (MODE == kModePack) {
+    // Contiguous payload, through the record's 256-byte padding.
+    const uint64_t padded = (L + kRecordAlign - 1) / kRecordAlign * kRecordAlign;
+    const uint64_t se = p1 < padded ? p1 : padded;
+    if (lane == 0 && se > p0) {
+      bulk_s2g(s.payload + p0, tile, static_cast<uint32_t>(se - p0));
+      bulk_commit();
+      issued = true;
+    }
+  } else if (MODE == kModeRestore || MODE == kModeRestoreV) {
+    const uint64_t lim = L < p1 ? L : p1;
+    if (s.layout == kContig) {
+      const uint64_t vend = lim & ~15ull;  // whole segments by bulk copy
+      if (lane == 0 && vend > p0) {
+        bulk_s2g(s.lbase + p0, tile, static_cast<uint32_t>(vend - p0));
+        bulk_commit();
+        issued = true;
+      }
+      for (uint64_t o = (vend > p0 ? vend : p0) + lane; o < lim; o += 32) s.lbase[o] = tile[o - p0];
+    } else {
+      uint8_t* rp = m.rowp[lane];
+      if (issue_runs<false>(m, rp, lim, tile, nullptr, lane)) {
+        bulk_commit();
+        issued = true;
+      }
+    }
+  }
+  if (T::kHash) {
+    // The tile's chunks, interleaved lane chains, read from shared memory.
+    const uint64_t c0 = p0 / kChunkBytes;
+    const int nc = static_cast<int>((p1 - p0) / kChunkBytes);
+    uint64_t h[kTileChunks];
+#pragma unroll
+    for (int q = 0; q < kTileChunks; ++q) h[q] = fmix(kSeed ^ ((c0 + q) * 32u + lane));
+#pragma unroll
+    for (int k = 0; k < kSegs; ++k) {
+#pragma unroll
+      for (int q = 0; q < kTileChunks; ++q) {
+        const uint4 v = q < nc ? *reinterpret_cast<const uint4*>(tile + q * kChunkBytes + 512 * k + 16 * lane)
+                               : zero;
+        h[q] = absorb(h[q], v);
+      }
+    }
+    // Moving passes are bound by DRAM; one tree per chunk paces the warps
+    // so that loads and stores interleave best (measured: the shared tree
+    // of tile_tree2 makes pack and restore slower).
+    uint64_t mine = 0;
+#pragma unroll
+    for (int q = 0; q < kTileChunks; ++q) {
+      const uint64_t x = __shfl_sync(kFull, warp_tree(fmix(h[q]), 32, lane), 0);
+      if (lane == q) mine = x;
+    }
+    const uint64_t root = warp_tree(mine, nc, lane);
+    if (lane == 0) nodes[m.node] = root;
+  }
+  return issued;
+}
+
+// The TMA kernel with static work: each warp moves a contiguous, balanced
+// range of the launch's tiles, kWarpStages in flight.
 template <int MODE>
 __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     k_bulk(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
            uint32_t* err) {
-  using T = ModeTraits<MODE>;
   constexpr int kBulkWarps = BulkShape<MODE>::kWarps;
   constexpr int kWarpStages = BulkShape<MODE>::kStages;
   extern __shared__ __align__(128) uint8_t smem_raw[];
@@ -672,7 +778,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
   const uint32_t t0 = static_cast<uint32_t>(T_all * gw / nw);
   const uint32_t t1 = static_cast<uint32_t>(T_all * (gw + 1) / nw);
   if (t0 >= t1) return;
-  int item = find_item(wl.begin, wl.n_items, t0, lane);  // item of the next tile to stage
+  int item = find_item(wl.begin, 0, wl.n_items, t0, lane);  // item of the next tile to stage
   auto item_of = [&](uint32_t t) {
     while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= t) ++item;
     return item;
@@ -681,7 +787,6 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
   for (int k = 0; k < pre; ++k)
     stage_tile<MODE>(secs, wl, item_of(t0 + k), t0 + k, sh.st[warp][k], sh.buf[warp][k],
                      &sh.bar[warp][k], err, lane);
-  const uint4 zero = make_uint4(0, 0, 0, 0);
   bool any_issued = false;
   for (uint32_t i = 0; t0 + i < t1; ++i) {
     const int sidx = static_cast<int>(i % kWarpStages);
@@ -696,84 +801,7 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
       if (lane == 0) atomicOr(err, kDevErrTimeout);
       break;
     }
-    const SecDesc& s = m.d;
-    const uint64_t L = s.bytes, p0 = m.p0, p1 = m.p1;
-    const uint64_t pe = staged_end<MODE>(s, p1);
-    // Complete the tile: [pe, p1) holds the stream's unaligned tail (layout
-    // side) and zeros past its end.
-    for (uint64_t o = pe + 16u * lane; o < p1; o += 512u) {
-      uint4 v = zero;
-      if (T::kLoadLayout && o < L) {
-        const uint64_t left = L - o;
-        v = ld_small(s.lbase + o, left < 16 ? static_cast<int>(left) : 16, true);
-      }
-      *reinterpret_cast<uint4*>(tile + (o - p0)) = v;
-    }
-    if (!T::kLoadLayout && (L & 15u) && L >= p0 && L < p1 && lane == 0) {
-      // Restore: payload bytes past the logical end read as zero.
-      const uint64_t o = L & ~15ull;
-      uint4* q = reinterpret_cast<uint4*>(tile + (o - p0));
-      *q = mask_tail(*q, static_cast<int>(L - o));
-    }
-    fence_async_smem();
-    __syncwarp();
-    bool issued = false;
-    if (MODE == kModePack) {
-      // Contiguous payload, through the record's 256-byte padding.
-      const uint64_t padded = (L + kRecordAlign - 1) / kRecordAlign * kRecordAlign;
-      const uint64_t se = p1 < padded ? p1 : padded;
-      if (lane == 0 && se > p0) {
-        bulk_s2g(s.payload + p0, tile, static_cast<uint32_t>(se - p0));
-        bulk_commit();
-        issued = true;
-      }
-    } else if (MODE == kModeRestore || MODE == kModeRestoreV) {
-      const uint64_t lim = L < p1 ? L : p1;
-      if (s.layout == kContig) {
-        const uint64_t vend = lim & ~15ull;  // whole segments by bulk copy
-        if (lane == 0 && vend > p0) {
-          bulk_s2g(s.lbase + p0, tile, static_cast<uint32_t>(vend - p0));
-          bulk_commit();
-          issued = true;
-        }
-        for (uint64_t o = (vend > p0 ? vend : p0) + lane; o < lim; o += 32) s.lbase[o] = tile[o - p0];
-      } else {
-        uint8_t* rp = m.rowp[lane];
-        if (issue_runs<false>(m, rp, lim, tile, nullptr, lane)) {
-          bulk_commit();
-          issued = true;
-        }
-      }
-    }
-    if (T::kHash) {
-      // The tile's chunks, interleaved lane chains, read from shared memory.
-      const uint64_t c0 = p0 / kChunkBytes;
-      const int nc = static_cast<int>((p1 - p0) / kChunkBytes);
-      uint64_t h[kTileChunks];
-#pragma unroll
-      for (int q = 0; q < kTileChunks; ++q) h[q] = fmix(kSeed ^ ((c0 + q) * 32u + lane));
-#pragma unroll
-      for (int k = 0; k < kSegs; ++k) {
-#pragma unroll
-        for (int q = 0; q < kTileChunks; ++q) {
-          const uint4 v = q < nc ? *reinterpret_cast<const uint4*>(tile + q * kChunkBytes + 512 * k + 16 * lane)
-                                 : zero;
-          h[q] = absorb(h[q], v);
-        }
-      }
-      // Moving passes are bound by DRAM; one tree per chunk paces the warps
-      // so that loads and stores interleave best (measured: the shared tree
-      // of tile_tree2 makes pack and restore slower).
-      uint64_t mine = 0;
-#pragma unroll
-      for (int q = 0; q < kTileChunks; ++q) {
-        const uint64_t x = __shfl_sync(kFull, warp_tree(fmix(h[q]), 32, lane), 0);
-        if (lane == q) mine = x;
-      }
-      const uint64_t root = warp_tree(mine, nc, lane);
-      if (lane == 0) nodes[m.node] = root;
-    }
-    if (issued) {
+    if (bulk_tile<MODE>(m, tile, nodes, lane)) {
       bulk_wait_read();
       any_issued = true;
     }
@@ -783,6 +811,123 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     if (tn < t1) stage_tile<MODE>(secs, wl, item_of(tn), tn, m, tile, bar, err, lane);
   }
   if (any_issued) bulk_wait_all();
+}
+
+// The TMA kernel with shared work, for launches of fewer than
+// kDynMaxTilesPerWarp tiles per warp: each warp first moves a contiguous,
+// balanced range of the first T_static tiles, then chunks of the rest
+// [T_static, T_all) handed out by an atomic counter (sched[0]) to whichever
+// warp asks first, so that warps that drew slower memory do not hold up the
+// end of the launch.  sched[0..1] are zero on entry; the last warp to finish
+// sets them back to zero.
+template <int MODE>
+__global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
+    k_bulk_shared(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
+                  uint32_t* err, uint32_t* sched) {
+  constexpr int kBulkWarps = BulkShape<MODE>::kWarps;
+  constexpr int kWarpStages = BulkShape<MODE>::kStages;
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  auto& sh = *reinterpret_cast<BulkShared<kBulkWarps, kWarpStages>*>(smem_raw);
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  if (lane < kWarpStages) {
+    mbar_init(&sh.bar[warp][lane], 1);
+    sh.st[warp][lane].sec = 0xFFFFFFFFu;
+  }
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  __syncwarp();
+
+  const uint32_t T_all = wl.n_tasks;
+  const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kBulkWarps + warp;
+  const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kBulkWarps;
+  const uint32_t T_dyn = T_all / kDynShare;
+  const uint32_t T_static = T_all - T_dyn;
+  const uint64_t per = T_dyn / (nw * kDynGrabsPerWarp);
+  const uint32_t chunk = static_cast<uint32_t>(per < 1 ? 1 : (per > kDynChunkMax ? kDynChunkMax : per));
+  const uint32_t t0 = static_cast<uint32_t>(T_static * gw / nw);
+  const uint32_t t1 = static_cast<uint32_t>(T_static * (gw + 1) / nw);
+  uint32_t next = t0, chunk_end = t1;  // tiles [next, chunk_end) are this warp's
+  int item = find_item(wl.begin, 0, wl.n_items, t0, lane);  // item of the last tile taken
+  // The next chunk, reserved ahead of need (where the warp would wait on a
+  // stage anyway) so that neither the atomic nor the search of its item
+  // delays a refill.
+  bool reserved = false, drained = false;
+  uint32_t res_next = 0, res_end = 0;
+  int res_item = 0;
+  auto reserve = [&]() {
+    if (reserved || drained) return;
+    uint32_t g = 0;
+    if (lane == 0) g = atomicAdd(sched, chunk);
+    g = __shfl_sync(kFull, g, 0);
+    if (g >= T_dyn) {
+      drained = true;
+      return;
+    }
+    res_next = T_static + g;
+    res_end = T_static + (g + chunk < T_dyn ? g + chunk : T_dyn);
+    res_item = item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= res_next
+                   ? find_item(wl.begin, item, wl.n_items, res_next, lane)
+                   : item;
+    reserved = true;
+  };
+  // The next tile of this warp (and `item`, its item); false once none is left.
+  auto take = [&](uint32_t* t) -> bool {
+    if (next >= chunk_end) {
+      reserve();
+      if (!reserved) return false;
+      next = res_next;
+      chunk_end = res_end;
+      item = res_item;
+      reserved = false;
+    }
+    *t = next++;
+    while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= *t) ++item;
+    return true;
+  };
+  int staged = 0;
+  for (int k = 0; k < kWarpStages; ++k) {
+    uint32_t t;
+    if (!take(&t)) break;
+    stage_tile<MODE>(secs, wl, item, t, sh.st[warp][k], sh.buf[warp][k], &sh.bar[warp][k], err,
+                     lane);
+    ++staged;
+  }
+  bool any_issued = false;
+  for (int i = 0; i < staged; ++i) {
+    const int sidx = i % kWarpStages;
+    const uint32_t use = static_cast<uint32_t>(i) / kWarpStages;
+    uint64_t* bar = &sh.bar[warp][sidx];
+    uint8_t* tile = sh.buf[warp][sidx];
+    WarpStage& m = sh.st[warp][sidx];
+    if (next + 1 >= chunk_end) reserve();  // the refill after next needs a new chunk
+    bool ok = true;
+    if (lane == 0) ok = mbar_wait(bar, use & 1);
+    ok = __shfl_sync(kFull, ok, 0);
+    if (!ok) {
+      if (lane == 0) atomicOr(err, kDevErrTimeout);
+      break;
+    }
+    if (bulk_tile<MODE>(m, tile, nodes, lane)) {
+      bulk_wait_read();
+      any_issued = true;
+    }
+    __syncwarp();
+    // Reuse the stage for this warp's next tile.
+    uint32_t tn;
+    if (take(&tn)) {
+      stage_tile<MODE>(secs, wl, item, tn, m, tile, bar, err, lane);
+      ++staged;
+    }
+  }
+  if (any_issued) bulk_wait_all();
+  // The last warp out leaves the counters at zero for the next launch.
+  if (lane == 0) {
+    __threadfence();
+    if (atomicAdd(sched + 1, 1u) == static_cast<uint32_t>(nw) - 1) {
+      atomicExch(sched, 0u);
+      atomicExch(sched + 1, 0u);
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -815,7 +960,7 @@ __global__ void __launch_bounds__(kHashThreads, 1)
   const uint32_t t0 = static_cast<uint32_t>(T_all * gw / nw);
   const uint32_t t1 = static_cast<uint32_t>(T_all * (gw + 1) / nw);
   if (t0 >= t1) return;
-  int item = find_item(wl.begin, wl.n_items, t0, lane);
+  int item = find_item(wl.begin, 0, wl.n_items, t0, lane);
   for (uint32_t t = t0; t < t1; ++t) {
     while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= t) ++item;
     const SecDesc* s = secs + __ldg(wl.ids + item);
@@ -2661,7 +2806,7 @@ int resident_blocks(const void* kernel) {
 
 template <int MODE>
 cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, uint32_t* err,
-                             int sm_count, cudaStream_t stream) {
+                             uint32_t* sched, int sm_count, cudaStream_t stream) {
   using Shape = BulkShape<MODE>;
   const size_t smem = sizeof(BulkShared<Shape::kWarps, Shape::kStages>);
   static uint64_t configured = 0;  // one bit per device (callers hold the context lock)
@@ -2672,12 +2817,18 @@ cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, 
   if (!(configured & bit)) {
     e = cudaFuncSetAttribute(k_bulk<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k_bulk_shared<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     configured |= bit;
   }
   const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + Shape::kWarps - 1) / Shape::kWarps;
   const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
-  k_bulk<MODE><<<blocks, Shape::kThreads, smem, stream>>>(secs, wl, nodes, err);
+  if (wl.n_tasks < static_cast<uint64_t>(kDynMaxTilesPerWarp) * blocks * Shape::kWarps)
+    k_bulk_shared<MODE><<<blocks, Shape::kThreads, smem, stream>>>(secs, wl, nodes, err, sched);
+  else
+    k_bulk<MODE><<<blocks, Shape::kThreads, smem, stream>>>(secs, wl, nodes, err);
   return cudaGetLastError();
 }
 
@@ -2714,7 +2865,7 @@ cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_
 }
 
 cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* nodes,
-                        uint32_t* dev_err, int sm_count, cudaStream_t stream) {
+                        uint32_t* dev_err, uint32_t* sched, int sm_count, cudaStream_t stream) {
   if (wl.n_tasks == 0) return cudaSuccess;
   switch (mode) {
     case kModeHash: {
@@ -2723,11 +2874,11 @@ cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* no
       k_hash<<<blocks, kHashThreads, 0, stream>>>(secs, wl, nodes);
       return cudaGetLastError();
     }
-    case kModePack: return launch_bulk_mode<kModePack>(secs, wl, nodes, dev_err, sm_count, stream);
+    case kModePack: return launch_bulk_mode<kModePack>(secs, wl, nodes, dev_err, sched, sm_count, stream);
     case kModeRestore:
-      return launch_bulk_mode<kModeRestore>(secs, wl, nodes, dev_err, sm_count, stream);
+      return launch_bulk_mode<kModeRestore>(secs, wl, nodes, dev_err, sched, sm_count, stream);
     case kModeRestoreV:
-      return launch_bulk_mode<kModeRestoreV>(secs, wl, nodes, dev_err, sm_count, stream);
+      return launch_bulk_mode<kModeRestoreV>(secs, wl, nodes, dev_err, sched, sm_count, stream);
     default: return cudaErrorInvalidValue;
   }
 }

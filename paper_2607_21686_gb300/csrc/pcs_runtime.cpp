@@ -343,7 +343,8 @@ struct pcs_ctx {
   std::unordered_set<pcs_snapshot*> live;
   // Workspaces, one per stream: the descriptors and tree nodes of a call,
   // after a header of per-call device words ([0] the fused kernel's ticket,
-  // [1] failures of a verify = 1 restore).  Calls on one stream are ordered
+  // [1] failures of a verify = 1 restore, [4] and [5] the TMA kernel's work
+  // sharing).  Calls on one stream are ordered
   // by the stream; calls on different streams do not share one, so they can
   // run side by side.
   struct Workspace {
@@ -464,6 +465,11 @@ Arena* arena_of(pcs_ctx* c, uint32_t placement) {
 }
 
 constexpr uint64_t kWsHeader = 256;  // per-call device words before the descriptors
+constexpr int kWordBulkSched = 4;    // header words [4], [5]: the TMA kernel's work sharing
+
+// The header words of a call: they sit just below its descriptors, in a
+// stream's workspace and in a prepared call's buffer alike.
+uint32_t* header_words(uint8_t* ws) { return reinterpret_cast<uint32_t*>(ws - kWsHeader); }
 
 // The workspace of `stream` for the call in progress: grown if needed (after
 // its last call has finished), else `stream` waits for its last call (a no-op
@@ -945,7 +951,8 @@ cudaError_t launch_streams(pcs_ctx* c, int mode, const SecDesc* dsecs, const Str
                 reinterpret_cast<const uint32_t*>(ws + L.bulk_begin),
                 static_cast<int>(P.bulk_ids.size()), P.bulk_tasks};
     LaunchScope ls(c, bulk_kind(mode), stream);
-    e = launch_bulk(mode, dsecs, wl, nodes, c->words, c->sm_count, stream);
+    e = launch_bulk(mode, dsecs, wl, nodes, c->words, header_words(ws) + kWordBulkSched, c->sm_count,
+                    stream);
     if (e != cudaSuccess) return e;
   }
   if (P.reg_tasks) {

@@ -258,8 +258,16 @@ def check(status: int, where: str) -> None:
         raise PcsError(status, where)
 
 
+_current_raw_stream = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
 def _stream_ptr(stream) -> int:
+    """The cudaStream_t of `stream` (a torch stream or an integer handle);
+    None means torch's current stream on the current device, read without
+    building a Stream object (a few microseconds per call otherwise)."""
     if stream is None:
+        if _current_raw_stream is not None:
+            return int(_current_raw_stream(torch.cuda.current_device()))
         stream = torch.cuda.current_stream()
     return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
 
