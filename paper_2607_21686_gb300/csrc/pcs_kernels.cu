@@ -69,6 +69,17 @@ __device__ __forceinline__ uint64_t comb(uint64_t a, uint64_t b) {
   return fmix(a * kP + rotl64(b, 31));
 }
 
+// Programmatic dependent launch (sm_90 and later).  The streaming, finalising,
+// scoring and top-k kernels are launched with programmatic stream
+// serialisation (launch_after), so the GPU may schedule one while the kernel
+// before it on the stream is still finishing.  Each begins here: wait until
+// that kernel has completed and its writes are visible, then let the next
+// kernel be scheduled.  Nothing before this point touches global memory.
+__device__ __forceinline__ void grid_dependency() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // Absorb one 16-byte segment (two little-endian words) into a lane chain.
 __device__ __forceinline__ uint64_t absorb(uint64_t h, uint4 v) {
   const uint64_t w0 = static_cast<uint64_t>(v.x) | (static_cast<uint64_t>(v.y) << 32);
@@ -387,6 +398,7 @@ template <int MODE>
 __global__ void __launch_bounds__(kThreads, 2)
     k_stream(const SecDesc* __restrict__ secs, WorkList wl, int glog2,
              uint64_t* __restrict__ nodes, uint32_t* err) {
+  grid_dependency();
   __shared__ SecDesc sdesc[kWarps];
   run_stream_tasks<MODE>(secs, wl, glog2, nodes, err, sdesc);
 }
@@ -758,6 +770,7 @@ template <int MODE>
 __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     k_bulk(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
            uint32_t* err) {
+  grid_dependency();
   constexpr int kBulkWarps = BulkShape<MODE>::kWarps;
   constexpr int kWarpStages = BulkShape<MODE>::kStages;
   extern __shared__ __align__(128) uint8_t smem_raw[];
@@ -824,6 +837,7 @@ template <int MODE>
 __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     k_bulk_shared(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
                   uint32_t* err, uint32_t* sched) {
+  grid_dependency();
   constexpr int kBulkWarps = BulkShape<MODE>::kWarps;
   constexpr int kWarpStages = BulkShape<MODE>::kStages;
   extern __shared__ __align__(128) uint8_t smem_raw[];
@@ -951,6 +965,7 @@ constexpr int kHashThreads = 32 * kHashWarps;
 
 __global__ void __launch_bounds__(kHashThreads, 1)
     k_hash(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes) {
+  grid_dependency();
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   // This warp's tiles: a contiguous, balanced range [t0, t1).
@@ -1011,6 +1026,7 @@ __device__ __forceinline__ uint64_t stream_fp(const SecDesc& s, uint64_t* nodes,
 __global__ void __launch_bounds__(kThreads)
     k_reduce_nodes(const NodeLevel* __restrict__ lv, int n_secs, uint64_t* nodes, uint32_t base,
                    uint32_t n_groups) {
+  grid_dependency();
   const int lane = threadIdx.x & 31;
   const uint32_t nw = gridDim.x * kWarps;
   for (uint32_t g = blockIdx.x * kWarps + (threadIdx.x >> 5); g < n_groups; g += nw) {
@@ -1049,6 +1065,7 @@ __device__ __forceinline__ void finalize_hash_warps(const SecDesc* __restrict__ 
 __global__ void __launch_bounds__(kThreads)
     k_finalize_hash(const SecDesc* __restrict__ secs, int n_secs, uint64_t* nodes,
                     uint64_t* fp_out, const uint64_t* fp_before, uint8_t* flags) {
+  grid_dependency();
   finalize_hash_warps(secs, n_secs, nodes, fp_out, fp_before, flags,
                       blockIdx.x * kWarps + (threadIdx.x >> 5), gridDim.x * kWarps);
 }
@@ -1143,6 +1160,7 @@ __global__ void __launch_bounds__(512)
     k_finalize_sessions(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
                         int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
                         uint8_t* corrupt, uint32_t* bad) {
+  grid_dependency();
   __shared__ uint64_t smem[kMaxSmemFps];
   __shared__ uint32_t s_bad;
   finalize_sessions_block<MODE>(secs, sess, n_sess, entries, nodes, corrupt, bad, blockIdx.x,
@@ -1156,6 +1174,7 @@ __global__ void __launch_bounds__(kThreads)
     k_finalize_sessions_warp(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
                              int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
                              uint8_t* corrupt, uint32_t* bad) {
+  grid_dependency();
   const int lane = threadIdx.x & 31;
   const int nw = gridDim.x * kWarps;
   for (int b = blockIdx.x * kWarps + (threadIdx.x >> 5); b < n_sess; b += nw) {
@@ -1218,6 +1237,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             uint32_t* err, uint32_t* ticket, int n_items, const SessDesc* __restrict__ sess,
             const Entry* __restrict__ entries, uint64_t* fp_out, const uint64_t* fp_before,
             uint8_t* flags, uint32_t* bad) {
+  grid_dependency();
   __shared__ SecDesc sdesc[kWarps];
   __shared__ uint64_t smem[64];  // up to 2048 sections per session
   __shared__ uint32_t s_bad;
@@ -1525,6 +1545,7 @@ template <int SPL, int DT, int HM>
 __global__ void __launch_bounds__(kThreads)
     k_score_fixed(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
                   float* __restrict__ scores, GHist gh) {
+  grid_dependency();
   __shared__ uint32_t s_cnt[HM ? kGBins : 1];
   __shared__ unsigned long long s_w[HM == 2 ? kGBins : 1];
   __shared__ bool s_last;
@@ -1545,6 +1566,7 @@ __global__ void __launch_bounds__(kThreads)
 __global__ void __launch_bounds__(kThreads)
     k_score_any(const BankDesc* __restrict__ banks, int n_banks, uint64_t n_entries,
                 float* __restrict__ scores) {
+  grid_dependency();
   const int lane = threadIdx.x & 31;
   const uint64_t gw = static_cast<uint64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
   const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kWarps;
@@ -1721,6 +1743,7 @@ __device__ void topk_bank_reg(const float* __restrict__ sc, int n, int k, int32_
 __global__ void __launch_bounds__(kThreads)
     k_topk(const BankDesc* __restrict__ banks, int n_banks, const float* __restrict__ scores,
            int32_t* __restrict__ kept_idx) {
+  grid_dependency();
   __shared__ uint32_t hist[256];
   __shared__ uint32_t warp_cnt[kWarps];
   __shared__ uint32_t s_prefix, s_mask, s_remaining;
@@ -2775,6 +2798,27 @@ __global__ void k_selftest_wait(int which, const uint32_t* never_set, uint32_t* 
   if (!ok) atomicOr(err, kDevErrTimeout);
 }
 
+// Launch `k` with programmatic stream serialisation: the GPU may schedule it
+// while the kernel before it on `stream` finishes (its blocks wait in
+// grid_dependency() until that kernel's writes are visible), instead of only
+// after that kernel has retired.  After a copy, an event or another kind of
+// stream operation the launch waits as usual.
+template <typename... P, typename... A>
+cudaError_t launch_after(void (*k)(P...), unsigned grid, unsigned block, size_t smem,
+                         cudaStream_t stream, A... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k, args...);
+}
+
 template <int MODE>
 int occupancy() {
   int b = 0;
@@ -2826,10 +2870,9 @@ cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, 
   const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + Shape::kWarps - 1) / Shape::kWarps;
   const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
   if (wl.n_tasks < static_cast<uint64_t>(kDynMaxTilesPerWarp) * blocks * Shape::kWarps)
-    k_bulk_shared<MODE><<<blocks, Shape::kThreads, smem, stream>>>(secs, wl, nodes, err, sched);
-  else
-    k_bulk<MODE><<<blocks, Shape::kThreads, smem, stream>>>(secs, wl, nodes, err);
-  return cudaGetLastError();
+    return launch_after(k_bulk_shared<MODE>, blocks, Shape::kThreads, smem, stream, secs, wl, nodes,
+                        err, sched);
+  return launch_after(k_bulk<MODE>, blocks, Shape::kThreads, smem, stream, secs, wl, nodes, err);
 }
 
 }  // namespace
@@ -2847,21 +2890,20 @@ cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_
   const int blocks = static_cast<int>(want < cap ? want : cap);
   switch (mode) {
     case kModeHash:
-      k_stream<kModeHash><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
-      break;
+      return launch_after(k_stream<kModeHash>, blocks, kThreads, 0, stream, secs, wl, group_log2,
+                          nodes, dev_err);
     case kModePack:
-      k_stream<kModePack><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
-      break;
+      return launch_after(k_stream<kModePack>, blocks, kThreads, 0, stream, secs, wl, group_log2,
+                          nodes, dev_err);
     case kModeRestore:
-      k_stream<kModeRestore><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
-      break;
+      return launch_after(k_stream<kModeRestore>, blocks, kThreads, 0, stream, secs, wl,
+                          group_log2, nodes, dev_err);
     case kModeRestoreV:
-      k_stream<kModeRestoreV><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err);
-      break;
+      return launch_after(k_stream<kModeRestoreV>, blocks, kThreads, 0, stream, secs, wl,
+                          group_log2, nodes, dev_err);
     default:
       return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* nodes,
@@ -2871,8 +2913,7 @@ cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* no
     case kModeHash: {
       const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + kHashWarps - 1) / kHashWarps;
       const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
-      k_hash<<<blocks, kHashThreads, 0, stream>>>(secs, wl, nodes);
-      return cudaGetLastError();
+      return launch_after(k_hash, blocks, kHashThreads, 0, stream, secs, wl, nodes);
     }
     case kModePack: return launch_bulk_mode<kModePack>(secs, wl, nodes, dev_err, sched, sm_count, stream);
     case kModeRestore:
@@ -2894,24 +2935,20 @@ cudaError_t launch_small(int mode, const SecDesc* secs, WorkList wl, int group_l
   const int blocks = static_cast<int>(want < cap ? want : cap);
   switch (mode) {
     case kModeHash:
-      k_small<kModeHash><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err, ticket,
-                                                          n_items, sess, entries, fp_out, fp_before,
-                                                          flags, bad);
-      break;
+      return launch_after(k_small<kModeHash>, blocks, kThreads, 0, stream, secs, wl, group_log2,
+                          nodes, dev_err, ticket, n_items, sess, entries, fp_out, fp_before, flags,
+                          bad);
     case kModePack:
-      k_small<kModePack><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err, ticket,
-                                                          n_items, sess, entries, fp_out, fp_before,
-                                                          flags, bad);
-      break;
+      return launch_after(k_small<kModePack>, blocks, kThreads, 0, stream, secs, wl, group_log2,
+                          nodes, dev_err, ticket, n_items, sess, entries, fp_out, fp_before, flags,
+                          bad);
     case kModeRestoreV:
-      k_small<kModeRestoreV><<<blocks, kThreads, 0, stream>>>(secs, wl, group_log2, nodes, dev_err,
-                                                              ticket, n_items, sess, entries, fp_out,
-                                                              fp_before, flags, bad);
-      break;
+      return launch_after(k_small<kModeRestoreV>, blocks, kThreads, 0, stream, secs, wl,
+                          group_log2, nodes, dev_err, ticket, n_items, sess, entries, fp_out,
+                          fp_before, flags, bad);
     default:
       return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess, int n_sess,
@@ -2924,34 +2961,30 @@ cudaError_t launch_finalize(int mode, const SecDesc* secs, const SessDesc* sess,
     const int want = (n_sess + kWarps - 1) / kWarps;
     const int blocks = want < 65535 ? want : 65535;
     if (mode == kModePack)
-      k_finalize_sessions_warp<kModePack><<<blocks, kThreads, 0, stream>>>(secs, sess, n_sess,
-                                                                          entries, nodes, flags, bad);
-    else if (mode == kModeRestoreV)
-      k_finalize_sessions_warp<kModeRestoreV><<<blocks, kThreads, 0, stream>>>(
-          secs, sess, n_sess, entries, nodes, flags, bad);
-    else
-      return cudaErrorInvalidValue;
-    return cudaGetLastError();
+      return launch_after(k_finalize_sessions_warp<kModePack>, blocks, kThreads, 0, stream, secs,
+                          sess, n_sess, entries, nodes, flags, bad);
+    if (mode == kModeRestoreV)
+      return launch_after(k_finalize_sessions_warp<kModeRestoreV>, blocks, kThreads, 0, stream,
+                          secs, sess, n_sess, entries, nodes, flags, bad);
+    return cudaErrorInvalidValue;
   }
   if (mode == kModeHash) {
     const int blocks = (n_sess + kWarps - 1) / kWarps;
-    k_finalize_hash<<<blocks < 4096 ? blocks : 4096, kThreads, 0, stream>>>(secs, n_sess, nodes, fp_out,
-                                                                            fp_before, flags);
-  } else if (mode == kModePack || mode == kModeRestoreV) {
+    return launch_after(k_finalize_hash, blocks < 4096 ? blocks : 4096, kThreads, 0, stream, secs,
+                        n_sess, nodes, fp_out, fp_before, flags);
+  }
+  if (mode == kModePack || mode == kModeRestoreV) {
     // A block per session, a warp per section (up to 16 at once: two
     // blocks of 64-register threads fit an SM).
     const int warps = max_secs < 8 ? 8 : max_secs > 16 ? 16 : max_secs;
     const int blocks = n_sess < 65535 ? n_sess : 65535;
     if (mode == kModePack)
-      k_finalize_sessions<kModePack><<<blocks, 32 * warps, 0, stream>>>(secs, sess, n_sess, entries,
-                                                                       nodes, flags, bad);
-    else
-      k_finalize_sessions<kModeRestoreV><<<blocks, 32 * warps, 0, stream>>>(
-          secs, sess, n_sess, entries, nodes, flags, bad);
-  } else {
-    return cudaErrorInvalidValue;
+      return launch_after(k_finalize_sessions<kModePack>, blocks, 32 * warps, 0, stream, secs, sess,
+                          n_sess, entries, nodes, flags, bad);
+    return launch_after(k_finalize_sessions<kModeRestoreV>, blocks, 32 * warps, 0, stream, secs,
+                        sess, n_sess, entries, nodes, flags, bad);
   }
-  return cudaGetLastError();
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_reduce_nodes(const NodeLevel* lv, int n_secs, uint64_t* nodes, uint32_t base,
@@ -2960,8 +2993,7 @@ cudaError_t launch_reduce_nodes(const NodeLevel* lv, int n_secs, uint64_t* nodes
   const uint64_t want = (static_cast<uint64_t>(n_groups) + kWarps - 1) / kWarps;
   const uint64_t cap = static_cast<uint64_t>(sm_count) * 8;
   const int blocks = static_cast<int>(want < cap ? want : cap);
-  k_reduce_nodes<<<blocks, kThreads, 0, stream>>>(lv, n_secs, nodes, base, n_groups);
-  return cudaGetLastError();
+  return launch_after(k_reduce_nodes, blocks, kThreads, 0, stream, lv, n_secs, nodes, base, n_groups);
 }
 
 cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries, int max_dim,
@@ -2977,15 +3009,16 @@ cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
   };
   // key_types: 0 = all fp16, 1 = all bf16, 2 = mixed.
   if (key_types == 2 || max_dim > 1024) {
-    k_score_any<<<grid(reinterpret_cast<const void*>(k_score_any)), kThreads, 0, stream>>>(
-        banks, n_banks, n_entries, scores);
-    return cudaGetLastError();
+    return launch_after(k_score_any, grid(reinterpret_cast<const void*>(k_score_any)), kThreads, 0,
+                        stream, banks, n_banks, n_entries, scores);
   }
   const int spl = max_dim <= 256 ? 1 : max_dim <= 512 ? 2 : 4;
   const int hm = gh.st ? gh.mode : 0;
-#define PCS_SCORE(S, D, H)                                                                    \
-  k_score_fixed<S, D, H><<<grid(reinterpret_cast<const void*>(k_score_fixed<S, D, H>)), kThreads, \
-                           0, stream>>>(banks, n_banks, n_entries, scores, gh)
+  cudaError_t e = cudaSuccess;
+#define PCS_SCORE(S, D, H)                                                                      \
+  e = launch_after(k_score_fixed<S, D, H>,                                                      \
+                   grid(reinterpret_cast<const void*>(k_score_fixed<S, D, H>)), kThreads, 0, stream, \
+                   banks, n_banks, n_entries, scores, gh)
 #define PCS_SCORE_H(S, D) (hm == 0 ? PCS_SCORE(S, D, 0) : hm == 1 ? PCS_SCORE(S, D, 1) : PCS_SCORE(S, D, 2))
   if (key_types == 1) {
     if (spl == 1) PCS_SCORE_H(1, 1);
@@ -2998,16 +3031,15 @@ cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
   }
 #undef PCS_SCORE_H
 #undef PCS_SCORE
-  if (fused) *fused = hm != 0;
-  return cudaGetLastError();
+  if (fused) *fused = hm != 0 && e == cudaSuccess;
+  return e;
 }
 
 cudaError_t launch_topk(const BankDesc* banks, int n_banks, const float* scores,
                         int32_t* kept_idx, cudaStream_t stream) {
   if (n_banks <= 0) return cudaSuccess;
-  k_topk<<<n_banks < 65535 ? n_banks : 65535, kThreads, 0, stream>>>(banks, n_banks, scores,
-                                                                     kept_idx);
-  return cudaGetLastError();
+  return launch_after(k_topk, n_banks < 65535 ? n_banks : 65535, kThreads, 0, stream, banks,
+                      n_banks, scores, kept_idx);
 }
 
 static int gblocks(const GPlan& p, int sm_count, const void* kernel) {
