@@ -1423,15 +1423,20 @@ __device__ __forceinline__ void score_range(const BankDesc* __restrict__ banks, 
   const uint64_t nw = static_cast<uint64_t>(gridDim.x) * kWarps;
   const uint64_t e_begin = n_entries * gw / nw, e_end = n_entries * (gw + 1) / nw;
   if (e_begin >= e_end) return;
+  // The last bank starting at or before e_begin, searched by the whole warp
+  // (32 probes a round, as in find_item).
   int b = 0;
   {
-    int lo = 0, hi = n_banks - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (__ldg(&banks[mid].entry_begin) <= e_begin) lo = mid;
-      else hi = mid - 1;
+    int span = n_banks;
+    while (span > 1) {
+      const int step = (span + 31) >> 5;
+      const int i = b + lane * step;
+      const bool le = i < b + span && __ldg(&banks[i].entry_begin) <= e_begin;
+      const unsigned m = __ballot_sync(kFull, le);  // lane 0 probes b: never empty
+      const int last = 31 - __clz(m);
+      b += last * step;
+      span = min(step, span - last * step);
     }
-    b = lo;
   }
   int qbank = -1, segs = 0;
   float qnorm = 0.f;
@@ -3001,8 +3006,10 @@ cudaError_t launch_score(const BankDesc* banks, int n_banks, uint64_t n_entries,
                          GHist gh, bool* fused) {
   if (fused) *fused = false;
   if (n_entries == 0) return cudaSuccess;
-  // At least eight rounds per warp; at most one resident wave.
-  const uint64_t want = (n_entries + kWarps * kScoreIlp * 8 - 1) / (kWarps * kScoreIlp * 8);
+  // At least two rounds of kScoreIlp entries per warp; at most one resident
+  // wave (large populations fill it).  Eight rounds per warp took the 64-bank
+  // population's score (16,164 entries) 15.5 us under ncu.
+  const uint64_t want = (n_entries + kWarps * kScoreIlp * 2 - 1) / (kWarps * kScoreIlp * 2);
   auto grid = [&](const void* k) {
     const uint64_t cap = static_cast<uint64_t>(sm_count) * resident_blocks(k);
     return static_cast<int>(want < cap ? want : cap);
