@@ -179,3 +179,28 @@ def test_small_unaligned_sources_in_large_calls(ctx, ctx_reg, dev):
         assert torch.equal(t, v)
     for sn in snaps:
         ctx.delete(sn)
+
+
+@pytest.mark.parametrize("sessions", [64, 2000, 3400])
+def test_markov_batches_static_and_shared_tma_kernels(ctx, dev, sessions):
+    """One checkpoint call of many Markov sessions, below and above the size
+    at which the TMA kernel stops handing out its last tiles at run time
+    (launches of fewer than 64 tiles per warp share them; on 152 SMs 2,000
+    sessions are 50,000 tiles, 3,400 sessions 85,000): every record equals
+    the oracle's, byte for byte, and a verified restore brings every byte back."""
+    g = torch.Generator(device=dev).manual_seed(77 + sessions)
+    obs = torch.randint(0, 256, (sessions, 3, 256, 256), generator=g, device=dev,
+                        dtype=torch.uint8)
+    rng = torch.randint(-2**62, 2**62, (sessions, 2), generator=g, device=dev, dtype=torch.int64)
+    arr = ctx.session_array([pcs.markov_session(s, obs[s], rng[s]) for s in range(sessions)])
+    hs = ctx.checkpoint_raw(arr, sessions)
+    obs_h, rng_h = obs.cpu().numpy(), rng.cpu().numpy().view(np.uint64)
+    for s in range(sessions):
+        ref = oracle.pack(oracle.markov_session(s, obs_h[s], rng_h[s]))
+        assert np.array_equal(ctx.record(pcs.Snapshot(ctx, hs[s])).numpy(), ref), s
+    o2, r2 = torch.zeros_like(obs), torch.zeros_like(rng)
+    tarr = ctx.session_array([pcs.markov_session(s, o2[s], r2[s]) for s in range(sessions)])
+    ctx.restore_raw(hs, sessions, tarr, verify=1)
+    torch.cuda.synchronize()
+    assert torch.equal(o2, obs) and torch.equal(r2, rng)
+    ctx.delete_raw(hs, sessions)
