@@ -7,6 +7,7 @@
 // turns a batch of sessions into one launch of the streaming kernel over
 // every section of every session, and owns the snapshots behind opaque
 // handles (Sec. 3 "The contract": checkpoint / restore / fork / delete).
+#include <nvtx3/nvToolsExt.h>
 #include <cuda_runtime.h>
 #include <fcntl.h>
 #include <unistd.h>
@@ -37,6 +38,18 @@ using namespace pcs;
 namespace {
 
 thread_local std::string g_err;
+
+// An NVTX range around each data-path call of the library, named after the
+// call, for Nsight tools (for example `ncu --nvtx --nvtx-include
+// "pcs_checkpoint/"` profiles only the kernels a checkpoint launched).
+// Without a tool attached a range costs a few nanoseconds.
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
+#define PCS_TRACE(name) TraceRange pcs_trace_range_(name)
 
 pcs_status fail(pcs_status s, const char* fmt, ...) {
   char buf[512];
@@ -1401,6 +1414,7 @@ pcs_status pcs_timing_read(pcs_ctx* c, pcs_kernel_time* out, int32_t max, int32_
 }
 
 pcs_status pcs_sync(pcs_ctx* c, void* stream) {
+  PCS_TRACE("pcs_sync");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   std::lock_guard<std::mutex> lk(c->mu);
   pcs_status st = set_device(c);
@@ -1443,6 +1457,7 @@ pcs_status pcs_selftest_wait(pcs_ctx* c, int32_t which, void* stream) {
 
 pcs_status pcs_fingerprint(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t* fp_out,
                            void* stream) {
+  PCS_TRACE("pcs_fingerprint");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   if (n > 0 && !fp_out) return fail(PCS_E_INVAL, "fp_out is null");
   std::lock_guard<std::mutex> lk(c->mu);
@@ -1453,6 +1468,7 @@ pcs_status pcs_fingerprint(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t*
 
 pcs_status pcs_classify(pcs_ctx* c, const pcs_buf* bufs, int32_t n, const uint64_t* fp_before,
                         uint64_t* fp_after, uint8_t* must_snapshot, void* stream) {
+  PCS_TRACE("pcs_classify");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   if (n > 0 && (!fp_before || !must_snapshot))
     return fail(PCS_E_INVAL, "fp_before and must_snapshot are required");
@@ -1564,6 +1580,7 @@ cudaError_t launch_bank_scores(pcs_ctx* c, const pcs_bank* banks, int32_t n,
 
 pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_prune_params* p,
                      float* scores, int32_t* kept_idx, int32_t* kept_off, void* stream_) {
+  PCS_TRACE("pcs_prune");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   std::vector<int32_t> k(std::max(n, 0));
@@ -1610,6 +1627,7 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
 
 pcs_status pcs_topk(pcs_ctx* c, const float* keys, const int32_t* n, const int32_t* k,
                     int32_t n_banks, int32_t* kept_idx, int32_t* kept_off, void* stream_) {
+  PCS_TRACE("pcs_topk");
   if (!c || n_banks < 0 || (n_banks > 0 && (!n || !k))) return fail(PCS_E_INVAL, "bad arguments");
   if (n_banks == 0) return PCS_OK;
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
@@ -1857,6 +1875,7 @@ static pcs_status prune_global_impl(pcs_ctx* c, const pcs_bank* banks, int32_t n
 
 pcs_status pcs_prune_global(pcs_ctx* c, const pcs_bank* banks, int32_t n, uint64_t budget,
                             float* scores, int32_t* kept_idx, int32_t* kept_off, void* stream) {
+  PCS_TRACE("pcs_prune_global");
   return prune_global_impl(c, banks, n, budget, scores, kept_idx, kept_off, stream, nullptr,
                            nullptr, 0);
 }
@@ -1865,6 +1884,7 @@ pcs_status pcs_prune_global_part(pcs_ctx* c, const pcs_bank* banks, int32_t n, u
                                  uint64_t pos_base, pcs_hist_exchange_fn exchange, void* user,
                                  float* scores, int32_t* kept_idx, int32_t* kept_off,
                                  void* stream) {
+  PCS_TRACE("pcs_prune_global_part");
   if (!exchange) return fail(PCS_E_INVAL, "exchange is null");
   return prune_global_impl(c, banks, n, budget, scores, kept_idx, kept_off, stream, exchange,
                            user, pos_base);
@@ -1928,6 +1948,7 @@ pcs_status pcs_record_bytes(const pcs_section* sections, int32_t n, uint64_t* ou
 
 pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, uint32_t placement,
                           pcs_snapshot** out, void* stream_) {
+  PCS_TRACE("pcs_checkpoint");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   if (n < 0 || (n > 0 && (!sessions || !out))) return fail(PCS_E_INVAL, "bad session list");
@@ -1965,6 +1986,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
 
 pcs_status pcs_fork_many(pcs_ctx* c, pcs_snapshot* const* parents, int32_t n,
                          pcs_snapshot** children, void* stream_) {
+  PCS_TRACE("pcs_fork_many");
   if (!c || n < 0 || (n > 0 && (!parents || !children))) return fail(PCS_E_INVAL, "bad arguments");
   if (n == 0) return PCS_OK;
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
@@ -2061,6 +2083,7 @@ pcs_status pcs_fork(pcs_ctx* c, const pcs_snapshot* parent, pcs_snapshot** child
 
 pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const pcs_session* targets,
                        int32_t verify, void* stream_) {
+  PCS_TRACE("pcs_restore");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   if (n < 0 || (n > 0 && (!snaps || !targets))) return fail(PCS_E_INVAL, "bad arguments");
@@ -2110,6 +2133,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
 pcs_status pcs_plan_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n,
                                uint32_t placement, pcs_snapshot** out, pcs_plan** plan,
                                void* stream_) {
+  PCS_TRACE("pcs_plan_checkpoint");
   if (!c || !plan) return fail(PCS_E_INVAL, "bad arguments");
   *plan = nullptr;
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
@@ -2143,6 +2167,7 @@ pcs_status pcs_plan_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t 
 
 pcs_status pcs_plan_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
                             const pcs_session* targets, int32_t verify, pcs_plan** plan) {
+  PCS_TRACE("pcs_plan_restore");
   if (!c || !plan) return fail(PCS_E_INVAL, "bad arguments");
   *plan = nullptr;
   if (n <= 0 || !snaps || !targets) return fail(PCS_E_INVAL, "bad arguments");
@@ -2172,6 +2197,7 @@ pcs_status pcs_plan_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
 }
 
 pcs_status pcs_plan_run(pcs_ctx* c, pcs_plan* p, void* stream_) {
+  PCS_TRACE("pcs_plan_run");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   std::lock_guard<std::mutex> lk(c->mu);
@@ -2216,6 +2242,7 @@ pcs_status pcs_plan_destroy(pcs_ctx* c, pcs_plan* p) {
 }
 
 pcs_status pcs_delete(pcs_ctx* c, pcs_snapshot* h) {
+  PCS_TRACE("pcs_delete");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   std::lock_guard<std::mutex> lk(c->mu);
   if (!check_handle(c, h)) return fail(PCS_E_HANDLE, "unknown snapshot handle");
@@ -2226,6 +2253,7 @@ pcs_status pcs_delete(pcs_ctx* c, pcs_snapshot* h) {
 }
 
 pcs_status pcs_delete_many(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n) {
+  PCS_TRACE("pcs_delete_many");
   if (!c || n < 0 || (n > 0 && !snaps)) return fail(PCS_E_INVAL, "bad arguments");
   std::lock_guard<std::mutex> lk(c->mu);
   for (int i = 0; i < n; ++i)
@@ -2294,6 +2322,7 @@ pcs_status pcs_snapshot_get_section(pcs_ctx* c, const pcs_snapshot* snap, int32_
 
 pcs_status pcs_snapshot_copy_out(pcs_ctx* c, const pcs_snapshot* snap, uint64_t offset,
                                  uint64_t bytes, void* dst, void* stream_) {
+  PCS_TRACE("pcs_snapshot_copy_out");
   if (!c || (bytes > 0 && !dst)) return fail(PCS_E_INVAL, "null argument");
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
   std::lock_guard<std::mutex> lk(c->mu);
@@ -2322,6 +2351,7 @@ static pcs_status ensure_stage(pcs_ctx* c) {
 }
 
 pcs_status pcs_snapshot_write_file(pcs_ctx* c, const pcs_snapshot* snap, const char* path) {
+  PCS_TRACE("pcs_snapshot_write_file");
   if (!c || !path) return fail(PCS_E_INVAL, "null argument");
   std::lock_guard<std::mutex> lk(c->mu);
   pcs_snapshot* h = check_handle(c, snap);
@@ -2359,6 +2389,7 @@ pcs_status pcs_snapshot_write_file(pcs_ctx* c, const pcs_snapshot* snap, const c
 
 pcs_status pcs_snapshot_read_file(pcs_ctx* c, const char* path, uint32_t placement,
                                   pcs_snapshot** out) {
+  PCS_TRACE("pcs_snapshot_read_file");
   if (!c || !path || !out) return fail(PCS_E_INVAL, "null argument");
   if (placement != PCS_PLACE_DEVICE && placement != PCS_PLACE_PINNED_HOST)
     return fail(PCS_E_INVAL, "unknown placement %u", placement);
@@ -2508,6 +2539,7 @@ pcs_status pool_check(pcs_ctx* c, pcs_pool* pl) {
 }  // namespace
 
 pcs_status pcs_pool_alloc(pcs_ctx* c, pcs_pool* pl, int32_t* ids, int32_t n, void* stream) {
+  PCS_TRACE("pcs_pool_alloc");
   if (n < 0 || (n > 0 && !ids)) return fail(PCS_E_INVAL, "bad arguments");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   std::lock_guard<std::mutex> lk(c->mu);
@@ -2521,6 +2553,7 @@ pcs_status pcs_pool_alloc(pcs_ctx* c, pcs_pool* pl, int32_t* ids, int32_t n, voi
 
 pcs_status pcs_pool_share(pcs_ctx* c, pcs_pool* pl, const int32_t* src, int32_t* dst, int32_t n,
                           void* stream) {
+  PCS_TRACE("pcs_pool_share");
   if (n < 0 || (n > 0 && !src)) return fail(PCS_E_INVAL, "bad arguments");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   std::lock_guard<std::mutex> lk(c->mu);
@@ -2534,6 +2567,7 @@ pcs_status pcs_pool_share(pcs_ctx* c, pcs_pool* pl, const int32_t* src, int32_t*
 
 pcs_status pcs_pool_prepare_write(pcs_ctx* c, pcs_pool* pl, int32_t* table, int64_t n_table,
                                   const int32_t* entries, int32_t n, void* stream) {
+  PCS_TRACE("pcs_pool_prepare_write");
   if (n < 0 || n_table < 0 || (n > 0 && !table)) return fail(PCS_E_INVAL, "bad arguments");
   if (!entries && n > n_table) return fail(PCS_E_INVAL, "n exceeds the table");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
@@ -2548,6 +2582,7 @@ pcs_status pcs_pool_prepare_write(pcs_ctx* c, pcs_pool* pl, int32_t* table, int6
 }
 
 pcs_status pcs_pool_release(pcs_ctx* c, pcs_pool* pl, const int32_t* ids, int32_t n, void* stream) {
+  PCS_TRACE("pcs_pool_release");
   if (n < 0 || (n > 0 && !ids)) return fail(PCS_E_INVAL, "bad arguments");
   if (!c) return fail(PCS_E_INVAL, "ctx is null");
   std::lock_guard<std::mutex> lk(c->mu);
@@ -2581,6 +2616,7 @@ pcs_status pcs_pool_query(pcs_ctx* c, pcs_pool* pl, int32_t* free_pages, uint32_
 
 pcs_status pcs_mismatch(pcs_ctx* c, const pcs_buf* a, const pcs_buf* b, int32_t n,
                         uint64_t* counts, void* stream_) {
+  PCS_TRACE("pcs_mismatch");
   if (!c || n < 0 || (n > 0 && (!a || !b || !counts))) return fail(PCS_E_INVAL, "bad arguments");
   if (n == 0) return PCS_OK;
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
@@ -2626,6 +2662,7 @@ pcs_status pcs_mismatch(pcs_ctx* c, const pcs_buf* a, const pcs_buf* b, int32_t 
 
 pcs_status pcs_classify_reads(pcs_ctx* c, const pcs_buf* bufs, int32_t n, const uint64_t* addr,
                               const uint64_t* bytes, int64_t m, uint8_t* flags, void* stream_) {
+  PCS_TRACE("pcs_classify_reads");
   if (!c || n < 0 || m < 0 || (n > 0 && (!bufs || !flags)) || (m > 0 && (!addr || !bytes)))
     return fail(PCS_E_INVAL, "bad arguments");
   if (n == 0) return PCS_OK;
