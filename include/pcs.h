@@ -242,7 +242,12 @@ pcs_status pcs_set_arena_limit(pcs_ctx *ctx, uint32_t placement, uint64_t bytes)
  * library's form of the session runtime's session table and PCS store
  * (Sec. 5, Figure fig:arch; Sec. 8), with the paged allocation that Sec. 3
  * "Boundary" leaves to the lower runtime.  PCS_E_CUDA if the device cannot
- * be used.
+ * be used.  Two environment variables, read here, change how the context
+ * works but never what it computes: PCS_CHECK=1 checks every call's plan on
+ * the host before launching it (node slots, work lists, layouts, payloads
+ * inside their records; a violation returns PCS_E_INVAL and launches
+ * nothing), and PCS_DISABLE_TMA=1 sends every stream through the register
+ * kernel instead of the TMA-staged one.
  */
 pcs_status pcs_create(int32_t device, pcs_ctx **out);
 /* Destroy a context (the end of the store of Sec. 5 / Sec. 8): waits for

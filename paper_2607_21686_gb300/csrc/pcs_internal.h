@@ -56,7 +56,8 @@ struct alignas(16) SecDesc {
   uint32_t align;          // CONTIG layout side: 16, 4 or 1 (largest that divides lbase)
   uint32_t fin_count;      // nodes the finaliser trees: [fin_begin, fin_begin + fin_count)
   uint32_t fin_begin;      // (the task nodes, or their 32-to-1 reduction)
-  uint32_t pad[3];
+  uint32_t sess;           // checkpoint / restore: the session of this stream
+  uint32_t pad[2];
 };
 static_assert(sizeof(SecDesc) == 112, "SecDesc layout");
 

@@ -350,6 +350,7 @@ struct pcs_ctx {
   int sm_count = 0;
   int stream_bps = 1;          // resident blocks per SM of the streaming kernel
   bool use_bulk = true;        // TMA-staged kernel for eligible streams
+  bool check_plans = false;    // PCS_CHECK=1: check every plan before launching
   std::mutex mu;
   std::shared_ptr<EventPool> events = std::make_shared<EventPool>();
   std::unique_ptr<Arena> dev_arena, host_arena;
@@ -851,6 +852,130 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   return P.nodes_total < (1ull << 32);
 }
 
+// ---------------------------------------------------------------------------
+// Plan checks (PCS_CHECK=1 at pcs_create): before anything is uploaded or
+// launched, every descriptor, work list and reduction level of a call is
+// checked against the invariants the kernels rely on -- node slots inside
+// the call's node array, work lists that cover each stream's tasks exactly
+// once, layouts the kernels can address, and record payloads inside their
+// record and block.  A failure is a planner bug: the call returns
+// PCS_E_INVAL naming the broken invariant and launches nothing.  compute-
+// sanitizer being unavailable, this is the bounds check of host-planned
+// offsets; index values read on the device are bounds-checked by the
+// kernels themselves.
+// ---------------------------------------------------------------------------
+
+std::string check_streams(const std::vector<SecDesc>& d, const std::vector<char>& bulk,
+                          const StreamPlan& P) {
+  char msg[256];
+  auto bad = [&](const char* fmt, auto... a) {
+    std::snprintf(msg, sizeof msg, fmt, a...);
+    return std::string(msg);
+  };
+  std::vector<int> seen(d.size(), 0);
+  auto walk = [&](const std::vector<uint32_t>& ids, const std::vector<uint32_t>& begin,
+                  uint32_t total, bool is_bulk) -> std::string {
+    if (ids.size() != begin.size()) return bad("work list of %zu ids, %zu begins", ids.size(), begin.size());
+    uint64_t t = 0;
+    for (size_t j = 0; j < ids.size(); ++j) {
+      if (ids[j] >= d.size()) return bad("work list item %zu names stream %u of %zu", j, ids[j], d.size());
+      if (begin[j] != t) return bad("work list item %zu begins at task %u, expected %llu", j,
+                                    begin[j], static_cast<unsigned long long>(t));
+      if (static_cast<bool>(bulk[ids[j]]) != is_bulk) return bad("stream %u in the wrong kernel's list", ids[j]);
+      ++seen[ids[j]];
+      t += d[ids[j]].n_tasks;
+    }
+    if (t != total) return bad("work list covers %llu tasks, plan says %u",
+                               static_cast<unsigned long long>(t), total);
+    return {};
+  };
+  std::string e = walk(P.bulk_ids, P.bulk_begin, P.bulk_tasks, true);
+  if (e.empty()) e = walk(P.reg_ids, P.reg_begin, P.reg_tasks, false);
+  if (!e.empty()) return e;
+  for (size_t i = 0; i < d.size(); ++i) {
+    const SecDesc& x = d[i];
+    if (seen[i] != 1) return bad("stream %zu appears in %d work lists", i, seen[i]);
+    if (x.n_chunks != n_chunks_of(x.bytes)) return bad("stream %zu: %llu chunks for %llu bytes", i,
+                                                        static_cast<unsigned long long>(x.n_chunks),
+                                                        static_cast<unsigned long long>(x.bytes));
+    const uint64_t per = bulk[i] ? kBulkTileChunks : (1ull << P.glog2);
+    if (x.n_tasks != (x.n_chunks + per - 1) / per) return bad("stream %zu: %u tasks for %llu chunks", i,
+                                                              x.n_tasks,
+                                                              static_cast<unsigned long long>(x.n_chunks));
+    if (static_cast<uint64_t>(x.task_begin) + x.n_tasks > P.nodes)
+      return bad("stream %zu: task nodes end past the %llu nodes", i,
+                 static_cast<unsigned long long>(P.nodes));
+    if (x.fin_count < 1 || static_cast<uint64_t>(x.fin_begin) + x.fin_count > P.nodes_total)
+      return bad("stream %zu: finalisation nodes [%u, +%u) outside %llu", i, x.fin_begin, x.fin_count,
+                 static_cast<unsigned long long>(P.nodes_total));
+    if (x.layout == kContig) {
+      if (x.bytes && !x.lbase) return bad("stream %zu: no base", i);
+      if (reinterpret_cast<uintptr_t>(x.lbase) % x.align) return bad("stream %zu: alignment %u wrong", i, x.align);
+      if (bulk[i] && x.bytes && x.align != 16) return bad("stream %zu: TMA stream off 16 bytes", i);
+    } else {
+      if (x.layout != kRows && x.layout != kRing) return bad("stream %zu: layout %u", i, x.layout);
+      if (x.row_bytes == 0 || (x.bytes && !x.index) || x.base_rows == 0)
+        return bad("stream %zu: rows without size, index or bound", i);
+      if (bulk[i] && (x.row_bytes < kBulkMinRowBytes || x.row_bytes % 16))
+        return bad("stream %zu: TMA rows of %llu bytes", i, static_cast<unsigned long long>(x.row_bytes));
+      if (x.layout == kRing &&
+          (x.window == 0 || x.page_rows == 0 || x.window % x.page_rows || x.ring_start >= x.window ||
+           x.bytes > static_cast<uint64_t>(x.window) * x.row_bytes))
+        return bad("stream %zu: ring window %u, pages of %u rows, start %u", i, x.window, x.page_rows,
+                   x.ring_start);
+    }
+  }
+  const size_t ns = d.size();
+  for (size_t k = 0; k < P.level_groups.size(); ++k)
+    for (size_t i = 0; i < ns; ++i) {
+      const NodeLevel& L = P.levels[k * ns + i];
+      if (static_cast<uint64_t>(L.src) + L.count > P.nodes_total ||
+          static_cast<uint64_t>(L.dst) + (L.count + 31) / 32 > P.nodes_total ||
+          L.dst < P.level_base[k] || L.dst + (L.count + 31) / 32 > P.level_base[k] + P.level_groups[k])
+        return bad("reduction level %zu of stream %zu outside its nodes", k, i);
+    }
+  return {};
+}
+
+// Records of a checkpoint or restore: sessions cover the streams in order,
+// record s lies in its block [block[s].first, block[s].second), each payload
+// inside its record.
+std::string check_sessions(const std::vector<SecDesc>& d, const std::vector<SessDesc>& sd,
+                           const std::vector<std::pair<const uint8_t*, const uint8_t*>>& block) {
+  char msg[256];
+  uint32_t next = 0;
+  for (size_t s = 0; s < sd.size(); ++s) {
+    const SessDesc& S = sd[s];
+    if (S.sec_begin != next || S.n_sections < 1 || S.sec_begin + S.n_sections > d.size()) {
+      std::snprintf(msg, sizeof msg, "session %zu: sections [%u, +%u) out of order", s, S.sec_begin,
+                    S.n_sections);
+      return msg;
+    }
+    next = S.sec_begin + S.n_sections;
+    if (S.record < block[s].first || S.record + S.total_bytes > block[s].second ||
+        S.payload_start > S.total_bytes ||
+        S.payload_start % kRecordAlign ||
+        S.payload_start < kHeaderBytes + static_cast<uint64_t>(kEntryBytes) * S.n_sections) {
+      std::snprintf(msg, sizeof msg, "session %zu: record outside its block or table overlap", s);
+      return msg;
+    }
+    for (uint32_t j = 0; j < S.n_sections; ++j) {
+      const SecDesc& x = d[S.sec_begin + j];
+      const uint64_t off = static_cast<uint64_t>(x.payload - S.record);
+      if (x.payload < S.record + S.payload_start || off % kRecordAlign ||
+          off + round_up(x.bytes, kRecordAlign) > S.total_bytes || x.sess != s) {
+        std::snprintf(msg, sizeof msg, "session %zu section %u: payload outside its record", s, j);
+        return msg;
+      }
+    }
+  }
+  if (next != d.size()) {
+    std::snprintf(msg, sizeof msg, "sessions cover %u of %zu streams", next, d.size());
+    return msg;
+  }
+  return {};
+}
+
 // A small call whose streams all take the register kernel runs in one
 // launch (k_small): the streaming pass and its finalisation.
 constexpr int kSmallMaxItems = 64;
@@ -922,6 +1047,10 @@ pcs_status fingerprint_impl(pcs_ctx* c, const pcs_buf* bufs, int32_t n, uint64_t
   StreamPlan P;
   if (!plan_streams(c, d, bulk, P, !fused)) return fail(PCS_E_INVAL, "too much data in one call");
   P.link_bound = link_bound_call(d, bulk, std::vector<char>(n, 1), cache);
+  if (c->check_plans) {
+    const std::string e = check_streams(d, bulk, P);
+    if (!e.empty()) return fail(PCS_E_INVAL, "plan check: %s", e.c_str());
+  }
   WsLayout L;
   L.secs = 0;
   const ListLayout LL = list_layout(P, sizeof(SecDesc) * n);
@@ -1140,6 +1269,7 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
     for (int i = 0; i < S.n_sections; ++i) {
       const pcs_section& x = S.sections[i];
       d.push_back(make_desc(x, rec + off, x.ring_start));
+      d.back().sess = static_cast<uint32_t>(s);
       Entry e{};
       e.type = x.type;
       e.dtype = x.dtype;
@@ -1174,6 +1304,16 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
   }
   pr->P.link_bound =
       link_bound_call(d, bulk, std::vector<char>(d.size(), placement == PCS_PLACE_DEVICE), cache);
+  if (c->check_plans) {
+    std::string e = check_streams(d, bulk, pr->P);
+    if (e.empty())
+      e = check_sessions(d, sd, std::vector<std::pair<const uint8_t*, const uint8_t*>>(
+                                    n, {blk->ptr, blk->ptr + blk->size}));
+    if (!e.empty()) {
+      arena_of(c, placement)->free(blk);
+      return fail(PCS_E_INVAL, "plan check: %s", e.c_str());
+    }
+  }
   WsLayout& L = pr->L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
@@ -1225,6 +1365,7 @@ pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
         rs = static_cast<uint32_t>(e.aux);
       }
       d.push_back(make_desc(x, h->record() + e.offset, rs));
+      d.back().sess = static_cast<uint32_t>(s);
       payload_dev.push_back(h->block->placement == PCS_PLACE_DEVICE);
     }
   }
@@ -1242,6 +1383,14 @@ pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
   if (!plan_streams(c, d, bulk, pr->P, !pr->fused))
     return fail(PCS_E_INVAL, "too much data in one call");
   pr->P.link_bound = link_bound_call(d, bulk, payload_dev, cache);
+  if (c->check_plans) {
+    std::vector<std::pair<const uint8_t*, const uint8_t*>> blocks(n);
+    for (int s = 0; s < n; ++s)
+      blocks[s] = {snaps[s]->block->ptr, snaps[s]->block->ptr + snaps[s]->block->size};
+    std::string e = check_streams(d, bulk, pr->P);
+    if (e.empty()) e = check_sessions(d, sd, blocks);
+    if (!e.empty()) return fail(PCS_E_INVAL, "plan check: %s", e.c_str());
+  }
   WsLayout& L = pr->L;
   L.secs = 0;
   L.sess = round_up(sizeof(SecDesc) * d.size(), kRecordAlign);
@@ -1300,6 +1449,8 @@ pcs_status pcs_create(int32_t device, pcs_ctx** out) {
   c->stream_bps = stream_blocks_per_sm();
   const char* no_tma = std::getenv("PCS_DISABLE_TMA");
   c->use_bulk = !(no_tma && no_tma[0] == '1');
+  const char* check = std::getenv("PCS_CHECK");
+  c->check_plans = check && check[0] == '1';
   c->dev_arena = std::make_unique<Arena>(PCS_PLACE_DEVICE, c->events);
   c->host_arena = std::make_unique<Arena>(PCS_PLACE_PINNED_HOST, c->events);
   PCS_CUDA(cudaMalloc(&c->words, 256));
@@ -2040,6 +2191,10 @@ pcs_status pcs_fork_many(pcs_ctx* c, pcs_snapshot* const* parents, int32_t n,
     bulk[i] = c->use_bulk && !small && parents[i]->block->placement == PCS_PLACE_DEVICE;
   StreamPlan P;
   if (!plan_streams(c, d, bulk, P)) return undo(fail(PCS_E_INVAL, "too much data in one call"));
+  if (c->check_plans) {
+    const std::string e = check_streams(d, bulk, P);
+    if (!e.empty()) return undo(fail(PCS_E_INVAL, "plan check: %s", e.c_str()));
+  }
   const ListLayout LL = list_layout(P, sizeof(SecDesc) * n);
   const uint64_t total = round_up(LL.end, kRecordAlign);
   uint8_t* ws = nullptr;
