@@ -386,7 +386,11 @@ def run_pcs(a, rank, world, local_rank):
     # End to end through the public API with the state coming from host memory.
     e2e = None
     if not a.no_e2e:
+        if world > 1:
+            torch.distributed.barrier()
         e2e = run_e2e(a, ctx, kv, dst, stream, dev)
+        if world > 1:
+            e2e = e2e_over_ranks(a, e2e, world)
 
     rows = None
     if not a.no_rows and rank == 0:
@@ -865,6 +869,24 @@ class HostBuffer:
             except BufferError:  # views still alive; the mapping goes with them
                 pass
             self.mm = None
+
+
+def e2e_over_ranks(a, e2e: dict, world: int) -> dict:
+    """The whole job's end-to-end line: every rank's step bytes over the
+    slowest rank's time per step (all ranks ran their steps at once)."""
+    ms = e2e.get("ms_per_step")
+    if max_over_ranks(0.0 if ms is not None else 1.0) != 0.0:
+        return {"value": None, "unit": "GB/s",
+                "note": "a rank could not pin its host pools; no whole-job end-to-end number"}
+    ms_all = max_over_ranks(float(ms))
+    out = dict(e2e)
+    out.update({"value": round(step_bytes(a) * world / (ms_all / 1e3) / 1e9, 2),
+                "ms_per_step": round(ms_all, 3),
+                "sessions_per_s": round(a.sessions * world / (ms_all / 1e3), 2),
+                "h2d_bytes_per_step": e2e["h2d_bytes_per_step"] * world,
+                "d2h_bytes_per_step": e2e["d2h_bytes_per_step"] * world,
+                "ranks": world, "rank0_value": e2e["value"]})
+    return out
 
 
 def run_e2e(a, ctx, kv, dst, stream, dev):

@@ -28,6 +28,24 @@ def _worker(rank, world, port, out):
     torch.distributed.destroy_process_group()
 
 
+def _e2e_worker(rank, world, port, out, fail_rank):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    torch.distributed.init_process_group("gloo", rank=rank, world_size=world)
+    sys.path.insert(0, ROOT)
+    import bench
+
+    class A:
+        sessions, layers, heads, head_dim, window, page_rows = 256, 24, 16, 64, 1024, 16
+    if rank == fail_rank:
+        mine = {"value": None, "unit": "GB/s", "note": "pinned allocation failed"}
+    else:
+        ms = 120.0 + 10.0 * rank
+        mine = {"value": round(bench.step_bytes(A) / (ms / 1e3) / 1e9, 2), "unit": "GB/s",
+                "ms_per_step": ms, "h2d_bytes_per_step": 100, "d2h_bytes_per_step": 8}
+    out[rank] = bench.e2e_over_ranks(A, mine, world)
+    torch.distributed.destroy_process_group()
+
+
 def _budget_worker(rank, world, port, out):
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     torch.distributed.init_process_group("gloo", rank=rank, world_size=world)
@@ -106,3 +124,29 @@ def test_sharded_budget_matches_one_process():
     E = rnd.choice([3072, 1024, 5000], 2048)
     want = oracle.k_budget(n, E.astype(np.uint64), 8 << 30)
     assert [k[s] for s in range(2048)] == want.tolist()
+
+
+@pytest.mark.parametrize("fail_rank", [-1, 1])
+def test_e2e_over_ranks_gloo(fail_rank):
+    """The whole-job end-to-end line: both ranks' step bytes over the slower
+    rank's time; no number at all when a rank could not run its end to end."""
+    ctx = mp.get_context("spawn")
+    with ctx.Manager() as m:
+        out = m.dict()
+        port = _free_port()
+        procs = [ctx.Process(target=_e2e_worker, args=(r, 2, port, out, fail_rank))
+                 for r in range(2)]
+        for p in procs:
+            p.start()
+        for p in procs:
+            p.join(120)
+            assert p.exitcode == 0
+        res = {r: {k: v for k, v in d.items() if k != "rank0_value"} for r, d in dict(out).items()}
+    assert res[0] == res[1]
+    if fail_rank >= 0:
+        assert res[0]["value"] is None
+    else:
+        step = 4 * 256 * (2 * 24 * 1024 * 16 * 64 * 2 + 32)
+        assert res[0]["ms_per_step"] == 130.0
+        assert res[0]["value"] == round(2 * step / 0.130 / 1e9, 2)
+        assert res[0]["h2d_bytes_per_step"] == 200 and res[0]["ranks"] == 2
