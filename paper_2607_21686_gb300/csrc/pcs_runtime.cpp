@@ -1258,6 +1258,7 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
     h->payload_start = pstart[s];
     h->session_id = S.session_id;
     h->kind = S.kind;
+    h->table.reserve(S.n_sections);
     sd[s].record = rec;
     sd[s].total_bytes = h->total_bytes;
     sd[s].payload_start = pstart[s];
@@ -2128,6 +2129,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   st = ws_release(c, stream, blk->written);
   if (st) return undo(st);
   blk->refs = n;
+  c->live.reserve(c->live.size() + n);
   for (int s = 0; s < n; ++s) {
     out[s] = handles[s].release();
     c->live.insert(out[s]);
@@ -2218,6 +2220,7 @@ pcs_status pcs_fork_many(pcs_ctx* c, pcs_snapshot* const* parents, int32_t n,
     blk[pl]->written = done;
     blk[pl]->refs = 0;
   }
+  c->live.reserve(c->live.size() + n);
   for (int i = 0; i < n; ++i) {
     Block* b = blk[parents[i]->block->placement];
     auto h = std::make_unique<pcs_snapshot>(*parents[i]);
@@ -2311,6 +2314,7 @@ pcs_status pcs_plan_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t 
   blk->written = record_event(c->events, stream);
   blk->refs = n + 1;  // the snapshots and the plan
   p->blocks.push_back(blk);
+  c->live.reserve(c->live.size() + n);
   for (int s = 0; s < n; ++s) {
     out[s] = handles[s].release();
     c->live.insert(out[s]);
