@@ -40,10 +40,10 @@ METRIC = "snapshot+restore GB/s and sessions/s on 1 GB300; % of HBM (PCIe) roofl
 # capture summarised in profiles/k_bulk_kv8x24_full.md (8 sessions, scaled by
 # sessions / 8), valid only for the streaming-kernel source it was taken on.
 NCU_TRAFFIC = {
-    "source_sha256_prefix": "34ca6aae9c996982",
+    "source_sha256_prefix": "453311c07109f60d",
     "sessions": 8,
-    "k_bulk<pack>": 805713664 + 754127616,
-    "k_bulk<restore_verify>": 805734144 + 754489344,
+    "k_bulk<pack>": 805864960 + 754253312,
+    "k_bulk<restore_verify>": 805719808 + 754248960,
 }
 
 

@@ -119,29 +119,39 @@ __device__ uint64_t warp_tree_inplace(uint64_t* a, uint32_t n, int lane) {
   return a[0];
 }
 
-// The same tree for n <= 1024: up to eight groups of 32 are read at once,
-// group g's root is kept in lane g, then the roots' tree.  Nothing is
-// written.  Called by one whole warp; every lane returns the root.
+// The same tree for n <= 1024, nothing written; called by one whole warp,
+// every lane returns the root.  Up to 32 items: one warp tree.  Beyond,
+// in blocks of 256 items: lane l reads items 8l .. 8l+7 of the block and
+// reduces them in its registers (the tree's first three levels over that
+// aligned group of eight, an odd last item carried up), the warp then
+// reduces the 32 group roots (five more levels), and the roots of up to four
+// blocks end the tree.  Aligned groups of 2^m items reduce to the nodes of
+// the global pairwise tree, so the root is the same; all 32 lanes combine
+// at once, where trees of 32-item groups leave half the lanes idle at each
+// level (a 256-item tree took 1,790 warp instructions that way).
 __device__ uint64_t warp_tree_regs(const uint64_t* a, uint32_t n, int lane) {
-  const uint32_t groups = (n + 31) / 32;
-  uint64_t mine = 0;
-  for (uint32_t g0 = 0; g0 < groups; g0 += 8) {
+  if (n <= 32) {
+    const uint64_t v = lane < static_cast<int>(n) ? a[lane] : 0;
+    return __shfl_sync(kFull, warp_tree(v, static_cast<int>(n), lane), 0);
+  }
+  const uint32_t blocks = (n + 255) / 256;
+  uint64_t block_root = 0;  // root of block b, kept in lane b
+  for (uint32_t b = 0; b < blocks; ++b) {
+    const uint32_t base = 256 * b;
+    const uint32_t nb = min(256u, n - base);
+    const int m = max(0, min(8, static_cast<int>(nb) - 8 * lane));  // this lane's items
     uint64_t v[8];
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const uint32_t i = 32 * (g0 + q) + lane;
-      v[q] = i < n ? a[i] : 0;
-    }
+    for (int i = 0; i < 8; ++i) v[i] = i < m ? a[base + 8 * lane + i] : 0;
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const uint32_t g = g0 + q;
-      if (g < groups) {  // the same for the whole warp
-        const uint64_t r = __shfl_sync(kFull, warp_tree(v[q], static_cast<int>(min(32u, n - 32 * g)), lane), 0);
-        if (lane == static_cast<int>(g)) mine = r;
-      }
-    }
+    for (int w = 1; w < 8; w <<= 1)
+#pragma unroll
+      for (int i = 0; i + w < 8; i += 2 * w)
+        if (i + w < m) v[i] = comb(v[i], v[i + w]);
+    const uint64_t r = __shfl_sync(kFull, warp_tree(v[0], static_cast<int>((nb + 7) / 8), lane), 0);
+    if (lane == static_cast<int>(b)) block_root = r;
   }
-  const uint64_t root = groups > 1 ? warp_tree(mine, static_cast<int>(groups), lane) : mine;
+  const uint64_t root = blocks > 1 ? warp_tree(block_root, static_cast<int>(blocks), lane) : block_root;
   return __shfl_sync(kFull, root, 0);
 }
 

@@ -813,11 +813,12 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   // A stream with many task nodes would leave one finalising warp a long
   // serial tree: reduce aligned groups of 32 nodes across the GPU, level by
   // level, until no stream has more than 32 nodes left.  Aligned groups of
-  // 32^k nodes reduce to the nodes of the global pairwise tree.  Up to 256
-  // nodes (eight groups) the finalising warp is quicker than another launch;
-  // reducing only down to 1,024 nodes (one level fewer for the 256 MiB
-  // buffers of the classify sweep) made the sweep's finalisation 14 us
-  // slower than the level it saved.
+  // 32^k nodes reduce to the nodes of the global pairwise tree.  Up to
+  // kFinRegNodes (1,024) nodes the finalising warp trees them from its
+  // registers quicker than another launch (measured with the lane-local
+  // register tree: the 64-bank step, whose latent sections have up to 512
+  // tiles, 0.236 -> 0.234 ms without its two reduction launches; with the
+  // earlier tree of 32-node groups a threshold of 256 was the better one).
   for (auto& x : d) {
     x.fin_begin = x.task_begin;
     x.fin_count = x.n_tasks;
@@ -825,7 +826,7 @@ bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<c
   uint64_t max_count = 0;
   for (const auto& x : d) max_count = std::max<uint64_t>(max_count, x.n_tasks);
   uint64_t groups = 0;
-  if (allow_reduce && max_count > 256) {
+  if (allow_reduce && max_count > kFinRegNodes) {
     while (max_count > 32) {
       const uint64_t level_base = node + groups;
       uint64_t level_groups = 0;
