@@ -1191,22 +1191,42 @@ __global__ void __launch_bounds__(kThreads)
     const SessDesc S = sess[b];
     Entry* table = reinterpret_cast<Entry*>(S.record + kHeaderBytes);
     const int ns = static_cast<int>(S.n_sections);
+    // Lane j reads section j's node range, length and (restore) stored fp,
+    // all sections at once; each section's tree then starts from its node
+    // loads, and a checkpoint's entry is read before the tree.
+    uint32_t fin_begin = 0, fin_count = 0;
+    uint64_t sec_bytes = 0, stored = 0;
+    if (lane < ns) {
+      const SecDesc* sj = secs + S.sec_begin + lane;
+      fin_begin = __ldg(&sj->fin_begin);
+      fin_count = __ldg(&sj->fin_count);
+      sec_bytes = __ldg(reinterpret_cast<const unsigned long long*>(&sj->bytes));
+      if (MODE != kModePack) stored = table[lane].fp;
+    }
     uint64_t mine = 0;
     bool bad_sec = false;
     for (int j = 0; j < ns; ++j) {
-      const SecDesc s = secs[S.sec_begin + j];
-      const uint64_t fp = stream_fp(s, nodes, lane);
+      uint4 ew = make_uint4(0, 0, 0, 0);  // pack: lanes 0..3 hold the entry, read before the tree
+      if (MODE == kModePack && lane < 4)
+        ew = reinterpret_cast<const uint4*>(&entries[S.sec_begin + j])[lane];
+      const uint32_t nb = __shfl_sync(kFull, fin_begin, j);
+      const uint32_t nc = __shfl_sync(kFull, fin_count, j);
+      const uint64_t by = __shfl_sync(kFull, sec_bytes, j);
+      const uint64_t root = nc <= kFinRegNodes ? warp_tree_regs(nodes + nb, nc, lane)
+                                               : warp_tree_inplace(nodes + nb, nc, lane);
+      const uint64_t fp = fmix(root ^ (by * kP));
       if (MODE == kModePack) {
-        if (lane < 4) {
-          Entry e = entries[S.sec_begin + j];
-          e.fp = fp;
-          reinterpret_cast<uint4*>(&table[j])[lane] = reinterpret_cast<const uint4*>(&e)[lane];
+        // The fp (bytes 32..39 of the entry) is the first half of lane 2's word.
+        if (lane == 2) {
+          ew.x = static_cast<uint32_t>(fp);
+          ew.y = static_cast<uint32_t>(fp >> 32);
         }
+        if (lane < 4) reinterpret_cast<uint4*>(&table[j])[lane] = ew;
         if (lane == j) mine = fp;
       } else {
         if (lane == j) {
-          mine = table[j].fp;
-          bad_sec = mine != fp;
+          mine = stored;
+          bad_sec = stored != fp;
         }
       }
     }
