@@ -712,13 +712,15 @@ def measure_banks_config2(ctx, dev, stream, peak):
     keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
     vals = [b.values[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
     banks = ctx.banks_array(keys, [b.queries[s] for s in range(S)], 512 + b.value_bytes)
-    params = ctx.params(pcs.PCS_K_FIXED, k_max=128)
+    # Each bank's kept list starts on a 16-byte boundary (kept_align 4), so the
+    # checkpoint moves the lists with the other sections' bulk copies.
+    params = ctx.params(pcs.PCS_K_FIXED, k_max=128, kept_align=4)
     ks = ctx.prune_counts(banks, S, params)
     koff = [0]
     for k in ks:
-        koff.append(koff[-1] + k)
+        koff.append(koff[-1] + (k + 3) // 4 * 4)
     kept = torch.empty(koff[-1], dtype=torch.int32, device=dev)
-    sess = [pcs.bank_session(s, keys[s], vals[s], kept[koff[s]:koff[s + 1]]) for s in range(S)]
+    sess = [pcs.bank_session(s, keys[s], vals[s], kept[koff[s]:koff[s] + ks[s]]) for s in range(S)]
     outs = [(torch.empty(ks[s], dtype=torch.int32, device=dev),
              torch.empty(ks[s], 256, dtype=torch.float16, device=dev),
              torch.empty((ks[s],) + tuple(b.values.shape[1:]), dtype=b.values.dtype, device=dev))
@@ -737,7 +739,7 @@ def measure_banks_config2(ctx, dev, stream, peak):
     kept_h = kept.cpu()
     ok = True
     for s in (0, S // 2, S - 1):
-        ki = kept_h[koff[s]:koff[s + 1]]
+        ki = kept_h[koff[s]:koff[s] + ks[s]]
         ok &= bool(torch.equal(outs[s][0].cpu(), ki)) and bool(torch.all(ki[1:] > ki[:-1]))
         ok &= bool(torch.equal(outs[s][2], vals[s][ki.long().to(dev)]))
     # Planned once, then launches only (prune, checkpoint, restore).
@@ -754,11 +756,11 @@ def measure_banks_config2(ctx, dev, stream, peak):
     ctx.plan_destroy(cplan)
     ctx.delete_raw(phs, S)
     kb = sum(b.n) * 512
-    payload = koff[-1] * (4 + 512 + b.value_bytes)
+    payload = sum(ks) * (4 + 512 + b.value_bytes)
     moved = kb + 4 * payload
     return {"population": "64 banks, n ~ U[1,512], key fp16[256], latent bf16[16,32,32], "
-                          "k = min(n,128)",
-            "entries": sum(b.n), "kept": koff[-1], "key_bytes_read": kb,
+                          "k = min(n,128); kept lists 16-byte aligned",
+            "entries": sum(b.n), "kept": sum(ks), "key_bytes_read": kb,
             "bytes_per_step": moved, "how": "prune + checkpoint to HBM + verified restore + "
             "delete, 20 back-to-back steps between one pair of events",
             "ms": round(med, 4), "GBs": round(moved / (med / 1e3) / 1e9, 1),

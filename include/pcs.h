@@ -185,6 +185,12 @@ typedef struct pcs_prune_params {
                            /* its banks are split over calls or processes   */
                            /* (the sum of every part's T); 0 = the T of the */
                            /* banks of this call                            */
+    uint32_t kept_align;   /* pcs_prune: 0 or 1 = kept lists back to back;  */
+                           /* 4 = each bank's list starts at a multiple of  */
+                           /* 4 entries (16 bytes of a 16-byte aligned      */
+                           /* kept_idx), so a checkpoint moves the lists    */
+                           /* with bulk copies                              */
+    uint32_t reserved;     /* 0                                             */
 } pcs_prune_params;
 
 typedef struct pcs_snapshot_info {
@@ -335,8 +341,13 @@ pcs_status pcs_prune_counts(const pcs_bank *banks, int32_t n, const pcs_prune_pa
  * largest (score, -index) -- ties to the lower index, NaN lowest, -0 == +0 --
  * and write their indices in ascending order.
  *   scores:   device float[sum n] (CSR by bank) or NULL
- *   kept_idx: device int32[sum k] (CSR by bank, k from pcs_prune_counts)
- *   kept_off: device int32[n + 1] or NULL: CSR offsets of kept_idx
+ *   kept_idx: device int32[sum k] (CSR by bank, k from pcs_prune_counts);
+ *             with kept_align = 4, int32[sum round_up(k, 4)]: bank b's list
+ *             starts at the sum of round_up(k, 4) over the banks before it
+ *             (the entries between lists are left as they were)
+ *   kept_off: device int32[n + 1] or NULL: offsets of the lists in kept_idx
+ *             (the last one: the entries kept_idx spans)
+ * PCS_E_INVAL for a kept_align other than 0, 1 or 4.
  */
 pcs_status pcs_prune(pcs_ctx *ctx, const pcs_bank *banks, int32_t n,
                      const pcs_prune_params *params, float *scores, int32_t *kept_idx,

@@ -1683,7 +1683,7 @@ pcs_status pcs_prune_counts(const pcs_bank* banks, int32_t n, const pcs_prune_pa
 // Validated scoring descriptors of n banks (k per bank, or all 0 if k is
 // NULL), entry offsets bank-major; *entries = total entries.
 pcs_status bank_descs(const pcs_bank* banks, int32_t n, const int32_t* k,
-                      std::vector<BankDesc>* d, uint64_t* entries_out) {
+                      std::vector<BankDesc>* d, uint64_t* entries_out, uint32_t kept_align = 1) {
   d->assign(std::max(n, 0), BankDesc{});
   uint64_t entries = 0, kept = 0;
   for (int s = 0; s < n; ++s) {
@@ -1708,7 +1708,7 @@ pcs_status bank_descs(const pcs_bank* banks, int32_t n, const int32_t* k,
     x.is_bf16 = b.key_dtype == PCS_DT_BF16;
     x.entry_bytes = b.entry_bytes;
     entries += b.n_entries;
-    kept += x.k;
+    kept += round_up(static_cast<uint64_t>(x.k), kept_align);
   }
   if (entries > 0x7FFFFFFFull) return fail(PCS_E_INVAL, "too many entries in one call");
   *entries_out = entries;
@@ -1740,14 +1740,16 @@ pcs_status pcs_prune(pcs_ctx* c, const pcs_bank* banks, int32_t n, const pcs_pru
   pcs_status st = pcs_prune_counts(banks, n, p, k.data());
   if (st) return st;
   if (n == 0) return PCS_OK;
+  const uint32_t align = p->kept_align == 0 ? 1u : p->kept_align;
+  if (align != 1 && align != 4) return fail(PCS_E_INVAL, "kept_align must be 0, 1 or 4");
   std::vector<BankDesc> d;
   uint64_t entries = 0;
-  st = bank_descs(banks, n, k.data(), &d, &entries);
+  st = bank_descs(banks, n, k.data(), &d, &entries, align);
   if (st) return st;
   std::vector<int32_t> koff(n + 1, 0);
   uint64_t kept = 0;
   for (int s = 0; s < n; ++s) {
-    kept += k[s];
+    kept += round_up(static_cast<uint64_t>(k[s]), align);
     koff[s + 1] = static_cast<int32_t>(kept);
   }
   if (kept > 0 && !kept_idx) return fail(PCS_E_INVAL, "kept_idx is null");

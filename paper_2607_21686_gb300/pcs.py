@@ -77,7 +77,8 @@ class pcs_bank(ctypes.Structure):
 class pcs_prune_params(ctypes.Structure):
     _fields_ = [("rule", ctypes.c_int32), ("k_max", ctypes.c_int32),
                 ("budget_bytes", ctypes.c_uint64), ("fraction", ctypes.c_double),
-                ("total_bytes", ctypes.c_uint64)]
+                ("total_bytes", ctypes.c_uint64), ("kept_align", ctypes.c_uint32),
+                ("reserved", ctypes.c_uint32)]
 
 
 class pcs_snapshot_info(ctypes.Structure):
@@ -590,9 +591,9 @@ class Context:
 
     @staticmethod
     def params(rule: int, k_max: int = 0, budget: int = 0, fraction: float = 0.0,
-               total_bytes: int = 0):
+               total_bytes: int = 0, kept_align: int = 0):
         return pcs_prune_params(rule=rule, k_max=k_max, budget_bytes=budget, fraction=fraction,
-                                total_bytes=total_bytes)
+                                total_bytes=total_bytes, kept_align=kept_align)
 
     @staticmethod
     def prune_counts(banks, n: int, params) -> list:

@@ -118,13 +118,14 @@ def case_banks2(ctx, a, dev):
     keys = [b.keys[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
     vals = [b.values[b.entry_off[s]:b.entry_off[s + 1]] for s in range(S)]
     banks = ctx.banks_array(keys, [b.queries[s] for s in range(S)], 512 + b.value_bytes)
-    params = ctx.params(pcs.PCS_K_FIXED, k_max=128)
+    # Kept lists on 16-byte boundaries, as in bench.py's bank row.
+    params = ctx.params(pcs.PCS_K_FIXED, k_max=128, kept_align=4)
     ks = ctx.prune_counts(banks, S, params)
     koff = [0]
     for k in ks:
-        koff.append(koff[-1] + k)
+        koff.append(koff[-1] + (k + 3) // 4 * 4)
     kept = torch.empty(koff[-1], dtype=torch.int32, device=dev)
-    sarr = ctx.session_array([pcs.bank_session(s, keys[s], vals[s], kept[koff[s]:koff[s + 1]])
+    sarr = ctx.session_array([pcs.bank_session(s, keys[s], vals[s], kept[koff[s]:koff[s] + ks[s]])
                               for s in range(S)])
     outs = [(torch.empty(ks[s], dtype=torch.int32, device=dev),
              torch.empty(ks[s], 256, dtype=torch.float16, device=dev),

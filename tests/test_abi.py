@@ -62,7 +62,7 @@ int main(void) {
   S(pcs_session) O(pcs_session, n_sections) O(pcs_session, sections)
   S(pcs_bank) O(pcs_bank, n_entries) O(pcs_bank, key_dtype) O(pcs_bank, entry_bytes)
   S(pcs_prune_params) O(pcs_prune_params, budget_bytes) O(pcs_prune_params, fraction)
-  O(pcs_prune_params, total_bytes)
+  O(pcs_prune_params, total_bytes) O(pcs_prune_params, kept_align)
   S(pcs_snapshot_info) O(pcs_snapshot_info, total_bytes) O(pcs_snapshot_info, data)
   S(pcs_section_info) O(pcs_section_info, offset) O(pcs_section_info, aux)
   S(pcs_stats) O(pcs_stats, live_snapshots)

@@ -533,3 +533,41 @@ def test_fork_many_mixed_placements(ctx, dev):
     ctx.delete_raw(kids, 6)
     for x in parents:
         ctx.delete(x)
+
+
+def test_prune_kept_align_16_bytes(ctx, dev):
+    """kept_align = 4: each bank's kept list starts at a multiple of four
+    entries; the lists are the oracle's top-k, kept_off gives the padded
+    offsets, and a checkpoint of the banks equals the oracle's records."""
+    b = synth.banks_config2(seed=91, sessions=12)
+    keys, vals, qs = _bank_views(b, dev)
+    banks = ctx.banks_array(keys, qs, 512 + b.value_bytes)
+    for bad in (2, 3, 8):
+        with pytest.raises(pcs.PcsError) as e:
+            ctx.prune(banks, b.sessions, ctx.params(pcs.PCS_K_FIXED, k_max=7, kept_align=bad),
+                      torch.empty(1024, dtype=torch.int32, device=dev))
+        assert e.value.status == pcs.PCS_E_INVAL
+    params = ctx.params(pcs.PCS_K_FIXED, k_max=37, kept_align=4)
+    ks = ctx.prune_counts(banks, b.sessions, params)
+    off = np.concatenate([[0], np.cumsum([(k + 3) // 4 * 4 for k in ks])]).astype(np.int64)
+    kept = torch.full((int(off[-1]),), -7, dtype=torch.int32, device=dev)
+    koff = torch.empty(b.sessions + 1, dtype=torch.int32, device=dev)
+    ctx.prune(banks, b.sessions, params, kept, koff)
+    assert koff.cpu().numpy().tolist() == off.tolist()
+    kept_h = kept.cpu().numpy()
+    for s in range(b.sessions):
+        sc = oracle.scores(np_view(b.queries[s]), np_view(keys[s].cpu()))
+        assert kept_h[off[s]:off[s] + ks[s]].tolist() == oracle.topk(sc, 37).tolist(), s
+        assert (kept_h[off[s] + ks[s]:off[s + 1]] == -7).all()  # padding untouched
+    sess = [pcs.bank_session(s, keys[s], vals[s], kept[int(off[s]):int(off[s]) + ks[s]])
+            for s in range(b.sessions)]
+    snaps = ctx.checkpoint(sess)
+    kdt = oracle.DT_F16 if b.keys.dtype == torch.float16 else oracle.DT_BF16
+    vdt = oracle.DT_BF16 if b.values.dtype == torch.bfloat16 else oracle.DT_U8
+    for s in range(b.sessions):
+        lo, hi = b.entry_off[s], b.entry_off[s + 1]
+        ref = oracle.pack(oracle.bank_session(s, np_view(b.keys[lo:hi]), np_view(b.values[lo:hi]),
+                                              np.ascontiguousarray(kept_h[off[s]:off[s] + ks[s]]),
+                                              kdt, vdt))
+        assert np.array_equal(ctx.record(snaps[s]).numpy(), ref), s
+        ctx.delete(snaps[s])
