@@ -1,6 +1,7 @@
 """Run one workload of the PCS hot path once (for profiling a single kernel).
 
     python profile_cases.py kv --sessions 8
+    python profile_cases.py suspend --sessions 8
     python profile_cases.py classify --n 200 --hi-mib 32
     python profile_cases.py prune --sessions 256
     python profile_cases.py markov --sessions 4096
@@ -52,6 +53,26 @@ def case_kv(ctx, a, dev):
 
     def step():
         hs = ctx.checkpoint_raw(src, kv.sessions)
+        ctx.restore_raw(hs, kv.sessions, dst, verify=2)
+        ctx.delete_raw(hs, kv.sessions)
+    return _timed(step, a.warmup)
+
+
+def case_suspend(ctx, a, dev):
+    """The KV sessions across the host link: checkpoint into records in
+    pinned host memory, then a verified restore from them into a freshly
+    permuted pool."""
+    kv = synth.kv(sessions=a.sessions, device=dev)
+    pt2 = synth.page_permutation(7, kv.sessions, kv.layers, kv.window // kv.page_rows, device=dev)
+    k2, v2, m2 = torch.empty_like(kv.k_pool), torch.empty_like(kv.v_pool), torch.empty_like(kv.meta)
+    src = ctx.session_array([pcs.kv_session(s, kv.meta[s], kv.k_pool, kv.v_pool, kv.page_table[s],
+                                            kv.ring_start[s], kv.window) for s in range(kv.sessions)])
+    dst = ctx.session_array([pcs.kv_session(s, m2[s], k2, v2, pt2[s],
+                                            pcs.PCS_RING_START_FROM_SNAPSHOT, kv.window)
+                             for s in range(kv.sessions)])
+
+    def step():
+        hs = ctx.checkpoint_raw(src, kv.sessions, pcs.PCS_PLACE_PINNED_HOST)
         ctx.restore_raw(hs, kv.sessions, dst, verify=2)
         ctx.delete_raw(hs, kv.sessions)
     return _timed(step, a.warmup)
@@ -230,7 +251,7 @@ def case_topk(ctx, a, dev):
     return _timed(lambda: ctx.topk(keys, na, ka, kept), a.warmup)
 
 
-CASES = {"kv": case_kv, "classify": case_classify, "prune": case_prune, "markov": case_markov,
+CASES = {"kv": case_kv, "suspend": case_suspend, "classify": case_classify, "prune": case_prune, "markov": case_markov,
          "markov_prepared": case_markov_prepared, "banks2": case_banks2,
          "markov_layouts": case_markov_layouts,
          "mismatch": case_mismatch, "prune_global": case_prune_global, "cow": case_cow,
