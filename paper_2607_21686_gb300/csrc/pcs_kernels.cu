@@ -69,12 +69,20 @@ __device__ __forceinline__ uint64_t comb(uint64_t a, uint64_t b) {
   return fmix(a * kP + rotl64(b, 31));
 }
 
+// A hint to bring the 128-byte line holding `p` into this SM's L1.
+__device__ __forceinline__ void prefetch_l1(const void* p) {
+  asm volatile("prefetch.global.L1 [%0];" ::"l"(p));
+}
+
 // Programmatic dependent launch (sm_90 and later).  The streaming, finalising,
 // scoring and top-k kernels are launched with programmatic stream
 // serialisation (launch_after), so the GPU may schedule one while the kernel
-// before it on the stream is still finishing.  Each begins here: wait until
-// that kernel has completed and its writes are visible, then let the next
-// kernel be scheduled.  Nothing before this point touches global memory.
+// before it on the stream is still finishing.  Each calls this before it
+// touches anything another kernel may write: wait until that kernel has
+// completed and its writes are visible, then let the next kernel be
+// scheduled.  Before this point a kernel reads only what the host wrote
+// before the launch (work lists and section, session and bank
+// descriptors), which no kernel writes.
 __device__ __forceinline__ void grid_dependency() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -608,6 +616,19 @@ __device__ __forceinline__ uint32_t issue_runs(const WarpStage& m, uint8_t* rp, 
   return static_cast<uint32_t>(b - a);
 }
 
+// Copy the descriptor of section `sec` into a stage (a whole warp; nothing
+// is read when the stage already holds it).
+__device__ __forceinline__ void stage_desc(const SecDesc* __restrict__ secs, uint32_t sec,
+                                           WarpStage& st, int lane) {
+  if (st.sec != sec) {  // warp-uniform
+    __syncwarp();
+    if (lane < static_cast<int>(sizeof(SecDesc) / 16))
+      reinterpret_cast<uint4*>(&st.d)[lane] = __ldg(reinterpret_cast<const uint4*>(secs + sec) + lane);
+    if (lane == 0) st.sec = sec;
+  }
+  __syncwarp();
+}
+
 // Stage tile t (of work list item `item`) into stage `st` / barrier `bar`.
 template <int MODE>
 __device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, const WorkList& wl,
@@ -616,13 +637,7 @@ __device__ __forceinline__ void stage_tile(const SecDesc* __restrict__ secs, con
   using T = ModeTraits<MODE>;
   const uint32_t sec = __ldg(wl.ids + item);
   const uint32_t loc = t - __ldg(wl.begin + item);
-  if (st.sec != sec) {  // warp-uniform
-    __syncwarp();
-    if (lane < static_cast<int>(sizeof(SecDesc) / 16))
-      reinterpret_cast<uint4*>(&st.d)[lane] = __ldg(reinterpret_cast<const uint4*>(secs + sec) + lane);
-    if (lane == 0) st.sec = sec;
-  }
-  __syncwarp();
+  stage_desc(secs, sec, st, lane);
   const SecDesc& s = st.d;
   const uint64_t L = s.bytes;
   const uint64_t p0 = static_cast<uint64_t>(loc) * kTileBytes;
@@ -780,7 +795,6 @@ template <int MODE>
 __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     k_bulk(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
            uint32_t* err) {
-  grid_dependency();
   constexpr int kBulkWarps = BulkShape<MODE>::kWarps;
   constexpr int kWarpStages = BulkShape<MODE>::kStages;
   extern __shared__ __align__(128) uint8_t smem_raw[];
@@ -801,7 +815,12 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
   const uint32_t t0 = static_cast<uint32_t>(T_all * gw / nw);
   const uint32_t t1 = static_cast<uint32_t>(T_all * (gw + 1) / nw);
   if (t0 >= t1) return;
+  // The work list and the descriptors are the host's, written before the
+  // launch: the first tile's item and section are found while the kernel
+  // ahead on the stream drains.
   int item = find_item(wl.begin, 0, wl.n_items, t0, lane);  // item of the next tile to stage
+  stage_desc(secs, __ldg(wl.ids + item), sh.st[warp][0], lane);
+  grid_dependency();
   auto item_of = [&](uint32_t t) {
     while (item + 1 < wl.n_items && __ldg(wl.begin + item + 1) <= t) ++item;
     return item;
@@ -847,7 +866,6 @@ template <int MODE>
 __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
     k_bulk_shared(const SecDesc* __restrict__ secs, WorkList wl, uint64_t* __restrict__ nodes,
                   uint32_t* err, uint32_t* sched) {
-  grid_dependency();
   constexpr int kBulkWarps = BulkShape<MODE>::kWarps;
   constexpr int kWarpStages = BulkShape<MODE>::kStages;
   extern __shared__ __align__(128) uint8_t smem_raw[];
@@ -872,6 +890,11 @@ __global__ void __launch_bounds__(BulkShape<MODE>::kThreads, 1)
   const uint32_t t1 = static_cast<uint32_t>(T_static * (gw + 1) / nw);
   uint32_t next = t0, chunk_end = t1;  // tiles [next, chunk_end) are this warp's
   int item = find_item(wl.begin, 0, wl.n_items, t0, lane);  // item of the last tile taken
+  // The work list and the descriptors are the host's: the first static
+  // tile's section is read before waiting for the kernel ahead.  The
+  // counters in `sched` are touched only after the wait.
+  if (t0 < t1) stage_desc(secs, __ldg(wl.ids + item), sh.st[warp][0], lane);
+  grid_dependency();
   // The next chunk, reserved ahead of need (where the warp would wait on a
   // stage anyway) so that neither the atomic nor the search of its item
   // delays a refill.
@@ -1170,9 +1193,22 @@ __global__ void __launch_bounds__(512)
     k_finalize_sessions(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
                         int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
                         uint8_t* corrupt, uint32_t* bad) {
-  grid_dependency();
   __shared__ uint64_t smem[kMaxSmemFps];
   __shared__ uint32_t s_bad;
+  // The host's descriptors of the block's first session (each warp's first
+  // section and, for a checkpoint, its table entry) are brought into L1
+  // while the kernel ahead on the stream drains.
+  if (static_cast<int>(blockIdx.x) < n_sess) {
+    const SessDesc* S0 = sess + blockIdx.x;
+    const uint32_t j = threadIdx.x >> 5;
+    if (j < __ldg(&S0->n_sections) && (threadIdx.x & 31) == 0) {
+      const uint32_t i = __ldg(&S0->sec_begin) + j;
+      prefetch_l1(secs + i);
+      prefetch_l1(reinterpret_cast<const uint8_t*>(secs + i) + sizeof(SecDesc) - 1);
+      if (MODE == kModePack) prefetch_l1(entries + i);
+    }
+  }
+  grid_dependency();
   finalize_sessions_block<MODE>(secs, sess, n_sess, entries, nodes, corrupt, bad, blockIdx.x,
                                 gridDim.x, smem, &s_bad);
 }
@@ -1184,25 +1220,37 @@ __global__ void __launch_bounds__(kThreads)
     k_finalize_sessions_warp(const SecDesc* __restrict__ secs, const SessDesc* __restrict__ sess,
                              int n_sess, const Entry* __restrict__ entries, uint64_t* nodes,
                              uint8_t* corrupt, uint32_t* bad) {
-  grid_dependency();
   const int lane = threadIdx.x & 31;
   const int nw = gridDim.x * kWarps;
-  for (int b = blockIdx.x * kWarps + (threadIdx.x >> 5); b < n_sess; b += nw) {
-    const SessDesc S = sess[b];
-    Entry* table = reinterpret_cast<Entry*>(S.record + kHeaderBytes);
-    const int ns = static_cast<int>(S.n_sections);
-    // Lane j reads section j's node range, length and (restore) stored fp,
-    // all sections at once; each section's tree then starts from its node
-    // loads, and a checkpoint's entry is read before the tree.
-    uint32_t fin_begin = 0, fin_count = 0;
-    uint64_t sec_bytes = 0, stored = 0;
-    if (lane < ns) {
+  // Lane j reads section j's node range and length, all sections at once.
+  // These are the host's descriptors: the warp's first session reads them
+  // while the kernel ahead on the stream drains.
+  SessDesc S;
+  uint32_t fin_begin = 0, fin_count = 0;
+  uint64_t sec_bytes = 0;
+  auto load_session = [&](int b) {
+    S = sess[b];
+    fin_begin = fin_count = 0;
+    sec_bytes = 0;
+    if (lane < static_cast<int>(S.n_sections)) {
       const SecDesc* sj = secs + S.sec_begin + lane;
       fin_begin = __ldg(&sj->fin_begin);
       fin_count = __ldg(&sj->fin_count);
       sec_bytes = __ldg(reinterpret_cast<const unsigned long long*>(&sj->bytes));
-      if (MODE != kModePack) stored = table[lane].fp;
     }
+  };
+  const int b_first = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (b_first < n_sess) load_session(b_first);
+  grid_dependency();
+  for (int b = b_first; b < n_sess; b += nw) {
+    if (b != b_first) load_session(b);
+    Entry* table = reinterpret_cast<Entry*>(S.record + kHeaderBytes);
+    const int ns = static_cast<int>(S.n_sections);
+    // A restore's stored fps (lane j: section j's), read once; each
+    // section's tree then starts from its node loads, and a checkpoint's
+    // entry is read before the tree.
+    uint64_t stored = 0;
+    if (MODE != kModePack && lane < ns) stored = table[lane].fp;
     uint64_t mine = 0;
     bool bad_sec = false;
     for (int j = 0; j < ns; ++j) {
