@@ -40,10 +40,10 @@ METRIC = "snapshot+restore GB/s and sessions/s on 1 GB300; % of HBM (PCIe) roofl
 # capture summarised in profiles/k_bulk_kv8x24_full.md (8 sessions, scaled by
 # sessions / 8), valid only for the streaming-kernel source it was taken on.
 NCU_TRAFFIC = {
-    "source_sha256_prefix": "453311c07109f60d",
+    "source_sha256_prefix": "82fadcb44e34aaa7",
     "sessions": 8,
-    "k_bulk<pack>": 805864960 + 754253312,
-    "k_bulk<restore_verify>": 805719808 + 754248960,
+    "k_bulk<pack>": 805706752 + 754244352,
+    "k_bulk<restore_verify>": 805732608 + 754476544,
 }
 
 
