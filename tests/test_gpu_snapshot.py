@@ -144,6 +144,35 @@ def test_bank_prune_ties_and_degenerate(ctx, dev):
         _check_prune(ctx, b, [keys.to(dev)], [q.to(dev)], p, dev)
 
 
+@pytest.mark.parametrize("largest", [512, 513])
+def test_prune_ties_at_every_bank_size(ctx, dev, largest):
+    """Relevance pruning where every threshold falls in a run of exact ties:
+    banks of 0, 1, 2, 31, 32, 33, 255, 511 and `largest` entries drawn from a
+    few distinct keys, with zero keys (score 0) and negated queries (negative
+    scores) among them; k from 0 to past n, and a fraction.  Scores, kept
+    sets and offsets equal the oracle's."""
+    D = 128
+    g = torch.Generator().manual_seed(largest)
+    sizes = [0, 1, 2, 31, 32, 33, 255, 511, largest, 0, 7]
+    q = [torch.randn(D, generator=g).half() for _ in sizes]
+    keys = []
+    for i, n in enumerate(sizes):
+        pool = torch.randn(5, D, generator=g).half()
+        pool[1] = 0
+        pool[2] = -q[i]
+        pick = torch.randint(0, 5, (n,), generator=g)
+        keys.append(pool[pick])
+    n_tot = sum(sizes)
+    b = synth.Banks(n=sizes, entry_off=np.concatenate([[0], np.cumsum(sizes)]).tolist(),
+                    keys=torch.cat(keys), values=torch.zeros(n_tot, 16, dtype=torch.uint8),
+                    queries=torch.stack(q), key_dim=D, value_bytes=16)
+    kd = [x.to(dev) for x in keys]
+    qd = [x.to(dev) for x in q]
+    for k in [0, 1, 2, 17, 32, 100, 256, 511, 600]:
+        _check_prune(ctx, b, kd, qd, ctx.params(pcs.PCS_K_FIXED, k_max=k), dev)
+    _check_prune(ctx, b, kd, qd, ctx.params(pcs.PCS_K_FRACTION, fraction=0.37), dev)
+
+
 def _bank_round_trip(ctx, b, dev, params, placement):
     keys, vals, qs = _bank_views(b, dev)
     ks, kept, koff = _check_prune(ctx, b, keys, qs, params, dev)
