@@ -3,6 +3,7 @@
 // device once per call; no torch types.
 #pragma once
 
+#include <atomic>
 #include <cstdint>
 
 #include <cuda_runtime.h>

@@ -2936,19 +2936,21 @@ cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, 
                              uint32_t* sched, int sm_count, cudaStream_t stream) {
   using Shape = BulkShape<MODE>;
   const size_t smem = sizeof(BulkShared<Shape::kWarps, Shape::kStages>);
-  static uint64_t configured = 0;  // one bit per device (callers hold the context lock)
+  // One bit per device.  Contexts on other threads may set the attribute at
+  // the same time; setting it twice is harmless.
+  static std::atomic<uint64_t> configured{0};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
-  if (!(configured & bit)) {
+  if (!(configured.load(std::memory_order_acquire) & bit)) {
     e = cudaFuncSetAttribute(k_bulk<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(k_bulk_shared<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    configured |= bit;
+    configured.fetch_or(bit, std::memory_order_release);
   }
   const uint64_t want = (static_cast<uint64_t>(wl.n_tasks) + Shape::kWarps - 1) / Shape::kWarps;
   const int blocks = static_cast<int>(want < static_cast<uint64_t>(sm_count) ? want : sm_count);
