@@ -127,7 +127,6 @@ cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_
 // ordered.  (Hash mode runs k_hash and does not use them.)
 cudaError_t launch_bulk(int mode, const SecDesc* secs, WorkList wl, uint64_t* nodes,
                         uint32_t* dev_err, uint32_t* sched, int sm_count, cudaStream_t stream);
-size_t bulk_shared_bytes();
 
 // One launch for a small call: the register streaming pass over wl (no
 // node reduction), then the finaliser of `mode` run by the last block to

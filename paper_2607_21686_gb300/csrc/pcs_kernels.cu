@@ -2964,8 +2964,6 @@ cudaError_t launch_bulk_mode(const SecDesc* secs, WorkList wl, uint64_t* nodes, 
 
 int stream_blocks_per_sm() { return occupancy<kModePack>(); }
 
-size_t bulk_shared_bytes() { return sizeof(BulkShared<BulkShape<kModePack>::kWarps, BulkShape<kModePack>::kStages>); }
-
 cudaError_t launch_stream(int mode, const SecDesc* secs, WorkList wl, int group_log2,
                           uint64_t* nodes, uint32_t* dev_err, int sm_count, int blocks_per_sm,
                           cudaStream_t stream) {
