@@ -321,6 +321,90 @@ class Arena {
   std::map<void*, void*> host_of_;
 };
 
+// A set of pointers in one open-addressed table (linear probing, erased
+// slots marked): no allocation per insert, and a membership test never
+// dereferences the pointer it is asked about, so any value a caller passes
+// as a handle can be checked.
+template <class T>
+class PtrSet {
+ public:
+  size_t size() const { return n_; }
+  bool count(const T* p) const {
+    if (slot_.empty() || !p) return false;
+    const uintptr_t k = reinterpret_cast<uintptr_t>(p);
+    for (size_t i = hash(k) & mask();; i = (i + 1) & mask()) {
+      if (slot_[i] == k) return true;
+      if (slot_[i] == kEmpty) return false;
+    }
+  }
+  void reserve(size_t n) {
+    if ((used_ + n) * 2 > slot_.size()) rehash(n_ + n);
+  }
+  void insert(T* p) {
+    reserve(1);
+    const uintptr_t k = reinterpret_cast<uintptr_t>(p);
+    size_t gone = SIZE_MAX;
+    for (size_t i = hash(k) & mask();; i = (i + 1) & mask()) {
+      if (slot_[i] == k) return;
+      if (slot_[i] == kGone && gone == SIZE_MAX) gone = i;
+      if (slot_[i] == kEmpty) {
+        if (gone != SIZE_MAX) {
+          i = gone;
+        } else {
+          ++used_;
+        }
+        slot_[i] = k;
+        ++n_;
+        return;
+      }
+    }
+  }
+  bool erase(const T* p) {
+    if (slot_.empty() || !p) return false;
+    const uintptr_t k = reinterpret_cast<uintptr_t>(p);
+    for (size_t i = hash(k) & mask();; i = (i + 1) & mask()) {
+      if (slot_[i] == k) {
+        slot_[i] = kGone;
+        --n_;
+        return true;
+      }
+      if (slot_[i] == kEmpty) return false;
+    }
+  }
+  template <class F>
+  void for_each(F f) const {
+    for (uintptr_t k : slot_)
+      if (k != kEmpty && k != kGone) f(reinterpret_cast<T*>(k));
+  }
+  void clear() {
+    slot_.clear();
+    n_ = used_ = 0;
+  }
+
+ private:
+  static constexpr uintptr_t kEmpty = 0, kGone = 1;  // never valid object addresses
+  std::vector<uintptr_t> slot_;  // a power of two of slots, at most half in use
+  size_t n_ = 0, used_ = 0;      // live entries; live + erased slots
+  size_t mask() const { return slot_.size() - 1; }
+  static size_t hash(uintptr_t x) {
+    uint64_t z = static_cast<uint64_t>(x);
+    z ^= z >> 33;
+    z *= 0xFF51AFD7ED558CCDull;  // MurmurHash3's 64-bit finaliser constant
+    z ^= z >> 33;
+    return static_cast<size_t>(z);
+  }
+  void rehash(size_t want) {
+    size_t cap = 16;
+    while (cap < want * 2 + 2) cap <<= 1;
+    std::vector<uintptr_t> old;
+    old.swap(slot_);
+    slot_.assign(cap, kEmpty);
+    n_ = used_ = 0;
+    for (uintptr_t k : old)
+      if (k != kEmpty && k != kGone) insert(reinterpret_cast<T*>(k));
+  }
+};
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -334,7 +418,12 @@ struct pcs_snapshot {
   uint64_t payload_start = 0;
   uint32_t session_id = 0;
   uint32_t kind = 0;
-  std::vector<Entry> table;    // host copy of the section table (fp = 0)
+  // Host copy of the section table (fp = 0): n_sections entries from
+  // `first` of an array shared by the snapshots of one call and their forks.
+  std::shared_ptr<const std::vector<Entry>> tables;
+  uint32_t first = 0;
+  uint32_t n_sections = 0;
+  const Entry* table() const { return tables->data() + first; }
   uint8_t* record() const { return block->ptr + offset; }
 };
 
@@ -354,7 +443,8 @@ struct pcs_ctx {
   std::mutex mu;
   std::shared_ptr<EventPool> events = std::make_shared<EventPool>();
   std::unique_ptr<Arena> dev_arena, host_arena;
-  std::unordered_set<pcs_snapshot*> live;
+  PtrSet<pcs_snapshot> live;
+  std::vector<pcs_snapshot*> spare;  // deleted handles' objects, for the next ones
   // Workspaces, one per stream: the descriptors and tree nodes of a call,
   // after a header of per-call device words ([0] the fused kernel's ticket,
   // [1] failures of a verify = 1 restore, [4] and [5] the TMA kernel's work
@@ -1120,8 +1210,27 @@ cudaError_t launch_streams(pcs_ctx* c, int mode, const SecDesc* dsecs, const Str
 }
 
 pcs_snapshot* check_handle(pcs_ctx* c, const pcs_snapshot* h) {
-  auto* p = const_cast<pcs_snapshot*>(h);
-  return c->live.count(p) ? p : nullptr;
+  return c->live.count(h) ? const_cast<pcs_snapshot*>(h) : nullptr;
+}
+
+// Handle objects: a deleted handle's object serves the next snapshot (calls
+// on thousands of sessions make and drop that many handles each).
+constexpr size_t kMaxSpareHandles = 1 << 20;
+
+std::unique_ptr<pcs_snapshot> new_snapshot(pcs_ctx* c) {
+  if (c->spare.empty()) return std::make_unique<pcs_snapshot>();
+  pcs_snapshot* h = c->spare.back();
+  c->spare.pop_back();
+  return std::unique_ptr<pcs_snapshot>(h);
+}
+
+void drop_snapshot(pcs_ctx* c, pcs_snapshot* h) {
+  *h = pcs_snapshot{};
+  if (c->spare.size() < kMaxSpareHandles) {
+    c->spare.push_back(h);
+  } else {
+    delete h;
+  }
 }
 
 // A checkpoint or a restore, planned: the descriptors (host bytes, uploaded
@@ -1245,21 +1354,23 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
   if (st) return st;
   std::vector<SecDesc> d;
   std::vector<SessDesc> sd(n);
-  std::vector<Entry> ent;
+  auto ent_shared = std::make_shared<std::vector<Entry>>();
+  std::vector<Entry>& ent = *ent_shared;  // the section tables of every record
   d.reserve(total_secs);
   ent.reserve(total_secs);
   handles->resize(n);
   for (int s = 0; s < n; ++s) {
     const pcs_session& S = sessions[s];
     uint8_t* rec = blk->ptr + rec_off[s];
-    auto h = std::make_unique<pcs_snapshot>();
+    auto h = new_snapshot(c);
     h->block = blk;
     h->offset = rec_off[s];
     h->total_bytes = rec_off[s + 1] - rec_off[s];
     h->payload_start = pstart[s];
     h->session_id = S.session_id;
     h->kind = S.kind;
-    h->table.reserve(S.n_sections);
+    h->first = static_cast<uint32_t>(ent.size());
+    h->n_sections = static_cast<uint32_t>(S.n_sections);
     sd[s].record = rec;
     sd[s].total_bytes = h->total_bytes;
     sd[s].payload_start = pstart[s];
@@ -1284,11 +1395,11 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
       e.dim1 = x.dim1;
       e.aux = x.layout == PCS_LAYOUT_RING ? x.ring_start : 0;
       ent.push_back(e);
-      h->table.push_back(e);
       off = round_up(off + x.bytes, kRecordAlign);
     }
     (*handles)[s] = std::move(h);
   }
+  for (auto& h : *handles) h->tables = ent_shared;
   PtrCache cache;
   std::vector<char> bulk(d.size());
   const bool small = total_bytes(d) <= kSmallCallBytes;
@@ -1338,13 +1449,17 @@ pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
   std::vector<SecDesc> d;
   std::vector<SessDesc> sd(n);
   std::vector<char> payload_dev;
+  uint64_t want = 0;
+  for (int s = 0; s < n; ++s) want += targets[s].n_sections > 0 ? targets[s].n_sections : 0;
+  d.reserve(std::min<uint64_t>(want, 1ull << 24));
+  payload_dev.reserve(d.capacity());
   for (int s = 0; s < n; ++s) {
     pcs_snapshot* h = check_handle(c, snaps[s]);
     if (!h) return fail(PCS_E_HANDLE, "snapshot %d: unknown handle", s);
     const pcs_session& T = targets[s];
-    if (T.n_sections != static_cast<int32_t>(h->table.size()) || !T.sections)
+    if (T.n_sections != static_cast<int32_t>(h->n_sections) || !T.sections)
       return fail(PCS_E_INVAL, "session %d: target has %d sections, snapshot %zu", s,
-                  T.n_sections, h->table.size());
+                  T.n_sections, h->n_sections);
     sd[s].record = h->record();
     sd[s].total_bytes = h->total_bytes;
     sd[s].payload_start = h->payload_start;
@@ -1356,7 +1471,7 @@ pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
       const pcs_section& x = T.sections[i];
       pcs_status st = check_section(x, s, i, true);
       if (st) return st;
-      const Entry& e = h->table[i];
+      const Entry& e = h->table()[i];
       if (x.bytes != e.bytes)
         return fail(PCS_E_INVAL, "session %d section %d: target bytes %llu != snapshot %llu", s, i,
                     static_cast<unsigned long long>(x.bytes), static_cast<unsigned long long>(e.bytes));
@@ -1467,11 +1582,13 @@ pcs_status pcs_destroy(pcs_ctx* c) {
     std::lock_guard<std::mutex> lk(c->mu);
     cudaSetDevice(c->device);
     cudaDeviceSynchronize();
-    for (auto* h : c->live) {
+    c->live.for_each([&](pcs_snapshot* h) {
       release_block(c, h->block);
       delete h;
-    }
+    });
     c->live.clear();
+    for (auto* h : c->spare) delete h;
+    c->spare.clear();
     for (auto* pl : c->pools) {
       cudaFree(pl->meta);
       delete pl;
@@ -2132,7 +2249,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   st = ws_release(c, stream, blk->written);
   if (st) return undo(st);
   blk->refs = n;
-  c->live.reserve(c->live.size() + n);
+  c->live.reserve(n);
   for (int s = 0; s < n; ++s) {
     out[s] = handles[s].release();
     c->live.insert(out[s]);
@@ -2223,10 +2340,11 @@ pcs_status pcs_fork_many(pcs_ctx* c, pcs_snapshot* const* parents, int32_t n,
     blk[pl]->written = done;
     blk[pl]->refs = 0;
   }
-  c->live.reserve(c->live.size() + n);
+  c->live.reserve(n);
   for (int i = 0; i < n; ++i) {
     Block* b = blk[parents[i]->block->placement];
-    auto h = std::make_unique<pcs_snapshot>(*parents[i]);
+    auto h = new_snapshot(c);
+    *h = *parents[i];
     h->block = b;
     h->offset = off[i];
     b->refs += 1;
@@ -2317,7 +2435,7 @@ pcs_status pcs_plan_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t 
   blk->written = record_event(c->events, stream);
   blk->refs = n + 1;  // the snapshots and the plan
   p->blocks.push_back(blk);
-  c->live.reserve(c->live.size() + n);
+  c->live.reserve(n);
   for (int s = 0; s < n; ++s) {
     out[s] = handles[s].release();
     c->live.insert(out[s]);
@@ -2410,7 +2528,7 @@ pcs_status pcs_delete(pcs_ctx* c, pcs_snapshot* h) {
   if (!check_handle(c, h)) return fail(PCS_E_HANDLE, "unknown snapshot handle");
   c->live.erase(h);
   release_block(c, h->block);
-  delete h;
+  drop_snapshot(c, h);
   return PCS_OK;
 }
 
@@ -2424,7 +2542,7 @@ pcs_status pcs_delete_many(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n) {
     pcs_snapshot* h = snaps[i];
     if (!c->live.erase(h)) return fail(PCS_E_HANDLE, "snapshot %d: listed twice", i);
     release_block(c, h->block);
-    delete h;
+    drop_snapshot(c, h);
   }
   return PCS_OK;
 }
@@ -2448,7 +2566,7 @@ pcs_status pcs_snapshot_get_info(pcs_ctx* c, const pcs_snapshot* snap, pcs_snaps
   if (st) return st;
   out->session_id = h->session_id;
   out->kind = h->kind;
-  out->n_sections = static_cast<int32_t>(h->table.size());
+  out->n_sections = static_cast<int32_t>(h->n_sections);
   out->placement = h->block->placement;
   out->total_bytes = h->total_bytes;
   std::memcpy(&out->session_fp, hdr + 24, 8);
@@ -2462,7 +2580,7 @@ pcs_status pcs_snapshot_get_section(pcs_ctx* c, const pcs_snapshot* snap, int32_
   std::lock_guard<std::mutex> lk(c->mu);
   pcs_snapshot* h = check_handle(c, snap);
   if (!h) return fail(PCS_E_HANDLE, "unknown snapshot handle");
-  if (i < 0 || i >= static_cast<int32_t>(h->table.size()))
+  if (i < 0 || i >= static_cast<int32_t>(h->n_sections))
     return fail(PCS_E_INVAL, "section %d out of range", i);
   pcs_status st = set_device(c);
   if (st) return st;
@@ -2622,15 +2740,16 @@ pcs_status pcs_snapshot_read_file(pcs_ctx* c, const char* path, uint32_t placeme
   }
   std::fclose(f);
   blk->refs = 1;
-  auto h = std::make_unique<pcs_snapshot>();
+  auto h = new_snapshot(c);
   h->block = blk;
   h->offset = 0;
   h->total_bytes = total;
   h->payload_start = pstart;
   h->session_id = sid;
   h->kind = kind;
-  h->table = table;
-  for (auto& e : h->table) e.fp = 0;
+  for (auto& e : table) e.fp = 0;
+  h->n_sections = static_cast<uint32_t>(table.size());
+  h->tables = std::make_shared<const std::vector<Entry>>(std::move(table));
   *out = h.release();
   c->live.insert(*out);
   return PCS_OK;
