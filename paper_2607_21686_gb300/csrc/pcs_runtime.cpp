@@ -611,12 +611,13 @@ constexpr uint64_t kPlanSlotBytes = 256 << 10;  // smallest pinned plan slot
 constexpr uint64_t kPlanSlotMax = 64ull << 20;  // larger plans are copied from pageable memory
 constexpr int kPlanSlots = 8;
 
-// Copy the call's descriptors (c->plan, `bytes`) into the workspace.  Plans
-// go through a pinned slot (round robin over kPlanSlots), reusable once the
-// call that last used it has passed its end event; a slot too small for the
-// plan is replaced by a larger one.  When the slot is still busy, or the plan
-// is huge, it is copied from pageable memory.
-cudaError_t plan_copy(pcs_ctx* c, uint8_t* ws, uint64_t bytes, cudaStream_t stream) {
+// A free pinned plan slot for `bytes` of descriptors (round robin over
+// kPlanSlots, grown to the largest plan it carries), which the call then
+// holds until ws_release records its end -- a call that fails before then
+// leaves the slot held for good, never reused early; null when the next slot
+// is still busy or the plan is huge.
+uint8_t* plan_slot(pcs_ctx* c, uint64_t bytes) {
+  c->plan_slot_used = -1;
   if (bytes <= kPlanSlotMax) {
     const int i = c->plan_slot;
     Ev& busy = c->plan_slot_busy[i];
@@ -636,19 +637,36 @@ cudaError_t plan_copy(pcs_ctx* c, uint8_t* ws, uint64_t bytes, cudaStream_t stre
         }
       }
       if (c->plan_slot_buf[i]) {
-        uint8_t* slot = c->plan_slot_buf[i];
-        std::memcpy(slot, c->plan.data(), bytes);
         c->plan_slot = (i + 1) % kPlanSlots;
-        // Held until ws_release records the call's end; a call that fails
-        // before then leaves the slot held for good (never reused early).
         busy = std::make_shared<Event>();
         c->plan_slot_used = i;
-        return cudaMemcpyAsync(ws, slot, bytes, cudaMemcpyHostToDevice, stream);
+        return c->plan_slot_buf[i];
       }
     }
   }
-  c->plan_slot_used = -1;
-  return cudaMemcpyAsync(ws, c->plan.data(), bytes, cudaMemcpyHostToDevice, stream);
+  return nullptr;
+}
+
+// Where a call writes `bytes` of descriptors: a pinned plan slot, else
+// `fallback` (pageable memory).
+uint8_t* plan_dst(pcs_ctx* c, uint64_t bytes, std::vector<uint8_t>& fallback) {
+  if (uint8_t* slot = plan_slot(c, bytes)) return slot;
+  fallback.resize(bytes);
+  return fallback.data();
+}
+
+// Send descriptors written where plan_dst said into the workspace.
+cudaError_t plan_send(pcs_ctx* c, uint8_t* ws, uint64_t bytes,
+                        const std::vector<uint8_t>& fallback, cudaStream_t stream) {
+  const uint8_t* src = c->plan_slot_used >= 0 ? c->plan_slot_buf[c->plan_slot_used] : fallback.data();
+  return cudaMemcpyAsync(ws, src, bytes, cudaMemcpyHostToDevice, stream);
+}
+
+// Copy the call's descriptors (c->plan, `bytes`) into the workspace, through
+// a pinned slot when one is free.
+cudaError_t plan_copy(pcs_ctx* c, uint8_t* ws, uint64_t bytes, cudaStream_t stream) {
+  if (uint8_t* slot = plan_slot(c, bytes)) std::memcpy(slot, c->plan.data(), bytes);
+  return plan_send(c, ws, bytes, c->plan, stream);
 }
 
 // End of a call's use of the workspace (and of its plan slot): `done`, if
@@ -1095,16 +1113,23 @@ ListLayout list_layout(const StreamPlan& P, uint64_t base) {
 }
 
 template <class T>
+void put(uint8_t* plan, uint64_t off, const std::vector<T>& v) {
+  if (!v.empty()) std::memcpy(plan + off, v.data(), v.size() * sizeof(T));
+}
+template <class T>
 void put(std::vector<uint8_t>& plan, uint64_t off, const std::vector<T>& v) {
-  if (!v.empty()) std::memcpy(plan.data() + off, v.data(), v.size() * sizeof(T));
+  put(plan.data(), off, v);
 }
 
-void put_lists(std::vector<uint8_t>& plan, const StreamPlan& P, const ListLayout& L) {
+void put_lists(uint8_t* plan, const StreamPlan& P, const ListLayout& L) {
   put(plan, L.bulk_ids, P.bulk_ids);
   put(plan, L.bulk_begin, P.bulk_begin);
   put(plan, L.reg_ids, P.reg_ids);
   put(plan, L.reg_begin, P.reg_begin);
   put(plan, L.levels, P.levels);
+}
+void put_lists(std::vector<uint8_t>& plan, const StreamPlan& P, const ListLayout& L) {
+  put_lists(plan.data(), P, L);
 }
 
 // Launch both streaming kernels of a plan (TMA-staged first).
@@ -1247,6 +1272,15 @@ struct Prepared {
   std::vector<uint8_t> plan;
 };
 
+// The bytes [0, L.nodes) of a plan's descriptors: a plain call writes them
+// straight into a pinned plan slot (one copy less; plan_send then sends
+// them), a prepared call into pr->plan, which it keeps.
+uint8_t* plan_target(pcs_ctx* c, Prepared* pr, bool to_slot) {
+  if (to_slot) return plan_dst(c, pr->L.nodes, pr->plan);
+  pr->plan.resize(pr->L.nodes);
+  return pr->plan.data();
+}
+
 }  // namespace
 
 // A prepared call: its descriptors in a device buffer of its own, and one
@@ -1328,7 +1362,8 @@ cudaError_t launch_prepared(pcs_ctx* c, const Prepared& pr, uint8_t* ws, uint32_
 // descriptors.  On failure nothing is left reserved.
 pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, uint32_t placement,
                             cudaStream_t stream, Prepared* pr, Block** blk_out,
-                            std::vector<std::unique_ptr<pcs_snapshot>>* handles) {
+                            std::vector<std::unique_ptr<pcs_snapshot>>* handles,
+                            bool to_slot = false) {
   if (placement != PCS_PLACE_DEVICE && placement != PCS_PLACE_PINNED_HOST)
     return fail(PCS_E_INVAL, "unknown placement %u", placement);
   // Plan records: sizes, offsets, entries.
@@ -1434,18 +1469,19 @@ pcs_status build_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, 
   pr->LL = list_layout(pr->P, L.entries + sizeof(Entry) * ent.size());
   L.nodes = round_up(pr->LL.end, kRecordAlign);
   L.total = L.nodes + 8 * pr->P.nodes_total;
-  pr->plan.resize(L.nodes);
-  put(pr->plan, L.secs, d);
-  put(pr->plan, L.sess, sd);
-  put(pr->plan, L.entries, ent);
-  put_lists(pr->plan, pr->P, pr->LL);
+  uint8_t* dst = plan_target(c, pr, to_slot);
+  put(dst, L.secs, d);
+  put(dst, L.sess, sd);
+  put(dst, L.entries, ent);
+  put_lists(dst, pr->P, pr->LL);
   *blk_out = blk;
   return PCS_OK;
 }
 
 // Plan a restore of n snapshots into n target sessions.
 pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
-                         const pcs_session* targets, int verify, Prepared* pr) {
+                         const pcs_session* targets, int verify, Prepared* pr,
+                         bool to_slot = false) {
   std::vector<SecDesc> d;
   std::vector<SessDesc> sd(n);
   std::vector<char> payload_dev;
@@ -1514,10 +1550,10 @@ pcs_status build_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n,
   pr->LL = list_layout(pr->P, L.sess + sizeof(SessDesc) * n);
   L.nodes = round_up(pr->LL.end, kRecordAlign);
   L.total = L.nodes + (verify ? 8 * pr->P.nodes_total : 0);
-  pr->plan.resize(L.nodes);
-  put(pr->plan, L.secs, d);
-  put(pr->plan, L.sess, sd);
-  put_lists(pr->plan, pr->P, pr->LL);
+  uint8_t* dst = plan_target(c, pr, to_slot);
+  put(dst, L.secs, d);
+  put(dst, L.sess, sd);
+  put_lists(dst, pr->P, pr->LL);
   return PCS_OK;
 }
 
@@ -2231,7 +2267,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   Prepared pr;
   Block* blk = nullptr;
   std::vector<std::unique_ptr<pcs_snapshot>> handles;
-  st = build_checkpoint(c, sessions, n, placement, stream, &pr, &blk, &handles);
+  st = build_checkpoint(c, sessions, n, placement, stream, &pr, &blk, &handles, true);
   if (st) return st;
   auto undo = [&](pcs_status s) {
     arena_of(c, placement)->free(blk);
@@ -2240,9 +2276,7 @@ pcs_status pcs_checkpoint(pcs_ctx* c, const pcs_session* sessions, int32_t n, ui
   uint8_t* ws = nullptr;
   st = ws_acquire(c, pr.L.total, stream, &ws);
   if (st) return undo(st);
-  c->plan.swap(pr.plan);
-  cudaError_t e = plan_copy(c, ws, pr.L.nodes, stream);
-  c->plan.swap(pr.plan);
+  cudaError_t e = plan_send(c, ws, pr.L.nodes, pr.plan, stream);
   if (e == cudaSuccess) e = launch_prepared(c, pr, ws, c->call_words, stream);
   if (e != cudaSuccess) return undo(cuda_fail(e, "checkpoint launch"));
   blk->written = record_event(c->events, stream);
@@ -2372,7 +2406,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   pcs_status st = set_device(c);
   if (st) return st;
   Prepared pr;
-  st = build_restore(c, snaps, n, targets, verify, &pr);
+  st = build_restore(c, snaps, n, targets, verify, &pr, true);
   if (st) return st;
   for (int s = 0; s < n; ++s) {
     if (s > 0 && snaps[s]->block == snaps[s - 1]->block) continue;  // one wait per run of a block
@@ -2382,10 +2416,7 @@ pcs_status pcs_restore(pcs_ctx* c, pcs_snapshot* const* snaps, int32_t n, const 
   uint8_t* ws = nullptr;
   st = ws_acquire(c, pr.L.total, stream, &ws);
   if (st) return st;
-  c->plan.swap(pr.plan);
-  cudaError_t e = plan_copy(c, ws, pr.L.nodes, stream);
-  c->plan.swap(pr.plan);
-  PCS_CUDA(e);
+  PCS_CUDA(plan_send(c, ws, pr.L.nodes, pr.plan, stream));
   // verify == 1: count failures of this call in words[1] and wait for them;
   // verify == 2: accumulate them in words[2] for the next pcs_sync.
   uint32_t* words = c->call_words;
