@@ -782,6 +782,7 @@ SecDesc make_desc(const pcs_section& s, uint8_t* payload, uint32_t ring_start) {
 struct PtrCache {
   std::vector<std::pair<uintptr_t, uintptr_t>> dev;
   std::unordered_map<const void*, bool> other;
+  size_t last = 0;  // the range that answered last (sections of a call share a few)
 };
 
 // cuMemGetAddressRange, looked up once through the runtime (no libcuda link).
@@ -806,8 +807,15 @@ AddrRangeFn addr_range_fn() {
 bool is_device_ptr(const void* p, PtrCache& cache) {
   if (!p) return true;
   const uintptr_t u = reinterpret_cast<uintptr_t>(p);
-  for (const auto& r : cache.dev)
-    if (u >= r.first && u < r.second) return true;
+  if (cache.last < cache.dev.size() && u >= cache.dev[cache.last].first &&
+      u < cache.dev[cache.last].second)
+    return true;
+  for (size_t i = 0; i < cache.dev.size(); ++i) {
+    if (u >= cache.dev[i].first && u < cache.dev[i].second) {
+      cache.last = i;
+      return true;
+    }
+  }
   auto it = cache.other.find(p);
   if (it != cache.other.end()) return it->second;
   cudaPointerAttributes a{};
@@ -894,8 +902,15 @@ uint64_t total_bytes(const std::vector<SecDesc>& d) {
 bool plan_streams(const pcs_ctx* c, std::vector<SecDesc>& d, const std::vector<char>& bulk,
                   StreamPlan& P, bool allow_reduce = true) {
   uint64_t reg_chunks = 0;
-  for (size_t i = 0; i < d.size(); ++i)
+  size_t n_bulk = 0;
+  for (size_t i = 0; i < d.size(); ++i) {
     if (!bulk[i]) reg_chunks += d[i].n_chunks;
+    n_bulk += bulk[i] ? 1 : 0;
+  }
+  P.bulk_ids.reserve(n_bulk);
+  P.bulk_begin.reserve(n_bulk);
+  P.reg_ids.reserve(d.size() - n_bulk);
+  P.reg_begin.reserve(d.size() - n_bulk);
   P.glog2 = choose_group_log2(c, reg_chunks);
   uint64_t node = 0, tb = 0, tr = 0;
   for (size_t i = 0; i < d.size(); ++i) {
