@@ -42,3 +42,43 @@ def test_delete_while_restore_pending_then_reuse_on_other_stream(ctx, dev):
         assert ctx.section(b, 0).fp == oracle.fingerprint(np_bytes(z))
         ctx.delete(b)
         y.zero_()
+
+
+def test_many_handles_in_random_order(ctx, dev):
+    """Thousands of live handles made by several calls and forks, deleted in
+    a random order between further calls: the live count, each surviving
+    handle's info and record, and the refusal of handles that were never
+    made all hold while handle objects are reused."""
+    import ctypes
+    rnd = np.random.default_rng(5)
+    base = ctx.stats().live_snapshots
+    t = torch.arange(64, dtype=torch.uint8, device=dev)
+    arr = ctx.session_array([_sess(t, sid=s) for s in range(3000)])
+    live = {}
+    for rounds in range(4):
+        hs = ctx.checkpoint_raw(arr, 3000)
+        kids = ctx.fork_raw(hs, 3000)
+        for i in range(3000):
+            live[hs[i]] = i
+            live[kids[i]] = i
+        ctx.sync()
+        assert ctx.stats().live_snapshots == base + len(live)
+        doomed = rnd.choice(sorted(live), size=len(live) // 2, replace=False)
+        batch = (ctypes.c_void_p * len(doomed))(*[int(h) for h in doomed])
+        ctx.delete_raw(batch, len(doomed))
+        for h in doomed:
+            del live[int(h)]
+        assert ctx.stats().live_snapshots == base + len(live)
+    for h in rnd.choice(sorted(live), size=50, replace=False):
+        snap = pcs.Snapshot(ctx, int(h))
+        assert ctx.info(snap).session_id == live[int(h)]
+        assert ctx.info(snap).n_sections == 1
+        off = ctx.section(snap, 0).offset
+        assert np.array_equal(ctx.record(snap).numpy()[off:off + 64], np.arange(64, dtype=np.uint8))
+    for bad in (8, 1 << 40, max(live) + 8):
+        with pytest.raises(pcs.PcsError) as e:
+            ctx.info(pcs.Snapshot(ctx, bad))
+        assert e.value.status == pcs.PCS_E_HANDLE
+    rest = sorted(live)
+    ctx.delete_raw((ctypes.c_void_p * len(rest))(*rest), len(rest))
+    assert ctx.stats().live_snapshots == base
