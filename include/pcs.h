@@ -604,7 +604,10 @@ pcs_status pcs_plan_run(pcs_ctx *ctx, pcs_plan *plan, void *stream);
 pcs_status pcs_plan_destroy(pcs_ctx *ctx, pcs_plan *plan);
 
 /* delete(c) (Sec. 3 "The contract"): release a snapshot (its memory is
- * reused once pending work that reads it has finished). */
+ * reused once pending work that reads it has finished).  The handle is
+ * invalid afterwards: a call given it returns PCS_E_HANDLE until a later
+ * checkpoint, fork or read issues the same handle value again (handle
+ * objects are reused), after which it names that new snapshot. */
 pcs_status pcs_delete(pcs_ctx *ctx, pcs_snapshot *snap);
 
 /* delete(c) (Sec. 3 "The contract") for n snapshots at once; PCS_E_HANDLE
